@@ -1,0 +1,229 @@
+/*
+ * msi.h -- C ABI of the slot-addressed MoE layer forward for GB300 (sm_103a).
+ *
+ * The library runs the data-parallel hot path of storage-backed MoE inference
+ * from "Memory-Sovereign Inference: Output-Exact Execution Beyond Full
+ * Residency": a Plan maps each logical (layer, expert) object to a byte extent
+ * in pinned host windows and to a reusable GPU slot with a stable address and
+ * a generation (Sec. "A Shared Cross-Adapter Plan Core"); experts are staged
+ * window -> slot asynchronously and published per generation (Sec. "Stable
+ * Slots and Bundle Publication"; Sec. "Implementation", "Scheduling and
+ * copies"); the layer forward routes tokens (fp32 router, softmax, top-k),
+ * groups them per expert, runs each selected expert's complete gate, up and
+ * down projections from its slot, and combines the weighted results
+ * (Sec. "Output-Exact Execution Beyond the Full-Residency Envelope").  A
+ * generation mismatch fails closed: nothing stale becomes visible
+ * (Sec. "Lifetime Is Part of Correctness").
+ *
+ * Conventions
+ *  - Every call returns msi_status; nothing is thrown across the ABI.
+ *  - The caller owns every device and pinned host buffer passed in (slot pool,
+ *    host windows, hidden rows, outputs, route-event buffers, workspace).  A
+ *    plan owns only host metadata, CUDA events and a few device words per slot
+ *    (the published generation and object of each slot).
+ *  - Streams are cudaStream_t values passed as msi_stream; 0 is the legacy
+ *    default stream.  Calls on one plan must come from one host thread at a
+ *    time; forwards of one plan are meant to be issued on one compute stream.
+ *  - Layouts: hidden rows bf16 row-major [T, H]; router weight fp32 [E, H];
+ *    a bf16 expert extent is W13 [2I, H] (rows 0..I-1 gate, I..2I-1 up, each
+ *    row K-contiguous) followed by W2 [H, I] (K-contiguous); a 4-bit extent is
+ *    W13 codes [2I, H/2] | W2 codes [H, I/2] | W13 fp16 scales [2I, H/32] |
+ *    W2 fp16 scales [H, I/32], code q -> scale * (q - 8), even column in the
+ *    low nibble.
+ *  - Shape limits of this build: E <= 512, 1 <= k <= min(E, 32), H a multiple
+ *    of 256, I a multiple of 128, T >= 0.  Other shapes return
+ *    MSI_ERR_UNSUPPORTED.
+ */
+#ifndef MSI_H_
+#define MSI_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* msi_stream; /* a cudaStream_t */
+
+typedef enum {
+  MSI_OK = 0,
+  MSI_ERR_INVALID_ARG = 1,       /* bad pointer, index, size or shape */
+  MSI_ERR_STALE_GENERATION = 2,  /* expected generation differs from the published one */
+  MSI_ERR_WRONG_OBJECT = 3,      /* the slot holds a different (layer, expert) object */
+  MSI_ERR_SLOT_BUSY = 4,         /* a live consumer still holds the slot */
+  MSI_ERR_NOT_RESIDENT = 5,      /* a needed expert has no slot */
+  MSI_ERR_TIMEOUT = 6,           /* a bounded host or device wait ran out */
+  MSI_ERR_CUDA = 7,              /* a CUDA runtime call failed (see msi_last_cuda_error) */
+  MSI_ERR_SHUT_DOWN = 8,         /* the plan is being destroyed */
+  MSI_ERR_UNSUPPORTED = 9,       /* shape outside this build's limits */
+  MSI_ERR_WORKSPACE = 10         /* workspace missing, misaligned or too small */
+} msi_status;
+
+enum { MSI_W_BF16 = 0, MSI_W_Q4G32 = 1 };
+
+enum { MSI_TRACE_HIT = 0, MSI_TRACE_STAGE = 1, MSI_TRACE_EVICT = 2 };
+
+/* GPU slot lifecycle states (Sec. "Separate Window and GPU-Slot Lifecycles"). */
+enum {
+  MSI_SLOT_VACANT = 0,        /* holds no object */
+  MSI_SLOT_LOADING = 1,       /* copy enqueued, readiness event not yet reached */
+  MSI_SLOT_DEVICE_READY = 2,  /* published, never consumed */
+  MSI_SLOT_IN_USE = 3,        /* a consumer (forward or caller ticket) is live */
+  MSI_SLOT_RECYCLABLE = 4     /* published and every consumer finished */
+};
+
+/* Forward flags. */
+enum {
+  MSI_FWD_RESIDUAL = 1  /* out = x + moe(x), rounded once to bf16 (decode stacks) */
+};
+
+/* Plan description (copied by msi_plan_create; pointers must outlive the plan). */
+typedef struct {
+  int n_layers;                 /* layers whose experts the plan manages (>= 1) */
+  int n_experts;                /* E routed experts per layer */
+  int top_k;                    /* k */
+  int hidden;                   /* H */
+  int inter;                    /* I, routed and shared expert intermediate size */
+  int has_shared;               /* 1: one always-resident shared expert per layer */
+  int wdtype;                   /* MSI_W_BF16 or MSI_W_Q4G32 (routed experts) */
+  int n_slots;                  /* S >= 2 GPU slots */
+  void* slot_pool;              /* device, S * extent_bytes, 128-byte aligned, caller-owned */
+  uint64_t extent_bytes;        /* must equal msi_extent_bytes(hidden, inter, wdtype) */
+  const void* host_windows;     /* pinned host memory holding the canonical extents */
+  const uint64_t* extent_off;   /* host [n_layers * E] byte offset of object (l, e) in
+                                   host_windows; NULL: (l * E + e) * extent_bytes */
+  const void* shared_w;         /* device, n_layers bf16 extents of the shared experts,
+                                   128-byte aligned (NULL when has_shared == 0) */
+  const float* shared_gate_w;   /* device fp32 [n_layers, H] shared-expert gate vectors */
+  int wave_capacity;            /* experts per LRU wave; 0: n_slots / 2 */
+  double wait_timeout_s;        /* bound on host waits for held consumers; 0: 1.0 s */
+} msi_plan_desc;
+
+typedef struct msi_plan msi_plan; /* opaque, owned by the library */
+
+/* Route event of one layer call (device buffers, caller-owned).  This is the
+ * router's top-k output recorded per layer and graph evaluation (Sec.
+ * "Output-Exact Execution Beyond the Full-Residency Envelope"). */
+typedef struct {
+  int32_t* ids;      /* [T, k] expert ids, descending logit, ties -> lower id */
+  float* weights;    /* [T, k] softmax over the selected k logits (sum to 1) */
+  int32_t* counts;   /* [E] routed rows per expert */
+  float* gap;        /* [T] logit of rank k-1 minus logit of rank k (+inf if k == E); may be NULL */
+} msi_route_event;
+
+/* One slot-trace record (telemetry of cache events and generations, Sec.
+ * "Implementation", "Telemetry").  call and wave are -1 for msi_slot_stage. */
+typedef struct {
+  uint64_t seq;
+  int32_t call, layer, expert, slot;
+  uint64_t generation;  /* new generation for STAGE; held generation for HIT and EVICT */
+  int32_t kind;         /* MSI_TRACE_* */
+  int32_t wave;
+} msi_trace_rec;
+
+/* Plan telemetry counters. */
+typedef struct {
+  uint64_t forwards, streamed_forwards, stages, hits, evicts;
+  uint64_t h2d_bytes;            /* extent bytes copied window -> slot */
+  uint64_t rejections;           /* host prechecks and device checks that failed closed */
+} msi_counters;
+
+/* Bytes of one expert extent for the given shape and weight type (0 on bad input). */
+uint64_t msi_extent_bytes(int hidden, int inter, int wdtype);
+
+/* Create a plan: validates the description, copies the manifest, creates the
+ * per-slot generation words (all slots Vacant, generation 0) and the TMA
+ * descriptors over the slot pool.  Needs a current CUDA device. */
+msi_status msi_plan_create(const msi_plan_desc* desc, msi_plan** out);
+
+/* Destroy a plan.  Fails with MSI_ERR_SLOT_BUSY (and destroys nothing) while a
+ * caller-held consumer ticket is live; otherwise drains all staging and
+ * forwards issued through the plan, then frees it (reset/shutdown drain,
+ * Sec. "Separate Window and GPU-Slot Lifecycles"). */
+msi_status msi_plan_destroy(msi_plan* plan);
+
+/* Device workspace bytes msi_moe_forward / msi_moe_forward_streamed need for T
+ * tokens.  The workspace is caller-owned, 256-byte aligned, and must not be
+ * shared by forwards that may run concurrently. */
+msi_status msi_workspace_size(const msi_plan* plan, int T, size_t* bytes);
+
+/* Stage object (layer, expert) into `slot`, asynchronously on `stage`:
+ * waits (on the GPU) for the slot's last consumer, invalidates the slot's
+ * published generation, copies the extent from the host window, publishes the
+ * new generation (old + 1) and records the slot's readiness event.  Returns
+ * MSI_ERR_TIMEOUT with nothing enqueued if a caller-held consumer ticket on the
+ * slot is not released within wait_timeout_s (no reuse before the last
+ * consumer, Sec. "Separate Window and GPU-Slot Lifecycles"). */
+msi_status msi_slot_stage(msi_plan* plan, int slot, int layer, int expert, msi_stream stage,
+                          uint64_t* new_generation);
+
+/* The plan's ledger for one layer: slot_of_expert[e] (-1 if not resident) and
+ * the generation published there (0 if not resident).  Host arrays [E]. */
+msi_status msi_slot_table(const msi_plan* plan, int layer, int32_t* slot_of_expert,
+                          uint64_t* gen_of_expert);
+
+/* Current lifecycle state of one slot (MSI_SLOT_*), derived from the ledger,
+ * its readiness and consumer events and caller-held tickets. */
+msi_status msi_slot_state(const msi_plan* plan, int slot, int* state);
+
+/* Layer forward over caller-managed residency (every needed expert already
+ * staged).  slot_table and expected_generations are host arrays [E]
+ * (slot -1: not resident).  Host precheck: if some e with slot_table[e] >= 0
+ * names a slot whose ledger object is not (layer, e) or whose generation is
+ * not expected_generations[e], nothing is enqueued and WRONG_OBJECT /
+ * STALE_GENERATION is returned for the lowest such e.  Device re-check: the
+ * forward re-reads the published generation of every needed expert's slot;
+ * on mismatch (or a needed expert without slot) no expert output and no `out`
+ * row is written, and msi_forward_status reports the failure.  Route events
+ * are always written (routing precedes the Plan).  Asynchronous on `compute`.
+ * hidden: device bf16 [T, H]; router_w: device fp32 [E, H]; out: device bf16
+ * [T, H]. */
+msi_status msi_moe_forward(msi_plan* plan, int layer, const void* hidden, int T,
+                           const float* router_w, const int32_t* slot_table,
+                           const uint64_t* expected_generations, void* out,
+                           const msi_route_event* ev, void* workspace, size_t workspace_bytes,
+                           unsigned flags, msi_stream compute);
+
+/* Layer forward with plan-managed residency (LRU waves).  Routes on `compute`,
+ * reads the per-expert counts back to the host (one synchronisation), then
+ * processes the needed experts as hits then misses in waves of wave_capacity:
+ * misses are staged on `stage` into victims chosen by least-recent use (slots
+ * of the current and previous wave pinned), each wave published by one event
+ * and consumed by the grouped expert FFN on `compute` while the next wave is
+ * staged.  Every hit, stage and eviction is appended to the slot trace.
+ * Returns after enqueueing the last wave and the combine. */
+msi_status msi_moe_forward_streamed(msi_plan* plan, int layer, const void* hidden, int T,
+                                    const float* router_w, void* out, const msi_route_event* ev,
+                                    void* workspace, size_t workspace_bytes, unsigned flags,
+                                    msi_stream compute, msi_stream stage);
+
+/* Wait for the most recent forward of the plan and return its device-side
+ * status (an msi_status value; MSI_OK when every needed expert passed the
+ * generation re-check and every bounded device wait completed). */
+msi_status msi_forward_status(msi_plan* plan, int* device_status);
+
+/* Host-side consumer tickets: a caller that reads slots outside a forward
+ * holds the slot while reading.  Staging into a held slot waits, bounded. */
+msi_status msi_consumer_hold(msi_plan* plan, int slot);
+msi_status msi_consumer_release(msi_plan* plan, int slot);
+
+/* Copy up to `cap` trace records (oldest first) into buf; *n receives the
+ * number copied.  msi_trace_clear empties the trace. */
+msi_status msi_trace_read(const msi_plan* plan, msi_trace_rec* buf, size_t cap, size_t* n);
+msi_status msi_trace_clear(msi_plan* plan);
+
+msi_status msi_get_counters(const msi_plan* plan, msi_counters* out);
+
+/* Number of kernels the library launched since the plan was created. */
+uint64_t msi_kernel_launches(const msi_plan* plan);
+
+/* Text of a status code; text of the last CUDA error seen by the library. */
+const char* msi_status_string(msi_status s);
+const char* msi_last_cuda_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MSI_H_ */

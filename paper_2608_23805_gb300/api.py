@@ -1,0 +1,175 @@
+"""Convenience wrapper over the C ABI for PyTorch callers.
+
+PyTorch supplies device memory, pinned host memory and streams; every step of
+the MoE layer forward runs in libmsi.so's CUDA kernels.  This module only
+marshals tensors into pointers and checks status codes.
+"""
+from __future__ import annotations
+
+import ctypes
+
+import numpy as np
+import torch
+
+from . import native as N
+
+
+def _ptr(t) -> int | None:
+    return None if t is None else t.data_ptr()
+
+
+def _stream(s) -> int | None:
+    s = torch.cuda.current_stream() if s is None else s
+    return s.cuda_stream
+
+
+class RouteEvent:
+    """Device buffers of one layer call's route event."""
+
+    def __init__(self, T: int, k: int, E: int, device="cuda"):
+        self.ids = torch.empty((T, k), dtype=torch.int32, device=device)
+        self.weights = torch.empty((T, k), dtype=torch.float32, device=device)
+        self.counts = torch.empty((E,), dtype=torch.int32, device=device)
+        self.gap = torch.empty((T,), dtype=torch.float32, device=device)
+        self.c = N.msi_route_event(_ptr(self.ids) if T else None, _ptr(self.weights) if T else None,
+                                   _ptr(self.counts), _ptr(self.gap) if T else None)
+
+
+class Plan:
+    """A Plan over one slot pool (see include/msi.h, msi_plan_desc)."""
+
+    def __init__(self, *, n_layers, n_experts, top_k, hidden, inter, n_slots, host_windows,
+                 has_shared=False, shared_w=None, shared_gate_w=None, wdtype=N.MSI_W_BF16,
+                 slot_pool=None, extent_off=None, wave_capacity=0, wait_timeout_s=0.0):
+        lib = N.lib()
+        self.E, self.k, self.H, self.I = n_experts, top_k, hidden, inter
+        self.n_layers, self.S = n_layers, n_slots
+        self.extent_bytes = int(lib.msi_extent_bytes(hidden, inter, wdtype))
+        if self.extent_bytes == 0:
+            raise ValueError("bad shape")
+        if slot_pool is None:
+            slot_pool = torch.empty(n_slots * self.extent_bytes, dtype=torch.uint8, device="cuda")
+        self._keep = [host_windows, slot_pool, shared_w, shared_gate_w]
+        self.slot_pool = slot_pool
+        self._off = None
+        if extent_off is not None:
+            self._off = np.ascontiguousarray(extent_off, dtype=np.uint64)
+        d = N.msi_plan_desc()
+        d.n_layers, d.n_experts, d.top_k = n_layers, n_experts, top_k
+        d.hidden, d.inter, d.has_shared, d.wdtype, d.n_slots = hidden, inter, int(has_shared), wdtype, n_slots
+        d.slot_pool = slot_pool.data_ptr()
+        d.extent_bytes = self.extent_bytes
+        d.host_windows = host_windows.data_ptr()
+        d.extent_off = self._off.ctypes.data if self._off is not None else None
+        d.shared_w = _ptr(shared_w)
+        d.shared_gate_w = _ptr(shared_gate_w)
+        d.wave_capacity = wave_capacity
+        d.wait_timeout_s = wait_timeout_s
+        h = ctypes.c_void_p()
+        N.check(lib.msi_plan_create(ctypes.byref(d), ctypes.byref(h)), "msi_plan_create")
+        self.h = h
+        self._ws = {}
+
+    # -- residency ---------------------------------------------------------
+    def stage(self, slot: int, layer: int, expert: int, stream=None) -> int:
+        g = ctypes.c_uint64()
+        N.check(N.lib().msi_slot_stage(self.h, slot, layer, expert, _stream(stream), ctypes.byref(g)),
+                "msi_slot_stage")
+        return g.value
+
+    def slot_table(self, layer: int):
+        st = np.empty(self.E, dtype=np.int32)
+        gt = np.empty(self.E, dtype=np.uint64)
+        N.check(N.lib().msi_slot_table(self.h, layer, st.ctypes.data, gt.ctypes.data), "msi_slot_table")
+        return st, gt
+
+    def slot_state(self, slot: int) -> int:
+        s = ctypes.c_int()
+        N.check(N.lib().msi_slot_state(self.h, slot, ctypes.byref(s)), "msi_slot_state")
+        return s.value
+
+    def hold(self, slot: int):
+        N.check(N.lib().msi_consumer_hold(self.h, slot), "msi_consumer_hold")
+
+    def release(self, slot: int):
+        N.check(N.lib().msi_consumer_release(self.h, slot), "msi_consumer_release")
+
+    # -- forward -------------------------------------------------------------
+    def workspace(self, T: int) -> torch.Tensor:
+        n = ctypes.c_size_t()
+        N.check(N.lib().msi_workspace_size(self.h, T, ctypes.byref(n)), "msi_workspace_size")
+        ws = self._ws.get("buf")
+        if ws is None or ws.numel() < n.value:
+            ws = torch.empty(max(n.value, 256), dtype=torch.uint8, device="cuda")
+            self._ws["buf"] = ws
+        return ws
+
+    def forward(self, layer, x, router_w, slot_table, expected, out=None, ev=None, residual=False,
+                stream=None, check=True):
+        T = x.shape[0]
+        out = torch.empty_like(x) if out is None else out
+        ev = RouteEvent(T, self.k, self.E) if ev is None else ev
+        ws = self.workspace(T)
+        st = np.ascontiguousarray(slot_table, dtype=np.int32)
+        ex = np.ascontiguousarray(expected, dtype=np.uint64)
+        rc = N.lib().msi_moe_forward(self.h, layer, _ptr(x), T, _ptr(router_w), st.ctypes.data,
+                                     ex.ctypes.data, _ptr(out), ctypes.byref(ev.c), _ptr(ws),
+                                     ws.numel(), N.MSI_FWD_RESIDUAL if residual else 0, _stream(stream))
+        if check:
+            N.check(rc, "msi_moe_forward")
+            return out, ev
+        return rc, out, ev
+
+    def forward_streamed(self, layer, x, router_w, out=None, ev=None, residual=False, stream=None,
+                         stage_stream=None, check=True):
+        T = x.shape[0]
+        out = torch.empty_like(x) if out is None else out
+        ev = RouteEvent(T, self.k, self.E) if ev is None else ev
+        ws = self.workspace(T)
+        rc = N.lib().msi_moe_forward_streamed(self.h, layer, _ptr(x), T, _ptr(router_w), _ptr(out),
+                                              ctypes.byref(ev.c), _ptr(ws), ws.numel(),
+                                              N.MSI_FWD_RESIDUAL if residual else 0, _stream(stream),
+                                              _stream(stage_stream))
+        if check:
+            N.check(rc, "msi_moe_forward_streamed")
+            return out, ev
+        return rc, out, ev
+
+    def status(self) -> int:
+        s = ctypes.c_int()
+        N.check(N.lib().msi_forward_status(self.h, ctypes.byref(s)), "msi_forward_status")
+        return s.value
+
+    # -- telemetry -------------------------------------------------------------
+    def trace(self, clear: bool = False):
+        """Slot trace as (call, layer, expert, slot, generation, kind, wave) tuples."""
+        cap = 1 << 20
+        buf = (N.msi_trace_rec * cap)()
+        n = ctypes.c_size_t()
+        N.check(N.lib().msi_trace_read(self.h, buf, cap, ctypes.byref(n)), "msi_trace_read")
+        kinds = {N.MSI_TRACE_HIT: "hit", N.MSI_TRACE_STAGE: "stage", N.MSI_TRACE_EVICT: "evict"}
+        out = [(r.call, r.layer, r.expert, r.slot, int(r.generation), kinds[r.kind], r.wave)
+               for r in buf[:n.value]]
+        if clear:
+            N.check(N.lib().msi_trace_clear(self.h), "msi_trace_clear")
+        return out
+
+    def counters(self) -> dict:
+        c = N.msi_counters()
+        N.check(N.lib().msi_get_counters(self.h, ctypes.byref(c)), "msi_get_counters")
+        return {f: getattr(c, f) for f, _ in c._fields_}
+
+    def launches(self) -> int:
+        return int(N.lib().msi_kernel_launches(self.h))
+
+    def close(self):
+        if getattr(self, "h", None) is not None and self.h.value:
+            N.check(N.lib().msi_plan_destroy(self.h), "msi_plan_destroy")
+            self.h = None
+
+    def __del__(self):
+        try:
+            if getattr(self, "h", None) is not None and self.h.value:
+                N.lib().msi_plan_destroy(self.h)
+        except Exception:
+            pass

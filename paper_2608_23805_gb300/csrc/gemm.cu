@@ -1,0 +1,342 @@
+// Grouped expert GEMMs on tcgen05 tensor cores (sm_103a).
+//
+// Each selected expert runs its complete gate, up and down projections
+// (paper, Sec. "Output-Exact Execution Beyond the Full-Residency Envelope"),
+// reading its weights from the stable address of the GPU slot the Plan
+// published for it (Sec. "Stable Slots and Bundle Publication").
+//
+// One persistent kernel per projection pair:
+//   gate-up (kGateUpGather / kGateUpTma):  h = silu(x Wg^T) * (x Wu^T)   -> bf16
+//   down    (kDown):                        y = h W2^T                     -> bf16
+// Tile: 128 token rows x 256 weight rows x 64 K per stage, 4-stage smem ring,
+// fp32 accumulators double-buffered in TMEM (2 x 256 columns).  Weights (B)
+// come by TMA from the slot pool viewed as one 2-D tensor per operand; the
+// routed token rows (A) of the gate-up GEMM are gathered through the
+// permutation with cp.async into the same 128-byte-swizzled layout TMA
+// writes; the down GEMM's A (h, already in permuted order) comes by TMA.
+//
+// Roles (warp-specialised):  warps 0-3 epilogue (TMEM -> registers -> global,
+// one token row per thread), warp 4 MMA issue + TMEM allocation, warp 5 TMA
+// producer, warps 6-9 row gather (gather mode only).  Every wait is bounded;
+// on expiry the CTA raises its abort flag, all roles drain and the kernel
+// reports MSI_ERR_TIMEOUT in the status word.
+#include "internal.cuh"
+
+namespace msi {
+
+namespace {
+
+constexpr int kEpiWarps = 4;
+constexpr int kGatherWarps = 4;
+constexpr int kLag = 2;  // gather stages in flight before signalling
+constexpr uint32_t kIdesc = idesc_bf16(kBM, kBN);
+
+template <int MODE>
+struct Cfg {
+  static constexpr bool kGather = (MODE == kGateUpGather);
+  static constexpr bool kTmaA = !kGather;
+  static constexpr bool kGateUp = (MODE != kDown);
+  static constexpr int kThreads = (6 + (kGather ? kGatherWarps : 0)) * 32;
+  static constexpr uint32_t kTxBytes = kBBytes + (kTmaA ? kABytes : 0);
+};
+
+struct TileCoord {
+  int g, m, n;
+};
+
+__device__ __forceinline__ TileCoord decode_tile(const GemmArgs& a, int t) {
+  int lo = 0, hi = a.num_groups - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (__ldg(&a.groups[mid].mt_begin) * a.nt <= t) lo = mid; else hi = mid - 1;
+  }
+  const int cnt = __ldg(&a.groups[lo].row_count);
+  const int mt = (cnt + kBM - 1) / kBM;
+  const int local = t - __ldg(&a.groups[lo].mt_begin) * a.nt;
+  TileCoord c;
+  c.g = lo;
+  c.n = local / mt;
+  c.m = local - c.n * mt;
+  return c;
+}
+
+}  // namespace
+
+int gemm_smem_bytes() {
+  return 1024 /* alignment slack */ + kStages * (kABytes + kBBytes) + 256 /* barriers */;
+}
+
+template <int MODE>
+__global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
+    grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA,
+                        const __grid_constant__ CUtensorMap tmB, const GemmArgs a) {
+  using C = Cfg<MODE>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + kStages * kABytes;
+  uint64_t* full = reinterpret_cast<uint64_t*>(sB + kStages * kBBytes);
+  uint64_t* empty = full + kStages;
+  uint64_t* tfull = empty + kStages;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* drain = tempty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&full[s], 1 + (C::kGather ? kGatherWarps : 0));
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&tfull[b], 1);
+      mbar_init(&tempty[b], kEpiWarps);
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    mbar_fence_init();
+  }
+  if (warp == 4) {
+    tmem_alloc(tmem_slot, 512);
+    tmem_relinquish();
+  }
+  if (warp == 5 && lane == 0) {
+    tma_prefetch(&tmB);
+    if (C::kTmaA) tma_prefetch(&tmA);
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  const int total = __ldg(a.total_mtiles) * a.nt;
+  const long long lim = a.wait_limit;
+
+  if (warp == 5) {
+    // ------------------------------------------------------------- TMA producer
+    if (lane == 0) {
+      uint32_t it = 0;
+      for (int t = blockIdx.x; t < total; t += gridDim.x) {
+        const TileCoord tc = decode_tile(a, t);
+        const Group* G = &a.groups[tc.g];
+        const int brow = __ldg(&G->slot) * a.b_rows_per_slot + a.b_row_off;
+        const int arow = __ldg(&G->row_begin) + tc.m * kBM;
+        bool ok = true;
+        for (int kb = 0; kb < a.kblocks; ++kb, ++it) {
+          const int s = it % kStages;
+          const uint32_t ph = (it / kStages) & 1;
+          if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, lim)) { ok = false; break; }
+          mbar_arrive_expect_tx(&full[s], C::kTxBytes);
+          uint8_t* b = sB + s * kBBytes;
+          if (C::kGateUp) {
+            tma_load_2d(b, &tmB, &full[s], kb * kBK, brow + tc.n * 128);
+            tma_load_2d(b + kBBytes / 2, &tmB, &full[s], kb * kBK, brow + a.up_off + tc.n * 128);
+          } else {
+            tma_load_2d(b, &tmB, &full[s], kb * kBK, brow + tc.n * kBN);
+            tma_load_2d(b + kBBytes / 2, &tmB, &full[s], kb * kBK, brow + tc.n * kBN + 128);
+          }
+          if (C::kTmaA) tma_load_2d(sA + s * kABytes, &tmA, &full[s], kb * kBK, arow);
+        }
+        if (!ok) break;
+      }
+      // On abort, wait (bounded) for the copies this thread armed to land
+      // before the CTA's shared memory is released.
+      if (*abort_flag) {
+        for (int d = 0; d < kStages && it > 0; ++d) {
+          const uint32_t j = it - 1 - d;
+          if ((int)j < 0) break;
+          const long long t0 = clock64();
+          while (!mbar_try_wait(&full[j % kStages], (j / kStages) & 1) && clock64() - t0 < lim) {
+          }
+        }
+      }
+    }
+  } else if (warp == 4) {
+    // ------------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      uint32_t it = 0, jt = 0;
+      for (int t = blockIdx.x; t < total; t += gridDim.x, ++jt) {
+        const uint32_t acc = jt & 1, aph = (jt >> 1) & 1;
+        if (!mbar_wait(&tempty[acc], aph ^ 1, abort_flag, lim)) break;
+        tc_fence_after();
+        const uint32_t d = tmem_base + acc * kBN;
+        bool ok = true;
+        for (int kb = 0; kb < a.kblocks; ++kb, ++it) {
+          const int s = it % kStages;
+          const uint32_t ph = (it / kStages) & 1;
+          if (!mbar_wait(&full[s], ph, abort_flag, lim)) { ok = false; break; }
+          tc_fence_after();
+          const uint64_t ad = sw128_desc(smem_u32(sA + s * kABytes));
+          const uint64_t bd = sw128_desc(smem_u32(sB + s * kBBytes));
+#pragma unroll
+          for (int k = 0; k < kBK / 16; ++k) {
+            // advance 16 bf16 (32 bytes) along K inside the 128-byte swizzle atom
+            umma_bf16(d, ad + 2 * k, bd + 2 * k, kIdesc, (kb | k) != 0);
+          }
+          umma_commit(&empty[s]);
+        }
+        if (!ok) break;
+        umma_commit(&tfull[acc]);
+      }
+      // every MMA this thread issued has completed before TMEM is released
+      umma_commit(drain);
+      const long long t0 = clock64();
+      while (!mbar_try_wait(drain, 0) && clock64() - t0 < lim) {
+      }
+    }
+  } else if (warp < kEpiWarps) {
+    // ------------------------------------------------------------- epilogue
+    uint32_t jt = 0;
+    const int r = warp * 32 + lane;
+    for (int t = blockIdx.x; t < total; t += gridDim.x, ++jt) {
+      const TileCoord tc = decode_tile(a, t);
+      const Group* G = &a.groups[tc.g];
+      const int cnt = __ldg(&G->row_count);
+      const bool valid = tc.m * kBM + r < cnt;
+      const size_t orow = (size_t)__ldg(&G->row_begin) + (size_t)tc.m * kBM + r;
+      const uint32_t acc = jt & 1, aph = (jt >> 1) & 1;
+      if (!mbar_wait(&tfull[acc], aph, abort_flag, lim)) break;
+      tc_fence_after();
+      const uint32_t tb = tmem_base + ((uint32_t)(warp * 32) << 16) + acc * kBN;
+      if (C::kGateUp) {
+        __nv_bfloat16* dst = a.out + orow * a.out_ld + tc.n * 128;
+#pragma unroll 1
+        for (int c = 0; c < 128; c += 16) {
+          uint32_t g[16], u[16];
+          tmem_ld16(tb + c, g);
+          tmem_ld16(tb + 128 + c, u);
+          tmem_ld_wait(g);
+          tmem_ld_wait(u);
+          uint32_t p[8];
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const float g0 = __uint_as_float(g[2 * i]), g1 = __uint_as_float(g[2 * i + 1]);
+            const float u0 = __uint_as_float(u[2 * i]), u1 = __uint_as_float(u[2 * i + 1]);
+            const float h0 = g0 / (1.0f + __expf(-g0)) * u0;
+            const float h1 = g1 / (1.0f + __expf(-g1)) * u1;
+            p[i] = pack_bf16x2(h0, h1);
+          }
+          if (valid) {
+            uint4* o = reinterpret_cast<uint4*>(dst + c);
+            o[0] = make_uint4(p[0], p[1], p[2], p[3]);
+            o[1] = make_uint4(p[4], p[5], p[6], p[7]);
+          }
+        }
+      } else {
+        __nv_bfloat16* dst = a.out + orow * a.out_ld + tc.n * kBN;
+#pragma unroll 1
+        for (int c = 0; c < kBN; c += 16) {
+          uint32_t v[16];
+          tmem_ld16(tb + c, v);
+          tmem_ld_wait(v);
+          uint32_t p[8];
+#pragma unroll
+          for (int i = 0; i < 8; ++i)
+            p[i] = pack_bf16x2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1]));
+          if (valid) {
+            uint4* o = reinterpret_cast<uint4*>(dst + c);
+            o[0] = make_uint4(p[0], p[1], p[2], p[3]);
+            o[1] = make_uint4(p[4], p[5], p[6], p[7]);
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&tempty[acc]);
+    }
+  } else if (C::kGather) {
+    // ------------------------------------------------------------- row gather
+    const int gt = threadIdx.x - 6 * 32;  // 0..127
+    const int chunk = gt & 7;             // 16-byte chunk of a 128-byte row slice
+    const int r0 = gt >> 3;               // rows r0 + 16 i
+    uint32_t it = 0, arrived = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+      const TileCoord tc = decode_tile(a, t);
+      const Group* G = &a.groups[tc.g];
+      const int cnt = __ldg(&G->row_count);
+      const int rb = __ldg(&G->row_begin);
+      const __nv_bfloat16* src[8];
+      uint32_t nbytes[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const int rr = tc.m * kBM + r0 + 16 * i;
+        if (rr < cnt) {
+          const int tok = __ldg(&a.perm[rb + rr]) / a.top_k;
+          src[i] = a.x + (size_t)tok * a.x_ld + chunk * 8;
+          nbytes[i] = 16;
+        } else {
+          src[i] = a.x;
+          nbytes[i] = 0;  // zero-fill rows past the expert's segment
+        }
+      }
+      for (int kb = 0; kb < a.kblocks; ++kb, ++it) {
+        const int s = it % kStages;
+        const uint32_t ph = (it / kStages) & 1;
+        if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, lim)) { ok = false; break; }
+        uint8_t* dstA = sA + s * kABytes;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const int rr = r0 + 16 * i;
+          cp_async16(dstA + rr * 128 + ((chunk ^ (rr & 7)) << 4), src[i] + kb * kBK, nbytes[i]);
+        }
+        cp_async_commit();
+        if (it + 1 - arrived > kLag) {
+          cp_async_wait<kLag>();
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&full[arrived % kStages]);
+          ++arrived;
+        }
+      }
+    }
+    cp_async_wait<0>();
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (ok) {
+      while (arrived < it) {
+        if (lane == 0) mbar_arrive(&full[arrived % kStages]);
+        ++arrived;
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 4) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem_base, 512);
+  }
+  if (threadIdx.x == 0 && *abort_flag) atomicCAS(a.status, 0, (int)MSI_ERR_TIMEOUT);
+}
+
+template <int MODE>
+static cudaError_t launch_mode(const CUtensorMap& tmA, const CUtensorMap& tmB, const GemmArgs& a,
+                               int grid, cudaStream_t s) {
+  static bool attr_done = false;
+  const int smem = gemm_smem_bytes();
+  if (!attr_done) {
+    cudaError_t e = cudaFuncSetAttribute(grouped_gemm_kernel<MODE>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    attr_done = true;
+  }
+  grouped_gemm_kernel<MODE><<<grid, Cfg<MODE>::kThreads, smem, s>>>(tmA, tmB, a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gemm(int mode, const CUtensorMap& tmA, const CUtensorMap& tmB, const GemmArgs& a,
+                        int grid, cudaStream_t s) {
+  switch (mode) {
+    case kGateUpGather: return launch_mode<kGateUpGather>(tmA, tmB, a, grid, s);
+    case kGateUpTma: return launch_mode<kGateUpTma>(tmA, tmB, a, grid, s);
+    case kDown: return launch_mode<kDown>(tmA, tmB, a, grid, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace msi

@@ -1,0 +1,348 @@
+// Internal declarations shared by the library's translation units: device
+// structs, PTX wrappers for sm_103a (mbarrier, TMA, tcgen05, cp.async) and the
+// kernel launchers.  Nothing here is part of the public C ABI (include/msi.h).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/msi.h"
+
+namespace msi {
+
+// ---------------------------------------------------------------------------
+// Limits of this build
+// ---------------------------------------------------------------------------
+constexpr int kMaxExperts = 512;
+constexpr int kMaxTopK = 32;
+constexpr int kMaxWave = 256;
+
+// ---------------------------------------------------------------------------
+// Device-side records
+// ---------------------------------------------------------------------------
+
+// Published identity of one slot: written on the staging stream after the
+// extent copy (obj = 0 while a copy is in flight or the slot is vacant).
+struct GenWord {
+  unsigned long long gen;
+  unsigned long long obj;  // ((layer + 1) << 32) | expert
+};
+
+__host__ __device__ inline unsigned long long obj_key(int layer, int expert) {
+  return ((unsigned long long)(layer + 1) << 32) | (unsigned)expert;
+}
+
+// One expert group of a grouped GEMM launch.
+struct Group {
+  int row_begin;   // first permuted row
+  int row_count;   // rows routed to the expert
+  int slot;        // weight block index in the B tensor maps
+  int mt_begin;    // prefix of 128-row tiles over the preceding groups
+  int ok;          // generation re-check passed
+  int expert;
+  int pad0, pad1;
+};
+
+// ---------------------------------------------------------------------------
+// Kernel argument blocks
+// ---------------------------------------------------------------------------
+
+struct RouterArgs {
+  const __nv_bfloat16* x;  // [T, H]
+  const float* wr;         // [E, H]
+  const float* wsg;        // [H] or nullptr
+  int T, H, E, k;
+  int* ids;                // [T, k]
+  float* weights;          // [T, k]
+  float* gap;              // [T] or nullptr
+  float* sg;               // [T] (when wsg)
+  int* bcount;             // [nb, E] routed ids per router block and expert
+};
+
+struct ScanArgs {
+  const int* bcount;
+  int nb, E;
+  int* bbase;    // [nb, E] exclusive prefix over blocks within each expert
+  int* counts;   // [E]
+};
+
+struct ScatterArgs {
+  const int* ids;     // [T*k]
+  const int* counts;  // [E]
+  const int* bbase;   // [nb, E]
+  int T, k, E, nb;
+  int* perm;          // [T*k]
+  int* inv;           // [T*k]
+  int* offsets;       // [E+1]
+};
+
+// Per-call tables uploaded by value (kernel parameters, < 32 KB).
+struct TableParams {
+  int E;
+  int layer;
+  int T;
+  int shared_slot;                 // shared-expert weight block (layer) or -1
+  int slot[kMaxExperts];
+  unsigned long long expected[kMaxExperts];
+};
+
+struct WaveParams {
+  int n;
+  int layer;
+  int slot[kMaxWave];
+  int expert[kMaxWave];
+  unsigned long long expected[kMaxWave];
+};
+
+struct PublishParams {
+  int n;
+  int slot[kMaxWave];
+  unsigned long long gen[kMaxWave];
+  unsigned long long obj[kMaxWave];
+};
+
+struct SetupArgs {
+  const int* counts;
+  const int* offsets;
+  const GenWord* genwords;
+  const int* table;                       // resident mode
+  const unsigned long long* expected;     // resident mode
+  int E, layer;
+  Group* groups;
+  int* total_mtiles;
+  int* status;
+};
+
+struct GemmArgs {
+  const Group* groups;
+  int num_groups;
+  const int* total_mtiles;  // device
+  int nt;                   // N tiles per group
+  int kblocks;              // K / 64
+  int b_rows_per_slot;      // rows of one weight block in the B tensor map
+  int b_row_off;            // row offset of the operand inside the block
+  int up_off;               // gate-up: row offset of the up rows (I)
+  int out_ld;               // output row length (elements)
+  __nv_bfloat16* out;
+  const __nv_bfloat16* x;   // gather source rows [T, H]
+  int x_ld;
+  const int* perm;          // permuted row -> t*k + j
+  int top_k;
+  int* status;
+  long long wait_limit;     // clock64 cycles per bounded wait
+};
+
+struct CombineArgs {
+  const __nv_bfloat16* yp;   // [T*k, H]
+  const float* weights;      // [T, k]
+  const int* inv;            // [T*k]
+  const float* sg;           // [T] or nullptr
+  const __nv_bfloat16* ys;   // [T, H] or nullptr
+  const __nv_bfloat16* x;    // residual or nullptr
+  __nv_bfloat16* out;        // [T, H]
+  int T, H, k;
+  const int* status;
+};
+
+enum GemmMode { kGateUpGather = 0, kGateUpTma = 1, kDown = 2 };
+
+// ---------------------------------------------------------------------------
+// Launchers (return cudaError_t of the launch)
+// ---------------------------------------------------------------------------
+cudaError_t launch_router(const RouterArgs& a, cudaStream_t s);
+cudaError_t launch_colscan(const ScanArgs& a, cudaStream_t s);
+cudaError_t launch_scatter(const ScatterArgs& a, cudaStream_t s);
+cudaError_t launch_upload(const TableParams& p, int* table, unsigned long long* expected,
+                          int* status, Group* shared_group, int* shared_total, cudaStream_t s);
+cudaError_t launch_setup_resident(const SetupArgs& a, cudaStream_t s);
+cudaError_t launch_setup_wave(const SetupArgs& a, const WaveParams& w, cudaStream_t s);
+cudaError_t launch_publish(const PublishParams& p, GenWord* genwords, cudaStream_t s);
+cudaError_t launch_gemm(int mode, const CUtensorMap& tmA, const CUtensorMap& tmB,
+                        const GemmArgs& a, int grid, cudaStream_t s);
+cudaError_t launch_combine(const CombineArgs& a, cudaStream_t s);
+cudaError_t launch_zero_counts(int* counts, int E, cudaStream_t s);
+
+constexpr int kRouterTM = 32;  // tokens per router block
+
+// GEMM tiling
+constexpr int kBM = 128;
+constexpr int kBN = 256;
+constexpr int kBK = 64;
+constexpr int kStages = 4;
+constexpr int kABytes = kBM * kBK * 2;
+constexpr int kBBytes = kBN * kBK * 2;
+int gemm_smem_bytes();
+
+// ---------------------------------------------------------------------------
+// PTX wrappers (device)
+// ---------------------------------------------------------------------------
+#if defined(__CUDACC__)
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_fence_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+               "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Bounded wait: returns false (and raises the CTA's abort flag) when the wait
+// exceeds `limit` clock64 cycles or another role already aborted.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                          long long limit) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const long long t0 = clock64();
+  while (true) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (*abort_flag) return false;
+    if (clock64() - t0 > limit) {
+      *abort_flag = 1;
+      return false;
+    }
+  }
+}
+
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__device__ __forceinline__ void tma_prefetch(const CUtensorMap* map) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+
+// 2-D tiled TMA load global -> shared, completion counted on `bar` (bytes).
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar, int c0,
+                                            int c1) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, "
+      "%4}], [%2];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(c0), "r"(c1)
+      : "memory");
+}
+
+__device__ __forceinline__ void cp_async16(void* dst, const void* src, uint32_t src_bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_u32(dst)), "l"(src),
+               "r"(src_bytes)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+// --- tcgen05 (5th-generation tensor cores, accumulators in TMEM) ---
+__device__ __forceinline__ void tmem_alloc(uint32_t* dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                   smem_u32(dst_smem)),
+               "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+// D[tmem] (+)= A[smem] * B[smem]^T, bf16 inputs, fp32 accumulate.
+__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
+                                          uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Arrive on `bar` once all previously issued tcgen05 ops of this thread complete.
+__device__ __forceinline__ void umma_commit(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+          smem_u32(bar))
+      : "memory");
+}
+
+// 32 lanes x 16 consecutive 32-bit columns; the wait carries the registers so
+// that no use can be scheduled before the load completes.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, "
+      "%12, %13, %14, %15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_ld_wait(uint32_t (&r)[16]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]),
+                 "+r"(r[6]), "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]),
+                 "+r"(r[12]), "+r"(r[13]), "+r"(r[14]), "+r"(r[15])
+               :
+               : "memory");
+}
+
+// Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, rows of
+// 128 bytes grouped in 8-row (1024-byte) atoms.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+  return (uint64_t)((saddr & 0x3FFFFu) >> 4)      // start address
+         | ((uint64_t)1 << 16)                    // leading byte offset (unused for SW128 K-major)
+         | ((uint64_t)(1024 >> 4) << 32)          // stride byte offset: 8 rows x 128 B
+         | ((uint64_t)1 << 46)                    // descriptor version (sm_100 family)
+         | ((uint64_t)2 << 61);                   // swizzle mode: 128 B
+}
+
+// Instruction descriptor of kind::f16: D fp32, A and B bf16, both K-major.
+__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+__device__ __forceinline__ float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xFFFF0000u); }
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+
+#endif  // __CUDACC__
+
+}  // namespace msi

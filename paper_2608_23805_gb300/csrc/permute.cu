@@ -1,0 +1,326 @@
+// Token grouping (histogram, scan, stable permutation), the per-call table
+// upload, the generation re-check that builds the GEMM groups, the slot
+// generation publication, and the weighted combine.
+//
+// Permutation: row r in [offsets[e], offsets[e+1]) holds the (t, j) pairs
+// routed to expert e in (t, j) order; perm[r] = t*k + j, inv[t*k + j] = r.
+// Atomic-free: per-router-block counts (written by the router kernel) ->
+// column prefix over blocks -> per-warp stable ranks from __match_any_sync.
+//
+// Generation re-check (fail closed): a published version must denote the
+// requested object and version, and a mismatch is rejected before any
+// consumer reads the slot (paper, Sec. "Lifetime Is Part of Correctness";
+// Sec. "Stable Slots and Bundle Publication").
+#include "internal.cuh"
+
+namespace msi {
+
+namespace {
+
+// ---- column prefix over router blocks: bbase[b][e], counts[e] ----
+__global__ void __launch_bounds__(1024) colscan_kernel(const ScanArgs a) {
+  __shared__ int part[32][33];
+  const int tx = threadIdx.x, ty = threadIdx.y;
+  const int e = blockIdx.x * 32 + tx;
+  const int sz = (a.nb + 31) / 32;
+  const int b0 = min(a.nb, ty * sz), b1 = min(a.nb, b0 + sz);
+  int sum = 0;
+  if (e < a.E)
+    for (int b = b0; b < b1; ++b) sum += a.bcount[(size_t)b * a.E + e];
+  part[ty][tx] = sum;
+  __syncthreads();
+  int run = 0;
+  for (int y = 0; y < ty; ++y) run += part[y][tx];
+  if (e < a.E) {
+    for (int b = b0; b < b1; ++b) {
+      const int v = a.bcount[(size_t)b * a.E + e];
+      a.bbase[(size_t)b * a.E + e] = run;
+      run += v;
+    }
+    if (ty == 31) a.counts[e] = run;
+  }
+}
+
+// ---- scatter: one warp per router block ----
+constexpr int kScatterWarps = 4;
+
+__global__ void __launch_bounds__(kScatterWarps * 32) scatter_kernel(const ScatterArgs a) {
+  __shared__ int offs[kMaxExperts + 1];
+  __shared__ int run[kScatterWarps][kMaxExperts];
+  __shared__ int wsum[kScatterWarps];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+
+  // exclusive scan of counts (E <= 512, 128 threads x 4 values)
+  int v[4], s = 0;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int e = tid * 4 + i;
+    v[i] = (e < a.E) ? a.counts[e] : 0;
+    s += v[i];
+  }
+  int incl = s;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const int o = __shfl_up_sync(0xffffffffu, incl, off);
+    if (lane >= off) incl += o;
+  }
+  if (lane == 31) wsum[warp] = incl;
+  __syncthreads();
+  int base = incl - s;
+  for (int w = 0; w < warp; ++w) base += wsum[w];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int e = tid * 4 + i;
+    if (e <= a.E) offs[e] = base;
+    base += v[i];
+  }
+  if (tid == kScatterWarps * 32 - 1 && a.E == kMaxExperts) offs[kMaxExperts] = base;
+  __syncthreads();
+  if (blockIdx.x == 0)
+    for (int e = tid; e <= a.E; e += blockDim.x) a.offsets[e] = offs[e];
+
+  const int b = blockIdx.x * kScatterWarps + warp;
+  if (b >= a.nb) return;
+  for (int e = lane; e < a.E; e += 32) run[warp][e] = 0;
+  __syncwarp();
+  const int f0 = b * kRouterTM * a.k;
+  const int f1 = min(a.T, (b + 1) * kRouterTM) * a.k;
+  const unsigned lt = (1u << lane) - 1u;
+  for (int f = f0 + lane; f - lane < f1; f += 32) {
+    const bool valid = f < f1;
+    const int e = valid ? a.ids[f] : -1;
+    const unsigned mask = __match_any_sync(0xffffffffu, e);
+    int before = 0;
+    if (valid) {
+      before = run[warp][e];
+      const int pos = offs[e] + a.bbase[(size_t)b * a.E + e] + before + __popc(mask & lt);
+      a.perm[pos] = f;
+      a.inv[f] = pos;
+    }
+    __syncwarp();
+    if (valid && lane == 31 - __clz(mask)) run[warp][e] = before + __popc(mask);
+    __syncwarp();
+  }
+}
+
+// ---- per-call table upload + forward begin ----
+__global__ void upload_kernel(const TableParams p, int* table, unsigned long long* expected,
+                              int* status, Group* sh, int* sh_total) {
+  for (int e = threadIdx.x; e < p.E; e += blockDim.x) {
+    table[e] = p.slot[e];
+    expected[e] = p.expected[e];
+  }
+  if (threadIdx.x == 0) {
+    *status = 0;
+    if (sh != nullptr) {
+      Group g;
+      g.row_begin = 0;
+      g.row_count = p.T;
+      g.slot = p.shared_slot;
+      g.mt_begin = 0;
+      g.ok = 1;
+      g.expert = -1;
+      g.pad0 = g.pad1 = 0;
+      *sh = g;
+      *sh_total = (p.T + kBM - 1) / kBM;
+    }
+  }
+}
+
+// ---- generation re-check + GEMM groups (one block) ----
+__device__ __forceinline__ int block_excl_scan(int v, int* tmp, int* total) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  int incl = v;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const int o = __shfl_up_sync(0xffffffffu, incl, off);
+    if (lane >= off) incl += o;
+  }
+  if (lane == 31) tmp[warp] = incl;
+  __syncthreads();
+  const int nw = blockDim.x >> 5;
+  int base = 0, tot = 0;
+  for (int w = 0; w < nw; ++w) {
+    if (w < warp) base += tmp[w];
+    tot += tmp[w];
+  }
+  *total = tot;
+  return base + incl - v;
+}
+
+__device__ __forceinline__ int block_min(int v, int* tmp) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) v = min(v, __shfl_xor_sync(0xffffffffu, v, off));
+  __syncthreads();
+  if (lane == 0) tmp[warp] = v;
+  __syncthreads();
+  int m = 0x7fffffff;
+  for (int w = 0; w < (int)(blockDim.x >> 5); ++w) m = min(m, tmp[w]);
+  return m;
+}
+
+__device__ __forceinline__ int check_code(const GenWord* gw, int slot, int layer, int e,
+                                          unsigned long long expected) {
+  if (slot < 0) return MSI_ERR_NOT_RESIDENT;
+  const unsigned long long obj = gw[slot].obj;
+  const unsigned long long gen = gw[slot].gen;
+  if (obj != obj_key(layer, e)) return MSI_ERR_WRONG_OBJECT;
+  if (gen != expected) return MSI_ERR_STALE_GENERATION;
+  return 0;
+}
+
+template <bool WAVE>
+__global__ void __launch_bounds__(kMaxExperts) setup_kernel(const SetupArgs a, const WaveParams w) {
+  __shared__ int tmp[32];
+  const int i = threadIdx.x;
+  const int n = WAVE ? w.n : a.E;
+  int e = -1, cnt = 0, slot = -1, code = 0;
+  if (i < n) {
+    e = WAVE ? w.expert[i] : i;
+    cnt = a.counts[e];
+    slot = WAVE ? w.slot[i] : a.table[e];
+    const unsigned long long exp = WAVE ? w.expected[i] : a.expected[e];
+    if (cnt > 0) code = check_code(a.genwords, slot, a.layer, e, exp);
+  }
+  const int mt = (i < n && code == 0) ? (cnt + kBM - 1) / kBM : 0;
+  int total = 0;
+  const int mt_begin = block_excl_scan(mt, tmp, &total);
+  if (i < n) {
+    Group g;
+    g.row_begin = a.offsets[e];
+    g.row_count = cnt;
+    g.slot = slot < 0 ? 0 : slot;
+    g.mt_begin = mt_begin;
+    g.ok = code == 0;
+    g.expert = e;
+    g.pad0 = g.pad1 = 0;
+    a.groups[i] = g;
+  }
+  const int key = code ? (e << 4) | code : 0x7fffffff;
+  const int m = block_min(key, tmp);
+  if (i == 0) {
+    *a.total_mtiles = total;
+    if (m != 0x7fffffff) atomicCAS(a.status, 0, m & 15);
+  }
+}
+
+__global__ void publish_kernel(const PublishParams p, GenWord* gw) {
+  const int i = threadIdx.x;
+  if (i < p.n) {
+    GenWord g;
+    g.gen = p.gen[i];
+    g.obj = p.obj[i];
+    gw[p.slot[i]] = g;
+  }
+}
+
+// ---- combine: out[t] = sum_j w[t,j] yp[inv[t*k+j]] (+ sg[t] ys[t]) (+ x[t]) ----
+__global__ void __launch_bounds__(256) combine_kernel(const CombineArgs a) {
+  if (*a.status != 0) return;  // fail closed: nothing stale becomes visible
+  const int t = blockIdx.x;
+  const int nchunk = a.H >> 3;
+  for (int c = threadIdx.x; c < nchunk; c += blockDim.x) {
+    float acc[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) acc[i] = 0.f;
+    for (int j = 0; j < a.k; ++j) {
+      const int r = __ldg(&a.inv[(size_t)t * a.k + j]);
+      const float w = __ldg(&a.weights[(size_t)t * a.k + j]);
+      const uint4 y = __ldg(reinterpret_cast<const uint4*>(a.yp + (size_t)r * a.H) + c);
+      acc[0] = fmaf(w, bf16_lo(y.x), acc[0]);
+      acc[1] = fmaf(w, bf16_hi(y.x), acc[1]);
+      acc[2] = fmaf(w, bf16_lo(y.y), acc[2]);
+      acc[3] = fmaf(w, bf16_hi(y.y), acc[3]);
+      acc[4] = fmaf(w, bf16_lo(y.z), acc[4]);
+      acc[5] = fmaf(w, bf16_hi(y.z), acc[5]);
+      acc[6] = fmaf(w, bf16_lo(y.w), acc[6]);
+      acc[7] = fmaf(w, bf16_hi(y.w), acc[7]);
+    }
+    if (a.ys != nullptr) {
+      const float g = a.sg[t];
+      const uint4 y = __ldg(reinterpret_cast<const uint4*>(a.ys + (size_t)t * a.H) + c);
+      acc[0] = fmaf(g, bf16_lo(y.x), acc[0]);
+      acc[1] = fmaf(g, bf16_hi(y.x), acc[1]);
+      acc[2] = fmaf(g, bf16_lo(y.y), acc[2]);
+      acc[3] = fmaf(g, bf16_hi(y.y), acc[3]);
+      acc[4] = fmaf(g, bf16_lo(y.z), acc[4]);
+      acc[5] = fmaf(g, bf16_hi(y.z), acc[5]);
+      acc[6] = fmaf(g, bf16_lo(y.w), acc[6]);
+      acc[7] = fmaf(g, bf16_hi(y.w), acc[7]);
+    }
+    if (a.x != nullptr) {
+      const uint4 y = __ldg(reinterpret_cast<const uint4*>(a.x + (size_t)t * a.H) + c);
+      acc[0] += bf16_lo(y.x);
+      acc[1] += bf16_hi(y.x);
+      acc[2] += bf16_lo(y.y);
+      acc[3] += bf16_hi(y.y);
+      acc[4] += bf16_lo(y.z);
+      acc[5] += bf16_hi(y.z);
+      acc[6] += bf16_lo(y.w);
+      acc[7] += bf16_hi(y.w);
+    }
+    uint4 o;
+    o.x = pack_bf16x2(acc[0], acc[1]);
+    o.y = pack_bf16x2(acc[2], acc[3]);
+    o.z = pack_bf16x2(acc[4], acc[5]);
+    o.w = pack_bf16x2(acc[6], acc[7]);
+    reinterpret_cast<uint4*>(a.out + (size_t)t * a.H)[c] = o;
+  }
+}
+
+__global__ void zero_kernel(int* p, int n) {
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x) p[i] = 0;
+}
+
+}  // namespace
+
+cudaError_t launch_colscan(const ScanArgs& a, cudaStream_t s) {
+  colscan_kernel<<<(a.E + 31) / 32, dim3(32, 32), 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_scatter(const ScatterArgs& a, cudaStream_t s) {
+  const int grid = (a.nb + kScatterWarps - 1) / kScatterWarps;
+  scatter_kernel<<<grid, kScatterWarps * 32, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_upload(const TableParams& p, int* table, unsigned long long* expected, int* status,
+                          Group* shared_group, int* shared_total, cudaStream_t s) {
+  upload_kernel<<<1, 512, 0, s>>>(p, table, expected, status, shared_group, shared_total);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_setup_resident(const SetupArgs& a, cudaStream_t s) {
+  WaveParams none;
+  none.n = 0;
+  none.layer = a.layer;
+  setup_kernel<false><<<1, kMaxExperts, 0, s>>>(a, none);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_setup_wave(const SetupArgs& a, const WaveParams& w, cudaStream_t s) {
+  setup_kernel<true><<<1, kMaxExperts, 0, s>>>(a, w);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_publish(const PublishParams& p, GenWord* genwords, cudaStream_t s) {
+  if (p.n == 0) return cudaSuccess;
+  publish_kernel<<<1, kMaxWave, 0, s>>>(p, genwords);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_combine(const CombineArgs& a, cudaStream_t s) {
+  if (a.T == 0) return cudaSuccess;
+  const int nthreads = min(256, a.H / 8);
+  combine_kernel<<<a.T, nthreads, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_zero_counts(int* counts, int E, cudaStream_t s) {
+  zero_kernel<<<1, 256, 0, s>>>(counts, E);
+  return cudaGetLastError();
+}
+
+}  // namespace msi

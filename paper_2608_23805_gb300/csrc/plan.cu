@@ -1,0 +1,952 @@
+// Host runtime of the C ABI: the Plan (immutable manifest + mutable slot
+// ledger), slot staging with generation publication, the LRU-wave residency
+// driver, and the two layer-forward entry points.
+//
+// Paper basis:
+//  - Plan = manifest (object -> extent, slot compatibility, stable device
+//    addresses) + mutable state (object, generation, readiness event and
+//    consumers per slot); replacement policy kept separate from the lifecycle
+//    (Sec. "A Shared Cross-Adapter Plan Core").
+//  - Slot lifecycle Vacant -> Loading -> DeviceReady -> InUse -> Recyclable ->
+//    Vacant; no reuse before the last consumer finishes (Sec. "Separate Window
+//    and GPU-Slot Lifecycles").
+//  - Bundle publication: all components checked before one publication
+//    transition; a device event publishes readiness; layer exit releases the
+//    consumer ticket (Sec. "Stable Slots and Bundle Publication";
+//    Sec. "Implementation", "Scheduling and copies").
+//  - Telemetry: stages, cache events, generations, H2D bytes, rejections
+//    (Sec. "Implementation", "Telemetry").
+//  - Per-layer LRU over 64 slots (Sec. "Evaluation", "Cache and storage
+//    state").  The wave policy (hits then misses, waves of half the pool, the
+//    previous wave pinned, least-recent victim, lowest index on ties) is the
+//    reading this library takes where the paper gives no rule.
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <atomic>
+#include <chrono>
+#include <cstring>
+#include <mutex>
+#include <string>
+#include <thread>
+#include <vector>
+
+#include "internal.cuh"
+
+using namespace msi;
+
+namespace {
+
+thread_local std::string g_last_cuda = "no error";
+
+msi_status cuda_fail(cudaError_t e, const char* what) {
+  g_last_cuda = std::string(what) + ": " + cudaGetErrorString(e);
+  return MSI_ERR_CUDA;
+}
+
+#define CK(call)                                               \
+  do {                                                         \
+    cudaError_t e_ = (call);                                   \
+    if (e_ != cudaSuccess) return cuda_fail(e_, #call);        \
+  } while (0)
+
+#define LAUNCH(plan, call)                                     \
+  do {                                                         \
+    cudaError_t e_ = (call);                                   \
+    if (e_ != cudaSuccess) return cuda_fail(e_, #call);        \
+    (plan)->launches++;                                        \
+  } while (0)
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (fn == nullptr) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+// 2-D bf16 tensor [rows, inner] (inner contiguous), box 64 x box_rows, 128-byte swizzle.
+bool make_tmap(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, uint32_t box_rows) {
+  auto fn = encode_fn();
+  if (fn == nullptr || rows == 0) return false;
+  cuuint64_t dims[2] = {inner, rows};
+  cuuint64_t strides[1] = {inner * 2};
+  cuuint32_t box[2] = {64, box_rows};
+  cuuint32_t es[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Reference-counted pool of CUDA events (readiness and consumer fences).
+struct EventPool {
+  std::vector<cudaEvent_t> ev;
+  std::vector<int> refs;
+  std::vector<int> freel;
+
+  msi_status acquire(int* id) {
+    if (freel.empty()) {
+      cudaEvent_t e;
+      CK(cudaEventCreateWithFlags(&e, cudaEventDisableTiming));
+      ev.push_back(e);
+      refs.push_back(0);
+      freel.push_back((int)ev.size() - 1);
+    }
+    *id = freel.back();
+    freel.pop_back();
+    refs[*id] = 1;
+    return MSI_OK;
+  }
+  void ref(int id) {
+    if (id >= 0) refs[id]++;
+  }
+  void unref(int id) {
+    if (id >= 0 && --refs[id] == 0) freel.push_back(id);
+  }
+  // true once the recorded work completed (or the event never recorded)
+  bool done(int id) {
+    if (id < 0) return true;
+    const cudaError_t e = cudaEventQuery(ev[id]);
+    if (e == cudaErrorNotReady) {
+      (void)cudaGetLastError();  // "not ready" is a state, not an error to report later
+      return false;
+    }
+    return true;
+  }
+};
+
+struct Slot {
+  int layer = -1, expert = -1;  // object held; -1: vacant
+  uint64_t gen = 0;             // generation of the current object
+  int ready = -1;               // event publishing the last stage
+  int consumer = -1;            // event of the last consumer
+  int64_t last_use = -1;        // LRU tick of the last consumption
+};
+
+struct WaveEntry {
+  int expert, slot;
+  bool miss;
+  uint64_t gen;
+};
+
+struct WsLayout {
+  size_t status, table, expected, groups, total, sh_group, sh_total, bcount, bbase, offsets, perm,
+      inv, sg, h, yp, hs, ys, bytes;
+};
+
+constexpr long long kDeviceWaitCycles = 4000000000LL;  // ~2 s at GB300 clocks
+
+}  // namespace
+
+struct msi_plan {
+  msi_plan_desc d{};
+  std::vector<uint64_t> off;
+  int sms = 0;
+  std::vector<Slot> slots;
+  std::vector<int> where;  // [L * E]: slot holding (l, e) or -1
+  std::vector<std::atomic<int>> holds;
+  GenWord* d_gen = nullptr;
+  int* h_status = nullptr;
+  int* h_counts = nullptr;
+  EventPool pool;
+  int fwd_ev = -1;
+  CUtensorMap tm_w13{}, tm_w2{}, tm_sh13{}, tm_sh2{};
+  std::vector<msi_trace_rec> trace;
+  uint64_t seq = 0;
+  msi_counters ctr{};
+  uint64_t launches = 0;
+  int64_t tick = 0;
+  int calls = 0;
+  int C = 1;
+  bool dying = false;
+  std::mutex mu;
+
+  explicit msi_plan(int S) : holds(S) {
+    for (auto& h : holds) h.store(0);
+  }
+};
+
+namespace {
+
+bool shape_ok(const msi_plan_desc& d) {
+  return d.n_experts >= 1 && d.n_experts <= kMaxExperts && d.top_k >= 1 &&
+         d.top_k <= std::min(d.n_experts, kMaxTopK) && d.hidden >= 256 && d.hidden % 256 == 0 &&
+         d.inter >= 128 && d.inter % 128 == 0 && d.wdtype == MSI_W_BF16;
+}
+
+WsLayout layout(const msi_plan* p, int T) {
+  WsLayout L{};
+  size_t o = 0;
+  auto take = [&](size_t bytes) {
+    const size_t r = o;
+    o += (bytes + 255) & ~(size_t)255;
+    return r;
+  };
+  const size_t E = p->d.n_experts, k = p->d.top_k, H = p->d.hidden, I = p->d.inter;
+  const size_t nb = ((size_t)T + kRouterTM - 1) / kRouterTM, Tk = (size_t)T * k;
+  L.status = take(4);
+  L.table = take(4 * E);
+  L.expected = take(8 * E);
+  L.groups = take(sizeof(Group) * std::max<size_t>(E, kMaxWave));
+  L.total = take(4);
+  L.sh_group = take(sizeof(Group));
+  L.sh_total = take(4);
+  L.bcount = take(4 * nb * E);
+  L.bbase = take(4 * nb * E);
+  L.offsets = take(4 * (E + 1));
+  L.perm = take(4 * Tk);
+  L.inv = take(4 * Tk);
+  L.sg = take(4 * (size_t)T);
+  L.h = take(2 * Tk * I);
+  L.yp = take(2 * Tk * H);
+  if (p->d.has_shared) {
+    L.hs = take(2 * (size_t)T * I);
+    L.ys = take(2 * (size_t)T * H);
+  }
+  L.bytes = o;
+  return L;
+}
+
+template <typename T>
+T* at(void* ws, size_t off) {
+  return reinterpret_cast<T*>(static_cast<char*>(ws) + off);
+}
+
+void add_trace(msi_plan* p, int call, int layer, int expert, int slot, uint64_t gen, int kind,
+               int wave) {
+  msi_trace_rec r;
+  r.seq = p->seq++;
+  r.call = call;
+  r.layer = layer;
+  r.expert = expert;
+  r.slot = slot;
+  r.generation = gen;
+  r.kind = kind;
+  r.wave = wave;
+  p->trace.push_back(r);
+}
+
+// Occupy `s` with (layer, e): records the eviction, bumps the generation.
+void ledger_stage(msi_plan* p, int s, int layer, int e, int call, int wave) {
+  Slot& sl = p->slots[s];
+  const int E = p->d.n_experts;
+  if (sl.layer >= 0) {
+    add_trace(p, call, sl.layer, sl.expert, s, sl.gen, MSI_TRACE_EVICT, wave);
+    p->where[(size_t)sl.layer * E + sl.expert] = -1;
+    p->ctr.evicts++;
+  }
+  sl.gen += 1;
+  sl.layer = layer;
+  sl.expert = e;
+  p->where[(size_t)layer * E + e] = s;
+  add_trace(p, call, layer, e, s, sl.gen, MSI_TRACE_STAGE, wave);
+  p->ctr.stages++;
+  p->ctr.h2d_bytes += p->d.extent_bytes;
+}
+
+// Wait on `stream` for every not-yet-complete event in ids (deduplicated).
+msi_status wait_events(msi_plan* p, std::vector<int>& ids, cudaStream_t stream) {
+  std::sort(ids.begin(), ids.end());
+  ids.erase(std::unique(ids.begin(), ids.end()), ids.end());
+  for (int id : ids)
+    if (id >= 0 && !p->pool.done(id)) CK(cudaStreamWaitEvent(stream, p->pool.ev[id], 0));
+  return MSI_OK;
+}
+
+// Enqueue the copies of `misses` on `stage` and publish them with one event.
+msi_status stage_enqueue(msi_plan* p, int layer, const std::vector<WaveEntry>& misses,
+                         cudaStream_t stage) {
+  if (misses.empty()) return MSI_OK;
+  std::vector<int> waits;
+  for (const auto& m : misses) {
+    waits.push_back(p->slots[m.slot].consumer);
+    waits.push_back(p->slots[m.slot].ready);
+  }
+  msi_status st = wait_events(p, waits, stage);
+  if (st != MSI_OK) return st;
+  PublishParams inv{}, pub{};
+  inv.n = pub.n = (int)misses.size();
+  for (size_t i = 0; i < misses.size(); ++i) {
+    inv.slot[i] = pub.slot[i] = misses[i].slot;
+    inv.gen[i] = 0;
+    inv.obj[i] = 0;
+    pub.gen[i] = misses[i].gen;
+    pub.obj[i] = obj_key(layer, misses[i].expert);
+  }
+  LAUNCH(p, launch_publish(inv, p->d_gen, stage));
+  const uint64_t eb = p->d.extent_bytes;
+  for (const auto& m : misses) {
+    const char* src = static_cast<const char*>(p->d.host_windows) +
+                      p->off[(size_t)layer * p->d.n_experts + m.expert];
+    char* dst = static_cast<char*>(p->d.slot_pool) + (size_t)m.slot * eb;
+    CK(cudaMemcpyAsync(dst, src, eb, cudaMemcpyHostToDevice, stage));
+  }
+  LAUNCH(p, launch_publish(pub, p->d_gen, stage));
+  int ev;
+  st = p->pool.acquire(&ev);
+  if (st != MSI_OK) return st;
+  CK(cudaEventRecord(p->pool.ev[ev], stage));
+  for (const auto& m : misses) {
+    p->pool.unref(p->slots[m.slot].ready);
+    p->slots[m.slot].ready = ev;
+    p->pool.ref(ev);
+  }
+  p->pool.unref(ev);
+  return MSI_OK;
+}
+
+// Record a consumer event on `s` for the slots in `used`.
+msi_status consumer_record(msi_plan* p, const std::vector<int>& used, cudaStream_t s) {
+  if (used.empty()) return MSI_OK;
+  int ev;
+  msi_status st = p->pool.acquire(&ev);
+  if (st != MSI_OK) return st;
+  CK(cudaEventRecord(p->pool.ev[ev], s));
+  for (int slot : used) {
+    p->pool.unref(p->slots[slot].consumer);
+    p->slots[slot].consumer = ev;
+    p->pool.ref(ev);
+  }
+  p->pool.unref(ev);
+  return MSI_OK;
+}
+
+struct FwdCtx {
+  int layer, T;
+  const void* x;
+  const float* router_w;
+  void* out;
+  const msi_route_event* ev;
+  void* ws;
+  WsLayout L;
+  unsigned flags;
+  cudaStream_t cs;
+  CUtensorMap tm_h, tm_x, tm_hs;
+};
+
+msi_status validate_fwd(msi_plan* p, int layer, const void* x, int T, const float* rw, void* out,
+                        const msi_route_event* ev, void* ws, size_t ws_bytes) {
+  if (p == nullptr || ev == nullptr) return MSI_ERR_INVALID_ARG;
+  if (p->dying) return MSI_ERR_SHUT_DOWN;
+  if (layer < 0 || layer >= p->d.n_layers || T < 0) return MSI_ERR_INVALID_ARG;
+  if (T > 0 && (x == nullptr || rw == nullptr || out == nullptr || ev->ids == nullptr ||
+                ev->weights == nullptr))
+    return MSI_ERR_INVALID_ARG;
+  if (ev->counts == nullptr) return MSI_ERR_INVALID_ARG;
+  if ((uintptr_t)x % 16 || (uintptr_t)out % 16) return MSI_ERR_INVALID_ARG;
+  const WsLayout L = layout(p, T);
+  if (ws == nullptr || (uintptr_t)ws % 256 || ws_bytes < L.bytes) return MSI_ERR_WORKSPACE;
+  return MSI_OK;
+}
+
+// Forward begin + router + histogram + permutation.
+msi_status front(msi_plan* p, FwdCtx& f, const TableParams& tp) {
+  const auto& d = p->d;
+  const int E = d.n_experts, k = d.top_k, H = d.hidden, I = d.inter;
+  void* ws = f.ws;
+  const WsLayout& L = f.L;
+  LAUNCH(p, launch_upload(tp, at<int>(ws, L.table), at<unsigned long long>(ws, L.expected),
+                          at<int>(ws, L.status), d.has_shared ? at<Group>(ws, L.sh_group) : nullptr,
+                          at<int>(ws, L.sh_total), f.cs));
+  if (f.T == 0) {
+    LAUNCH(p, launch_zero_counts(f.ev->counts, E, f.cs));
+    return MSI_OK;
+  }
+  const int nb = (f.T + kRouterTM - 1) / kRouterTM;
+  RouterArgs ra{};
+  ra.x = static_cast<const __nv_bfloat16*>(f.x);
+  ra.wr = f.router_w;
+  ra.wsg = d.has_shared ? d.shared_gate_w + (size_t)f.layer * H : nullptr;
+  ra.T = f.T;
+  ra.H = H;
+  ra.E = E;
+  ra.k = k;
+  ra.ids = f.ev->ids;
+  ra.weights = f.ev->weights;
+  ra.gap = f.ev->gap;
+  ra.sg = at<float>(ws, L.sg);
+  ra.bcount = at<int>(ws, L.bcount);
+  LAUNCH(p, launch_router(ra, f.cs));
+  ScanArgs sa{at<int>(ws, L.bcount), nb, E, at<int>(ws, L.bbase), f.ev->counts};
+  LAUNCH(p, launch_colscan(sa, f.cs));
+  ScatterArgs xa{f.ev->ids, f.ev->counts, at<int>(ws, L.bbase), f.T, k, E, nb,
+                 at<int>(ws, L.perm), at<int>(ws, L.inv), at<int>(ws, L.offsets)};
+  LAUNCH(p, launch_scatter(xa, f.cs));
+  const size_t Tk = (size_t)f.T * k;
+  if (!make_tmap(&f.tm_h, at<char>(ws, L.h), I, Tk, 128)) return MSI_ERR_CUDA;
+  if (d.has_shared) {
+    if (!make_tmap(&f.tm_x, f.x, H, f.T, 128)) return MSI_ERR_CUDA;
+    if (!make_tmap(&f.tm_hs, at<char>(ws, L.hs), I, f.T, 128)) return MSI_ERR_CUDA;
+  }
+  return MSI_OK;
+}
+
+GemmArgs gateup_args(msi_plan* p, FwdCtx& f, const Group* groups, int ng, const int* total,
+                     __nv_bfloat16* out) {
+  const auto& d = p->d;
+  GemmArgs g{};
+  g.groups = groups;
+  g.num_groups = ng;
+  g.total_mtiles = total;
+  g.nt = d.inter / 128;
+  g.kblocks = d.hidden / kBK;
+  g.b_rows_per_slot = 3 * d.inter;
+  g.b_row_off = 0;
+  g.up_off = d.inter;
+  g.out_ld = d.inter;
+  g.out = out;
+  g.x = static_cast<const __nv_bfloat16*>(f.x);
+  g.x_ld = d.hidden;
+  g.perm = at<int>(f.ws, f.L.perm);
+  g.top_k = d.top_k;
+  g.status = at<int>(f.ws, f.L.status);
+  g.wait_limit = kDeviceWaitCycles;
+  return g;
+}
+
+GemmArgs down_args(msi_plan* p, FwdCtx& f, const Group* groups, int ng, const int* total,
+                   __nv_bfloat16* out) {
+  const auto& d = p->d;
+  GemmArgs g = gateup_args(p, f, groups, ng, total, out);
+  g.nt = d.hidden / kBN;
+  g.kblocks = d.inter / kBK;
+  g.b_rows_per_slot = 3 * d.hidden;
+  g.b_row_off = 2 * d.hidden;
+  g.up_off = 0;
+  g.out_ld = d.hidden;
+  return g;
+}
+
+msi_status routed_ffn(msi_plan* p, FwdCtx& f, int ng, int grid1, int grid2) {
+  const Group* groups = at<Group>(f.ws, f.L.groups);
+  const int* total = at<int>(f.ws, f.L.total);
+  GemmArgs g1 = gateup_args(p, f, groups, ng, total, at<__nv_bfloat16>(f.ws, f.L.h));
+  LAUNCH(p, launch_gemm(kGateUpGather, p->tm_w13, p->tm_w13, g1, grid1, f.cs));
+  GemmArgs g2 = down_args(p, f, groups, ng, total, at<__nv_bfloat16>(f.ws, f.L.yp));
+  LAUNCH(p, launch_gemm(kDown, f.tm_h, p->tm_w2, g2, grid2, f.cs));
+  return MSI_OK;
+}
+
+msi_status shared_ffn(msi_plan* p, FwdCtx& f) {
+  if (!p->d.has_shared || f.T == 0) return MSI_OK;
+  const Group* g = at<Group>(f.ws, f.L.sh_group);
+  const int* total = at<int>(f.ws, f.L.sh_total);
+  const int mt = (f.T + kBM - 1) / kBM;
+  GemmArgs s1 = gateup_args(p, f, g, 1, total, at<__nv_bfloat16>(f.ws, f.L.hs));
+  LAUNCH(p, launch_gemm(kGateUpTma, f.tm_x, p->tm_sh13, s1, std::min(p->sms, mt * s1.nt), f.cs));
+  GemmArgs s2 = down_args(p, f, g, 1, total, at<__nv_bfloat16>(f.ws, f.L.ys));
+  LAUNCH(p, launch_gemm(kDown, f.tm_hs, p->tm_sh2, s2, std::min(p->sms, mt * s2.nt), f.cs));
+  return MSI_OK;
+}
+
+msi_status finish(msi_plan* p, FwdCtx& f) {
+  const auto& d = p->d;
+  if (f.T > 0) {
+    CombineArgs c{};
+    c.yp = at<__nv_bfloat16>(f.ws, f.L.yp);
+    c.weights = f.ev->weights;
+    c.inv = at<int>(f.ws, f.L.inv);
+    c.sg = d.has_shared ? at<float>(f.ws, f.L.sg) : nullptr;
+    c.ys = d.has_shared ? at<__nv_bfloat16>(f.ws, f.L.ys) : nullptr;
+    c.x = (f.flags & MSI_FWD_RESIDUAL) ? static_cast<const __nv_bfloat16*>(f.x) : nullptr;
+    c.out = static_cast<__nv_bfloat16*>(f.out);
+    c.T = f.T;
+    c.H = d.hidden;
+    c.k = d.top_k;
+    c.status = at<int>(f.ws, f.L.status);
+    LAUNCH(p, launch_combine(c, f.cs));
+  }
+  CK(cudaMemcpyAsync(p->h_status, at<int>(f.ws, f.L.status), sizeof(int), cudaMemcpyDeviceToHost,
+                     f.cs));
+  int ev;
+  msi_status st = p->pool.acquire(&ev);
+  if (st != MSI_OK) return st;
+  CK(cudaEventRecord(p->pool.ev[ev], f.cs));
+  p->pool.unref(p->fwd_ev);
+  p->fwd_ev = ev;
+  return MSI_OK;
+}
+
+bool wait_unheld(msi_plan* p, int slot) {
+  const double lim = p->d.wait_timeout_s > 0 ? p->d.wait_timeout_s : 1.0;
+  const auto t0 = std::chrono::steady_clock::now();
+  while (p->holds[slot].load() > 0) {
+    const double el = std::chrono::duration<double>(std::chrono::steady_clock::now() - t0).count();
+    if (el > lim) return false;
+    std::this_thread::sleep_for(std::chrono::microseconds(200));
+  }
+  return true;
+}
+
+}  // namespace
+
+// ===========================================================================
+// C ABI
+// ===========================================================================
+extern "C" {
+
+uint64_t msi_extent_bytes(int hidden, int inter, int wdtype) {
+  if (hidden <= 0 || inter <= 0) return 0;
+  const uint64_t HI = (uint64_t)hidden * inter;
+  if (wdtype == MSI_W_BF16) return 3 * HI * 2;
+  if (wdtype == MSI_W_Q4G32) {
+    if (hidden % 32 || inter % 32) return 0;
+    return 3 * HI / 2 + 3 * HI / 32 * 2;
+  }
+  return 0;
+}
+
+const char* msi_status_string(msi_status s) {
+  switch (s) {
+    case MSI_OK: return "ok";
+    case MSI_ERR_INVALID_ARG: return "invalid argument";
+    case MSI_ERR_STALE_GENERATION: return "stale generation";
+    case MSI_ERR_WRONG_OBJECT: return "wrong object in slot";
+    case MSI_ERR_SLOT_BUSY: return "slot busy (live consumer)";
+    case MSI_ERR_NOT_RESIDENT: return "needed expert not resident";
+    case MSI_ERR_TIMEOUT: return "bounded wait timed out";
+    case MSI_ERR_CUDA: return "CUDA error";
+    case MSI_ERR_SHUT_DOWN: return "plan shut down";
+    case MSI_ERR_UNSUPPORTED: return "unsupported shape";
+    case MSI_ERR_WORKSPACE: return "workspace missing, misaligned or too small";
+  }
+  return "unknown status";
+}
+
+const char* msi_last_cuda_error(void) { return g_last_cuda.c_str(); }
+
+msi_status msi_plan_create(const msi_plan_desc* desc, msi_plan** out) {
+  if (desc == nullptr || out == nullptr) return MSI_ERR_INVALID_ARG;
+  *out = nullptr;
+  const msi_plan_desc& d = *desc;
+  if (d.n_layers < 1 || d.n_slots < 2 || d.slot_pool == nullptr || d.host_windows == nullptr)
+    return MSI_ERR_INVALID_ARG;
+  if (d.wdtype != MSI_W_BF16 && d.wdtype != MSI_W_Q4G32) return MSI_ERR_INVALID_ARG;
+  if (!shape_ok(d)) return MSI_ERR_UNSUPPORTED;
+  if (d.extent_bytes != msi_extent_bytes(d.hidden, d.inter, d.wdtype)) return MSI_ERR_INVALID_ARG;
+  if ((uintptr_t)d.slot_pool % 128) return MSI_ERR_INVALID_ARG;
+  if (d.has_shared && (d.shared_w == nullptr || d.shared_gate_w == nullptr ||
+                       (uintptr_t)d.shared_w % 128 || (uintptr_t)d.shared_gate_w % 16))
+    return MSI_ERR_INVALID_ARG;
+  const int C = d.wave_capacity > 0 ? d.wave_capacity : d.n_slots / 2;
+  if (C < 1 || 2 * C > d.n_slots || C > kMaxWave) return MSI_ERR_INVALID_ARG;
+
+  msi_plan* p = new msi_plan(d.n_slots);
+  p->d = d;
+  p->C = C;
+  const size_t nobj = (size_t)d.n_layers * d.n_experts;
+  p->off.resize(nobj);
+  for (size_t i = 0; i < nobj; ++i) p->off[i] = d.extent_off ? d.extent_off[i] : i * d.extent_bytes;
+  p->slots.resize(d.n_slots);
+  p->where.assign(nobj, -1);
+  auto fail = [&](msi_status s) {
+    if (p->d_gen) cudaFree(p->d_gen);
+    if (p->h_status) cudaFreeHost(p->h_status);
+    if (p->h_counts) cudaFreeHost(p->h_counts);
+    delete p;
+    return s;
+  };
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&p->sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e == cudaSuccess) e = cudaMalloc(&p->d_gen, sizeof(GenWord) * d.n_slots);
+  if (e == cudaSuccess) e = cudaMemset(p->d_gen, 0, sizeof(GenWord) * d.n_slots);
+  if (e == cudaSuccess) e = cudaMallocHost(&p->h_status, sizeof(int));
+  if (e == cudaSuccess) e = cudaMallocHost(&p->h_counts, sizeof(int) * d.n_experts);
+  if (e != cudaSuccess) return fail(cuda_fail(e, "msi_plan_create"));
+  *p->h_status = 0;
+  const uint64_t H = d.hidden, I = d.inter, S = d.n_slots;
+  if (d.wdtype == MSI_W_BF16) {
+    if (!make_tmap(&p->tm_w13, d.slot_pool, H, S * 3 * I, 128) ||
+        !make_tmap(&p->tm_w2, d.slot_pool, I, S * 3 * H, 128))
+      return fail(MSI_ERR_CUDA);
+  }
+  if (d.has_shared) {
+    if (!make_tmap(&p->tm_sh13, d.shared_w, H, (uint64_t)d.n_layers * 3 * I, 128) ||
+        !make_tmap(&p->tm_sh2, d.shared_w, I, (uint64_t)d.n_layers * 3 * H, 128))
+      return fail(MSI_ERR_CUDA);
+  }
+  *out = p;
+  return MSI_OK;
+}
+
+msi_status msi_plan_destroy(msi_plan* p) {
+  if (p == nullptr) return MSI_ERR_INVALID_ARG;
+  {
+    std::lock_guard<std::mutex> g(p->mu);
+    for (auto& h : p->holds)
+      if (h.load() > 0) return MSI_ERR_SLOT_BUSY;
+    p->dying = true;
+    // drain: every readiness, consumer and forward event still referenced
+    for (auto& s : p->slots) {
+      if (s.ready >= 0) cudaEventSynchronize(p->pool.ev[s.ready]);
+      if (s.consumer >= 0) cudaEventSynchronize(p->pool.ev[s.consumer]);
+    }
+    if (p->fwd_ev >= 0) cudaEventSynchronize(p->pool.ev[p->fwd_ev]);
+    for (auto ev : p->pool.ev) cudaEventDestroy(ev);
+    cudaFree(p->d_gen);
+    cudaFreeHost(p->h_status);
+    cudaFreeHost(p->h_counts);
+  }
+  delete p;
+  return MSI_OK;
+}
+
+msi_status msi_workspace_size(const msi_plan* p, int T, size_t* bytes) {
+  if (p == nullptr || bytes == nullptr || T < 0) return MSI_ERR_INVALID_ARG;
+  *bytes = layout(p, T).bytes;
+  return MSI_OK;
+}
+
+msi_status msi_slot_stage(msi_plan* p, int slot, int layer, int expert, msi_stream stage,
+                          uint64_t* new_generation) {
+  if (p == nullptr) return MSI_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> g(p->mu);
+  if (p->dying) return MSI_ERR_SHUT_DOWN;
+  const auto& d = p->d;
+  if (slot < 0 || slot >= d.n_slots || layer < 0 || layer >= d.n_layers || expert < 0 ||
+      expert >= d.n_experts)
+    return MSI_ERR_INVALID_ARG;
+  const int cur = p->where[(size_t)layer * d.n_experts + expert];
+  if (cur >= 0 && cur != slot) return MSI_ERR_INVALID_ARG;  // one slot per object
+  if (!wait_unheld(p, slot)) {
+    p->ctr.rejections++;
+    return MSI_ERR_TIMEOUT;
+  }
+  Slot& sl = p->slots[slot];
+  const uint64_t gen = sl.gen + 1;
+  std::vector<WaveEntry> m{{expert, slot, true, gen}};
+  msi_status st = stage_enqueue(p, layer, m, reinterpret_cast<cudaStream_t>(stage));
+  if (st != MSI_OK) return st;
+  ledger_stage(p, slot, layer, expert, -1, -1);
+  if (new_generation) *new_generation = sl.gen;
+  return MSI_OK;
+}
+
+msi_status msi_slot_table(const msi_plan* cp, int layer, int32_t* slot_of, uint64_t* gen_of) {
+  msi_plan* p = const_cast<msi_plan*>(cp);
+  if (p == nullptr || slot_of == nullptr || gen_of == nullptr) return MSI_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> g(p->mu);
+  if (layer < 0 || layer >= p->d.n_layers) return MSI_ERR_INVALID_ARG;
+  const int E = p->d.n_experts;
+  for (int e = 0; e < E; ++e) {
+    const int s = p->where[(size_t)layer * E + e];
+    slot_of[e] = s;
+    gen_of[e] = s >= 0 ? p->slots[s].gen : 0;
+  }
+  return MSI_OK;
+}
+
+msi_status msi_slot_state(const msi_plan* cp, int slot, int* state) {
+  msi_plan* p = const_cast<msi_plan*>(cp);
+  if (p == nullptr || state == nullptr || slot < 0 || slot >= p->d.n_slots)
+    return MSI_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> g(p->mu);
+  const Slot& s = p->slots[slot];
+  if (s.layer < 0) *state = MSI_SLOT_VACANT;
+  else if (!p->pool.done(s.ready)) *state = MSI_SLOT_LOADING;
+  else if (p->holds[slot].load() > 0 || !p->pool.done(s.consumer)) *state = MSI_SLOT_IN_USE;
+  else if (s.consumer < 0) *state = MSI_SLOT_DEVICE_READY;
+  else *state = MSI_SLOT_RECYCLABLE;
+  return MSI_OK;
+}
+
+msi_status msi_moe_forward(msi_plan* p, int layer, const void* x, int T, const float* rw,
+                           const int32_t* table, const uint64_t* expected, void* out,
+                           const msi_route_event* ev, void* ws, size_t ws_bytes, unsigned flags,
+                           msi_stream compute) {
+  if (p == nullptr) return MSI_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> g(p->mu);
+  msi_status st = validate_fwd(p, layer, x, T, rw, out, ev, ws, ws_bytes);
+  if (st != MSI_OK) return st;
+  if (table == nullptr || expected == nullptr) return MSI_ERR_INVALID_ARG;
+  const auto& d = p->d;
+  const int E = d.n_experts;
+  // host precheck: nothing is enqueued when a named slot does not hold the
+  // requested object and version
+  std::vector<int> used;
+  for (int e = 0; e < E; ++e) {
+    const int s = table[e];
+    if (s < -1 || s >= d.n_slots) return MSI_ERR_INVALID_ARG;
+    if (s < 0) continue;
+    const Slot& sl = p->slots[s];
+    if (sl.layer != layer || sl.expert != e) {
+      p->ctr.rejections++;
+      return MSI_ERR_WRONG_OBJECT;
+    }
+    if (sl.gen != expected[e]) {
+      p->ctr.rejections++;
+      return MSI_ERR_STALE_GENERATION;
+    }
+    used.push_back(s);
+  }
+  FwdCtx f{};
+  f.layer = layer;
+  f.T = T;
+  f.x = x;
+  f.router_w = rw;
+  f.out = out;
+  f.ev = ev;
+  f.ws = ws;
+  f.L = layout(p, T);
+  f.flags = flags;
+  f.cs = reinterpret_cast<cudaStream_t>(compute);
+  // readiness: the compute stream waits for every pending publication it reads
+  std::vector<int> waits;
+  for (int s : used) waits.push_back(p->slots[s].ready);
+  st = wait_events(p, waits, f.cs);
+  if (st != MSI_OK) return st;
+  static thread_local TableParams tp;
+  tp.E = E;
+  tp.layer = layer;
+  tp.T = T;
+  tp.shared_slot = d.has_shared ? layer : -1;
+  for (int e = 0; e < E; ++e) {
+    tp.slot[e] = table[e];
+    tp.expected[e] = expected[e];
+  }
+  st = front(p, f, tp);
+  if (st != MSI_OK) return st;
+  if (T > 0) {
+    SetupArgs sa{};
+    sa.counts = ev->counts;
+    sa.offsets = at<int>(ws, f.L.offsets);
+    sa.genwords = p->d_gen;
+    sa.table = at<int>(ws, f.L.table);
+    sa.expected = at<unsigned long long>(ws, f.L.expected);
+    sa.E = E;
+    sa.layer = layer;
+    sa.groups = at<Group>(ws, f.L.groups);
+    sa.total_mtiles = at<int>(ws, f.L.total);
+    sa.status = at<int>(ws, f.L.status);
+    LAUNCH(p, launch_setup_resident(sa, f.cs));
+    const long long mt_max = ((long long)T * d.top_k + kBM - 1) / kBM + E;
+    const int g1 = (int)std::min<long long>(p->sms, mt_max * (d.inter / 128));
+    const int g2 = (int)std::min<long long>(p->sms, mt_max * (d.hidden / kBN));
+    st = routed_ffn(p, f, E, g1, g2);
+    if (st != MSI_OK) return st;
+    st = consumer_record(p, used, f.cs);
+    if (st != MSI_OK) return st;
+    st = shared_ffn(p, f);
+    if (st != MSI_OK) return st;
+  }
+  st = finish(p, f);
+  if (st != MSI_OK) return st;
+  p->ctr.forwards++;
+  return MSI_OK;
+}
+
+msi_status msi_moe_forward_streamed(msi_plan* p, int layer, const void* x, int T, const float* rw,
+                                    void* out, const msi_route_event* ev, void* ws, size_t ws_bytes,
+                                    unsigned flags, msi_stream compute, msi_stream stage) {
+  if (p == nullptr) return MSI_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> g(p->mu);
+  msi_status st = validate_fwd(p, layer, x, T, rw, out, ev, ws, ws_bytes);
+  if (st != MSI_OK) return st;
+  const auto& d = p->d;
+  const int E = d.n_experts;
+  FwdCtx f{};
+  f.layer = layer;
+  f.T = T;
+  f.x = x;
+  f.router_w = rw;
+  f.out = out;
+  f.ev = ev;
+  f.ws = ws;
+  f.L = layout(p, T);
+  f.flags = flags;
+  f.cs = reinterpret_cast<cudaStream_t>(compute);
+  cudaStream_t ss = reinterpret_cast<cudaStream_t>(stage);
+  static thread_local TableParams tp;
+  tp.E = 0;
+  tp.layer = layer;
+  tp.T = T;
+  tp.shared_slot = d.has_shared ? layer : -1;
+  st = front(p, f, tp);
+  if (st != MSI_OK) return st;
+  // counts back to the host: the needed set decides the staging
+  CK(cudaMemcpyAsync(p->h_counts, ev->counts, sizeof(int) * E, cudaMemcpyDeviceToHost, f.cs));
+  int cev;
+  st = p->pool.acquire(&cev);
+  if (st != MSI_OK) return st;
+  CK(cudaEventRecord(p->pool.ev[cev], f.cs));
+  st = shared_ffn(p, f);  // overlaps the host planning and the first wave's copies
+  if (st != MSI_OK) return st;
+  const cudaError_t se = cudaEventSynchronize(p->pool.ev[cev]);
+  p->pool.unref(cev);
+  if (se != cudaSuccess) return cuda_fail(se, "counts readback");
+
+  // held slots: wait (bounded) before planning so the plan never picks them
+  for (int s = 0; s < d.n_slots; ++s)
+    if (!wait_unheld(p, s)) {
+      p->ctr.rejections++;
+      return MSI_ERR_TIMEOUT;
+    }
+
+  // ---- LRU-wave plan (host ledger; identical rules to the slot simulator) ----
+  const int call = p->calls++;
+  std::vector<int> hits, misses;
+  for (int e = 0; e < E; ++e) {
+    if (p->h_counts[e] <= 0) continue;
+    (p->where[(size_t)layer * E + e] >= 0 ? hits : misses).push_back(e);
+  }
+  std::vector<int> order(hits);
+  order.insert(order.end(), misses.begin(), misses.end());
+  std::vector<std::vector<WaveEntry>> waves;
+  std::vector<char> pinned(d.n_slots, 0);
+  std::vector<int> prev;
+  for (size_t w0 = 0; w0 < order.size(); w0 += p->C) {
+    const int w = (int)waves.size();
+    std::vector<WaveEntry> wave;
+    std::fill(pinned.begin(), pinned.end(), 0);
+    for (int s : prev) pinned[s] = 1;
+    for (size_t i = w0; i < std::min(order.size(), w0 + p->C); ++i) {
+      const int e = order[i];
+      int s = p->where[(size_t)layer * E + e];
+      bool miss = false;
+      if (s >= 0) {
+        add_trace(p, call, layer, e, s, p->slots[s].gen, MSI_TRACE_HIT, w);
+        p->ctr.hits++;
+      } else {
+        int victim = -1;
+        for (int c = 0; c < d.n_slots && victim < 0; ++c)
+          if (!pinned[c] && p->slots[c].layer < 0) victim = c;
+        if (victim < 0) {
+          for (int c = 0; c < d.n_slots; ++c) {
+            if (pinned[c]) continue;
+            if (victim < 0 || p->slots[c].last_use < p->slots[victim].last_use) victim = c;
+          }
+        }
+        s = victim;
+        ledger_stage(p, s, layer, e, call, w);
+        miss = true;
+      }
+      pinned[s] = 1;
+      wave.push_back({e, s, miss, p->slots[s].gen});
+    }
+    prev.clear();
+    for (const auto& we : wave) {
+      p->tick += 1;
+      p->slots[we.slot].last_use = p->tick;
+      prev.push_back(we.slot);
+    }
+    waves.push_back(std::move(wave));
+  }
+
+  // ---- issue: stage(w + 1) overlaps compute(w) ----
+  auto stage_wave = [&](size_t w) -> msi_status {
+    std::vector<WaveEntry> m;
+    for (const auto& we : waves[w])
+      if (we.miss) m.push_back(we);
+    return stage_enqueue(p, layer, m, ss);
+  };
+  if (!waves.empty()) {
+    st = stage_wave(0);
+    if (st != MSI_OK) return st;
+  }
+  static thread_local WaveParams wp;
+  for (size_t w = 0; w < waves.size(); ++w) {
+    if (w + 1 < waves.size()) {
+      st = stage_wave(w + 1);
+      if (st != MSI_OK) return st;
+    }
+    std::vector<int> waits, used;
+    int mtiles = 0;
+    wp.n = (int)waves[w].size();
+    wp.layer = layer;
+    for (int i = 0; i < wp.n; ++i) {
+      const WaveEntry& we = waves[w][i];
+      waits.push_back(p->slots[we.slot].ready);
+      used.push_back(we.slot);
+      wp.slot[i] = we.slot;
+      wp.expert[i] = we.expert;
+      wp.expected[i] = we.gen;
+      mtiles += (p->h_counts[we.expert] + kBM - 1) / kBM;
+    }
+    st = wait_events(p, waits, f.cs);
+    if (st != MSI_OK) return st;
+    SetupArgs sa{};
+    sa.counts = ev->counts;
+    sa.offsets = at<int>(ws, f.L.offsets);
+    sa.genwords = p->d_gen;
+    sa.E = E;
+    sa.layer = layer;
+    sa.groups = at<Group>(ws, f.L.groups);
+    sa.total_mtiles = at<int>(ws, f.L.total);
+    sa.status = at<int>(ws, f.L.status);
+    LAUNCH(p, launch_setup_wave(sa, wp, f.cs));
+    const int g1 = std::max(1, std::min(p->sms, mtiles * (d.inter / 128)));
+    const int g2 = std::max(1, std::min(p->sms, mtiles * (d.hidden / kBN)));
+    st = routed_ffn(p, f, wp.n, g1, g2);
+    if (st != MSI_OK) return st;
+    st = consumer_record(p, used, f.cs);
+    if (st != MSI_OK) return st;
+  }
+  st = finish(p, f);
+  if (st != MSI_OK) return st;
+  p->ctr.forwards++;
+  p->ctr.streamed_forwards++;
+  return MSI_OK;
+}
+
+msi_status msi_forward_status(msi_plan* p, int* device_status) {
+  if (p == nullptr || device_status == nullptr) return MSI_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> g(p->mu);
+  if (p->fwd_ev < 0) {
+    *device_status = MSI_OK;
+    return MSI_OK;
+  }
+  CK(cudaEventSynchronize(p->pool.ev[p->fwd_ev]));
+  *device_status = *p->h_status;
+  if (*device_status != MSI_OK) p->ctr.rejections++;
+  return MSI_OK;
+}
+
+msi_status msi_consumer_hold(msi_plan* p, int slot) {
+  if (p == nullptr || slot < 0 || slot >= p->d.n_slots) return MSI_ERR_INVALID_ARG;
+  if (p->dying) return MSI_ERR_SHUT_DOWN;
+  p->holds[slot].fetch_add(1);
+  return MSI_OK;
+}
+
+msi_status msi_consumer_release(msi_plan* p, int slot) {
+  if (p == nullptr || slot < 0 || slot >= p->d.n_slots) return MSI_ERR_INVALID_ARG;
+  int cur = p->holds[slot].load();
+  while (cur > 0 && !p->holds[slot].compare_exchange_weak(cur, cur - 1)) {
+  }
+  return cur > 0 ? MSI_OK : MSI_ERR_INVALID_ARG;
+}
+
+msi_status msi_trace_read(const msi_plan* cp, msi_trace_rec* buf, size_t cap, size_t* n) {
+  msi_plan* p = const_cast<msi_plan*>(cp);
+  if (p == nullptr || n == nullptr || (buf == nullptr && cap > 0)) return MSI_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> g(p->mu);
+  const size_t m = std::min(cap, p->trace.size());
+  if (m) std::memcpy(buf, p->trace.data(), m * sizeof(msi_trace_rec));
+  *n = m;
+  return MSI_OK;
+}
+
+msi_status msi_trace_clear(msi_plan* p) {
+  if (p == nullptr) return MSI_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> g(p->mu);
+  p->trace.clear();
+  return MSI_OK;
+}
+
+msi_status msi_get_counters(const msi_plan* cp, msi_counters* out) {
+  msi_plan* p = const_cast<msi_plan*>(cp);
+  if (p == nullptr || out == nullptr) return MSI_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> g(p->mu);
+  *out = p->ctr;
+  return MSI_OK;
+}
+
+uint64_t msi_kernel_launches(const msi_plan* p) { return p ? p->launches : 0; }
+
+}  // extern "C"

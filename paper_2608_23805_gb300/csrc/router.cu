@@ -1,0 +1,213 @@
+// Router: fp32 logits, top-k, softmax weights, shared-expert gate and the
+// per-block expert histogram, fused in one kernel (logits never reach HBM).
+//
+// The router's top-k output is the route event the paper records once per
+// layer and graph evaluation, before any Plan action (Sec. "Output-Exact
+// Execution Beyond the Full-Residency Envelope").  Readings where the paper is
+// silent: weights are the softmax over the selected k logits (they sum to 1);
+// equal logits rank the lower expert id first.
+//
+// Block = 32 tokens x all E (<= 512) experts, 256 threads.  Each thread owns
+// an 8-token x 8-expert fp32 register tile (experts strided by 64 so a warp
+// reads 32 consecutive expert rows).  K is staged 32 at a time with cp.async:
+// x as bf16 [32 tok][32 k]; Wr as fp32 [512 e][32 k] with the eight 16-byte
+// chunks of each row XOR-swizzled by (e & 7), so a warp's 16-byte reads of
+// one k-quad hit all 32 banks once per 8 lanes.  Accumulation runs over h in
+// ascending order.  Top-k: one warp per token, k+1 rounds of a warp-shuffle
+// argmax over (logit desc, id asc).
+#include "internal.cuh"
+
+namespace msi {
+
+namespace {
+constexpr int TM = kRouterTM;
+constexpr int BK = 32;
+constexpr int EP = 512;                      // experts per pass (this build: one pass)
+constexpr int NTH = 256;
+constexpr int XS_BYTES = TM * BK * 2;        // 2 KB
+constexpr int WS_BYTES = EP * BK * 4;        // 64 KB
+constexpr int STAGE_BYTES = XS_BYTES + WS_BYTES;
+constexpr int NSTAGE = 2;
+constexpr int LLD = EP + 4;                  // logits row stride (floats)
+constexpr int SMEM = NSTAGE * STAGE_BYTES;   // 132 KB (logits and ids reuse it)
+static_assert(TM * LLD * 4 + TM * kMaxTopK * 4 <= SMEM, "logits do not fit");
+
+__device__ __forceinline__ void load_stage(const RouterArgs& a, uint8_t* st, int t0, int kb) {
+  const int tid = threadIdx.x;
+  uint8_t* xs = st;
+  uint8_t* ws = st + XS_BYTES;
+  if (tid < TM * 4) {
+    const int tok = tid >> 2, c = tid & 3;
+    const bool v = (t0 + tok) < a.T;
+    const __nv_bfloat16* src = a.x + (size_t)(v ? t0 + tok : 0) * a.H + kb * BK + c * 8;
+    cp_async16(xs + tok * 64 + c * 16, src, v ? 16u : 0u);
+  }
+#pragma unroll
+  for (int i = 0; i < (EP * 8) / NTH; ++i) {
+    const int idx = tid + NTH * i;
+    const int e = idx >> 3, c = idx & 7;
+    const bool v = e < a.E;
+    const float* src = a.wr + (size_t)(v ? e : 0) * a.H + kb * BK + c * 4;
+    cp_async16(ws + e * 128 + ((c ^ (e & 7)) << 4), src, v ? 16u : 0u);
+  }
+}
+
+__global__ void __launch_bounds__(NTH, 1) router_kernel(const RouterArgs a) {
+  extern __shared__ __align__(128) uint8_t smem[];
+  const int tid = threadIdx.x;
+  const int t0 = blockIdx.x * TM;
+  const int tg = tid >> 6;   // token group: tokens tg*8 .. tg*8+7
+  const int el = tid & 63;   // experts el + 64 j
+  float acc[8][8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i)
+#pragma unroll
+    for (int j = 0; j < 8; ++j) acc[i][j] = 0.f;
+
+  const int nk = a.H / BK;
+  load_stage(a, smem, t0, 0);
+  cp_async_commit();
+  for (int kb = 0; kb < nk; ++kb) {
+    if (kb + 1 < nk) load_stage(a, smem + ((kb + 1) % NSTAGE) * STAGE_BYTES, t0, kb + 1);
+    cp_async_commit();
+    cp_async_wait<1>();
+    __syncthreads();
+    const uint8_t* xs = smem + (kb % NSTAGE) * STAGE_BYTES;
+    const uint8_t* ws = xs + XS_BYTES;
+#pragma unroll
+    for (int kq = 0; kq < BK / 4; ++kq) {
+      float4 w[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int e = el + 64 * j;
+        w[j] = *reinterpret_cast<const float4*>(ws + e * 128 + ((kq ^ (e & 7)) << 4));
+      }
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const uint2 xv = *reinterpret_cast<const uint2*>(xs + (tg * 8 + i) * 64 + kq * 8);
+        const float x0 = bf16_lo(xv.x), x1 = bf16_hi(xv.x), x2 = bf16_lo(xv.y), x3 = bf16_hi(xv.y);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          float s = acc[i][j];
+          s = fmaf(x0, w[j].x, s);
+          s = fmaf(x1, w[j].y, s);
+          s = fmaf(x2, w[j].z, s);
+          s = fmaf(x3, w[j].w, s);
+          acc[i][j] = s;
+        }
+      }
+    }
+    __syncthreads();
+  }
+
+  // logits -> shared memory [TM][LLD]
+  float* L = reinterpret_cast<float*>(smem);
+  int* ids_s = reinterpret_cast<int*>(smem + TM * LLD * 4);
+#pragma unroll
+  for (int i = 0; i < 8; ++i)
+#pragma unroll
+    for (int j = 0; j < 8; ++j) L[(tg * 8 + i) * LLD + el + 64 * j] = acc[i][j];
+  __syncthreads();
+
+  // top-k: warp w handles tokens w*4 .. w*4+3
+  const int warp = tid >> 5, lane = tid & 31;
+  const int nvalid = min(TM, a.T - t0);
+  const int k = a.k;
+  const int per_lane = (a.E + 31) >> 5;  // <= 16
+  for (int q = 0; q < TM / 8; ++q) {
+    const int tok = warp * (TM / 8) + q;
+    if (tok >= nvalid) break;
+    float v[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      const int e = lane + 32 * i;
+      v[i] = (i < per_lane && e < a.E) ? L[tok * LLD + e] : -INFINITY;
+    }
+    uint32_t removed = 0;
+    float my_v = -INFINITY;
+    int my_i = 0;
+    float next_v = -INFINITY;  // logit of rank k (when k < E)
+    const int rounds = min(k + 1, a.E);
+    for (int r = 0; r < rounds; ++r) {
+      float bv = -INFINITY;
+      int bi = 0x7fffffff;
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const int e = lane + 32 * i;
+        if (i < per_lane && e < a.E && !((removed >> i) & 1u)) {
+          if (v[i] > bv || (v[i] == bv && e < bi)) { bv = v[i]; bi = e; }
+        }
+      }
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) {
+        const float ov = __shfl_xor_sync(0xffffffffu, bv, off);
+        const int oi = __shfl_xor_sync(0xffffffffu, bi, off);
+        if (ov > bv || (ov == bv && oi < bi)) { bv = ov; bi = oi; }
+      }
+      if ((bi & 31) == lane) removed |= 1u << (bi >> 5);
+      if (r == lane) { my_v = bv; my_i = bi; }
+      if (r == k) next_v = bv;
+    }
+    const float l0 = __shfl_sync(0xffffffffu, my_v, 0);
+    float ex = (lane < k) ? expf(my_v - l0) : 0.f;
+    float sum = ex;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
+    const size_t t = (size_t)t0 + tok;
+    if (lane < k) {
+      a.ids[t * k + lane] = my_i;
+      a.weights[t * k + lane] = ex / sum;
+      ids_s[tok * k + lane] = my_i;
+    }
+    if (a.gap != nullptr) {
+      const float lk1 = __shfl_sync(0xffffffffu, my_v, k - 1);
+      if (lane == 0) a.gap[t] = (k < a.E) ? (lk1 - next_v) : INFINITY;
+    }
+    if (a.wsg != nullptr) {
+      const __nv_bfloat16* xr = a.x + t * a.H;
+      float s = 0.f;
+      for (int h = lane * 8; h < a.H; h += 256) {
+        const uint4 xv = *reinterpret_cast<const uint4*>(xr + h);
+        const float4 w0 = *reinterpret_cast<const float4*>(a.wsg + h);
+        const float4 w1 = *reinterpret_cast<const float4*>(a.wsg + h + 4);
+        s = fmaf(bf16_lo(xv.x), w0.x, s);
+        s = fmaf(bf16_hi(xv.x), w0.y, s);
+        s = fmaf(bf16_lo(xv.y), w0.z, s);
+        s = fmaf(bf16_hi(xv.y), w0.w, s);
+        s = fmaf(bf16_lo(xv.z), w1.x, s);
+        s = fmaf(bf16_hi(xv.z), w1.y, s);
+        s = fmaf(bf16_lo(xv.w), w1.z, s);
+        s = fmaf(bf16_hi(xv.w), w1.w, s);
+      }
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+      if (lane == 0) a.sg[t] = 1.0f / (1.0f + expf(-s));
+    }
+  }
+  __syncthreads();
+
+  // per-block histogram of the routed ids (deterministic, no atomics)
+  const int nids = nvalid * k;
+  for (int e = tid; e < a.E; e += NTH) {
+    int c = 0;
+    for (int i = 0; i < nids; ++i) c += (ids_s[i] == e);
+    a.bcount[(size_t)blockIdx.x * a.E + e] = c;
+  }
+}
+}  // namespace
+
+cudaError_t launch_router(const RouterArgs& a, cudaStream_t s) {
+  static bool attr_done = false;
+  if (!attr_done) {
+    cudaError_t e =
+        cudaFuncSetAttribute(router_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM);
+    if (e != cudaSuccess) return e;
+    attr_done = true;
+  }
+  const int nb = (a.T + TM - 1) / TM;
+  if (nb == 0) return cudaSuccess;
+  router_kernel<<<nb, NTH, SMEM, s>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace msi
