@@ -1,0 +1,480 @@
+"""Benchmark of the slot-addressed MoE layer forward on GB300.
+
+python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl ours|reference]
+
+A step is one MoE layer forward over one batch of synthetic tokens: router
+(fp32 logits, softmax, top-k), histogram and permutation, expert staging into
+GPU slots (LRU waves, generation-fenced) where the workload streams, grouped
+SwiGLU expert FFN reading weights from slots, shared expert, combine.
+Default workload: the Qwen3-Next-shaped layer (hidden 2048, 512 experts,
+top-10, intermediate 512, shared expert) over 4,096 tokens with all 512
+experts resident in slots.  --workload prefill32k_lru64 runs the same layer
+at 32,768 tokens with a 64-slot pool: 448 of the 512 experts are staged from
+pinned host windows per call in LRU waves.
+
+Prints one JSON line (rank 0).  `value` is whole-job tokens/s over the timed
+steps (device time, CUDA events on the compute stream); `e2e` repeats the
+metric with the hidden rows copied from pinned host memory and the outputs
+read back inside the timed region; `roofline` is the dominant kernel's
+algorithmic work per launch over its event-timed duration; `cpu_baseline` is
+the fp64 oracle timed on a bounded sample on this host's cores.
+Multi-GPU (torchrun): independent replicas, one per GPU, no collective in the
+data path; the timing is the max over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "MoE-layer prefill tokens/s"
+PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+                  "sm_max_mhz": 2070.0}
+N_SMS = 152
+FP32_LANES_PER_SM = 128
+L2_BYTES = 129 * 1024 * 1024
+
+# dram__bytes_read.sum + dram__bytes_write.sum per launch from one ncu capture,
+# keyed by (workload, kernel kind); valid only while the kernel source hash matches.
+TRAFFIC = {}
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    return dict(PEAKS_FALLBACK), "fallback"
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    for name in ("gemm.cu", "router.cu", "permute.cu", "internal.cuh"):
+        with open(os.path.join(ROOT, "paper_2608_23805_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+# ---------------------------------------------------------------------------
+# Distributed plumbing (replicas only)
+# ---------------------------------------------------------------------------
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def aggregate(units_per_rank: float, seconds: float, world: int, backend_ready: bool):
+    """Whole-job throughput for independent replicas: the units all ranks
+    processed over the slowest rank's time (max over ranks)."""
+    if world > 1 and backend_ready:
+        import torch
+        import torch.distributed as dist
+        dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+        t = torch.tensor([seconds, units_per_rank], dtype=torch.float64, device=dev)
+        mx = t[:1].clone()
+        dist.all_reduce(mx, op=dist.ReduceOp.MAX)
+        tot = t[1:].clone()
+        dist.all_reduce(tot, op=dist.ReduceOp.SUM)
+        return float(tot.item()) / float(mx.item()), float(mx.item())
+    return units_per_rank / seconds, seconds
+
+
+# ---------------------------------------------------------------------------
+# Clock sampling during the timed region
+# ---------------------------------------------------------------------------
+
+class ClockSampler:
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.idx = gpu_index
+        self.proc = None
+        self.path = os.path.join("/tmp", "msi_clocks_%d_%d.csv" % (os.getpid(), gpu_index))
+
+    def start(self):
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.idx), "--query-gpu=" + self.Q,
+                                          "--format=csv,noheader,nounits", "-lms", os.environ.get("MSI_CLOCK_MS", "100")],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.f.close()
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx = float(parts[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        os.unlink(self.path)
+        return {"sm_mhz": float(np.median(sm)) if sm else None, "sm_max_mhz": mx,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# Workload setup (synthetic, seeded)
+# ---------------------------------------------------------------------------
+
+class Workload:
+    def __init__(self, name: str):
+        import torch
+
+        import synth
+        from paper_2608_23805_gb300 import api
+        self.cfg = cfg = synth.config(name)
+        self.name = name
+        E, H, I, eb = cfg.n_experts, cfg.hidden, cfg.inter, cfg.extent_bytes
+        self.windows = torch.empty(E * eb, dtype=torch.uint8, pin_memory=True)
+        synth.fill_extents(cfg, 0, self.windows.numpy())
+        self.router_np = synth.router_weight(cfg)
+        self.router = torch.from_numpy(self.router_np).cuda()
+        self.x_bits = synth.hidden(cfg)
+        self.x_host = torch.from_numpy(self.x_bits.view(np.int16)).view(torch.bfloat16).pin_memory()
+        self.x = self.x_host.cuda()
+        shared_w = gate_w = None
+        self.shared_np = self.gate_np = None
+        if cfg.has_shared:
+            self.shared_np = synth.shared_extent(cfg)
+            self.gate_np = synth.shared_gate_weight(cfg)
+            shared_w = torch.from_numpy(self.shared_np).cuda()
+            gate_w = torch.from_numpy(self.gate_np[None, :].copy()).cuda()
+        self.plan = api.Plan(n_layers=1, n_experts=E, top_k=cfg.top_k, hidden=H, inter=I,
+                             n_slots=cfg.n_slots, host_windows=self.windows,
+                             has_shared=cfg.has_shared, shared_w=shared_w, shared_gate_w=gate_w,
+                             wdtype=cfg.wdtype)
+        self.cs = torch.cuda.Stream()
+        self.ss = torch.cuda.Stream()
+        self.out = torch.empty_like(self.x)
+        self.ev = api.RouteEvent(cfg.tokens, cfg.top_k, E)
+        self.table = self.gens = None
+        if not cfg.lru:
+            for e in range(E):
+                self.plan.stage(e, 0, e, self.ss)
+            torch.cuda.synchronize()
+            self.table, self.gens = self.plan.slot_table(0)
+
+    def step(self, x=None):
+        x = self.x if x is None else x
+        if self.cfg.lru:
+            self.plan.forward_streamed(0, x, self.router, out=self.out, ev=self.ev, stream=self.cs,
+                                       stage_stream=self.ss)
+        else:
+            self.plan.forward(0, x, self.router, self.table, self.gens, out=self.out, ev=self.ev,
+                              stream=self.cs)
+
+
+def algorithmic(cfg, kind: str, units: dict):
+    """Algorithmic work per step of one kernel kind: (bound, flops, bytes).
+
+    rows = T*k routed rows; per routed row the gate-up GEMM does 2*H*2I flops
+    and the down GEMM 2*I*H; weights are read once per expert per step."""
+    T, H, I, E, k = cfg.tokens, cfg.hidden, cfg.inter, cfg.n_experts, cfg.top_k
+    rows = T * k
+    eb_w13 = 2 * I * H * 2
+    eb_w2 = H * I * 2
+    if kind == "gateup":
+        return 2.0 * rows * H * 2 * I, E * eb_w13 + rows * H * 2 + rows * I * 2
+    if kind == "down":
+        return 2.0 * rows * I * H, E * eb_w2 + rows * I * 2 + rows * H * 2
+    if kind == "shared_gateup":
+        return 2.0 * T * H * 2 * I, eb_w13 + T * H * 2 + T * I * 2
+    if kind == "shared_down":
+        return 2.0 * T * I * H, eb_w2 + T * I * 2 + T * H * 2
+    if kind == "router":
+        return 2.0 * T * H * E, T * H * 2 + E * H * 4 + T * k * 8
+    if kind == "combine":
+        return 2.0 * rows * H, rows * H * 2 + T * H * 2 * (2 if cfg.has_shared else 1) + T * k * 8
+    if kind in ("scan", "scatter"):
+        return 0.0, T * k * 4 * 3
+    return 0.0, 0.0
+
+
+def roofline(cfg, kt: dict, steps: int, peaks: dict, clocks: dict, workload: str):
+    """Roofline object of the dominant (largest summed time) kernel kind."""
+    kind = max(kt, key=lambda k: kt[k][0])
+    ms, launches = kt[kind]
+    flops, nbytes = algorithmic(cfg, kind, {})
+    per_launch_s = ms / 1e3 / max(launches, 1)
+    per_launch_flops = flops * steps / max(launches, 1)
+    per_launch_bytes = nbytes * steps / max(launches, 1)
+    ridge = peaks["bf16_tflops_sustained"] * 1e12 / (peaks["hbm_gbs"] * 1e9)
+    if kind == "router":
+        mhz = clocks.get("sm_mhz") or peaks.get("sm_max_mhz", 2070.0)
+        peak = N_SMS * FP32_LANES_PER_SM * 2 * mhz * 1e6 / 1e12
+        ach = per_launch_flops / per_launch_s / 1e12
+        r = {"bound": "alu", "achieved": ach, "peak": peak, "unit": "TFLOP/s",
+             "peak_source": "152 SMs x 128 FP32 lanes x 2 flop x median SM clock %.0f MHz" % mhz}
+    elif flops > 0 and flops / max(nbytes, 1) >= ridge:
+        ach = per_launch_flops / per_launch_s / 1e12
+        peak = peaks["bf16_tflops_sustained"]
+        r = {"bound": "tensor", "achieved": ach, "peak": peak, "unit": "TFLOP/s",
+             "peak_source": "bf16_tflops_sustained of measured (kernel timed inside the step)"}
+    else:
+        ach = per_launch_bytes / per_launch_s / 1e9
+        peak = peaks["hbm_gbs"]
+        r = {"bound": "hbm", "achieved": ach, "peak": peak, "unit": "GB/s",
+             "peak_source": "hbm_gbs of measured"}
+    r["frac"] = r["achieved"] / r["peak"]
+    r["kernel"] = kind
+    r["launches_per_step"] = launches / steps
+    r["ms_per_launch"] = ms / max(launches, 1)
+    t = TRAFFIC.get((workload, kind))
+    r["traffic"] = t["bytes_per_launch"] if (t and t.get("src_hash") == kernel_source_hash()) else None
+    return r
+
+
+def cpu_baseline(w: "Workload", tokens: int):
+    """The fp64 oracle, as it stands, on the first `tokens` tokens of the same
+    workload, on this host's cores; tokens/s."""
+    import oracle
+    cfg = w.cfg
+    eb = cfg.extent_bytes
+    wnp = w.windows.numpy()
+    kw = {}
+    if cfg.has_shared:
+        kw = dict(shared_extent=w.shared_np, w_sg=w.gate_np)
+    t0 = time.perf_counter()
+    oracle.moe_layer(w.x_bits[:tokens], w.router_np, cfg.top_k, lambda e: wnp[e * eb:(e + 1) * eb],
+                     cfg.hidden, cfg.inter, cfg.wdtype, **kw)
+    if cfg.lru:
+        sim = oracle.LRUWaveSim(cfg.n_slots)
+        sim.call(0, range(cfg.n_experts))
+    dt = time.perf_counter() - t0
+    cores = int(os.environ.get("OMP_NUM_THREADS", os.environ.get("OPENBLAS_NUM_THREADS", os.cpu_count() or 1)))
+    return {"value": tokens / dt, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+            "sample": "fp64 oracle forward of the first %d of %d tokens (router over all %d experts, "
+                      "expert FFNs, shared expert, combine, LRU-wave plan), %.1f s" %
+                      (tokens, cfg.tokens, cfg.n_experts, dt)}
+
+
+SAMPLE_TOKENS = {"prefill32k_lru64": 4096, "qwen3next_4k": 4096, "tiny": 64}
+
+
+# ---------------------------------------------------------------------------
+# Arms
+# ---------------------------------------------------------------------------
+
+def run_ours(args):
+    import torch
+    world, rank, local = dist_env()
+    backend = False
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", init_method="env://")
+        backend = True
+    else:
+        torch.cuda.set_device(0)
+    import __graft_entry__
+    __graft_entry__.build()
+    w = Workload(args.workload)
+    cfg = w.cfg
+    peaks, peak_kind = load_peaks()
+
+    flush = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device="cuda")
+    sampler = ClockSampler(local)
+    sampler.start()
+    w.plan.timing(True)
+    # warm-up immediately precedes the timed steps (an idle GPU drops its clocks and link state)
+    for _ in range(args.warmup):
+        flush.zero_()
+        torch.cuda.current_stream().synchronize()
+        w.step()
+    torch.cuda.synchronize()
+    w.plan.timing_read(reset=True)
+    if backend:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    launches0 = w.plan.launches()
+    staged0 = w.plan.counters()["h2d_bytes"]
+    evs = []
+    wall0 = time.perf_counter()
+    for _ in range(args.steps):
+        flush.zero_()                                # L2 flushed between timed steps (untimed)
+        torch.cuda.current_stream().synchronize()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(w.cs)
+        w.step()
+        b.record(w.cs)
+        evs.append((a, b))
+    torch.cuda.synchronize()
+    wall = time.perf_counter() - wall0
+    launches = w.plan.launches() - launches0
+    staged = (w.plan.counters()["h2d_bytes"] - staged0) // args.steps
+    dev_s = sum(a.elapsed_time(b) for a, b in evs) / 1e3
+    kt = w.plan.timing_read(reset=True)
+    w.plan.timing(False)
+    assert w.plan.status() == 0, "device status %d" % w.plan.status()
+
+    # e2e: hidden rows from pinned host memory in, outputs and route ids out
+    out_host = torch.empty_like(w.out, device="cpu").pin_memory()
+    ids_host = torch.empty_like(w.ev.ids, device="cpu").pin_memory()
+    x_dev = torch.empty_like(w.x)
+    e2e_evs = []
+    for _ in range(args.steps):
+        flush.zero_()
+        torch.cuda.current_stream().synchronize()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(w.cs)
+        with torch.cuda.stream(w.cs):
+            x_dev.copy_(w.x_host, non_blocking=True)
+        w.step(x_dev)
+        with torch.cuda.stream(w.cs):
+            out_host.copy_(w.out, non_blocking=True)
+            ids_host.copy_(w.ev.ids, non_blocking=True)
+        b.record(w.cs)
+        b.synchronize()
+        e2e_evs.append((a, b))
+    e2e_s = sum(a.elapsed_time(b) for a, b in e2e_evs) / 1e3
+    if backend:
+        torch.distributed.barrier()
+    clocks = sampler.stop()
+
+    units = cfg.tokens * args.steps
+    value, tmax = aggregate(units, dev_s, world, backend)
+    e2e_value, _ = aggregate(units, e2e_s, world, backend)
+    if rank != 0:
+        return
+    rl = roofline(cfg, {k: v for k, v in kt.items() if v[1] > 0}, args.steps, peaks, clocks,
+                  args.workload)
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": tmax / args.steps * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic: seeded N(0,1) bf16 hidden rows, N(0,0.02) bf16 expert weights, "
+                "N(0,0.02) fp32 router",
+        "config": {"workload": args.workload, "tokens": cfg.tokens, "hidden": cfg.hidden,
+                   "experts": cfg.n_experts, "top_k": cfg.top_k, "inter": cfg.inter,
+                   "shared_expert": cfg.has_shared, "slots": cfg.n_slots,
+                   "residency": "LRU waves of %d, staged from pinned host windows" % (cfg.n_slots // 2)
+                   if cfg.lru else "all experts resident",
+                   "weights": "bf16" if cfg.wdtype == 0 else "q4g32",
+                   "parallelism": "replicas" if world > 1 else "single GPU",
+                   "l2": "flushed between timed steps (2x L2 write, untimed)"},
+        "roofline": rl,
+        "e2e": {"value": e2e_value, "unit": "tokens/s",
+                "h2d_bytes_per_step": int(w.x.numel() * 2),
+                "d2h_bytes_per_step": int(w.out.numel() * 2 + w.ev.ids.numel() * 4),
+                "staged_h2d_bytes_per_step": int(staged)},
+        "gpu_launches": int(launches),
+        "clocks": clocks,
+        "kernels_ms_per_step": {k: round(v[0] / args.steps, 4) for k, v in kt.items() if v[1] > 0},
+        "wall_s_timed": wall,
+        "step_ms": [round(a.elapsed_time(b), 3) for a, b in evs],
+        "peaks": peak_kind,
+    }
+    if world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(w, SAMPLE_TOKENS.get(args.workload, 256))
+    print(json.dumps(line), flush=True)
+
+
+def run_reference(args):
+    """Reference arm: the fp64 CPU oracle as it stands, each step a bounded
+    sample (REF_TOKENS tokens) of the same workload, on this host's cores."""
+    world, rank, _ = dist_env()
+    if rank != 0:
+        return
+    import oracle
+    import synth
+    cfg = synth.config(args.workload)
+    ntok = REF_TOKENS.get(args.workload, 128)
+    eb = cfg.extent_bytes
+    x = synth.hidden(cfg, tokens=ntok)
+    wr = synth.router_weight(cfg)
+    cache = {}
+
+    def extent(e):
+        if e not in cache:
+            cache[e] = synth.expert_extent(cfg, 0, e)
+        return cache[e]
+
+    kw = {}
+    if cfg.has_shared:
+        kw = dict(shared_extent=synth.shared_extent(cfg), w_sg=synth.shared_gate_weight(cfg))
+    for e in range(cfg.n_experts):
+        extent(e)
+
+    def step():
+        oracle.moe_layer(x, wr, cfg.top_k, extent, cfg.hidden, cfg.inter, cfg.wdtype, **kw)
+        if cfg.lru:
+            oracle.LRUWaveSim(cfg.n_slots).call(0, range(cfg.n_experts))
+
+    for _ in range(args.warmup):
+        step()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    dt = time.perf_counter() - t0
+    value = ntok * args.steps / dt
+    cores = os.cpu_count() or 1
+    sample = ("fp64 oracle forward of %d of the %d tokens per step (router over all %d experts, "
+              "expert FFNs, shared expert, combine, LRU-wave plan)" % (ntok, cfg.tokens, cfg.n_experts))
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt / args.steps * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (same seeded inputs)",
+        "config": {"workload": args.workload, "tokens": cfg.tokens, "sample_tokens": ntok},
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }), flush=True)
+
+
+REF_TOKENS = {"prefill32k_lru64": 256, "qwen3next_4k": 256, "tiny": 64}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--workload", default="qwen3next_4k",
+                    choices=["prefill32k_lru64", "qwen3next_4k", "tiny"])
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -215,6 +215,29 @@ msi_status msi_trace_clear(msi_plan* plan);
 
 msi_status msi_get_counters(const msi_plan* plan, msi_counters* out);
 
+/* Kernel kinds for per-kernel timing. */
+enum {
+  MSI_K_UPLOAD = 0,        /* per-call tables / forward begin */
+  MSI_K_ROUTER = 1,        /* fp32 logits + top-k + weights + block histogram */
+  MSI_K_SCAN = 2,          /* column prefix over router blocks */
+  MSI_K_SCATTER = 3,       /* stable permutation */
+  MSI_K_SETUP = 4,         /* generation re-check + GEMM groups */
+  MSI_K_GATEUP = 5,        /* routed gate-up GEMM with SwiGLU epilogue */
+  MSI_K_DOWN = 6,          /* routed down GEMM */
+  MSI_K_SHARED_GATEUP = 7, /* shared-expert gate-up GEMM */
+  MSI_K_SHARED_DOWN = 8,   /* shared-expert down GEMM */
+  MSI_K_COMBINE = 9,       /* weighted combine */
+  MSI_K_PUBLISH = 10,      /* slot generation publication (staging stream) */
+  MSI_K_COUNT = 11
+};
+
+/* Per-kernel timing: when enabled, every launch is bracketed by CUDA events on
+ * its own stream.  msi_timing_read waits for the recorded launches and returns
+ * per kind the summed milliseconds and launch counts (arrays [MSI_K_COUNT]);
+ * reset != 0 clears the accumulators. */
+msi_status msi_timing_enable(msi_plan* plan, int on);
+msi_status msi_timing_read(msi_plan* plan, double* ms, uint64_t* launches, int reset);
+
 /* Number of kernels the library launched since the plan was created. */
 uint64_t msi_kernel_launches(const msi_plan* plan);
 

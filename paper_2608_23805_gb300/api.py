@@ -159,6 +159,17 @@ class Plan:
         N.check(N.lib().msi_get_counters(self.h, ctypes.byref(c)), "msi_get_counters")
         return {f: getattr(c, f) for f, _ in c._fields_}
 
+    def timing(self, on: bool = True):
+        N.check(N.lib().msi_timing_enable(self.h, int(on)), "msi_timing_enable")
+
+    def timing_read(self, reset: bool = True) -> dict:
+        """{kind: (milliseconds summed, launches)} of the timed launches."""
+        ms = np.zeros(len(N.KERNEL_KINDS), dtype=np.float64)
+        n = np.zeros(len(N.KERNEL_KINDS), dtype=np.uint64)
+        N.check(N.lib().msi_timing_read(self.h, ms.ctypes.data, n.ctypes.data, int(reset)),
+                "msi_timing_read")
+        return {k: (float(ms[i]), int(n[i])) for i, k in enumerate(N.KERNEL_KINDS)}
+
     def launches(self) -> int:
         return int(N.lib().msi_kernel_launches(self.h))
 

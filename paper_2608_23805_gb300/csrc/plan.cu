@@ -50,11 +50,22 @@ msi_status cuda_fail(cudaError_t e, const char* what) {
     if (e_ != cudaSuccess) return cuda_fail(e_, #call);        \
   } while (0)
 
-#define LAUNCH(plan, call)                                     \
-  do {                                                         \
-    cudaError_t e_ = (call);                                   \
-    if (e_ != cudaSuccess) return cuda_fail(e_, #call);        \
-    (plan)->launches++;                                        \
+// Launch one kernel of kind `kind` on `strm`, counted and (optionally) timed.
+#define LAUNCH(plan, kind, strm, call)                                   \
+  do {                                                                   \
+    cudaEvent_t ea_ = nullptr, eb_ = nullptr;                            \
+    if ((plan)->timer.on) {                                              \
+      ea_ = (plan)->timer.get();                                         \
+      eb_ = (plan)->timer.get();                                         \
+      cudaEventRecord(ea_, (strm));                                      \
+    }                                                                    \
+    cudaError_t e_ = (call);                                             \
+    if (e_ != cudaSuccess) return cuda_fail(e_, #call);                  \
+    if (ea_ != nullptr) {                                                \
+      cudaEventRecord(eb_, (strm));                                      \
+      (plan)->timer.pending.push_back({(kind), ea_, eb_});               \
+    }                                                                    \
+    (plan)->launches++;                                                  \
   } while (0)
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
@@ -141,6 +152,43 @@ struct WsLayout {
 
 constexpr long long kDeviceWaitCycles = 4000000000LL;  // ~2 s at GB300 clocks
 
+// Opt-in per-kernel timing: event pairs around each launch, resolved on read.
+struct KernelTimer {
+  bool on = false;
+  std::vector<cudaEvent_t> freel;
+  struct Rec { int kind; cudaEvent_t a, b; };
+  std::vector<Rec> pending;
+  double ms[MSI_K_COUNT] = {};
+  uint64_t n[MSI_K_COUNT] = {};
+
+  cudaEvent_t get() {
+    if (!freel.empty()) {
+      cudaEvent_t e = freel.back();
+      freel.pop_back();
+      return e;
+    }
+    cudaEvent_t e = nullptr;
+    cudaEventCreate(&e);
+    return e;
+  }
+  void resolve() {
+    for (auto& r : pending) {
+      float t = 0.f;
+      cudaEventSynchronize(r.b);
+      if (cudaEventElapsedTime(&t, r.a, r.b) == cudaSuccess) ms[r.kind] += t;
+      n[r.kind]++;
+      freel.push_back(r.a);
+      freel.push_back(r.b);
+    }
+    pending.clear();
+  }
+  void destroy() {
+    resolve();
+    for (auto e : freel) cudaEventDestroy(e);
+    freel.clear();
+  }
+};
+
 }  // namespace
 
 struct msi_plan {
@@ -164,6 +212,7 @@ struct msi_plan {
   int calls = 0;
   int C = 1;
   bool dying = false;
+  KernelTimer timer;
   std::mutex mu;
 
   explicit msi_plan(int S) : holds(S) {
@@ -278,7 +327,7 @@ msi_status stage_enqueue(msi_plan* p, int layer, const std::vector<WaveEntry>& m
     pub.gen[i] = misses[i].gen;
     pub.obj[i] = obj_key(layer, misses[i].expert);
   }
-  LAUNCH(p, launch_publish(inv, p->d_gen, stage));
+  LAUNCH(p, MSI_K_PUBLISH, stage, launch_publish(inv, p->d_gen, stage));
   const uint64_t eb = p->d.extent_bytes;
   for (const auto& m : misses) {
     const char* src = static_cast<const char*>(p->d.host_windows) +
@@ -286,7 +335,7 @@ msi_status stage_enqueue(msi_plan* p, int layer, const std::vector<WaveEntry>& m
     char* dst = static_cast<char*>(p->d.slot_pool) + (size_t)m.slot * eb;
     CK(cudaMemcpyAsync(dst, src, eb, cudaMemcpyHostToDevice, stage));
   }
-  LAUNCH(p, launch_publish(pub, p->d_gen, stage));
+  LAUNCH(p, MSI_K_PUBLISH, stage, launch_publish(pub, p->d_gen, stage));
   int ev;
   st = p->pool.acquire(&ev);
   if (st != MSI_OK) return st;
@@ -350,11 +399,11 @@ msi_status front(msi_plan* p, FwdCtx& f, const TableParams& tp) {
   const int E = d.n_experts, k = d.top_k, H = d.hidden, I = d.inter;
   void* ws = f.ws;
   const WsLayout& L = f.L;
-  LAUNCH(p, launch_upload(tp, at<int>(ws, L.table), at<unsigned long long>(ws, L.expected),
+  LAUNCH(p, MSI_K_UPLOAD, f.cs, launch_upload(tp, at<int>(ws, L.table), at<unsigned long long>(ws, L.expected),
                           at<int>(ws, L.status), d.has_shared ? at<Group>(ws, L.sh_group) : nullptr,
                           at<int>(ws, L.sh_total), f.cs));
   if (f.T == 0) {
-    LAUNCH(p, launch_zero_counts(f.ev->counts, E, f.cs));
+    LAUNCH(p, MSI_K_UPLOAD, f.cs, launch_zero_counts(f.ev->counts, E, f.cs));
     return MSI_OK;
   }
   const int nb = (f.T + kRouterTM - 1) / kRouterTM;
@@ -371,12 +420,12 @@ msi_status front(msi_plan* p, FwdCtx& f, const TableParams& tp) {
   ra.gap = f.ev->gap;
   ra.sg = at<float>(ws, L.sg);
   ra.bcount = at<int>(ws, L.bcount);
-  LAUNCH(p, launch_router(ra, f.cs));
+  LAUNCH(p, MSI_K_ROUTER, f.cs, launch_router(ra, f.cs));
   ScanArgs sa{at<int>(ws, L.bcount), nb, E, at<int>(ws, L.bbase), f.ev->counts};
-  LAUNCH(p, launch_colscan(sa, f.cs));
+  LAUNCH(p, MSI_K_SCAN, f.cs, launch_colscan(sa, f.cs));
   ScatterArgs xa{f.ev->ids, f.ev->counts, at<int>(ws, L.bbase), f.T, k, E, nb,
                  at<int>(ws, L.perm), at<int>(ws, L.inv), at<int>(ws, L.offsets)};
-  LAUNCH(p, launch_scatter(xa, f.cs));
+  LAUNCH(p, MSI_K_SCATTER, f.cs, launch_scatter(xa, f.cs));
   const size_t Tk = (size_t)f.T * k;
   if (!make_tmap(&f.tm_h, at<char>(ws, L.h), I, Tk, 128)) return MSI_ERR_CUDA;
   if (d.has_shared) {
@@ -426,9 +475,9 @@ msi_status routed_ffn(msi_plan* p, FwdCtx& f, int ng, int grid1, int grid2) {
   const Group* groups = at<Group>(f.ws, f.L.groups);
   const int* total = at<int>(f.ws, f.L.total);
   GemmArgs g1 = gateup_args(p, f, groups, ng, total, at<__nv_bfloat16>(f.ws, f.L.h));
-  LAUNCH(p, launch_gemm(kGateUpGather, p->tm_w13, p->tm_w13, g1, grid1, f.cs));
+  LAUNCH(p, MSI_K_GATEUP, f.cs, launch_gemm(kGateUpGather, p->tm_w13, p->tm_w13, g1, grid1, f.cs));
   GemmArgs g2 = down_args(p, f, groups, ng, total, at<__nv_bfloat16>(f.ws, f.L.yp));
-  LAUNCH(p, launch_gemm(kDown, f.tm_h, p->tm_w2, g2, grid2, f.cs));
+  LAUNCH(p, MSI_K_DOWN, f.cs, launch_gemm(kDown, f.tm_h, p->tm_w2, g2, grid2, f.cs));
   return MSI_OK;
 }
 
@@ -438,9 +487,9 @@ msi_status shared_ffn(msi_plan* p, FwdCtx& f) {
   const int* total = at<int>(f.ws, f.L.sh_total);
   const int mt = (f.T + kBM - 1) / kBM;
   GemmArgs s1 = gateup_args(p, f, g, 1, total, at<__nv_bfloat16>(f.ws, f.L.hs));
-  LAUNCH(p, launch_gemm(kGateUpTma, f.tm_x, p->tm_sh13, s1, std::min(p->sms, mt * s1.nt), f.cs));
+  LAUNCH(p, MSI_K_SHARED_GATEUP, f.cs, launch_gemm(kGateUpTma, f.tm_x, p->tm_sh13, s1, std::min(p->sms, mt * s1.nt), f.cs));
   GemmArgs s2 = down_args(p, f, g, 1, total, at<__nv_bfloat16>(f.ws, f.L.ys));
-  LAUNCH(p, launch_gemm(kDown, f.tm_hs, p->tm_sh2, s2, std::min(p->sms, mt * s2.nt), f.cs));
+  LAUNCH(p, MSI_K_SHARED_DOWN, f.cs, launch_gemm(kDown, f.tm_hs, p->tm_sh2, s2, std::min(p->sms, mt * s2.nt), f.cs));
   return MSI_OK;
 }
 
@@ -459,7 +508,7 @@ msi_status finish(msi_plan* p, FwdCtx& f) {
     c.H = d.hidden;
     c.k = d.top_k;
     c.status = at<int>(f.ws, f.L.status);
-    LAUNCH(p, launch_combine(c, f.cs));
+    LAUNCH(p, MSI_K_COMBINE, f.cs, launch_combine(c, f.cs));
   }
   CK(cudaMemcpyAsync(p->h_status, at<int>(f.ws, f.L.status), sizeof(int), cudaMemcpyDeviceToHost,
                      f.cs));
@@ -588,6 +637,7 @@ msi_status msi_plan_destroy(msi_plan* p) {
       if (s.consumer >= 0) cudaEventSynchronize(p->pool.ev[s.consumer]);
     }
     if (p->fwd_ev >= 0) cudaEventSynchronize(p->pool.ev[p->fwd_ev]);
+    p->timer.destroy();
     for (auto ev : p->pool.ev) cudaEventDestroy(ev);
     cudaFree(p->d_gen);
     cudaFreeHost(p->h_status);
@@ -724,7 +774,7 @@ msi_status msi_moe_forward(msi_plan* p, int layer, const void* x, int T, const f
     sa.groups = at<Group>(ws, f.L.groups);
     sa.total_mtiles = at<int>(ws, f.L.total);
     sa.status = at<int>(ws, f.L.status);
-    LAUNCH(p, launch_setup_resident(sa, f.cs));
+    LAUNCH(p, MSI_K_SETUP, f.cs, launch_setup_resident(sa, f.cs));
     const long long mt_max = ((long long)T * d.top_k + kBM - 1) / kBM + E;
     const int g1 = (int)std::min<long long>(p->sms, mt_max * (d.inter / 128));
     const int g2 = (int)std::min<long long>(p->sms, mt_max * (d.hidden / kBN));
@@ -879,7 +929,7 @@ msi_status msi_moe_forward_streamed(msi_plan* p, int layer, const void* x, int T
     sa.groups = at<Group>(ws, f.L.groups);
     sa.total_mtiles = at<int>(ws, f.L.total);
     sa.status = at<int>(ws, f.L.status);
-    LAUNCH(p, launch_setup_wave(sa, wp, f.cs));
+    LAUNCH(p, MSI_K_SETUP, f.cs, launch_setup_wave(sa, wp, f.cs));
     const int g1 = std::max(1, std::min(p->sms, mtiles * (d.inter / 128)));
     const int g2 = std::max(1, std::min(p->sms, mtiles * (d.hidden / kBN)));
     st = routed_ffn(p, f, wp.n, g1, g2);
@@ -948,5 +998,27 @@ msi_status msi_get_counters(const msi_plan* cp, msi_counters* out) {
 }
 
 uint64_t msi_kernel_launches(const msi_plan* p) { return p ? p->launches : 0; }
+
+msi_status msi_timing_enable(msi_plan* p, int on) {
+  if (p == nullptr) return MSI_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> g(p->mu);
+  p->timer.on = on != 0;
+  return MSI_OK;
+}
+
+msi_status msi_timing_read(msi_plan* p, double* ms, uint64_t* launches, int reset) {
+  if (p == nullptr || ms == nullptr || launches == nullptr) return MSI_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> g(p->mu);
+  p->timer.resolve();
+  for (int k = 0; k < MSI_K_COUNT; ++k) {
+    ms[k] = p->timer.ms[k];
+    launches[k] = p->timer.n[k];
+    if (reset) {
+      p->timer.ms[k] = 0.0;
+      p->timer.n[k] = 0;
+    }
+  }
+  return MSI_OK;
+}
 
 }  // extern "C"

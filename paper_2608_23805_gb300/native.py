@@ -28,6 +28,8 @@ MSI_W_Q4G32 = 1
 MSI_TRACE_HIT, MSI_TRACE_STAGE, MSI_TRACE_EVICT = 0, 1, 2
 MSI_SLOT_VACANT, MSI_SLOT_LOADING, MSI_SLOT_DEVICE_READY, MSI_SLOT_IN_USE, MSI_SLOT_RECYCLABLE = range(5)
 MSI_FWD_RESIDUAL = 1
+KERNEL_KINDS = ["upload", "router", "scan", "scatter", "setup", "gateup", "down", "shared_gateup",
+                "shared_down", "combine", "publish"]
 
 
 class msi_plan_desc(ctypes.Structure):
@@ -83,6 +85,8 @@ _SIGS = {
     "msi_trace_clear": (ctypes.c_int, [_P]),
     "msi_get_counters": (ctypes.c_int, [_P, ctypes.POINTER(msi_counters)]),
     "msi_kernel_launches": (ctypes.c_uint64, [_P]),
+    "msi_timing_enable": (ctypes.c_int, [_P, ctypes.c_int]),
+    "msi_timing_read": (ctypes.c_int, [_P, _P, _P, ctypes.c_int]),
     "msi_status_string": (ctypes.c_char_p, [ctypes.c_int]),
     "msi_last_cuda_error": (ctypes.c_char_p, []),
 }
