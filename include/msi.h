@@ -185,6 +185,22 @@ msi_status msi_moe_forward(msi_plan* plan, int layer, const void* hidden, int T,
                            const msi_route_event* ev, void* workspace, size_t workspace_bytes,
                            unsigned flags, msi_stream compute);
 
+/* msi_moe_forward for callers that cannot allocate device memory (code inside
+ * another runtime's memory budget without an allocator handle, plugins whose
+ * host framework owns every allocation, loops that forbid allocation after
+ * start-up).  The paper has no counterpart: this is a library convenience.
+ * Same arguments and behaviour as msi_moe_forward minus the workspace, which
+ * is a fixed 32 MiB device array inside the library, reserved on every GPU
+ * that loads the library until exit.  Returns MSI_ERR_WORKSPACE, enqueueing
+ * nothing, when msi_workspace_size(plan, T) exceeds 32 MiB.  The first call on
+ * a device resolves the array's address (make it before any stream capture).
+ * All calls share the array: calls whose kernels overlap on the GPU race, so
+ * serialise them.  The call itself allocates nothing. */
+msi_status msi_moe_forward_static(msi_plan* plan, int layer, const void* hidden, int T,
+                                  const float* router_w, const int32_t* slot_table,
+                                  const uint64_t* expected_generations, void* out,
+                                  const msi_route_event* ev, unsigned flags, msi_stream compute);
+
 /* Layer forward with plan-managed residency (LRU waves).  Routes on `compute`,
  * reads the per-expert counts back to the host (one synchronisation), then
  * processes the needed experts as hits then misses in waves of wave_capacity:

@@ -77,6 +77,8 @@ _SIGS = {
     "msi_moe_forward_streamed": (ctypes.c_int, [_P, ctypes.c_int, _P, ctypes.c_int, _P, _P,
                                                 ctypes.POINTER(msi_route_event), _P, ctypes.c_size_t,
                                                 ctypes.c_uint, _P, _P]),
+    "msi_moe_forward_static": (ctypes.c_int, [_P, ctypes.c_int, _P, ctypes.c_int, _P, _P, _P, _P,
+                                              ctypes.POINTER(msi_route_event), ctypes.c_uint, _P]),
     "msi_forward_status": (ctypes.c_int, [_P, ctypes.POINTER(ctypes.c_int)]),
     "msi_consumer_hold": (ctypes.c_int, [_P, ctypes.c_int]),
     "msi_consumer_release": (ctypes.c_int, [_P, ctypes.c_int]),
