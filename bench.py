@@ -202,8 +202,9 @@ def algorithmic(cfg, kind: str, units: dict):
     and the down GEMM 2*I*H; weights are read once per expert per step."""
     T, H, I, E, k = cfg.tokens, cfg.hidden, cfg.inter, cfg.n_experts, cfg.top_k
     rows = T * k
-    eb_w13 = 2 * I * H * 2
-    eb_w2 = H * I * 2
+    wb = 2.0 if cfg.wdtype == 0 else 0.5625      # bytes per weight (bf16, or 4-bit + fp16 scale / 32)
+    eb_w13 = 2 * I * H * wb
+    eb_w2 = H * I * wb
     if kind == "gateup":
         return 2.0 * rows * H * 2 * I, E * eb_w13 + rows * H * 2 + rows * I * 2
     if kind == "down":
@@ -279,7 +280,8 @@ def cpu_baseline(w: "Workload", tokens: int):
                       (tokens, cfg.tokens, cfg.n_experts, dt)}
 
 
-SAMPLE_TOKENS = {"prefill32k_lru64": 4096, "qwen3next_4k": 4096, "tiny": 64}
+SAMPLE_TOKENS = {"prefill32k_lru64": 4096, "prefill32k_q4_lru64": 4096, "qwen3next_4k": 4096,
+                 "tiny": 64}
 
 
 # ---------------------------------------------------------------------------
@@ -455,7 +457,7 @@ def run_reference(args):
     }), flush=True)
 
 
-REF_TOKENS = {"prefill32k_lru64": 256, "qwen3next_4k": 256, "tiny": 64}
+REF_TOKENS = {"prefill32k_lru64": 256, "prefill32k_q4_lru64": 256, "qwen3next_4k": 256, "tiny": 64}
 
 
 def main():
@@ -464,7 +466,7 @@ def main():
     ap.add_argument("--steps", type=int, default=10)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--workload", default="qwen3next_4k",
-                    choices=["prefill32k_lru64", "qwen3next_4k", "tiny"])
+                    choices=["qwen3next_4k", "prefill32k_lru64", "prefill32k_q4_lru64", "tiny"])
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()

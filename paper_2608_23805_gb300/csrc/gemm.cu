@@ -6,8 +6,14 @@
 // published for it (Sec. "Stable Slots and Bundle Publication").
 //
 // One persistent kernel per projection pair:
-//   gate-up (kGateUpGather / kGateUpTma):  h = silu(x Wg^T) * (x Wu^T)   -> bf16
-//   down    (kDown):                        y = h W2^T                     -> bf16
+//   gate-up (kGateUpGather / kGateUpTma / kGateUpGatherQ4):  h = silu(x Wg^T) * (x Wu^T) -> bf16
+//   down    (kDown / kDownQ4):                                y = h W2^T                  -> bf16
+// The q4 modes read 4-bit weights (one fp16 scale per 32 weights of a row)
+// from the slot and dequantise them to bf16 in shared memory inside the
+// producer: eight warps prefetch codes and scales with cp.async into a
+// three-stage raw ring and each thread converts its own B row
+// (w = scale * (q - 8), rounded once to bf16) into the swizzled layout the
+// MMA reads, so the weights cross HBM at 0.5625 bytes each.
 // Tile: 128 token rows x 256 weight rows x 64 K per stage, 4-stage smem ring,
 // fp32 accumulators double-buffered in TMEM (2 x 256 columns).  Weights (B)
 // come by TMA from the slot pool viewed as one 2-D tensor per operand; the
@@ -17,9 +23,12 @@
 //
 // Roles (warp-specialised):  warps 0-3 epilogue (TMEM -> registers -> global,
 // one token row per thread), warp 4 MMA issue + TMEM allocation, warp 5 TMA
-// producer, warps 6-9 row gather (gather mode only).  Every wait is bounded;
+// producer, warps 6-9 row gather (gather modes), then eight dequant warps
+// (q4 modes).  Every wait is bounded;
 // on expiry the CTA raises its abort flag, all roles drain and the kernel
 // reports MSI_ERR_TIMEOUT in the status word.
+#include <cuda_fp16.h>
+
 #include "internal.cuh"
 
 namespace msi {
@@ -31,13 +40,25 @@ constexpr int kGatherWarps = 4;
 constexpr int kLag = 2;  // gather stages in flight before signalling
 constexpr uint32_t kIdesc = idesc_bf16(kBM, kBN);
 
+constexpr int kDqWarps = 8;   // one thread per B row (256 rows)
+constexpr int kRaw = 3;       // raw (packed) stages in flight ahead of conversion
+constexpr int kRawRowBytes = 32;  // 64 codes of one B row per stage
+
 template <int MODE>
 struct Cfg {
-  static constexpr bool kGather = (MODE == kGateUpGather);
+  static constexpr bool kQ4 = (MODE == kGateUpGatherQ4 || MODE == kDownQ4);
+  static constexpr bool kGather = (MODE == kGateUpGather || MODE == kGateUpGatherQ4);
+  static constexpr bool kGateUp = (MODE == kGateUpGather || MODE == kGateUpTma || MODE == kGateUpGatherQ4);
   static constexpr bool kTmaA = !kGather;
-  static constexpr bool kGateUp = (MODE != kDown);
-  static constexpr int kThreads = (6 + (kGather ? kGatherWarps : 0)) * 32;
-  static constexpr uint32_t kTxBytes = kBBytes + (kTmaA ? kABytes : 0);
+  static constexpr bool kTmaB = !kQ4;
+  static constexpr bool kTmaAny = kTmaA || kTmaB;
+  static constexpr int kGatherWarp0 = 6;
+  static constexpr int kDqWarp0 = 6 + (kGather ? kGatherWarps : 0);
+  static constexpr int kThreads = (kDqWarp0 + (kQ4 ? kDqWarps : 0)) * 32;
+  static constexpr uint32_t kTxBytes = (kTmaB ? kBBytes : 0) + (kTmaA ? kABytes : 0);
+  static constexpr int kFullCount = (kTmaAny ? 1 : 0) + (kGather ? kGatherWarps : 0) + (kQ4 ? kDqWarps : 0);
+  static constexpr int kRawBytes = kQ4 ? kRaw * kBN * (kRawRowBytes + 4) : 0;
+  static constexpr int kSmem = 1024 + kStages * (kABytes + kBBytes) + kRawBytes + 256;
 };
 
 struct TileCoord {
@@ -62,10 +83,6 @@ __device__ __forceinline__ TileCoord decode_tile(const GemmArgs& a, int t) {
 
 }  // namespace
 
-int gemm_smem_bytes() {
-  return 1024 /* alignment slack */ + kStages * (kABytes + kBBytes) + 256 /* barriers */;
-}
-
 template <int MODE>
 __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
     grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA,
@@ -76,7 +93,9 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
                                              ~static_cast<uintptr_t>(1023));
   uint8_t* sA = smem;
   uint8_t* sB = smem + kStages * kABytes;
-  uint64_t* full = reinterpret_cast<uint64_t*>(sB + kStages * kBBytes);
+  uint8_t* raw_codes = sB + kStages * kBBytes;                    // q4: [kRaw][256][32]
+  uint32_t* raw_scales = reinterpret_cast<uint32_t*>(raw_codes + (C::kQ4 ? kRaw * kBN * kRawRowBytes : 0));
+  uint64_t* full = reinterpret_cast<uint64_t*>(raw_codes + C::kRawBytes);
   uint64_t* empty = full + kStages;
   uint64_t* tfull = empty + kStages;
   uint64_t* tempty = tfull + 2;
@@ -89,7 +108,7 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
-      mbar_init(&full[s], 1 + (C::kGather ? kGatherWarps : 0));
+      mbar_init(&full[s], C::kFullCount);
       mbar_init(&empty[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
@@ -105,7 +124,7 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
     tmem_relinquish();
   }
   if (warp == 5 && lane == 0) {
-    tma_prefetch(&tmB);
+    if (C::kTmaB) tma_prefetch(&tmB);
     if (C::kTmaA) tma_prefetch(&tmA);
   }
   tc_fence_before();
@@ -117,7 +136,7 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
 
   if (warp == 5) {
     // ------------------------------------------------------------- TMA producer
-    if (lane == 0) {
+    if (lane == 0 && C::kTmaAny) {
       uint32_t it = 0;
       for (int t = blockIdx.x; t < total; t += gridDim.x) {
         const TileCoord tc = decode_tile(a, t);
@@ -131,10 +150,10 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
           if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, lim)) { ok = false; break; }
           mbar_arrive_expect_tx(&full[s], C::kTxBytes);
           uint8_t* b = sB + s * kBBytes;
-          if (C::kGateUp) {
+          if (C::kTmaB && C::kGateUp) {
             tma_load_2d(b, &tmB, &full[s], kb * kBK, brow + tc.n * 128);
             tma_load_2d(b + kBBytes / 2, &tmB, &full[s], kb * kBK, brow + a.up_off + tc.n * 128);
-          } else {
+          } else if (C::kTmaB) {
             tma_load_2d(b, &tmB, &full[s], kb * kBK, brow + tc.n * kBN);
             tma_load_2d(b + kBBytes / 2, &tmB, &full[s], kb * kBK, brow + tc.n * kBN + 128);
           }
@@ -247,9 +266,9 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(&tempty[acc]);
     }
-  } else if (C::kGather) {
+  } else if (C::kGather && warp < C::kGatherWarp0 + kGatherWarps) {
     // ------------------------------------------------------------- row gather
-    const int gt = threadIdx.x - 6 * 32;  // 0..127
+    const int gt = threadIdx.x - C::kGatherWarp0 * 32;  // 0..127
     const int chunk = gt & 7;             // 16-byte chunk of a 128-byte row slice
     const int r0 = gt >> 3;               // rows r0 + 16 i
     uint32_t it = 0, arrived = 0;
@@ -302,6 +321,78 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
         ++arrived;
       }
     }
+  } else if (C::kQ4) {
+    // ------------------------------------------------------------- q4 dequant
+    const int d = threadIdx.x - C::kDqWarp0 * 32;  // B row of this thread, 0..255
+    const uint32_t my_tiles =
+        (uint32_t)blockIdx.x < (uint32_t)total ? (total - 1 - blockIdx.x) / gridDim.x + 1 : 0;
+    const uint32_t nstages = my_tiles * a.kblocks;
+    // prefetch cursor: (tile, kb) of the next raw stage, with this row's sources
+    uint32_t jp = 0;
+    int cur_tile = -1;
+    const uint8_t* code_row = nullptr;
+    const uint8_t* scale_row = nullptr;
+    auto issue = [&](uint32_t j) {
+      const int tile_idx = (int)(j / a.kblocks);
+      const int kb = (int)(j % a.kblocks);
+      if (tile_idx != cur_tile) {
+        cur_tile = tile_idx;
+        const TileCoord tc = decode_tile(a, blockIdx.x + tile_idx * gridDim.x);
+        const uint8_t* base =
+            a.q4_pool + (unsigned long long)__ldg(&a.groups[tc.g].slot) * a.q4_extent;
+        int row;
+        if (C::kGateUp) row = d < 128 ? tc.n * 128 + d : a.up_off + tc.n * 128 + (d - 128);
+        else row = tc.n * kBN + d;
+        code_row = base + a.q4_code_off + (size_t)row * a.q4_code_ld;
+        scale_row = base + a.q4_scale_off + (size_t)row * a.q4_scale_ld;
+      }
+      const int r = j % kRaw;
+      uint8_t* dst = raw_codes + (r * kBN + d) * kRawRowBytes;
+      cp_async16(dst, code_row + kb * 32, 16u);
+      cp_async16(dst + 16, code_row + kb * 32 + 16, 16u);
+      cp_async4(&raw_scales[r * kBN + d], scale_row + kb * 4);
+    };
+    for (int i = 0; i < kRaw - 1; ++i, ++jp) {
+      if (jp < nstages) issue(jp);
+      cp_async_commit();
+    }
+    bool ok = true;
+    for (uint32_t it = 0; it < nstages; ++it, ++jp) {
+      if (jp < nstages) issue(jp);
+      cp_async_commit();
+      cp_async_wait<kRaw - 1>();  // this thread's raw stage `it` has landed
+      const int s = it % kStages;
+      const uint32_t ph = (it / kStages) & 1;
+      if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, lim)) { ok = false; break; }
+      const int r = it % kRaw;
+      const uint4* rc = reinterpret_cast<const uint4*>(raw_codes + (r * kBN + d) * kRawRowBytes);
+      const uint4 c0 = rc[0], c1 = rc[1];
+      const uint32_t sc = raw_scales[r * kBN + d];
+      const float s0 = __half2float(__ushort_as_half((unsigned short)(sc & 0xFFFFu)));
+      const float s1 = __half2float(__ushort_as_half((unsigned short)(sc >> 16)));
+      uint8_t* dst_row = sB + s * kBBytes + d * 128;
+      const uint32_t words[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
+#pragma unroll
+      for (int c = 0; c < 8; ++c) {
+        const float sc_f = c < 4 ? s0 : s1;
+        const uint32_t w = words[c];
+        uint32_t o[4];
+#pragma unroll
+        for (int b = 0; b < 4; ++b) {
+          const uint32_t lo = (w >> (8 * b)) & 0xFu, hi = (w >> (8 * b + 4)) & 0xFu;
+          // exact small integers: 2^23 + q - (2^23 + 8) = q - 8
+          const float ql = __uint_as_float(0x4B000000u | lo) - 8388616.0f;
+          const float qh = __uint_as_float(0x4B000000u | hi) - 8388616.0f;
+          o[b] = pack_bf16x2(ql * sc_f, qh * sc_f);
+        }
+        *reinterpret_cast<uint4*>(dst_row + ((c ^ (d & 7)) << 4)) = make_uint4(o[0], o[1], o[2], o[3]);
+      }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&full[s]);
+    }
+    cp_async_wait<0>();
+    (void)ok;
   }
 
   tc_fence_before();
@@ -318,7 +409,7 @@ template <int MODE>
 static cudaError_t launch_mode(const CUtensorMap& tmA, const CUtensorMap& tmB, const GemmArgs& a,
                                int grid, cudaStream_t s) {
   static bool attr_done = false;
-  const int smem = gemm_smem_bytes();
+  const int smem = Cfg<MODE>::kSmem;
   if (!attr_done) {
     cudaError_t e = cudaFuncSetAttribute(grouped_gemm_kernel<MODE>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
@@ -335,6 +426,8 @@ cudaError_t launch_gemm(int mode, const CUtensorMap& tmA, const CUtensorMap& tmB
     case kGateUpGather: return launch_mode<kGateUpGather>(tmA, tmB, a, grid, s);
     case kGateUpTma: return launch_mode<kGateUpTma>(tmA, tmB, a, grid, s);
     case kDown: return launch_mode<kDown>(tmA, tmB, a, grid, s);
+    case kGateUpGatherQ4: return launch_mode<kGateUpGatherQ4>(tmA, tmB, a, grid, s);
+    case kDownQ4: return launch_mode<kDownQ4>(tmA, tmB, a, grid, s);
     default: return cudaErrorInvalidValue;
   }
 }

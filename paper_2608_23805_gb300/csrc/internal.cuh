@@ -132,6 +132,13 @@ struct GemmArgs {
   int top_k;
   int* status;
   long long wait_limit;     // clock64 cycles per bounded wait
+  // 4-bit weights (q4 modes): codes and fp16 scales read from the slot pool
+  const uint8_t* q4_pool;
+  unsigned long long q4_extent;  // bytes per slot
+  long long q4_code_off;         // byte offset of this operand's codes in an extent
+  int q4_code_ld;                // bytes per weight row of codes (K / 2)
+  long long q4_scale_off;        // byte offset of this operand's scales in an extent
+  int q4_scale_ld;               // bytes per weight row of scales (K / 16)
 };
 
 struct CombineArgs {
@@ -146,7 +153,7 @@ struct CombineArgs {
   const int* status;
 };
 
-enum GemmMode { kGateUpGather = 0, kGateUpTma = 1, kDown = 2 };
+enum GemmMode { kGateUpGather = 0, kGateUpTma = 1, kDown = 2, kGateUpGatherQ4 = 3, kDownQ4 = 4 };
 
 // ---------------------------------------------------------------------------
 // Launchers (return cudaError_t of the launch)
@@ -173,7 +180,6 @@ constexpr int kBK = 64;
 constexpr int kStages = 4;
 constexpr int kABytes = kBM * kBK * 2;
 constexpr int kBBytes = kBN * kBK * 2;
-int gemm_smem_bytes();
 
 // ---------------------------------------------------------------------------
 // PTX wrappers (device)
@@ -253,6 +259,9 @@ __device__ __forceinline__ void cp_async16(void* dst, const void* src, uint32_t 
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_u32(dst)), "l"(src),
                "r"(src_bytes)
                : "memory");
+}
+__device__ __forceinline__ void cp_async4(void* dst, const void* src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
 }
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
 template <int N>

@@ -225,7 +225,8 @@ namespace {
 bool shape_ok(const msi_plan_desc& d) {
   return d.n_experts >= 1 && d.n_experts <= kMaxExperts && d.top_k >= 1 &&
          d.top_k <= std::min(d.n_experts, kMaxTopK) && d.hidden >= 256 && d.hidden % 256 == 0 &&
-         d.inter >= 128 && d.inter % 128 == 0 && d.wdtype == MSI_W_BF16;
+         d.inter >= 128 && d.inter % 128 == 0 &&
+         (d.wdtype == MSI_W_BF16 || d.wdtype == MSI_W_Q4G32);
 }
 
 WsLayout layout(const msi_plan* p, int T) {
@@ -472,11 +473,31 @@ GemmArgs down_args(msi_plan* p, FwdCtx& f, const Group* groups, int ng, const in
 }
 
 msi_status routed_ffn(msi_plan* p, FwdCtx& f, int ng, int grid1, int grid2) {
+  const auto& d = p->d;
   const Group* groups = at<Group>(f.ws, f.L.groups);
   const int* total = at<int>(f.ws, f.L.total);
   GemmArgs g1 = gateup_args(p, f, groups, ng, total, at<__nv_bfloat16>(f.ws, f.L.h));
-  LAUNCH(p, MSI_K_GATEUP, f.cs, launch_gemm(kGateUpGather, p->tm_w13, p->tm_w13, g1, grid1, f.cs));
   GemmArgs g2 = down_args(p, f, groups, ng, total, at<__nv_bfloat16>(f.ws, f.L.yp));
+  if (d.wdtype == MSI_W_Q4G32) {
+    // 4-bit extent: W13 codes [2I, H/2] | W2 codes [H, I/2] | W13 scales [2I, H/32] | W2 scales [H, I/32]
+    const long long HI = (long long)d.hidden * d.inter;
+    for (GemmArgs* g : {&g1, &g2}) {
+      g->q4_pool = static_cast<const uint8_t*>(d.slot_pool);
+      g->q4_extent = d.extent_bytes;
+    }
+    g1.q4_code_off = 0;
+    g1.q4_code_ld = d.hidden / 2;
+    g1.q4_scale_off = 3 * HI / 2;
+    g1.q4_scale_ld = d.hidden / 16;
+    g2.q4_code_off = HI;
+    g2.q4_code_ld = d.inter / 2;
+    g2.q4_scale_off = 3 * HI / 2 + HI / 8;
+    g2.q4_scale_ld = d.inter / 16;
+    LAUNCH(p, MSI_K_GATEUP, f.cs, launch_gemm(kGateUpGatherQ4, f.tm_h, f.tm_h, g1, grid1, f.cs));
+    LAUNCH(p, MSI_K_DOWN, f.cs, launch_gemm(kDownQ4, f.tm_h, f.tm_h, g2, grid2, f.cs));
+    return MSI_OK;
+  }
+  LAUNCH(p, MSI_K_GATEUP, f.cs, launch_gemm(kGateUpGather, p->tm_w13, p->tm_w13, g1, grid1, f.cs));
   LAUNCH(p, MSI_K_DOWN, f.cs, launch_gemm(kDown, f.tm_h, p->tm_w2, g2, grid2, f.cs));
   return MSI_OK;
 }

@@ -71,6 +71,9 @@ def _load():
             lib.synth_normal_f32.restype = None
             lib.synth_normal_f32.argtypes = [ctypes.c_uint64, ctypes.c_uint64, ctypes.c_double,
                                              ctypes.c_void_p]
+            lib.synth_quantize_q4g32.restype = None
+            lib.synth_quantize_q4g32.argtypes = [ctypes.c_void_p, ctypes.c_uint64, ctypes.c_uint64,
+                                                 ctypes.c_void_p, ctypes.c_void_p]
             lib.synth_raw_u64.restype = None
             lib.synth_raw_u64.argtypes = [ctypes.c_uint64, ctypes.c_uint64, ctypes.c_void_p]
             _lib = lib
@@ -191,17 +194,13 @@ def quantize_q4g32(w_bf16: np.ndarray):
     scale = fp16(absmax / 7), q = clip(rint(w / scale) + 8, 0, 15).
     Returns (packed uint8 [rows, cols/2] with the even column in the low
     nibble, scales as fp16 bits uint16 [rows, cols/32])."""
-    rows, cols = w_bf16.shape
+    w = np.ascontiguousarray(w_bf16, dtype=np.uint16)
+    rows, cols = w.shape
     assert cols % 32 == 0
-    w = _bf16_bits_to_f32(w_bf16).astype(np.float64).reshape(rows, cols // 32, 32)
-    amax = np.abs(w).max(axis=2)
-    scale16 = (amax / 7.0).astype(np.float16)
-    s = scale16.astype(np.float64)[:, :, None]
-    with np.errstate(divide="ignore", invalid="ignore"):
-        q = np.where(s > 0, np.rint(w / np.where(s > 0, s, 1.0)), 0.0)
-    q = np.clip(q + 8, 0, 15).astype(np.uint8).reshape(rows, cols)
-    packed = (q[:, 0::2] | (q[:, 1::2] << 4)).astype(np.uint8)
-    return packed, scale16.view(np.uint16)
+    packed = np.empty((rows, cols // 2), dtype=np.uint8)
+    scales = np.empty((rows, cols // 32), dtype=np.uint16)
+    _load().synth_quantize_q4g32(w.ctypes.data, rows, cols, packed.ctypes.data, scales.ctypes.data)
+    return packed, scales
 
 
 def expert_extent(cfg: MoEConfig, layer: int, expert: int) -> np.ndarray:
@@ -234,7 +233,6 @@ def _extent(cfg, k13, k2, layer, index):
 def fill_extents(cfg: MoEConfig, layer: int, out: np.ndarray, experts=None, threads: int = 0):
     """Write the extents of `experts` (default: all) of `layer` into
     out[e * extent_bytes : (e + 1) * extent_bytes] (uint8, e.g. a pinned host buffer)."""
-    from concurrent.futures import ThreadPoolExecutor
     eb = cfg.extent_bytes
     experts = range(cfg.n_experts) if experts is None else experts
     assert out.dtype == np.uint8 and out.size >= cfg.n_experts * eb
@@ -242,10 +240,6 @@ def fill_extents(cfg: MoEConfig, layer: int, out: np.ndarray, experts=None, thre
     def one(e):
         out[e * eb:(e + 1) * eb] = expert_extent(cfg, layer, e)
 
-    if cfg.wdtype == W_BF16:
-        for e in experts:          # the C generator is already OpenMP-parallel
-            one(e)
-    else:
-        with ThreadPoolExecutor(max_workers=threads or min(16, os.cpu_count() or 1)) as ex:
-            list(ex.map(one, experts))
+    for e in experts:              # the C generator and quantiser are OpenMP-parallel
+        one(e)
     return out

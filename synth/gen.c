@@ -76,3 +76,45 @@ void synth_normal_f32(uint64_t key, uint64_t n, double std_dev, float* out) {
 void synth_raw_u64(uint64_t key, uint64_t n, uint64_t* out) {
   for (uint64_t i = 0; i < n; ++i) out[i] = mix64(key + (i + 1) * GOLDEN);
 }
+
+/*
+ * Input preparation of the 4-bit workload (not part of the method): quantise
+ * bf16 weights [rows, cols] per 32 consecutive weights of a row:
+ * scale = fp16(absmax / 7) (round to nearest even), q = clamp(rint(w / scale) + 8, 0, 15),
+ * two codes per byte with the even column in the low nibble.
+ */
+static inline double bf16_to_double(uint16_t b) {
+  union { uint32_t u; float f; } v;
+  v.u = (uint32_t)b << 16;
+  return (double)v.f;
+}
+
+void synth_quantize_q4g32(const uint16_t* w, uint64_t rows, uint64_t cols, uint8_t* packed,
+                          uint16_t* scales) {
+  const uint64_t groups = cols / 32;
+#pragma omp parallel for schedule(static)
+  for (int64_t r = 0; r < (int64_t)rows; ++r) {
+    for (uint64_t g = 0; g < groups; ++g) {
+      const uint16_t* src = w + (uint64_t)r * cols + g * 32;
+      double amax = 0.0;
+      for (int i = 0; i < 32; ++i) {
+        double a = fabs(bf16_to_double(src[i]));
+        if (a > amax) amax = a;
+      }
+      _Float16 s16 = (_Float16)(amax / 7.0);
+      union { _Float16 h; uint16_t u; } sv;
+      sv.h = s16;
+      scales[(uint64_t)r * groups + g] = sv.u;
+      const double s = (double)s16;
+      uint8_t q[32];
+      for (int i = 0; i < 32; ++i) {
+        double v = s > 0 ? rint(bf16_to_double(src[i]) / s) + 8.0 : 8.0;
+        if (v < 0) v = 0;
+        if (v > 15) v = 15;
+        q[i] = (uint8_t)v;
+      }
+      uint8_t* dst = packed + (uint64_t)r * (cols / 2) + g * 16;
+      for (int i = 0; i < 16; ++i) dst[i] = (uint8_t)(q[2 * i] | (q[2 * i + 1] << 4));
+    }
+  }
+}

@@ -198,3 +198,46 @@ def test_balanced_teardown_states():
     states = {case.plan.slot_state(s) for s in range(cfg.n_slots)}
     assert states <= {N.MSI_SLOT_VACANT, N.MSI_SLOT_RECYCLABLE, N.MSI_SLOT_DEVICE_READY}
     case.close()
+
+
+# ---------------------------------------------------------------------------
+# 4-bit block-quantised experts (group 32, fp16 scale), dequantised in the GEMM
+# ---------------------------------------------------------------------------
+
+def test_q4_tiny_streamed_lru():
+    cfg = synth.config("tiny", wdtype=synth.W_Q4G32)
+    case = Case(cfg)
+    sim = oracle.LRUWaveSim(cfg.n_slots)
+    for call in range(2):
+        x_bits = synth.hidden(cfg, 0, 20 + call)
+        out, ev = _run_streamed(case, x_bits)
+        assert case.plan.status() == N.MSI_OK
+        ref = case.oracle_layer(x_bits)
+        ids = ev.ids.cpu().numpy()
+        compare_routes(ids, ev.weights.cpu().numpy(), ref)
+        sim.call(0, _needed(ids, cfg.n_experts))
+        compare_out(bf16_bits(out), ref["out"], ~oracle.near_tie_tokens(ref["gap_k"]))
+    assert case.plan.trace() == sim.trace
+    case.close()
+
+
+def test_q4_qwen_shape_lru_waves():
+    """Qwen3-Next layer shape with 4-bit experts, 64-slot pool, 2,000 tokens
+    (all 512 experts needed: 8 waves of 32, 448 stages after the first call)."""
+    cfg = synth.config("prefill32k_q4_lru64", tokens=2000)
+    case = Case(cfg)
+    sim = oracle.LRUWaveSim(cfg.n_slots)
+    rng = np.random.default_rng(1)
+    for call in range(2):
+        x_bits = synth.hidden(cfg, 0, call)
+        out, ev = _run_streamed(case, x_bits)
+        assert case.plan.status() == N.MSI_OK
+        ids = ev.ids.cpu().numpy()
+        r = oracle.router(x_bits, case.router_np[0], cfg.top_k, case.gate_np[0])
+        compare_routes(ids, ev.weights.cpu().numpy(), r)
+        sim.call(0, _needed(ids, cfg.n_experts))
+        toks = np.sort(rng.choice(cfg.tokens, 48, replace=False))
+        ref = case.oracle_layer(x_bits, tokens=toks)
+        compare_out(bf16_bits(out)[toks], ref["out"], ~oracle.near_tie_tokens(ref["gap_k"]))
+    assert case.plan.trace() == sim.trace
+    case.close()
