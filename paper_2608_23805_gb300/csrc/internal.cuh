@@ -61,6 +61,20 @@ struct RouterArgs {
   int* bcount;             // [nb, E] routed ids per router block and expert
 };
 
+struct RouterTcArgs {
+  const __nv_bfloat16* x;  // [T, H] (shared-gate dot products)
+  const float* wsg;        // [H] or nullptr
+  int T, H, E, k;
+  int tmem_cols;           // power of two >= max(32, E)
+  int* ids;                // [T, k]
+  float* weights;          // [T, k]
+  float* gap;              // [T] or nullptr
+  float* sg;               // [T]
+  int* bcount;             // [ceil(T/128), E]
+  int* status;
+  long long wait_limit;
+};
+
 struct ScanArgs {
   const int* bcount;
   int nb, E;
@@ -73,6 +87,7 @@ struct ScatterArgs {
   const int* counts;  // [E]
   const int* bbase;   // [nb, E]
   int T, k, E, nb;
+  int tm;             // tokens per router block
   int* perm;          // [T*k]
   int* inv;           // [T*k]
   int* offsets;       // [E+1]
@@ -159,6 +174,9 @@ enum GemmMode { kGateUpGather = 0, kGateUpTma = 1, kDown = 2, kGateUpGatherQ4 = 
 // Launchers (return cudaError_t of the launch)
 // ---------------------------------------------------------------------------
 cudaError_t launch_router(const RouterArgs& a, cudaStream_t s);
+cudaError_t launch_split3(const float* w, long long n, __nv_bfloat16* out, cudaStream_t s);
+cudaError_t launch_router_tc(const CUtensorMap& tmX, const CUtensorMap& tmW, const RouterTcArgs& a,
+                             cudaStream_t s);
 cudaError_t launch_colscan(const ScanArgs& a, cudaStream_t s);
 cudaError_t launch_scatter(const ScatterArgs& a, cudaStream_t s);
 cudaError_t launch_upload(const TableParams& p, int* table, unsigned long long* expected,

@@ -83,8 +83,8 @@ __global__ void __launch_bounds__(kScatterWarps * 32) scatter_kernel(const Scatt
   if (b >= a.nb) return;
   for (int e = lane; e < a.E; e += 32) run[warp][e] = 0;
   __syncwarp();
-  const int f0 = b * kRouterTM * a.k;
-  const int f1 = min(a.T, (b + 1) * kRouterTM) * a.k;
+  const int f0 = b * a.tm * a.k;
+  const int f1 = min(a.T, (b + 1) * a.tm) * a.k;
   const unsigned lt = (1u << lane) - 1u;
   for (int f = f0 + lane; f - lane < f1; f += 32) {
     const bool valid = f < f1;

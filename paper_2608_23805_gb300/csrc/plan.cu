@@ -146,8 +146,9 @@ struct WaveEntry {
 };
 
 struct WsLayout {
-  size_t status, table, expected, groups, total, sh_group, sh_total, bcount, bbase, offsets, perm,
-      inv, sg, h, yp, hs, ys, bytes;
+  size_t status, table, expected, groups, total, sh_group, sh_total, w3, bcount, bbase, offsets,
+      perm, inv, sg, h, yp, hs, ys, bytes;
+  int tm;  // tokens per router block
 };
 
 constexpr long long kDeviceWaitCycles = 4000000000LL;  // ~2 s at GB300 clocks
@@ -222,6 +223,9 @@ struct msi_plan {
 
 namespace {
 
+// The tensor-core router needs E to be a multiple of 16 (MMA N granularity).
+bool tensor_router(const msi_plan_desc& d) { return d.n_experts % 16 == 0; }
+
 bool shape_ok(const msi_plan_desc& d) {
   return d.n_experts >= 1 && d.n_experts <= kMaxExperts && d.top_k >= 1 &&
          d.top_k <= std::min(d.n_experts, kMaxTopK) && d.hidden >= 256 && d.hidden % 256 == 0 &&
@@ -238,7 +242,8 @@ WsLayout layout(const msi_plan* p, int T) {
     return r;
   };
   const size_t E = p->d.n_experts, k = p->d.top_k, H = p->d.hidden, I = p->d.inter;
-  const size_t nb = ((size_t)T + kRouterTM - 1) / kRouterTM, Tk = (size_t)T * k;
+  L.tm = tensor_router(p->d) ? 128 : kRouterTM;
+  const size_t nb = ((size_t)T + L.tm - 1) / L.tm, Tk = (size_t)T * k;
   L.status = take(4);
   L.table = take(4 * E);
   L.expected = take(8 * E);
@@ -246,6 +251,7 @@ WsLayout layout(const msi_plan* p, int T) {
   L.total = take(4);
   L.sh_group = take(sizeof(Group));
   L.sh_total = take(4);
+  L.w3 = tensor_router(p->d) ? take(3 * E * H * 2) : 0;
   L.bcount = take(4 * nb * E);
   L.bbase = take(4 * nb * E);
   L.offsets = take(4 * (E + 1));
@@ -407,30 +413,55 @@ msi_status front(msi_plan* p, FwdCtx& f, const TableParams& tp) {
     LAUNCH(p, MSI_K_UPLOAD, f.cs, launch_zero_counts(f.ev->counts, E, f.cs));
     return MSI_OK;
   }
-  const int nb = (f.T + kRouterTM - 1) / kRouterTM;
-  RouterArgs ra{};
-  ra.x = static_cast<const __nv_bfloat16*>(f.x);
-  ra.wr = f.router_w;
-  ra.wsg = d.has_shared ? d.shared_gate_w + (size_t)f.layer * H : nullptr;
-  ra.T = f.T;
-  ra.H = H;
-  ra.E = E;
-  ra.k = k;
-  ra.ids = f.ev->ids;
-  ra.weights = f.ev->weights;
-  ra.gap = f.ev->gap;
-  ra.sg = at<float>(ws, L.sg);
-  ra.bcount = at<int>(ws, L.bcount);
-  LAUNCH(p, MSI_K_ROUTER, f.cs, launch_router(ra, f.cs));
+  const int nb = (f.T + L.tm - 1) / L.tm;
+  if (!make_tmap(&f.tm_x, f.x, H, f.T, 128)) return MSI_ERR_CUDA;
+  if (tensor_router(d)) {
+    __nv_bfloat16* w3 = at<__nv_bfloat16>(ws, L.w3);
+    LAUNCH(p, MSI_K_ROUTER, f.cs, launch_split3(f.router_w, (long long)E * H, w3, f.cs));
+    CUtensorMap tm_w3;
+    if (!make_tmap(&tm_w3, w3, H, (uint64_t)3 * E, 256)) return MSI_ERR_CUDA;
+    RouterTcArgs ra{};
+    ra.x = static_cast<const __nv_bfloat16*>(f.x);
+    ra.wsg = d.has_shared ? d.shared_gate_w + (size_t)f.layer * H : nullptr;
+    ra.T = f.T;
+    ra.H = H;
+    ra.E = E;
+    ra.k = k;
+    int cols = 32;
+    while (cols < E) cols <<= 1;
+    ra.tmem_cols = cols;
+    ra.ids = f.ev->ids;
+    ra.weights = f.ev->weights;
+    ra.gap = f.ev->gap;
+    ra.sg = at<float>(ws, L.sg);
+    ra.bcount = at<int>(ws, L.bcount);
+    ra.status = at<int>(ws, L.status);
+    ra.wait_limit = kDeviceWaitCycles;
+    LAUNCH(p, MSI_K_ROUTER, f.cs, launch_router_tc(f.tm_x, tm_w3, ra, f.cs));
+  } else {
+    RouterArgs ra{};
+    ra.x = static_cast<const __nv_bfloat16*>(f.x);
+    ra.wr = f.router_w;
+    ra.wsg = d.has_shared ? d.shared_gate_w + (size_t)f.layer * H : nullptr;
+    ra.T = f.T;
+    ra.H = H;
+    ra.E = E;
+    ra.k = k;
+    ra.ids = f.ev->ids;
+    ra.weights = f.ev->weights;
+    ra.gap = f.ev->gap;
+    ra.sg = at<float>(ws, L.sg);
+    ra.bcount = at<int>(ws, L.bcount);
+    LAUNCH(p, MSI_K_ROUTER, f.cs, launch_router(ra, f.cs));
+  }
   ScanArgs sa{at<int>(ws, L.bcount), nb, E, at<int>(ws, L.bbase), f.ev->counts};
   LAUNCH(p, MSI_K_SCAN, f.cs, launch_colscan(sa, f.cs));
-  ScatterArgs xa{f.ev->ids, f.ev->counts, at<int>(ws, L.bbase), f.T, k, E, nb,
+  ScatterArgs xa{f.ev->ids, f.ev->counts, at<int>(ws, L.bbase), f.T, k, E, nb, L.tm,
                  at<int>(ws, L.perm), at<int>(ws, L.inv), at<int>(ws, L.offsets)};
   LAUNCH(p, MSI_K_SCATTER, f.cs, launch_scatter(xa, f.cs));
   const size_t Tk = (size_t)f.T * k;
   if (!make_tmap(&f.tm_h, at<char>(ws, L.h), I, Tk, 128)) return MSI_ERR_CUDA;
   if (d.has_shared) {
-    if (!make_tmap(&f.tm_x, f.x, H, f.T, 128)) return MSI_ERR_CUDA;
     if (!make_tmap(&f.tm_hs, at<char>(ws, L.hs), I, f.T, 128)) return MSI_ERR_CUDA;
   }
   return MSI_OK;

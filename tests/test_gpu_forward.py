@@ -241,3 +241,20 @@ def test_q4_qwen_shape_lru_waves():
         compare_out(bf16_bits(out)[toks], ref["out"], ~oracle.near_tie_tokens(ref["gap_k"]))
     assert case.plan.trace() == sim.trace
     case.close()
+
+
+def test_simt_router_path_odd_expert_count():
+    """E = 20 (not a multiple of 16) routes through the fp32 FFMA router."""
+    cfg = synth.config("tiny", n_experts=20, n_slots=8)
+    case = Case(cfg)
+    sim = oracle.LRUWaveSim(cfg.n_slots)
+    x_bits = synth.hidden(cfg, 0, 5)
+    out, ev = _run_streamed(case, x_bits)
+    assert case.plan.status() == N.MSI_OK
+    ref = case.oracle_layer(x_bits)
+    ids = ev.ids.cpu().numpy()
+    compare_routes(ids, ev.weights.cpu().numpy(), ref)
+    sim.call(0, _needed(ids, cfg.n_experts))
+    compare_out(bf16_bits(out), ref["out"])
+    assert case.plan.trace() == sim.trace
+    case.close()
