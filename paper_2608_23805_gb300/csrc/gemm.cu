@@ -19,7 +19,9 @@
 // come by TMA from the slot pool viewed as one 2-D tensor per operand; the
 // routed token rows (A) of the gate-up GEMM are gathered through the
 // permutation with cp.async into the same 128-byte-swizzled layout TMA
-// writes; the down GEMM's A (h, already in permuted order) comes by TMA.
+// writes, each thread arriving on the stage barrier when its copies land
+// (cp.async.mbarrier.arrive.noinc); the down GEMM's A (h, already in permuted
+// order) comes by TMA.
 //
 // Roles (warp-specialised):  warps 0-3 epilogue (TMEM -> registers -> global,
 // one token row per thread), warp 4 MMA issue + TMEM allocation, warp 5 TMA
@@ -37,7 +39,6 @@ namespace {
 
 constexpr int kEpiWarps = 4;
 constexpr int kGatherWarps = 4;
-constexpr int kLag = 2;  // gather stages in flight before signalling
 constexpr uint32_t kIdesc = idesc_bf16(kBM, kBN);
 
 constexpr int kDqWarps = 8;   // one thread per B row (256 rows)
@@ -56,7 +57,8 @@ struct Cfg {
   static constexpr int kDqWarp0 = 6 + (kGather ? kGatherWarps : 0);
   static constexpr int kThreads = (kDqWarp0 + (kQ4 ? kDqWarps : 0)) * 32;
   static constexpr uint32_t kTxBytes = (kTmaB ? kBBytes : 0) + (kTmaA ? kABytes : 0);
-  static constexpr int kFullCount = (kTmaAny ? 1 : 0) + (kGather ? kGatherWarps : 0) + (kQ4 ? kDqWarps : 0);
+  // gather threads arrive one by one as their copies land (cp.async ... arrive.noinc)
+  static constexpr int kFullCount = (kTmaAny ? 1 : 0) + (kGather ? kGatherWarps * 32 : 0) + (kQ4 ? kDqWarps : 0);
   static constexpr int kRawBytes = kQ4 ? kRaw * kBN * (kRawRowBytes + 4) : 0;
   static constexpr int kSmem = 1024 + kStages * (kABytes + kBBytes) + kRawBytes + 256;
 };
@@ -187,6 +189,9 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
           const int s = it % kStages;
           const uint32_t ph = (it / kStages) & 1;
           if (!mbar_wait(&full[s], ph, abort_flag, lim)) { ok = false; break; }
+          // cp.async (generic proxy) wrote A in the gather modes: order those
+          // writes before this thread's tensor-core (async proxy) reads
+          if (C::kGather) fence_proxy_async_smem();
           tc_fence_after();
           const uint64_t ad = sw128_desc(smem_u32(sA + s * kABytes));
           const uint64_t bd = sw128_desc(smem_u32(sB + s * kBBytes));
@@ -271,7 +276,7 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
     const int gt = threadIdx.x - C::kGatherWarp0 * 32;  // 0..127
     const int chunk = gt & 7;             // 16-byte chunk of a 128-byte row slice
     const int r0 = gt >> 3;               // rows r0 + 16 i
-    uint32_t it = 0, arrived = 0;
+    uint32_t it = 0;
     bool ok = true;
     for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
       const TileCoord tc = decode_tile(a, t);
@@ -302,25 +307,10 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
           const int rr = r0 + 16 * i;
           cp_async16(dstA + rr * 128 + ((chunk ^ (rr & 7)) << 4), src[i] + kb * kBK, nbytes[i]);
         }
-        cp_async_commit();
-        if (it + 1 - arrived > kLag) {
-          cp_async_wait<kLag>();
-          fence_proxy_async_smem();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&full[arrived % kStages]);
-          ++arrived;
-        }
+        cp_async_arrive_noinc(&full[s]);  // arrives when this thread's copies land
       }
     }
     cp_async_wait<0>();
-    fence_proxy_async_smem();
-    __syncwarp();
-    if (ok) {
-      while (arrived < it) {
-        if (lane == 0) mbar_arrive(&full[arrived % kStages]);
-        ++arrived;
-      }
-    }
   } else if (C::kQ4) {
     // ------------------------------------------------------------- q4 dequant
     const int d = threadIdx.x - C::kDqWarp0 * 32;  // B row of this thread, 0..255
