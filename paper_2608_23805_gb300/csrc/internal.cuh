@@ -65,12 +65,17 @@ struct RouterTcArgs {
   const __nv_bfloat16* x;  // [T, H] (shared-gate dot products)
   const float* wsg;        // [H] or nullptr
   int T, H, E, k;
-  int tmem_cols;           // power of two >= max(32, E)
+  int chunk;               // experts per router CTA (<= kRouterChunk)
+  int nchunk;              // E / chunk
+  int kp;                  // candidates per chunk: min(k + 1, chunk)
+  int tmem_cols;           // power of two >= max(32, chunk)
+  float* cand_v;           // [T, nchunk, kp] candidate logits
+  int* cand_i;             // [T, nchunk, kp] candidate expert ids
   int* ids;                // [T, k]
   float* weights;          // [T, k]
   float* gap;              // [T] or nullptr
   float* sg;               // [T]
-  int* bcount;             // [ceil(T/128), E]
+  int* bcount;             // [ceil(T/32), E]
   int* status;
   long long wait_limit;
 };
@@ -189,7 +194,8 @@ cudaError_t launch_gemm(int mode, const CUtensorMap& tmA, const CUtensorMap& tmB
 cudaError_t launch_combine(const CombineArgs& a, cudaStream_t s);
 cudaError_t launch_zero_counts(int* counts, int E, cudaStream_t s);
 
-constexpr int kRouterTM = 32;  // tokens per router block
+constexpr int kRouterTM = 32;  // tokens per fp32 FFMA router block
+constexpr int kRouterChunk = 128;  // experts per tensor-core router CTA
 
 // GEMM tiling
 constexpr int kBM = 128;

@@ -146,8 +146,8 @@ struct WaveEntry {
 };
 
 struct WsLayout {
-  size_t status, table, expected, groups, total, sh_group, sh_total, w3, bcount, bbase, offsets,
-      perm, inv, sg, h, yp, hs, ys, bytes;
+  size_t status, table, expected, groups, total, sh_group, sh_total, w3, cand_v, cand_i, bcount,
+      bbase, offsets, perm, inv, sg, h, yp, hs, ys, bytes;
   int tm;  // tokens per router block
 };
 
@@ -223,8 +223,13 @@ struct msi_plan {
 
 namespace {
 
-// The tensor-core router needs E to be a multiple of 16 (MMA N granularity).
-bool tensor_router(const msi_plan_desc& d) { return d.n_experts % 16 == 0; }
+// The tensor-core router splits E into chunks of min(E, 128) experts (MMA N,
+// a multiple of 16) and keeps k + 1 <= 32 candidates per chunk and token.
+bool tensor_router(const msi_plan_desc& d) {
+  const int E = d.n_experts;
+  return E % 16 == 0 && (E <= kRouterChunk || E % kRouterChunk == 0) && d.top_k <= 31 &&
+         E / std::min(E, kRouterChunk) * std::min(d.top_k + 1, std::min(E, kRouterChunk)) <= 160;
+}
 
 bool shape_ok(const msi_plan_desc& d) {
   return d.n_experts >= 1 && d.n_experts <= kMaxExperts && d.top_k >= 1 &&
@@ -242,7 +247,7 @@ WsLayout layout(const msi_plan* p, int T) {
     return r;
   };
   const size_t E = p->d.n_experts, k = p->d.top_k, H = p->d.hidden, I = p->d.inter;
-  L.tm = tensor_router(p->d) ? 128 : kRouterTM;
+  L.tm = kRouterTM;  // both routers count ids per 32-token block
   const size_t nb = ((size_t)T + L.tm - 1) / L.tm, Tk = (size_t)T * k;
   L.status = take(4);
   L.table = take(4 * E);
@@ -252,6 +257,12 @@ WsLayout layout(const msi_plan* p, int T) {
   L.sh_group = take(sizeof(Group));
   L.sh_total = take(4);
   L.w3 = tensor_router(p->d) ? take(3 * E * H * 2) : 0;
+  if (tensor_router(p->d)) {
+    const size_t ch = std::min<size_t>(E, kRouterChunk);
+    const size_t ncand = (E / ch) * std::min<size_t>(k + 1, ch);
+    L.cand_v = take(4 * (size_t)T * ncand);
+    L.cand_i = take(4 * (size_t)T * ncand);
+  }
   L.bcount = take(4 * nb * E);
   L.bbase = take(4 * nb * E);
   L.offsets = take(4 * (E + 1));
@@ -418,8 +429,9 @@ msi_status front(msi_plan* p, FwdCtx& f, const TableParams& tp) {
   if (tensor_router(d)) {
     __nv_bfloat16* w3 = at<__nv_bfloat16>(ws, L.w3);
     LAUNCH(p, MSI_K_ROUTER, f.cs, launch_split3(f.router_w, (long long)E * H, w3, f.cs));
+    const int ch = std::min(E, kRouterChunk);
     CUtensorMap tm_w3;
-    if (!make_tmap(&tm_w3, w3, H, (uint64_t)3 * E, 256)) return MSI_ERR_CUDA;
+    if (!make_tmap(&tm_w3, w3, H, (uint64_t)3 * E, (uint32_t)ch)) return MSI_ERR_CUDA;
     RouterTcArgs ra{};
     ra.x = static_cast<const __nv_bfloat16*>(f.x);
     ra.wsg = d.has_shared ? d.shared_gate_w + (size_t)f.layer * H : nullptr;
@@ -427,9 +439,14 @@ msi_status front(msi_plan* p, FwdCtx& f, const TableParams& tp) {
     ra.H = H;
     ra.E = E;
     ra.k = k;
+    ra.chunk = ch;
+    ra.nchunk = E / ch;
+    ra.kp = std::min(k + 1, ch);
     int cols = 32;
-    while (cols < E) cols <<= 1;
+    while (cols < ch) cols <<= 1;
     ra.tmem_cols = cols;
+    ra.cand_v = at<float>(ws, L.cand_v);
+    ra.cand_i = at<int>(ws, L.cand_i);
     ra.ids = f.ev->ids;
     ra.weights = f.ev->weights;
     ra.gap = f.ev->gap;

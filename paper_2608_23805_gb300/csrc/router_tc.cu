@@ -1,6 +1,6 @@
 // Router on tcgen05 tensor cores with fp32-exact products: fp32 logits,
 // top-k, softmax weights, shared-expert gate and the per-block expert
-// histogram in one kernel (the logits stay in TMEM).
+// histogram (the logits never reach HBM).
 //
 // The router's top-k output is the route event recorded per layer and graph
 // evaluation (paper, Sec. "Output-Exact Execution Beyond the Full-Residency
@@ -14,12 +14,20 @@
 // logits = x Wr^T is three bf16 MMAs accumulating in fp32 -- the same value as
 // an fp32 GEMM up to accumulation order.
 //
-// One CTA = 128 tokens x all E experts (E <= 512 fp32 accumulators per row in
-// TMEM, in chunks of <= 256 columns).  Stage = 64 K of one plane of one
-// expert chunk: x tile (TMA, 16 KB) + 256 weight rows (TMA, 32 KB), 4 stages.
-// Warps 0-3: epilogue (one token row per thread: top-(k+1) insertion over the
-// row's E logits in ascending id order, weights, gap, histogram, shared gate),
-// warp 4: MMA + TMEM, warp 5: TMA producer.  All waits are bounded.
+// Two kernels:
+//  1. router_tc_kernel, one CTA per (128 tokens, chunk of <= 128 experts):
+//     logits of the chunk in TMEM (per stage one x tile and the chunk's rows
+//     of all three planes, by TMA, feeding 12 MMAs), then each token's
+//     top-(k+1) candidates within the chunk by warp-shuffle argmax (logit
+//     desc, id asc) from shared memory, four rows at a time per warp.
+//  2. router_merge_kernel, one warp per 8 tokens (four at a time): the
+//     top-(k+1) of the union of the chunks' candidates (it contains the global
+//     top-(k+1)), weights, gap, and the per-32-token expert histogram for the
+//     permutation; then shared_gate_kernel, one warp per token, computes the
+//     shared-expert gate sigmoid(x . w_sg).
+// Warps 0-3 epilogue, warp 4 MMA + TMEM, warp 5 TMA producer (one lane each
+// for the single-thread roles; every role claims its whole warp).  All waits
+// are bounded.
 #include "internal.cuh"
 
 namespace msi {
@@ -27,12 +35,13 @@ namespace msi {
 namespace {
 
 constexpr int NTH = 192;
-constexpr int RT_STAGES = 4;
-constexpr int RT_A = 128 * 64 * 2;
-constexpr int RT_B = 256 * 64 * 2;
-constexpr int RT_SMEM = 1024 + RT_STAGES * (RT_A + RT_B) + 256 + kMaxExperts * 4;
-constexpr int RT_LLD = kMaxExperts + 1;  // padded logits row (floats)
-static_assert(64 * RT_LLD * 4 <= RT_STAGES * (RT_A + RT_B), "logits half does not fit");
+constexpr int RT_STAGES = 3;
+constexpr int RT_A = 128 * 64 * 2;                   // x tile (64 K)
+constexpr int RT_B = kRouterChunk * 64 * 2;          // one plane's chunk weight rows (64 K)
+constexpr int RT_STAGE = RT_A + 3 * RT_B;            // x tile + the three planes
+constexpr int RT_LLD = kRouterChunk + 1;             // padded logits row (floats)
+constexpr int RT_SMEM = 1024 + RT_STAGES * RT_STAGE + 256;
+static_assert(128 * RT_LLD * 4 <= RT_STAGES * RT_STAGE, "logits tile does not fit");
 
 __global__ void split3_kernel(const float* __restrict__ w, long long n, __nv_bfloat16* __restrict__ out) {
   for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < n;
@@ -48,31 +57,62 @@ __global__ void split3_kernel(const float* __restrict__ w, long long n, __nv_bfl
   }
 }
 
+// Warp-wide argmax over per-lane candidates (value desc, id asc).
+__device__ __forceinline__ void warp_best(float& bv, int& bi) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    const float ov = __shfl_xor_sync(0xffffffffu, bv, off);
+    const int oi = __shfl_xor_sync(0xffffffffu, bi, off);
+    if (ov > bv || (ov == bv && oi < bi)) {
+      bv = ov;
+      bi = oi;
+    }
+  }
+}
+
+// Four independent warp-wide argmaxes interleaved (hides shuffle latency).
+__device__ __forceinline__ void warp_best4(float (&bv)[4], int (&bi)[4]) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    float ov[4];
+    int oi[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      ov[u] = __shfl_xor_sync(0xffffffffu, bv[u], off);
+      oi[u] = __shfl_xor_sync(0xffffffffu, bi[u], off);
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      if (ov[u] > bv[u] || (ov[u] == bv[u] && oi[u] < bi[u])) {
+        bv[u] = ov[u];
+        bi[u] = oi[u];
+      }
+    }
+  }
+}
+
 __global__ void __launch_bounds__(NTH, 1)
     router_tc_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmW,
                      const RouterTcArgs a) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint8_t* sA = smem;
-  uint8_t* sB = smem + RT_STAGES * RT_A;
-  uint64_t* full = reinterpret_cast<uint64_t*>(sB + RT_STAGES * RT_B);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + RT_STAGES * RT_STAGE);
   uint64_t* empty = full + RT_STAGES;
   uint64_t* tfull = empty + RT_STAGES;
   uint64_t* drain = tfull + 1;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  int* hist = reinterpret_cast<int*>(reinterpret_cast<uint8_t*>(full) + 256);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int E = a.E, k = a.k;
-  const int nchunk = (E + 255) / 256;
+  const int ch = a.chunk;                 // experts per chunk
+  const int c = blockIdx.y;               // chunk index
   const int kblocks = a.H / 64;
-  const int nstage = nchunk * kblocks * 3;
+  const int nstage = kblocks;
   const int m0 = blockIdx.x * 128;
   const long long lim = a.wait_limit;
 
-  for (int e = threadIdx.x; e < E; e += NTH) hist[e] = 0;
   if (threadIdx.x == 0) {
     for (int s = 0; s < RT_STAGES; ++s) {
       mbar_init(&full[s], 1);
@@ -97,18 +137,20 @@ __global__ void __launch_bounds__(NTH, 1)
   const uint32_t tmem_base = *tmem_slot;
 
   if (warp == 5) {
+    // ------------------------------------------------------------- TMA producer
     if (lane == 0) {
       int it = 0;
       for (; it < nstage; ++it) {
         const int s = it % RT_STAGES;
         const uint32_t ph = (it / RT_STAGES) & 1;
         if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, lim)) break;
-        const int c = it / (kblocks * 3);
-        const int rem = it - c * kblocks * 3;
-        const int kb = rem / 3, plane = rem - kb * 3;
-        mbar_arrive_expect_tx(&full[s], RT_A + RT_B);
-        tma_load_2d(sA + s * RT_A, &tmX, &full[s], kb * 64, m0);
-        tma_load_2d(sB + s * RT_B, &tmW, &full[s], kb * 64, plane * E + c * 256);
+        uint8_t* st = smem + s * RT_STAGE;
+        // x box: 128 rows of 64 bf16; weight boxes: `ch` rows of 64 bf16 per plane
+        mbar_arrive_expect_tx(&full[s], RT_A + 3 * ch * 128);
+        tma_load_2d(st, &tmX, &full[s], it * 64, m0);
+#pragma unroll
+        for (int plane = 0; plane < 3; ++plane)
+          tma_load_2d(st + RT_A + plane * RT_B, &tmW, &full[s], it * 64, plane * E + c * ch);
       }
       if (*abort_flag) {
         for (int d = 0; d < RT_STAGES && it - 1 - d >= 0; ++d) {
@@ -120,22 +162,24 @@ __global__ void __launch_bounds__(NTH, 1)
       }
     }
   } else if (warp == 4) {
+    // ------------------------------------------------------------- MMA issuer
     if (lane == 0) {
       bool ok = true;
+      const uint32_t idesc = idesc_bf16(128, ch);
       for (int it = 0; it < nstage; ++it) {
         const int s = it % RT_STAGES;
         const uint32_t ph = (it / RT_STAGES) & 1;
         if (!mbar_wait(&full[s], ph, abort_flag, lim)) { ok = false; break; }
         tc_fence_after();
-        const int c = it / (kblocks * 3);
-        const int rem = it - c * kblocks * 3;
-        const int n_c = min(256, E - c * 256);
-        const uint32_t idesc = idesc_bf16(128, n_c);
-        const uint64_t ad = sw128_desc(smem_u32(sA + s * RT_A));
-        const uint64_t bd = sw128_desc(smem_u32(sB + s * RT_B));
+        const uint8_t* st = smem + s * RT_STAGE;
+        const uint64_t ad = sw128_desc(smem_u32(st));
 #pragma unroll
-        for (int kk = 0; kk < 4; ++kk)
-          umma_bf16(tmem_base + c * 256, ad + 2 * kk, bd + 2 * kk, idesc, (rem | kk) != 0);
+        for (int plane = 0; plane < 3; ++plane) {
+          const uint64_t bd = sw128_desc(smem_u32(st + RT_A + plane * RT_B));
+#pragma unroll
+          for (int kk = 0; kk < 4; ++kk)
+            umma_bf16(tmem_base, ad + 2 * kk, bd + 2 * kk, idesc, (it | plane | kk) != 0);
+        }
         umma_commit(&empty[s]);
       }
       if (ok) umma_commit(tfull);
@@ -146,111 +190,81 @@ __global__ void __launch_bounds__(NTH, 1)
     }
   } else {
     // ------------------------------------------------------------- epilogue
-    // Logits TMEM -> shared memory (the stage buffers are free once the MMA
-    // loop is done), 64 rows at a time, rows padded to LLD floats so that the
-    // 32 lanes' column writes fall into distinct banks; then one warp per
-    // token picks the top k+1 by warp-shuffle argmax (logit desc, id asc).
+    // Chunk logits TMEM -> shared memory (the stage buffers are free once the
+    // MMA loop is done; rows padded so the 32 lanes' column writes fall into
+    // distinct banks), then one warp per token picks its top k+1 in the chunk.
     const bool ready = __all_sync(0xffffffffu, mbar_wait(tfull, 0, abort_flag, lim));
     tc_fence_after();
     float* L = reinterpret_cast<float*>(smem);
-    const int tid = threadIdx.x;  // 0..127
-    const int per_lane = (E + 31) >> 5;
-    for (int half = 0; half < 2; ++half) {
-      if (ready && (warp >> 1) == half) {
-        const uint32_t tb = tmem_base + ((uint32_t)(warp * 32) << 16);
-        float* row = L + (size_t)((warp & 1) * 32 + lane) * RT_LLD;
-        for (int e0 = 0; e0 < E; e0 += 16) {
-          uint32_t v[16];
-          tmem_ld16(tb + e0, v);
-          tmem_ld_wait(v);
+    if (ready) {
+      const uint32_t tb = tmem_base + ((uint32_t)(warp * 32) << 16);
+      float* row = L + (size_t)(warp * 32 + lane) * RT_LLD;
+      for (int e0 = 0; e0 < ch; e0 += 16) {
+        uint32_t v[16];
+        tmem_ld16(tb + e0, v);
+        tmem_ld_wait(v);
 #pragma unroll
-          for (int j = 0; j < 16; ++j) row[e0 + j] = __uint_as_float(v[j]);
-        }
+        for (int j = 0; j < 16; ++j) row[e0 + j] = __uint_as_float(v[j]);
       }
-      asm volatile("bar.sync 1, 128;" ::: "memory");
-      if (ready) {
-        for (int q = 0; q < 16; ++q) {
-          const int rl = warp * 16 + q;           // row within this half
-          const int t = m0 + half * 64 + rl;
-          if (t >= a.T) break;
-          const float* row = L + (size_t)rl * RT_LLD;
-          float v[16];
-#pragma unroll
-          for (int i = 0; i < 16; ++i) {
-            const int e = lane + 32 * i;
-            v[i] = (i < per_lane && e < E) ? row[e] : -INFINITY;
-          }
-          uint32_t removed = 0;
-          float my_v = -INFINITY, next_v = -INFINITY;
-          int my_i = 0;
-          const int rounds = min(k + 1, E);
-          for (int rr = 0; rr < rounds; ++rr) {
-            float bv = -INFINITY;
-            int bi = 0x7fffffff;
-#pragma unroll
-            for (int i = 0; i < 16; ++i) {
-              const int e = lane + 32 * i;
-              if (i < per_lane && e < E && !((removed >> i) & 1u)) {
-                if (v[i] > bv || (v[i] == bv && e < bi)) { bv = v[i]; bi = e; }
-              }
-            }
-#pragma unroll
-            for (int off = 16; off > 0; off >>= 1) {
-              const float ov = __shfl_xor_sync(0xffffffffu, bv, off);
-              const int oi = __shfl_xor_sync(0xffffffffu, bi, off);
-              if (ov > bv || (ov == bv && oi < bi)) { bv = ov; bi = oi; }
-            }
-            if ((bi & 31) == lane) removed |= 1u << (bi >> 5);
-            if (rr == lane) { my_v = bv; my_i = bi; }
-            if (rr == k) next_v = bv;
-          }
-          const float l0 = __shfl_sync(0xffffffffu, my_v, 0);
-          const float ex = (lane < k) ? expf(my_v - l0) : 0.f;
-          float sum = ex;
-#pragma unroll
-          for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
-          if (lane < k) {
-            a.ids[(size_t)t * k + lane] = my_i;
-            a.weights[(size_t)t * k + lane] = ex / sum;
-            atomicAdd(&hist[my_i], 1);
-          }
-          if (a.gap != nullptr) {
-            const float lk1 = __shfl_sync(0xffffffffu, my_v, k - 1);
-            if (lane == 0) a.gap[t] = (k < E) ? (lk1 - next_v) : INFINITY;
-          }
-        }
-      }
-      asm volatile("bar.sync 1, 128;" ::: "memory");
     }
     tc_fence_before();
-    if (a.wsg != nullptr) {
-      // shared-expert gate: warp w computes x . w_sg for rows w*32 .. w*32+31
-      for (int q = 0; q < 32; ++q) {
-        const int tt = m0 + warp * 32 + q;
-        if (tt >= a.T) break;
-        const __nv_bfloat16* xr = a.x + (size_t)tt * a.H;
-        float s = 0.f;
-#pragma unroll 8
-        for (int h = lane * 8; h < a.H; h += 256) {
-          const uint4 xv = __ldg(reinterpret_cast<const uint4*>(xr + h));
-          const float4 w0 = __ldg(reinterpret_cast<const float4*>(a.wsg + h));
-          const float4 w1 = __ldg(reinterpret_cast<const float4*>(a.wsg + h + 4));
-          s = fmaf(bf16_lo(xv.x), w0.x, s);
-          s = fmaf(bf16_hi(xv.x), w0.y, s);
-          s = fmaf(bf16_lo(xv.y), w0.z, s);
-          s = fmaf(bf16_hi(xv.y), w0.w, s);
-          s = fmaf(bf16_lo(xv.z), w1.x, s);
-          s = fmaf(bf16_hi(xv.z), w1.y, s);
-          s = fmaf(bf16_lo(xv.w), w1.z, s);
-          s = fmaf(bf16_hi(xv.w), w1.w, s);
+    asm volatile("bar.sync 1, 128;" ::: "memory");
+    const int kp = a.kp;  // candidates per chunk: min(k + 1, chunk)
+    if (ready) {
+      for (int q0 = 0; q0 < 32; q0 += 4) {  // four of this warp's rows at a time
+        float v[4][4];
+        uint32_t removed[4] = {0, 0, 0, 0};
+        float my_v[4];
+        int my_i[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const float* row = L + (size_t)(warp * 32 + q0 + u) * RT_LLD;
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const int e = lane + 32 * i;
+            v[u][i] = e < ch ? row[e] : -INFINITY;
+          }
+          my_v[u] = -INFINITY;
+          my_i[u] = 0x7fffffff;
+        }
+        for (int rr = 0; rr < kp; ++rr) {
+          float bv[4];
+          int bi[4];
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            bv[u] = -INFINITY;
+            bi[u] = 0x7fffffff;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              const int e = lane + 32 * i;
+              if (e < ch && !((removed[u] >> i) & 1u) &&
+                  (v[u][i] > bv[u] || (v[u][i] == bv[u] && e < bi[u]))) {
+                bv[u] = v[u][i];
+                bi[u] = e;
+              }
+            }
+          }
+          warp_best4(bv, bi);
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            if ((bi[u] & 31) == lane) removed[u] |= 1u << (bi[u] >> 5);
+            if (rr == lane) {
+              my_v[u] = bv[u];
+              my_i[u] = c * ch + bi[u];  // global expert id
+            }
+          }
         }
 #pragma unroll
-        for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
-        if (lane == 0) a.sg[tt] = 1.0f / (1.0f + expf(-s));
+        for (int u = 0; u < 4; ++u) {
+          const int t = m0 + warp * 32 + q0 + u;
+          if (lane < kp && t < a.T) {
+            const size_t o = ((size_t)t * a.nchunk + c) * kp + lane;
+            a.cand_v[o] = my_v[u];
+            a.cand_i[o] = my_i[u];
+          }
+        }
       }
     }
-    // histogram of this block's routed ids -> bcount[block][e]
-    for (int e = tid; e < E; e += 128) a.bcount[(size_t)blockIdx.x * E + e] = hist[e];
   }
 
   tc_fence_before();
@@ -261,6 +275,130 @@ __global__ void __launch_bounds__(NTH, 1)
     tmem_dealloc(tmem_base, a.tmem_cols);
   }
   if (threadIdx.x == 0 && *abort_flag) atomicCAS(a.status, 0, (int)MSI_ERR_TIMEOUT);
+}
+
+// One warp per token: top-(k+1) of the union of the chunks' candidates, the
+// route event (ids, weights, gap) and the block's expert histogram.
+__global__ void __launch_bounds__(512) router_merge_kernel(const RouterTcArgs a) {
+  __shared__ int hist[4][kMaxExperts];  // one histogram per 32-token sub-block
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int E = a.E, k = a.k;
+  const int ncand = a.nchunk * a.kp;  // <= 160
+  for (int e = threadIdx.x; e < 4 * kMaxExperts; e += blockDim.x) (&hist[0][0])[e] = 0;
+  __syncthreads();
+  const int m0 = blockIdx.x * 128;
+  const int sb = warp >> 2;  // this warp's 8 tokens lie in sub-block sb
+  for (int q0 = 0; q0 < 8; q0 += 4) {
+    float v[4][5];
+    int id[4][5];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int t = m0 + warp * 8 + q0 + u;
+#pragma unroll
+      for (int i = 0; i < 5; ++i) {
+        const int j = lane + 32 * i;
+        const bool in = t < a.T && j < ncand;
+        const int cid = in ? a.cand_i[(size_t)t * ncand + j] : -1;
+        const bool real = cid >= 0 && cid < E;  // an aborted router leaves no valid candidate
+        v[u][i] = real ? a.cand_v[(size_t)t * ncand + j] : -INFINITY;
+        id[u][i] = real ? cid : 0x7fffffff;
+      }
+    }
+    uint32_t removed[4] = {0, 0, 0, 0};
+    float my_v[4], next_v[4];
+    int my_i[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      my_v[u] = -INFINITY;
+      next_v[u] = -INFINITY;
+      my_i[u] = 0;
+    }
+    const int rounds = min(k + 1, E);
+    for (int rr = 0; rr < rounds; ++rr) {
+      float bv[4];
+      int bi[4], bslot[4], mine[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        bv[u] = -INFINITY;
+        bi[u] = 0x7fffffff;
+        bslot[u] = -1;
+#pragma unroll
+        for (int i = 0; i < 5; ++i) {
+          if (!((removed[u] >> i) & 1u) &&
+              (v[u][i] > bv[u] || (v[u][i] == bv[u] && id[u][i] < bi[u]))) {
+            bv[u] = v[u][i];
+            bi[u] = id[u][i];
+            bslot[u] = i;
+          }
+        }
+        mine[u] = bi[u];
+      }
+      warp_best4(bv, bi);
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        if (bslot[u] >= 0 && mine[u] == bi[u]) removed[u] |= 1u << bslot[u];  // ids are unique
+        if (rr == lane) {
+          my_v[u] = bv[u];
+          my_i[u] = bi[u];
+        }
+        if (rr == k) next_v[u] = bv[u];
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int t = m0 + warp * 8 + q0 + u;
+      const float l0 = __shfl_sync(0xffffffffu, my_v[u], 0);
+      const float ex = (lane < k) ? expf(my_v[u] - l0) : 0.f;
+      float sum = ex;
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
+      const float lk1 = __shfl_sync(0xffffffffu, my_v[u], k - 1);
+      if (t < a.T) {
+        if (lane < k) {
+          const bool real = my_i[u] >= 0 && my_i[u] < E;
+          a.ids[(size_t)t * k + lane] = real ? my_i[u] : 0;
+          a.weights[(size_t)t * k + lane] = ex / sum;
+          if (real) atomicAdd(&hist[sb][my_i[u]], 1);
+        }
+        if (a.gap != nullptr && lane == 0) a.gap[t] = (k < E) ? (lk1 - next_v[u]) : INFINITY;
+      }
+    }
+  }
+  __syncthreads();
+  const int nsub = (a.T + 31) / 32;  // rows of bcount (32-token sub-blocks)
+  for (int i = threadIdx.x; i < 4 * E; i += blockDim.x) {
+    const int s = i / E, e = i - s * E;
+    const int row = blockIdx.x * 4 + s;
+    if (row < nsub) a.bcount[(size_t)row * E + e] = hist[s][e];
+  }
+}
+
+// Shared-expert gate sigmoid(x . w_sg), one warp per token.
+__global__ void __launch_bounds__(256) shared_gate_kernel(const __nv_bfloat16* __restrict__ x,
+                                                          const float* __restrict__ wsg, int T, int H,
+                                                          float* __restrict__ sg) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int t = blockIdx.x * 8 + warp;
+  if (t >= T) return;
+  const __nv_bfloat16* xr = x + (size_t)t * H;
+  float s = 0.f;
+#pragma unroll 8
+  for (int h = lane * 8; h < H; h += 256) {
+    const uint4 xv = __ldg(reinterpret_cast<const uint4*>(xr + h));
+    const float4 w0 = __ldg(reinterpret_cast<const float4*>(wsg + h));
+    const float4 w1 = __ldg(reinterpret_cast<const float4*>(wsg + h + 4));
+    s = fmaf(bf16_lo(xv.x), w0.x, s);
+    s = fmaf(bf16_hi(xv.x), w0.y, s);
+    s = fmaf(bf16_lo(xv.y), w0.z, s);
+    s = fmaf(bf16_hi(xv.y), w0.w, s);
+    s = fmaf(bf16_lo(xv.z), w1.x, s);
+    s = fmaf(bf16_hi(xv.z), w1.y, s);
+    s = fmaf(bf16_lo(xv.w), w1.z, s);
+    s = fmaf(bf16_hi(xv.w), w1.w, s);
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+  if (lane == 0) sg[t] = 1.0f / (1.0f + expf(-s));
 }
 
 }  // namespace
@@ -283,7 +421,13 @@ cudaError_t launch_router_tc(const CUtensorMap& tmX, const CUtensorMap& tmW, con
   }
   const int nb = (a.T + 127) / 128;
   if (nb == 0) return cudaSuccess;
-  router_tc_kernel<<<nb, NTH, RT_SMEM, s>>>(tmX, tmW, a);
+  router_tc_kernel<<<dim3(nb, a.nchunk), NTH, RT_SMEM, s>>>(tmX, tmW, a);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  router_merge_kernel<<<nb, 512, 0, s>>>(a);
+  e = cudaGetLastError();
+  if (e != cudaSuccess || a.wsg == nullptr) return e;
+  shared_gate_kernel<<<(a.T + 7) / 8, 256, 0, s>>>(a.x, a.wsg, a.T, a.H, a.sg);
   return cudaGetLastError();
 }
 

@@ -258,3 +258,24 @@ def test_simt_router_path_odd_expert_count():
     compare_out(bf16_bits(out), ref["out"])
     assert case.plan.trace() == sim.trace
     case.close()
+
+
+@pytest.mark.parametrize("E,k", [(64, 31), (64, 32), (256, 8)])
+def test_router_limits_and_chunks(E, k):
+    """k = 31 is the largest top-k of the tensor-core router (k + 1 candidates
+    per chunk), k = 32 routes through the fp32 FFMA router, E = 256 merges two
+    128-expert chunks."""
+    cfg = synth.config("tiny", n_experts=E, top_k=k, n_slots=E, tokens=96)
+    case = Case(cfg)
+    table, gens = case.stage_all()
+    x_bits = synth.hidden(cfg, 0, 9)
+    out, ev = case.plan.forward(0, bf16_tensor(x_bits), case.router[0], table, gens)
+    torch.cuda.synchronize()
+    assert case.plan.status() == N.MSI_OK
+    ref = case.oracle_layer(x_bits)
+    compare_routes(ev.ids.cpu().numpy(), ev.weights.cpu().numpy(), ref)
+    g = ev.gap.cpu().numpy()
+    ok = ~oracle.near_tie_tokens(ref["gap_adj"])
+    np.testing.assert_allclose(g[ok], ref["gap_k"][ok], rtol=0, atol=2e-5)
+    compare_out(bf16_bits(out), ref["out"], ~oracle.near_tie_tokens(ref["gap_k"]))
+    case.close()
