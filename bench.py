@@ -43,9 +43,17 @@ N_SMS = 152
 FP32_LANES_PER_SM = 128
 L2_BYTES = 129 * 1024 * 1024
 
-# dram__bytes_read.sum + dram__bytes_write.sum per launch from one ncu capture,
-# keyed by (workload, kernel kind); valid only while the kernel source hash matches.
-TRAFFIC = {}
+# dram__bytes_read.sum + dram__bytes_write.sum per launch from one ncu capture
+# (the summaries under profiles/), keyed by (workload, kernel kind); reported
+# only while the GEMM source still hashes to the value the capture was taken at.
+TRAFFIC = {
+    ("qwen3next_4k", "gateup"): {"bytes_per_launch": 2269214000 + 41656832, "src_hash": "9d5993bb87cdfb4a",
+                                 "profile": "profiles/gemm_gateup_qwen3next_4k.md"},
+    ("prefill32k_lru64", "gateup"): {"bytes_per_launch": 206174208 + 13412864, "src_hash": "9d5993bb87cdfb4a",
+                                     "profile": "profiles/gemm_gateup_prefill32k_lru64.md"},
+    ("prefill32k_q4_lru64", "gateup"): {"bytes_per_launch": 104274176 + 7133440, "src_hash": "9d5993bb87cdfb4a",
+                                        "profile": "profiles/gemm_gateup_q4_prefill32k_q4_lru64.md"},
+}
 
 
 def load_peaks():
@@ -58,8 +66,9 @@ def load_peaks():
 
 
 def kernel_source_hash() -> str:
+    """Hash of the grouped-GEMM source (the dominant kernels' code)."""
     h = hashlib.sha256()
-    for name in ("gemm.cu", "router.cu", "permute.cu", "internal.cuh"):
+    for name in ("gemm.cu", "internal.cuh"):
         with open(os.path.join(ROOT, "paper_2608_23805_gb300", "csrc", name), "rb") as f:
             h.update(f.read())
     return h.hexdigest()[:16]
@@ -255,6 +264,8 @@ def roofline(cfg, kt: dict, steps: int, peaks: dict, clocks: dict, workload: str
     r["ms_per_launch"] = ms / max(launches, 1)
     t = TRAFFIC.get((workload, kind))
     r["traffic"] = t["bytes_per_launch"] if (t and t.get("src_hash") == kernel_source_hash()) else None
+    if r["traffic"] is not None:
+        r["traffic_source"] = t["profile"]
     return r
 
 
