@@ -57,7 +57,9 @@ typedef enum {
   MSI_ERR_CUDA = 7,              /* a CUDA runtime call failed (see msi_last_cuda_error) */
   MSI_ERR_SHUT_DOWN = 8,         /* the plan is being destroyed */
   MSI_ERR_UNSUPPORTED = 9,       /* shape outside this build's limits */
-  MSI_ERR_WORKSPACE = 10         /* workspace missing, misaligned or too small */
+  MSI_ERR_WORKSPACE = 10,        /* workspace missing, misaligned or too small */
+  MSI_ERR_SOURCE = 11            /* a source extent failed (short read / I/O error); its
+                                    bundle was not staged and nothing was published */
 } msi_status;
 
 enum { MSI_W_BF16 = 0, MSI_W_Q4G32 = 1 };
@@ -71,6 +73,15 @@ enum {
   MSI_SLOT_DEVICE_READY = 2,  /* published, never consumed */
   MSI_SLOT_IN_USE = 3,        /* a consumer (forward or caller ticket) is live */
   MSI_SLOT_RECYCLABLE = 4     /* published and every consumer finished */
+};
+
+/* Host-side fault hooks (msi_fault_inject), one-shot per (layer, expert). */
+enum {
+  MSI_FAULT_SHORT_READ = 1,        /* the object's next source delivery is short: staging it
+                                      (alone or inside a bundle) fails with MSI_ERR_SOURCE */
+  MSI_FAULT_STALE_COMPLETION = 2,  /* the object's next publication carries the previous
+                                      generation (a late stale completion) */
+  MSI_FAULT_WRONG_OBJECT = 3       /* the object's next publication names another object */
 };
 
 /* Forward flags. */
@@ -218,6 +229,26 @@ msi_status msi_moe_forward_streamed(msi_plan* plan, int layer, const void* hidde
  * status (an msi_status value; MSI_OK when every needed expert passed the
  * generation re-check and every bounded device wait completed). */
 msi_status msi_forward_status(msi_plan* plan, int* device_status);
+
+/* Reset: fails with MSI_ERR_SLOT_BUSY while a caller-held ticket is live;
+ * otherwise waits for every staging and forward issued through the plan,
+ * invalidates every slot (Vacant; its published generation word cleared, so
+ * no expectation from before the reset can pass a check), clears the LRU state
+ * and advances the request epoch.  Generations keep increasing across resets
+ * (Sec. "Separate Window and GPU-Slot Lifecycles": reset advances the epoch
+ * after the outstanding-work checks; drain or invalidate outstanding
+ * versions). */
+msi_status msi_plan_reset(msi_plan* plan, uint64_t* new_epoch);
+
+/* Deterministic fault hooks for lifecycle tests, applied on the host (no GPU
+ * fault is ever raised): see MSI_FAULT_*.  The paper's fault cells (its table
+ * of fault modes) check that a short or failed read publishes nothing and
+ * that a stale completion or wrong object is rejected before visibility.
+ * kind: one MSI_FAULT_* value; layer in [0, n_layers), expert in
+ * [0, n_experts).  Arming the same object again replaces its pending fault.
+ * Errors: MSI_ERR_INVALID_ARG for a null plan, an unknown kind or an index
+ * out of range.  Nothing is allocated; msi_plan_reset does not disarm. */
+msi_status msi_fault_inject(msi_plan* plan, int kind, int layer, int expert);
 
 /* Host-side consumer tickets: a caller that reads slots outside a forward
  * holds the slot while reading.  Staging into a held slot waits, bounded. */

@@ -88,6 +88,14 @@ class Plan:
         N.check(N.lib().msi_slot_state(self.h, slot, ctypes.byref(s)), "msi_slot_state")
         return s.value
 
+    def reset(self) -> int:
+        e = ctypes.c_uint64()
+        N.check(N.lib().msi_plan_reset(self.h, ctypes.byref(e)), "msi_plan_reset")
+        return e.value
+
+    def inject(self, kind: int, layer: int, expert: int):
+        N.check(N.lib().msi_fault_inject(self.h, kind, layer, expert), "msi_fault_inject")
+
     def hold(self, slot: int):
         N.check(N.lib().msi_consumer_hold(self.h, slot), "msi_consumer_hold")
 

@@ -26,6 +26,7 @@
 #include <atomic>
 #include <chrono>
 #include <cstring>
+#include <map>
 #include <mutex>
 #include <string>
 #include <thread>
@@ -213,6 +214,8 @@ struct msi_plan {
   int calls = 0;
   int C = 1;
   bool dying = false;
+  uint64_t epoch = 0;
+  std::map<uint64_t, int> faults;  // one-shot host-side fault hooks by object key
   KernelTimer timer;
   std::mutex mu;
 
@@ -344,6 +347,14 @@ msi_status stage_enqueue(msi_plan* p, int layer, const std::vector<WaveEntry>& m
     inv.obj[i] = 0;
     pub.gen[i] = misses[i].gen;
     pub.obj[i] = obj_key(layer, misses[i].expert);
+    auto f = p->faults.find(obj_key(layer, misses[i].expert));
+    if (f != p->faults.end() && f->second == MSI_FAULT_STALE_COMPLETION) {
+      pub.gen[i] = misses[i].gen - 1;  // a late completion of the previous version lands
+      p->faults.erase(f);
+    } else if (f != p->faults.end() && f->second == MSI_FAULT_WRONG_OBJECT) {
+      pub.obj[i] = obj_key(layer, (misses[i].expert + 1) % p->d.n_experts);
+      p->faults.erase(f);
+    }
   }
   LAUNCH(p, MSI_K_PUBLISH, stage, launch_publish(inv, p->d_gen, stage));
   const uint64_t eb = p->d.extent_bytes;
@@ -632,6 +643,7 @@ const char* msi_status_string(msi_status s) {
     case MSI_ERR_SHUT_DOWN: return "plan shut down";
     case MSI_ERR_UNSUPPORTED: return "unsupported shape";
     case MSI_ERR_WORKSPACE: return "workspace missing, misaligned or too small";
+    case MSI_ERR_SOURCE: return "source extent failed; nothing published";
   }
   return "unknown status";
 }
@@ -733,6 +745,14 @@ msi_status msi_slot_stage(msi_plan* p, int slot, int layer, int expert, msi_stre
     return MSI_ERR_INVALID_ARG;
   const int cur = p->where[(size_t)layer * d.n_experts + expert];
   if (cur >= 0 && cur != slot) return MSI_ERR_INVALID_ARG;  // one slot per object
+  {
+    auto f = p->faults.find(obj_key(layer, expert));
+    if (f != p->faults.end() && f->second == MSI_FAULT_SHORT_READ) {
+      p->faults.erase(f);  // the source delivered less than the extent: nothing is staged
+      p->ctr.rejections++;
+      return MSI_ERR_SOURCE;
+    }
+  }
   if (!wait_unheld(p, slot)) {
     p->ctr.rejections++;
     return MSI_ERR_TIMEOUT;
@@ -907,6 +927,17 @@ msi_status msi_moe_forward_streamed(msi_plan* p, int layer, const void* x, int T
       return MSI_ERR_TIMEOUT;
     }
 
+  // every miss's source must be whole before any bundle is planned or published
+  for (int e = 0; e < E; ++e) {
+    if (p->h_counts[e] <= 0 || p->where[(size_t)layer * E + e] >= 0) continue;
+    auto f = p->faults.find(obj_key(layer, e));
+    if (f != p->faults.end() && f->second == MSI_FAULT_SHORT_READ) {
+      p->faults.erase(f);
+      p->ctr.rejections++;
+      return MSI_ERR_SOURCE;
+    }
+  }
+
   // ---- LRU-wave plan (host ledger; identical rules to the slot simulator) ----
   const int call = p->calls++;
   std::vector<int> hits, misses;
@@ -1023,6 +1054,52 @@ msi_status msi_forward_status(msi_plan* p, int* device_status) {
   CK(cudaEventSynchronize(p->pool.ev[p->fwd_ev]));
   *device_status = *p->h_status;
   if (*device_status != MSI_OK) p->ctr.rejections++;
+  return MSI_OK;
+}
+
+msi_status msi_plan_reset(msi_plan* p, uint64_t* new_epoch) {
+  if (p == nullptr) return MSI_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> g(p->mu);
+  if (p->dying) return MSI_ERR_SHUT_DOWN;
+  for (auto& h : p->holds)
+    if (h.load() > 0) return MSI_ERR_SLOT_BUSY;
+  // drain: every outstanding stage, consumer and forward
+  for (auto& sl : p->slots) {
+    if (sl.ready >= 0) CK(cudaEventSynchronize(p->pool.ev[sl.ready]));
+    if (sl.consumer >= 0) CK(cudaEventSynchronize(p->pool.ev[sl.consumer]));
+  }
+  if (p->fwd_ev >= 0) CK(cudaEventSynchronize(p->pool.ev[p->fwd_ev]));
+  // invalidate: nothing published before the reset can pass a check after it
+  CK(cudaMemset(p->d_gen, 0, sizeof(GenWord) * p->d.n_slots));
+  const int E = p->d.n_experts;
+  for (int s = 0; s < p->d.n_slots; ++s) {
+    Slot& sl = p->slots[s];
+    if (sl.layer >= 0) {
+      add_trace(p, -1, sl.layer, sl.expert, s, sl.gen, MSI_TRACE_EVICT, -1);
+      p->where[(size_t)sl.layer * E + sl.expert] = -1;
+      p->ctr.evicts++;
+    }
+    sl.layer = sl.expert = -1;
+    sl.last_use = -1;
+    p->pool.unref(sl.ready);
+    p->pool.unref(sl.consumer);
+    sl.ready = sl.consumer = -1;
+  }
+  p->tick = 0;
+  p->epoch++;
+  if (new_epoch) *new_epoch = p->epoch;
+  return MSI_OK;
+}
+
+msi_status msi_fault_inject(msi_plan* p, int kind, int layer, int expert) {
+  if (p == nullptr || layer < 0 || layer >= p->d.n_layers || expert < 0 ||
+      expert >= p->d.n_experts)
+    return MSI_ERR_INVALID_ARG;
+  if (kind != MSI_FAULT_SHORT_READ && kind != MSI_FAULT_STALE_COMPLETION &&
+      kind != MSI_FAULT_WRONG_OBJECT)
+    return MSI_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> g(p->mu);
+  p->faults[obj_key(layer, expert)] = kind;
   return MSI_OK;
 }
 

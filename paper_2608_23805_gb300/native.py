@@ -22,6 +22,8 @@ MSI_ERR_CUDA = 7
 MSI_ERR_SHUT_DOWN = 8
 MSI_ERR_UNSUPPORTED = 9
 MSI_ERR_WORKSPACE = 10
+MSI_ERR_SOURCE = 11
+MSI_FAULT_SHORT_READ, MSI_FAULT_STALE_COMPLETION, MSI_FAULT_WRONG_OBJECT = 1, 2, 3
 
 MSI_W_BF16 = 0
 MSI_W_Q4G32 = 1
@@ -80,6 +82,8 @@ _SIGS = {
     "msi_moe_forward_static": (ctypes.c_int, [_P, ctypes.c_int, _P, ctypes.c_int, _P, _P, _P, _P,
                                               ctypes.POINTER(msi_route_event), ctypes.c_uint, _P]),
     "msi_forward_status": (ctypes.c_int, [_P, ctypes.POINTER(ctypes.c_int)]),
+    "msi_plan_reset": (ctypes.c_int, [_P, ctypes.POINTER(ctypes.c_uint64)]),
+    "msi_fault_inject": (ctypes.c_int, [_P, ctypes.c_int, ctypes.c_int, ctypes.c_int]),
     "msi_consumer_hold": (ctypes.c_int, [_P, ctypes.c_int]),
     "msi_consumer_release": (ctypes.c_int, [_P, ctypes.c_int]),
     "msi_trace_read": (ctypes.c_int, [_P, ctypes.POINTER(msi_trace_rec), ctypes.c_size_t,
