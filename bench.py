@@ -47,11 +47,11 @@ L2_BYTES = 129 * 1024 * 1024
 # (the summaries under profiles/), keyed by (workload, kernel kind); reported
 # only while the GEMM source still hashes to the value the capture was taken at.
 TRAFFIC = {
-    ("qwen3next_4k", "gateup"): {"bytes_per_launch": 2269214000 + 41656832, "src_hash": "9d5993bb87cdfb4a",
+    ("qwen3next_4k", "gateup"): {"bytes_per_launch": 2269214000 + 41656832, "src_hash": "3c748c6041a2f15a",
                                  "profile": "profiles/gemm_gateup_qwen3next_4k.md"},
-    ("prefill32k_lru64", "gateup"): {"bytes_per_launch": 206174208 + 13412864, "src_hash": "9d5993bb87cdfb4a",
+    ("prefill32k_lru64", "gateup"): {"bytes_per_launch": 206174208 + 13412864, "src_hash": "3c748c6041a2f15a",
                                      "profile": "profiles/gemm_gateup_prefill32k_lru64.md"},
-    ("prefill32k_q4_lru64", "gateup"): {"bytes_per_launch": 104274176 + 7133440, "src_hash": "9d5993bb87cdfb4a",
+    ("prefill32k_q4_lru64", "gateup"): {"bytes_per_launch": 104274176 + 7133440, "src_hash": "3c748c6041a2f15a",
                                         "profile": "profiles/gemm_gateup_q4_prefill32k_q4_lru64.md"},
 }
 
@@ -125,6 +125,15 @@ class ClockSampler:
                                          stdout=self.f, stderr=subprocess.DEVNULL)
         except (OSError, FileNotFoundError):
             self.proc = None
+            return
+        # the sampler's start-up (driver-library initialisation) must not fall
+        # inside the warm-up or timed region: wait for its first sample
+        t0 = time.time()
+        while time.time() - t0 < 10.0 and self.proc.poll() is None:
+            self.f.flush()
+            if os.path.getsize(self.path) > 0:
+                break
+            time.sleep(0.05)
 
     def stop(self):
         if self.proc is None:

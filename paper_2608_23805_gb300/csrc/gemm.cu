@@ -398,13 +398,11 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
 template <int MODE>
 static cudaError_t launch_mode(const CUtensorMap& tmA, const CUtensorMap& tmB, const GemmArgs& a,
                                int grid, cudaStream_t s) {
-  static bool attr_done = false;
+  static std::atomic<unsigned long long> attr_done{0};
   const int smem = Cfg<MODE>::kSmem;
-  if (!attr_done) {
-    cudaError_t e = cudaFuncSetAttribute(grouped_gemm_kernel<MODE>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  {
+    cudaError_t e = smem_attr_once(grouped_gemm_kernel<MODE>, smem, attr_done);
     if (e != cudaSuccess) return e;
-    attr_done = true;
   }
   grouped_gemm_kernel<MODE><<<grid, Cfg<MODE>::kThreads, smem, s>>>(tmA, tmB, a);
   return cudaGetLastError();

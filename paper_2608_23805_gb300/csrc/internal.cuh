@@ -3,6 +3,8 @@
 // kernel launchers.  Nothing here is part of the public C ABI (include/msi.h).
 #pragma once
 
+#include <atomic>
+
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -11,6 +13,21 @@
 #include "../../include/msi.h"
 
 namespace msi {
+
+// Raise a kernel's dynamic shared-memory limit once per device (the attribute
+// belongs to the device's context); `done` holds one bit per device ordinal.
+template <typename K>
+inline cudaError_t smem_attr_once(K* kernel, int bytes, std::atomic<unsigned long long>& done) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const unsigned long long bit = dev < 64 ? 1ull << dev : 0ull;
+  if (bit != 0 && (done.load(std::memory_order_acquire) & bit)) return cudaSuccess;
+  e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess && bit != 0) done.fetch_or(bit, std::memory_order_acq_rel);
+  return e;
+}
+
 
 // ---------------------------------------------------------------------------
 // Limits of this build

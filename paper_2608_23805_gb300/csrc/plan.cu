@@ -328,6 +328,30 @@ msi_status wait_events(msi_plan* p, std::vector<int>& ids, cudaStream_t stream) 
   return MSI_OK;
 }
 
+// Make `stream` wait for the publication of every slot in `slots`.  A slot
+// whose publication event has completed drops its reference to it, so later
+// calls (a resident pool is read by every forward) skip the query.
+msi_status wait_ready(msi_plan* p, const std::vector<int>& slots, cudaStream_t stream) {
+  std::vector<int> pending, complete;
+  auto has = [](const std::vector<int>& v, int id) {
+    return std::find(v.begin(), v.end(), id) != v.end();
+  };
+  for (int s : slots) {
+    Slot& sl = p->slots[s];
+    const int id = sl.ready;
+    if (id < 0 || has(pending, id)) continue;
+    if (has(complete, id) || p->pool.done(id)) {
+      if (!has(complete, id)) complete.push_back(id);
+      sl.ready = -1;
+      p->pool.unref(id);
+    } else {
+      pending.push_back(id);
+    }
+  }
+  for (int id : pending) CK(cudaStreamWaitEvent(stream, p->pool.ev[id], 0));
+  return MSI_OK;
+}
+
 // Enqueue the copies of `misses` on `stage` and publish them with one event.
 msi_status stage_enqueue(msi_plan* p, int layer, const std::vector<WaveEntry>& misses,
                          cudaStream_t stage) {
@@ -836,9 +860,7 @@ msi_status msi_moe_forward(msi_plan* p, int layer, const void* x, int T, const f
   f.flags = flags;
   f.cs = reinterpret_cast<cudaStream_t>(compute);
   // readiness: the compute stream waits for every pending publication it reads
-  std::vector<int> waits;
-  for (int s : used) waits.push_back(p->slots[s].ready);
-  st = wait_events(p, waits, f.cs);
+  st = wait_ready(p, used, f.cs);
   if (st != MSI_OK) return st;
   static thread_local TableParams tp;
   tp.E = E;
@@ -1005,20 +1027,19 @@ msi_status msi_moe_forward_streamed(msi_plan* p, int layer, const void* x, int T
       st = stage_wave(w + 1);
       if (st != MSI_OK) return st;
     }
-    std::vector<int> waits, used;
+    std::vector<int> used;
     int mtiles = 0;
     wp.n = (int)waves[w].size();
     wp.layer = layer;
     for (int i = 0; i < wp.n; ++i) {
       const WaveEntry& we = waves[w][i];
-      waits.push_back(p->slots[we.slot].ready);
       used.push_back(we.slot);
       wp.slot[i] = we.slot;
       wp.expert[i] = we.expert;
       wp.expected[i] = we.gen;
       mtiles += (p->h_counts[we.expert] + kBM - 1) / kBM;
     }
-    st = wait_events(p, waits, f.cs);
+    st = wait_ready(p, used, f.cs);
     if (st != MSI_OK) return st;
     SetupArgs sa{};
     sa.counts = ev->counts;

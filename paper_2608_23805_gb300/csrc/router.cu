@@ -197,12 +197,10 @@ __global__ void __launch_bounds__(NTH, 1) router_kernel(const RouterArgs a) {
 }  // namespace
 
 cudaError_t launch_router(const RouterArgs& a, cudaStream_t s) {
-  static bool attr_done = false;
-  if (!attr_done) {
-    cudaError_t e =
-        cudaFuncSetAttribute(router_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM);
+  static std::atomic<unsigned long long> attr_done{0};
+  {
+    cudaError_t e = smem_attr_once(router_kernel, SMEM, attr_done);
     if (e != cudaSuccess) return e;
-    attr_done = true;
   }
   const int nb = (a.T + TM - 1) / TM;
   if (nb == 0) return cudaSuccess;

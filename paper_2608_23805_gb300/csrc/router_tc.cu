@@ -412,12 +412,10 @@ cudaError_t launch_split3(const float* w, long long n, __nv_bfloat16* out, cudaS
 
 cudaError_t launch_router_tc(const CUtensorMap& tmX, const CUtensorMap& tmW, const RouterTcArgs& a,
                              cudaStream_t s) {
-  static bool attr_done = false;
-  if (!attr_done) {
-    cudaError_t e = cudaFuncSetAttribute(router_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         RT_SMEM);
+  static std::atomic<unsigned long long> attr_done{0};
+  {
+    cudaError_t e = smem_attr_once(router_tc_kernel, RT_SMEM, attr_done);
     if (e != cudaSuccess) return e;
-    attr_done = true;
   }
   const int nb = (a.T + 127) / 128;
   if (nb == 0) return cudaSuccess;
