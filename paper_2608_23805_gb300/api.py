@@ -18,6 +18,10 @@ def _ptr(t) -> int | None:
     return None if t is None else t.data_ptr()
 
 
+def _flags(residual: bool, single_cta: bool) -> int:
+    return (N.MSI_FWD_RESIDUAL if residual else 0) | (N.MSI_FWD_SINGLE_CTA if single_cta else 0)
+
+
 def _stream(s) -> int | None:
     s = torch.cuda.current_stream() if s is None else s
     return s.cuda_stream
@@ -113,7 +117,7 @@ class Plan:
         return ws
 
     def forward(self, layer, x, router_w, slot_table, expected, out=None, ev=None, residual=False,
-                stream=None, check=True):
+                stream=None, check=True, single_cta=False):
         T = x.shape[0]
         out = torch.empty_like(x) if out is None else out
         ev = RouteEvent(T, self.k, self.E) if ev is None else ev
@@ -122,21 +126,21 @@ class Plan:
         ex = np.ascontiguousarray(expected, dtype=np.uint64)
         rc = N.lib().msi_moe_forward(self.h, layer, _ptr(x), T, _ptr(router_w), st.ctypes.data,
                                      ex.ctypes.data, _ptr(out), ctypes.byref(ev.c), _ptr(ws),
-                                     ws.numel(), N.MSI_FWD_RESIDUAL if residual else 0, _stream(stream))
+                                     ws.numel(), _flags(residual, single_cta), _stream(stream))
         if check:
             N.check(rc, "msi_moe_forward")
             return out, ev
         return rc, out, ev
 
     def forward_streamed(self, layer, x, router_w, out=None, ev=None, residual=False, stream=None,
-                         stage_stream=None, check=True):
+                         stage_stream=None, check=True, single_cta=False):
         T = x.shape[0]
         out = torch.empty_like(x) if out is None else out
         ev = RouteEvent(T, self.k, self.E) if ev is None else ev
         ws = self.workspace(T)
         rc = N.lib().msi_moe_forward_streamed(self.h, layer, _ptr(x), T, _ptr(router_w), _ptr(out),
                                               ctypes.byref(ev.c), _ptr(ws), ws.numel(),
-                                              N.MSI_FWD_RESIDUAL if residual else 0, _stream(stream),
+                                              _flags(residual, single_cta), _stream(stream),
                                               _stream(stage_stream))
         if check:
             N.check(rc, "msi_moe_forward_streamed")

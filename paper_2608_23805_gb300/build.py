@@ -17,7 +17,7 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libmsi.so")
-SOURCES = ["plan.cu", "router.cu", "router_tc.cu", "permute.cu", "gemm.cu", "noalloc.cu"]
+SOURCES = ["plan.cu", "router.cu", "router_tc.cu", "permute.cu", "gemm.cu", "gemm_pair.cu", "noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -225,48 +225,7 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
       if (!mbar_wait(&tfull[acc], aph, abort_flag, lim)) break;
       tc_fence_after();
       const uint32_t tb = tmem_base + ((uint32_t)(warp * 32) << 16) + acc * kBN;
-      if (C::kGateUp) {
-        __nv_bfloat16* dst = a.out + orow * a.out_ld + tc.n * 128;
-#pragma unroll 1
-        for (int c = 0; c < 128; c += 16) {
-          uint32_t g[16], u[16];
-          tmem_ld16(tb + c, g);
-          tmem_ld16(tb + 128 + c, u);
-          tmem_ld_wait(g);
-          tmem_ld_wait(u);
-          uint32_t p[8];
-#pragma unroll
-          for (int i = 0; i < 8; ++i) {
-            const float g0 = __uint_as_float(g[2 * i]), g1 = __uint_as_float(g[2 * i + 1]);
-            const float u0 = __uint_as_float(u[2 * i]), u1 = __uint_as_float(u[2 * i + 1]);
-            const float h0 = g0 / (1.0f + __expf(-g0)) * u0;
-            const float h1 = g1 / (1.0f + __expf(-g1)) * u1;
-            p[i] = pack_bf16x2(h0, h1);
-          }
-          if (valid) {
-            uint4* o = reinterpret_cast<uint4*>(dst + c);
-            o[0] = make_uint4(p[0], p[1], p[2], p[3]);
-            o[1] = make_uint4(p[4], p[5], p[6], p[7]);
-          }
-        }
-      } else {
-        __nv_bfloat16* dst = a.out + orow * a.out_ld + tc.n * kBN;
-#pragma unroll 1
-        for (int c = 0; c < kBN; c += 16) {
-          uint32_t v[16];
-          tmem_ld16(tb + c, v);
-          tmem_ld_wait(v);
-          uint32_t p[8];
-#pragma unroll
-          for (int i = 0; i < 8; ++i)
-            p[i] = pack_bf16x2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1]));
-          if (valid) {
-            uint4* o = reinterpret_cast<uint4*>(dst + c);
-            o[0] = make_uint4(p[0], p[1], p[2], p[3]);
-            o[1] = make_uint4(p[4], p[5], p[6], p[7]);
-          }
-        }
-      }
+      epilogue_tile<C::kGateUp>(tb, a.out + orow * a.out_ld + tc.n * (C::kGateUp ? 128 : kBN), valid);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&tempty[acc]);

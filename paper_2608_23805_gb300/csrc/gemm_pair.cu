@@ -1,0 +1,362 @@
+// Grouped expert GEMMs on CTA pairs (tcgen05 cta_group::2, sm_103a).
+//
+// Same projections as the single-CTA kernel in gemm.cu (paper, Sec.
+// "Output-Exact Execution Beyond the Full-Residency Envelope": each selected
+// expert's gate, up and down projections over its routed rows, weights read
+// from the stable slot address the Plan published), for groups large enough
+// to fill 256-row tiles, as in a long prefill.
+//
+// Two CTAs on neighbouring SMs form a cluster and share one 256 x 256 output
+// tile.  CTA r holds A rows [128 r, 128 r + 128) of the tile and B rows
+// (output columns) [128 r, 128 r + 128) in its own shared memory; the even
+// CTA issues the pair MMA, which reads both halves of A and B at the same
+// shared-memory offsets and accumulates each CTA's 128 rows into that CTA's
+// TMEM.  Per K step of 64 each SM therefore fills 32 KB of shared memory for
+// 128 x 256 x 64 multiply-adds, against 48 KB in the single-CTA tile: the
+// reduction that lets the tensor pipe outrun the L2 -> SM feed.
+//
+// Tile: 256 token rows x 256 output columns x 64 K per stage, 6-stage ring per
+// CTA, fp32 accumulators double-buffered in TMEM (2 x 256 columns).
+//
+// Synchronisation (all waits bounded; on expiry the CTA raises its abort flag,
+// the roles drain and the status word reports MSI_ERR_TIMEOUT):
+//   * each CTA's TMA loads and row-gather copies complete on that CTA's own
+//     `full` barrier; in the odd CTA a relay thread forwards each completed
+//     stage to the even CTA's `full` barrier, so no copy ever signals a
+//     barrier in the other CTA (an aborted CTA never receives a late
+//     transaction count);
+//   * the even CTA's MMA thread waits its `full` barrier (own stage + relayed
+//     peer stage), issues four pair MMAs and commits to `empty` of both CTAs
+//     (multicast), and to `tfull` of both CTAs at the end of a tile;
+//   * the epilogue warps of both CTAs read their own TMEM and arrive on the
+//     even CTA's `tempty` barrier (eight arrivals free an accumulator);
+//   * teardown: the MMA issuer's final commit reaches `drain` in both CTAs,
+//     each CTA waits it, then a cluster barrier, then both release TMEM.
+// Cross-CTA arrivals are plain (CTA-scope release) remote arrives: a
+// cluster-scope release or acquire on every K step serialises the pipeline
+// behind a cluster-wide fence (measured: 1.5-1.9x slower).
+//
+// Roles per CTA: warps 0-3 epilogue, warp 4 MMA issue (even CTA) or stage
+// relay (odd CTA) and TMEM allocation, warp 5 TMA producer, warps 6-9 row
+// gather (gate-up over routed rows).
+#include <algorithm>
+
+#include "internal.cuh"
+
+namespace msi {
+
+namespace {
+
+constexpr int kPairRows = 2 * kBM;         // 256 token rows per pair tile
+constexpr int kPStages = 6;
+constexpr int kPA = kBM * kBK * 2;         // 16 KB: this CTA's 128 A rows of one K step
+constexpr int kPB = 128 * kBK * 2;         // 16 KB: this CTA's 128 B rows of one K step
+constexpr uint32_t kPIdesc = idesc_bf16(kPairRows, kBN);
+constexpr int kPEpiWarps = 4;
+constexpr int kPGatherWarps = 4;
+
+template <int MODE>
+struct PCfg {
+  static constexpr bool kGather = (MODE == kGateUpGather);
+  static constexpr bool kGateUp = (MODE == kGateUpGather || MODE == kGateUpTma);
+  static constexpr int kGatherWarp0 = 6;
+  static constexpr int kThreads = (kGatherWarp0 + (kGather ? kPGatherWarps : 0)) * 32;
+  static constexpr uint32_t kTx = kPB + (kGather ? 0 : kPA);
+  // own producer (expect_tx) + own gather threads (one arrival each as their copies land)
+  static constexpr int kFullLocal = 1 + (kGather ? kPGatherWarps * 32 : 0);
+  static constexpr int kSmem = 1024 + kPStages * (kPA + kPB) + 256;
+};
+
+struct PairTile {
+  int g, m2, n;
+};
+
+__device__ __forceinline__ PairTile decode_pair(const GemmArgs& a, int t) {
+  int lo = 0, hi = a.num_groups - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (__ldg(&a.groups[mid].pt_begin) * a.nt <= t) lo = mid; else hi = mid - 1;
+  }
+  const int cnt = __ldg(&a.groups[lo].row_count);
+  const int mt2 = (cnt + kPairRows - 1) / kPairRows;
+  const int local = t - __ldg(&a.groups[lo].pt_begin) * a.nt;
+  PairTile c;
+  c.g = lo;
+  c.n = local / mt2;
+  c.m2 = local - c.n * mt2;
+  return c;
+}
+
+}  // namespace
+
+template <int MODE>
+__global__ void __launch_bounds__(PCfg<MODE>::kThreads, 1)
+    grouped_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA,
+                             const __grid_constant__ CUtensorMap tmB, const GemmArgs a) {
+  using C = PCfg<MODE>;
+  extern __shared__ uint8_t smem_raw[];
+  // the same offsets in both CTAs: the pair MMA addresses the peer's operands
+  // through the even CTA's descriptors
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + kPStages * kPA;
+  uint64_t* full = reinterpret_cast<uint64_t*>(sB + kPStages * kPB);
+  uint64_t* empty = full + kPStages;
+  uint64_t* tfull = empty + kPStages;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* drain = tempty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();
+  const bool leader = rank == 0;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kPStages; ++s) {
+      mbar_init(&full[s], C::kFullLocal + (leader ? 1 : 0));  // + the peer's relay
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&tfull[b], 1);
+      mbar_init(&tempty[b], 2 * kPEpiWarps);  // the epilogue warps of both CTAs
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    mbar_fence_init();
+  }
+  if (warp == 4) {
+    tmem_alloc_pair(tmem_slot, 512);
+    tmem_relinquish_pair();
+  }
+  if (warp == 5 && lane == 0) {
+    tma_prefetch(&tmB);
+    if (!C::kGather) tma_prefetch(&tmA);
+  }
+  tc_fence_before();
+  cluster_sync_all();  // both CTAs' barriers initialised before any cross-CTA arrival
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  const int total = __ldg(a.total_mtiles + 1) * a.nt;
+  const int pair = blockIdx.x >> 1;
+  const int npairs = gridDim.x >> 1;
+  const long long lim = a.wait_limit;
+
+  if (warp == 5) {
+    // ------------------------------------------------------------- TMA producer
+    if (lane == 0) {
+      uint32_t it = 0;
+      for (int t = pair; t < total; t += npairs) {
+        const PairTile tc = decode_pair(a, t);
+        const Group* G = &a.groups[tc.g];
+        const int brow0 = __ldg(&G->slot) * a.b_rows_per_slot + a.b_row_off;
+        // gate-up: the even CTA holds 128 gate rows, the odd CTA the matching up rows
+        const int brow = C::kGateUp ? brow0 + (rank ? a.up_off : 0) + tc.n * 128
+                                    : brow0 + tc.n * kBN + (int)rank * 128;
+        const int arow = __ldg(&G->row_begin) + tc.m2 * kPairRows + (int)rank * kBM;
+        bool ok = true;
+        for (int kb = 0; kb < a.kblocks; ++kb, ++it) {
+          const int s = it % kPStages;
+          const uint32_t ph = (it / kPStages) & 1;
+          if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, lim)) { ok = false; break; }
+          mbar_arrive_expect_tx(&full[s], C::kTx);
+          tma_load_2d(sB + s * kPB, &tmB, &full[s], kb * kBK, brow);
+          if (!C::kGather) tma_load_2d(sA + s * kPA, &tmA, &full[s], kb * kBK, arow);
+        }
+        if (!ok) break;
+      }
+      // On abort, wait (bounded) for the copies this thread armed to land
+      // before the CTA's shared memory is released.
+      if (*abort_flag) {
+        for (int d = 0; d < kPStages && it > 0; ++d) {
+          const uint32_t j = it - 1 - d;
+          if ((int)j < 0) break;
+          const long long t0 = clock64();
+          while (!mbar_try_wait(&full[j % kPStages], (j / kPStages) & 1) && clock64() - t0 < lim) {
+          }
+        }
+      }
+    }
+  } else if (warp == 4) {
+    if (lane == 0 && leader) {
+      // ----------------------------------------------------------- MMA issuer
+      uint32_t it = 0, jt = 0;
+      for (int t = pair; t < total; t += npairs, ++jt) {
+        const uint32_t acc = jt & 1, aph = (jt >> 1) & 1;
+        if (!mbar_wait(&tempty[acc], aph ^ 1, abort_flag, lim)) break;
+        tc_fence_after();
+        const uint32_t d = tmem_base + acc * kBN;
+        bool ok = true;
+        for (int kb = 0; kb < a.kblocks; ++kb, ++it) {
+          const int s = it % kPStages;
+          const uint32_t ph = (it / kPStages) & 1;
+          if (!mbar_wait(&full[s], ph, abort_flag, lim)) { ok = false; break; }
+          // this CTA's gathered rows were written by cp.async (generic proxy);
+          // the relay fenced the peer's before forwarding its stage
+          if (C::kGather) fence_proxy_async_smem();
+          tc_fence_after();
+          const uint64_t ad = sw128_desc(smem_u32(sA + s * kPA));
+          const uint64_t bd = sw128_desc(smem_u32(sB + s * kPB));
+#pragma unroll
+          for (int k = 0; k < kBK / 16; ++k) {
+            umma_bf16_pair(d, ad + 2 * k, bd + 2 * k, kPIdesc, (kb | k) != 0);
+          }
+          umma_commit_pair(&empty[s]);
+        }
+        if (!ok) break;
+        umma_commit_pair(&tfull[acc]);
+      }
+      umma_commit_pair(drain);
+    } else if (lane == 0) {
+      // ------------------------------------------------------ stage relay (odd)
+      const uint32_t my_tiles = pair < total ? (uint32_t)((total - 1 - pair) / npairs + 1) : 0u;
+      const uint32_t nst = my_tiles * (uint32_t)a.kblocks;
+      for (uint32_t it = 0; it < nst; ++it) {
+        const int s = it % kPStages;
+        const uint32_t ph = (it / kPStages) & 1;
+        if (!mbar_wait(&full[s], ph, abort_flag, lim)) break;
+        if (C::kGather) fence_proxy_async_smem();
+        mbar_arrive_remote(mapa_shared(smem_u32(&full[s]), 0));
+      }
+    }
+    if (lane == 0) {
+      // every pair MMA that reads this CTA's shared memory or writes its TMEM
+      // has completed before either is released
+      const long long t0 = clock64();
+      while (!mbar_try_wait(drain, 0) && clock64() - t0 < lim) {
+      }
+    }
+  } else if (warp < kPEpiWarps) {
+    // ------------------------------------------------------------- epilogue
+    uint32_t jt = 0;
+    const int r = warp * 32 + lane;
+    const uint32_t lead_tempty[2] = {mapa_shared(smem_u32(&tempty[0]), 0),
+                                     mapa_shared(smem_u32(&tempty[1]), 0)};
+    for (int t = pair; t < total; t += npairs, ++jt) {
+      const PairTile tc = decode_pair(a, t);
+      const Group* G = &a.groups[tc.g];
+      const int cnt = __ldg(&G->row_count);
+      const int grow = tc.m2 * kPairRows + (int)rank * kBM + r;  // row inside the group
+      const bool valid = grow < cnt;
+      const size_t orow = (size_t)__ldg(&G->row_begin) + (size_t)grow;
+      const uint32_t acc = jt & 1, aph = (jt >> 1) & 1;
+      if (!mbar_wait(&tfull[acc], aph, abort_flag, lim)) break;
+      tc_fence_after();
+      const uint32_t tb = tmem_base + ((uint32_t)(warp * 32) << 16) + acc * kBN;
+      epilogue_tile<C::kGateUp>(tb, a.out + orow * a.out_ld + tc.n * (C::kGateUp ? 128 : kBN), valid);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_remote(lead_tempty[acc]);
+    }
+  } else if (C::kGather && warp < C::kGatherWarp0 + kPGatherWarps) {
+    // ------------------------------------------------------------- row gather
+    const int gt = threadIdx.x - C::kGatherWarp0 * 32;  // 0..127
+    const int chunk = gt & 7;             // 16-byte chunk of a 128-byte row slice
+    const int r0 = gt >> 3;               // rows r0 + 16 i of this CTA's 128
+    uint32_t it = 0;
+    bool ok = true;
+    for (int t = pair; t < total && ok; t += npairs) {
+      const PairTile tc = decode_pair(a, t);
+      const Group* G = &a.groups[tc.g];
+      const int cnt = __ldg(&G->row_count);
+      const int rb = __ldg(&G->row_begin);
+      const __nv_bfloat16* src[8];
+      uint32_t nbytes[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const int rr = tc.m2 * kPairRows + (int)rank * kBM + r0 + 16 * i;
+        if (rr < cnt) {
+          const int tok = __ldg(&a.perm[rb + rr]) / a.top_k;
+          src[i] = a.x + (size_t)tok * a.x_ld + chunk * 8;
+          nbytes[i] = 16;
+        } else {
+          src[i] = a.x;
+          nbytes[i] = 0;  // zero-fill rows past the expert's segment
+        }
+      }
+      for (int kb = 0; kb < a.kblocks; ++kb, ++it) {
+        const int s = it % kPStages;
+        const uint32_t ph = (it / kPStages) & 1;
+        if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, lim)) { ok = false; break; }
+        uint8_t* dstA = sA + s * kPA;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const int rr = r0 + 16 * i;
+          cp_async16(dstA + rr * 128 + ((chunk ^ (rr & 7)) << 4), src[i] + kb * kBK, nbytes[i]);
+        }
+        cp_async_arrive_noinc(&full[s]);  // arrives when this thread's copies land
+      }
+    }
+    cp_async_wait<0>();
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync_all();  // neither CTA leaves while the other may still reach it
+  if (warp == 4) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc_pair(tmem_base, 512);
+  }
+  if (threadIdx.x == 0 && *abort_flag) atomicCAS(a.status, 0, (int)MSI_ERR_TIMEOUT);
+}
+
+namespace {
+
+struct PairLaunchInfo {
+  std::atomic<unsigned long long> attr_done{0};
+  std::atomic<int> max_clusters[64] = {};
+};
+
+template <int MODE>
+cudaError_t launch_pair_mode(const CUtensorMap& tmA, const CUtensorMap& tmB, const GemmArgs& a,
+                             int max_pairs, cudaStream_t s) {
+  static PairLaunchInfo info;
+  const int smem = PCfg<MODE>::kSmem;
+  auto kernel = grouped_gemm_pair_kernel<MODE>;
+  cudaError_t e = smem_attr_once(kernel, smem, info.attr_done);
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.blockDim = dim3(PCfg<MODE>::kThreads, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int dev = 0;
+  e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  // pairs that can be resident at once (a persistent grid never waits for a
+  // pair to finish before another can start)
+  int mc = dev < 64 ? info.max_clusters[dev].load() : 0;
+  if (mc <= 0) {
+    cfg.gridDim = dim3(2, 1, 1);
+    e = cudaOccupancyMaxActiveClusters(&mc, kernel, &cfg);
+    if (e != cudaSuccess) return e;
+    if (mc <= 0) return cudaErrorInvalidConfiguration;
+    if (dev < 64) info.max_clusters[dev].store(mc);
+  }
+  const int pairs = std::max(1, std::min(mc, max_pairs));
+  cfg.gridDim = dim3(2 * pairs, 1, 1);
+  return cudaLaunchKernelEx(&cfg, kernel, tmA, tmB, a);
+}
+
+}  // namespace
+
+cudaError_t launch_gemm_pair(int mode, const CUtensorMap& tmA, const CUtensorMap& tmB,
+                             const GemmArgs& a, int max_pairs, cudaStream_t s) {
+  switch (mode) {
+    case kGateUpGather: return launch_pair_mode<kGateUpGather>(tmA, tmB, a, max_pairs, s);
+    case kGateUpTma: return launch_pair_mode<kGateUpTma>(tmA, tmB, a, max_pairs, s);
+    case kDown: return launch_pair_mode<kDown>(tmA, tmB, a, max_pairs, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace msi

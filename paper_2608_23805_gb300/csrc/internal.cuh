@@ -59,7 +59,8 @@ struct Group {
   int mt_begin;    // prefix of 128-row tiles over the preceding groups
   int ok;          // generation re-check passed
   int expert;
-  int pad0, pad1;
+  int pt_begin;    // prefix of 256-row (CTA-pair) tiles over the preceding groups
+  int pad1;
 };
 
 // ---------------------------------------------------------------------------
@@ -148,14 +149,14 @@ struct SetupArgs {
   const unsigned long long* expected;     // resident mode
   int E, layer;
   Group* groups;
-  int* total_mtiles;
+  int* total_mtiles;   // [0]: 128-row tiles, [1]: 256-row pair tiles
   int* status;
 };
 
 struct GemmArgs {
   const Group* groups;
   int num_groups;
-  const int* total_mtiles;  // device
+  const int* total_mtiles;  // device: [0] 128-row tiles, [1] 256-row pair tiles
   int nt;                   // N tiles per group
   int kblocks;              // K / 64
   int b_rows_per_slot;      // rows of one weight block in the B tensor map
@@ -208,6 +209,10 @@ cudaError_t launch_setup_wave(const SetupArgs& a, const WaveParams& w, cudaStrea
 cudaError_t launch_publish(const PublishParams& p, GenWord* genwords, cudaStream_t s);
 cudaError_t launch_gemm(int mode, const CUtensorMap& tmA, const CUtensorMap& tmB,
                         const GemmArgs& a, int grid, cudaStream_t s);
+// CTA-pair variant (tcgen05 cta_group::2, 256 x 256 tiles) of kGateUpGather,
+// kGateUpTma and kDown; `max_pairs` bounds the pairs launched.
+cudaError_t launch_gemm_pair(int mode, const CUtensorMap& tmA, const CUtensorMap& tmB,
+                             const GemmArgs& a, int max_pairs, cudaStream_t s);
 cudaError_t launch_combine(const CombineArgs& a, cudaStream_t s);
 cudaError_t launch_zero_counts(int* counts, int E, cudaStream_t s);
 
@@ -336,6 +341,67 @@ __device__ __forceinline__ void tc_fence_after() {
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 }
 
+// --- clusters of two CTAs (tcgen05 cta_group::2) ---
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// shared::cluster address of the object at `saddr` (shared::cta) in CTA `rank`
+__device__ __forceinline__ uint32_t mapa_shared(uint32_t saddr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
+  return r;
+}
+// Arrive on a barrier of a CTA of this cluster (shared::cluster address).
+// Default semantics (release, CTA scope), as for a local arrive: the pair
+// protocol orders data through the barriers' own completion mechanisms (TMA
+// transaction counts, tcgen05.commit), so no cluster-wide fence is needed on
+// the per-stage path.
+__device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_addr) {
+  asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+// Every thread of both CTAs of the cluster.
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// Issued by one warp in each CTA of the pair.
+__device__ __forceinline__ void tmem_alloc_pair(uint32_t* dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                   smem_u32(dst_smem)),
+               "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish_pair() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+// Pair MMA, issued by the even CTA: A rows and B rows (N) come half from each
+// CTA's shared memory at the same offsets; each CTA's TMEM receives its rows.
+__device__ __forceinline__ void umma_bf16_pair(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
+                                               uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// Arrive once on the barrier at `bar`'s offset in both CTAs when all earlier
+// pair MMAs of this thread complete.
+__device__ __forceinline__ void umma_commit_pair(uint64_t* bar) {
+  const uint16_t mask = 3;
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 "
+      "[%0], %1;" ::"r"(smem_u32(bar)),
+      "h"(mask)
+      : "memory");
+}
+
 // D[tmem] (+)= A[smem] * B[smem]^T, bf16 inputs, fp32 accumulate.
 __device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
                                           uint32_t idesc, uint32_t accumulate) {
@@ -375,6 +441,34 @@ __device__ __forceinline__ void tmem_ld_wait(uint32_t (&r)[16]) {
                : "memory");
 }
 
+// 32 lanes x 32 consecutive 32-bit columns.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, "
+      "%12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, "
+      "%30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]),
+        "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]),
+        "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+}
+// Wait for this thread's TMEM loads; the registers pass through the wait so
+// that no use is scheduled before it.
+template <int N>
+__device__ __forceinline__ void tmem_wait_regs(uint32_t (&r)[N]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < N; ++i) asm volatile("" : "+r"(r[i]));
+}
+// 32-byte global store (one full sector), 32-byte aligned address.
+__device__ __forceinline__ void st_global_v8(void* p, const uint32_t* v) {
+  asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(p), "r"(v[0]),
+               "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7])
+               : "memory");
+}
+
 // Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, rows of
 // 128 bytes grouped in 8-row (1024-byte) atoms.
 __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
@@ -396,6 +490,68 @@ __device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v 
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&h);
+}
+
+// Epilogue of one accumulator tile for the thread's token row, output
+// columns [c0, c1): TMEM columns at tb to bf16 at dst (32-byte aligned),
+// stored when `valid`.
+//   gate-up: TMEM columns 0-127 hold x.Wg^T and 128-255 x.Wu^T of the same
+//            128 intermediate units; h = silu(g) * u = g * u / (1 + e^-g);
+//            c0, c1 are h columns (multiples of 32, <= 128).
+//   down:    output column c is TMEM column c (multiples of 64, <= 256).
+// TMEM is read 64 columns per wait and each store fills a 32-byte sector.
+template <bool GATEUP>
+__device__ __forceinline__ void epilogue_cols(uint32_t tb, __nv_bfloat16* dst, bool valid, int c0,
+                                              int c1) {
+  if (GATEUP) {
+#pragma unroll 1
+    for (int c = c0; c < c1; c += 32) {
+      uint32_t g[32], u[32];
+      tmem_ld32(tb + c, g);
+      tmem_ld32(tb + 128 + c, u);
+      tmem_wait_regs(g);
+      tmem_wait_regs(u);
+      uint32_t p[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const float g0 = __uint_as_float(g[2 * i]), g1 = __uint_as_float(g[2 * i + 1]);
+        const float u0 = __uint_as_float(u[2 * i]), u1 = __uint_as_float(u[2 * i + 1]);
+        // approximate divide (2 ulp): far below the bf16 rounding of h; an
+        // infinite e^-g (g < -88) gives 0, the limit of silu
+        p[i] = pack_bf16x2(__fdividef(g0 * u0, 1.0f + __expf(-g0)),
+                           __fdividef(g1 * u1, 1.0f + __expf(-g1)));
+      }
+      if (valid) {
+        st_global_v8(dst + c, p);
+        st_global_v8(dst + c + 16, p + 8);
+      }
+    }
+  } else {
+#pragma unroll 1
+    for (int c = c0; c < c1; c += 64) {
+      uint32_t v[32], w[32];
+      tmem_ld32(tb + c, v);
+      tmem_ld32(tb + c + 32, w);
+      tmem_wait_regs(v);
+      tmem_wait_regs(w);
+      uint32_t p[32];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        p[i] = pack_bf16x2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1]));
+        p[16 + i] = pack_bf16x2(__uint_as_float(w[2 * i]), __uint_as_float(w[2 * i + 1]));
+      }
+      if (valid) {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) st_global_v8(dst + c + 16 * q, p + 8 * q);
+      }
+    }
+  }
+}
+
+// The whole tile for the thread's row.
+template <bool GATEUP>
+__device__ __forceinline__ void epilogue_tile(uint32_t tb, __nv_bfloat16* dst, bool valid) {
+  epilogue_cols<GATEUP>(tb, dst, valid, 0, GATEUP ? 128 : 256);
 }
 
 #endif  // __CUDACC__

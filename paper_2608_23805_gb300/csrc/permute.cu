@@ -120,9 +120,10 @@ __global__ void upload_kernel(const TableParams p, int* table, unsigned long lon
       g.mt_begin = 0;
       g.ok = 1;
       g.expert = -1;
-      g.pad0 = g.pad1 = 0;
+      g.pt_begin = g.pad1 = 0;
       *sh = g;
-      *sh_total = (p.T + kBM - 1) / kBM;
+      sh_total[0] = (p.T + kBM - 1) / kBM;
+      sh_total[1] = (p.T + 2 * kBM - 1) / (2 * kBM);
     }
   }
 }
@@ -184,8 +185,11 @@ __global__ void __launch_bounds__(kMaxExperts) setup_kernel(const SetupArgs a, c
     if (cnt > 0) code = check_code(a.genwords, slot, a.layer, e, exp);
   }
   const int mt = (i < n && code == 0) ? (cnt + kBM - 1) / kBM : 0;
-  int total = 0;
+  const int pt = (i < n && code == 0) ? (cnt + 2 * kBM - 1) / (2 * kBM) : 0;
+  int total = 0, ptotal = 0;
   const int mt_begin = block_excl_scan(mt, tmp, &total);
+  __syncthreads();
+  const int pt_begin = block_excl_scan(pt, tmp, &ptotal);
   if (i < n) {
     Group g;
     g.row_begin = a.offsets[e];
@@ -194,13 +198,15 @@ __global__ void __launch_bounds__(kMaxExperts) setup_kernel(const SetupArgs a, c
     g.mt_begin = mt_begin;
     g.ok = code == 0;
     g.expert = e;
-    g.pad0 = g.pad1 = 0;
+    g.pt_begin = pt_begin;
+    g.pad1 = 0;
     a.groups[i] = g;
   }
   const int key = code ? (e << 4) | code : 0x7fffffff;
   const int m = block_min(key, tmp);
   if (i == 0) {
-    *a.total_mtiles = total;
+    a.total_mtiles[0] = total;
+    a.total_mtiles[1] = ptotal;
     if (m != 0x7fffffff) atomicCAS(a.status, 0, m & 15);
   }
 }

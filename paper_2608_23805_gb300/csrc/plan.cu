@@ -256,9 +256,9 @@ WsLayout layout(const msi_plan* p, int T) {
   L.table = take(4 * E);
   L.expected = take(8 * E);
   L.groups = take(sizeof(Group) * std::max<size_t>(E, kMaxWave));
-  L.total = take(4);
+  L.total = take(8);      // 128-row tiles, 256-row pair tiles
   L.sh_group = take(sizeof(Group));
-  L.sh_total = take(4);
+  L.sh_total = take(8);
   L.w3 = tensor_router(p->d) ? take(3 * E * H * 2) : 0;
   if (tensor_router(p->d)) {
     const size_t ch = std::min<size_t>(E, kRouterChunk);
@@ -555,7 +555,16 @@ GemmArgs down_args(msi_plan* p, FwdCtx& f, const Group* groups, int ng, const in
   return g;
 }
 
-msi_status routed_ffn(msi_plan* p, FwdCtx& f, int ng, int grid1, int grid2) {
+// CTA-pair (256-row) tiles run ~2-7 % faster than 128-row tiles once a
+// launch's groups average >= 1,024 rows (long prefills, the shared expert);
+// below that their coarser row padding and tile rounds lose (measured at
+// ~680 rows per group: 90 us against 80 us).
+constexpr long long kPairMinRows = 1024;
+bool pair_tiles(const FwdCtx& f, long long rows, int groups) {
+  return !(f.flags & MSI_FWD_SINGLE_CTA) && groups > 0 && rows >= kPairMinRows * groups;
+}
+
+msi_status routed_ffn(msi_plan* p, FwdCtx& f, int ng, int grid1, int grid2, bool pair) {
   const auto& d = p->d;
   const Group* groups = at<Group>(f.ws, f.L.groups);
   const int* total = at<int>(f.ws, f.L.total);
@@ -580,6 +589,13 @@ msi_status routed_ffn(msi_plan* p, FwdCtx& f, int ng, int grid1, int grid2) {
     LAUNCH(p, MSI_K_DOWN, f.cs, launch_gemm(kDownQ4, f.tm_h, f.tm_h, g2, grid2, f.cs));
     return MSI_OK;
   }
+  if (pair) {
+    LAUNCH(p, MSI_K_GATEUP, f.cs,
+           launch_gemm_pair(kGateUpGather, p->tm_w13, p->tm_w13, g1, std::max(1, grid1 / 2), f.cs));
+    LAUNCH(p, MSI_K_DOWN, f.cs,
+           launch_gemm_pair(kDown, f.tm_h, p->tm_w2, g2, std::max(1, grid2 / 2), f.cs));
+    return MSI_OK;
+  }
   LAUNCH(p, MSI_K_GATEUP, f.cs, launch_gemm(kGateUpGather, p->tm_w13, p->tm_w13, g1, grid1, f.cs));
   LAUNCH(p, MSI_K_DOWN, f.cs, launch_gemm(kDown, f.tm_h, p->tm_w2, g2, grid2, f.cs));
   return MSI_OK;
@@ -591,8 +607,16 @@ msi_status shared_ffn(msi_plan* p, FwdCtx& f) {
   const int* total = at<int>(f.ws, f.L.sh_total);
   const int mt = (f.T + kBM - 1) / kBM;
   GemmArgs s1 = gateup_args(p, f, g, 1, total, at<__nv_bfloat16>(f.ws, f.L.hs));
-  LAUNCH(p, MSI_K_SHARED_GATEUP, f.cs, launch_gemm(kGateUpTma, f.tm_x, p->tm_sh13, s1, std::min(p->sms, mt * s1.nt), f.cs));
   GemmArgs s2 = down_args(p, f, g, 1, total, at<__nv_bfloat16>(f.ws, f.L.ys));
+  if (p->d.wdtype == MSI_W_BF16 && pair_tiles(f, f.T, 1)) {
+    const int pt = (f.T + 2 * kBM - 1) / (2 * kBM);
+    LAUNCH(p, MSI_K_SHARED_GATEUP, f.cs,
+           launch_gemm_pair(kGateUpTma, f.tm_x, p->tm_sh13, s1, pt * s1.nt, f.cs));
+    LAUNCH(p, MSI_K_SHARED_DOWN, f.cs,
+           launch_gemm_pair(kDown, f.tm_hs, p->tm_sh2, s2, pt * s2.nt, f.cs));
+    return MSI_OK;
+  }
+  LAUNCH(p, MSI_K_SHARED_GATEUP, f.cs, launch_gemm(kGateUpTma, f.tm_x, p->tm_sh13, s1, std::min(p->sms, mt * s1.nt), f.cs));
   LAUNCH(p, MSI_K_SHARED_DOWN, f.cs, launch_gemm(kDown, f.tm_hs, p->tm_sh2, s2, std::min(p->sms, mt * s2.nt), f.cs));
   return MSI_OK;
 }
@@ -889,7 +913,8 @@ msi_status msi_moe_forward(msi_plan* p, int layer, const void* x, int T, const f
     const long long mt_max = ((long long)T * d.top_k + kBM - 1) / kBM + E;
     const int g1 = (int)std::min<long long>(p->sms, mt_max * (d.inter / 128));
     const int g2 = (int)std::min<long long>(p->sms, mt_max * (d.hidden / kBN));
-    st = routed_ffn(p, f, E, g1, g2);
+    st = routed_ffn(p, f, E, g1, g2,
+                    d.wdtype == MSI_W_BF16 && pair_tiles(f, (long long)T * d.top_k, E));
     if (st != MSI_OK) return st;
     st = consumer_record(p, used, f.cs);
     if (st != MSI_OK) return st;
@@ -1029,6 +1054,7 @@ msi_status msi_moe_forward_streamed(msi_plan* p, int layer, const void* x, int T
     }
     std::vector<int> used;
     int mtiles = 0;
+    long long wave_rows = 0;
     wp.n = (int)waves[w].size();
     wp.layer = layer;
     for (int i = 0; i < wp.n; ++i) {
@@ -1038,6 +1064,7 @@ msi_status msi_moe_forward_streamed(msi_plan* p, int layer, const void* x, int T
       wp.expert[i] = we.expert;
       wp.expected[i] = we.gen;
       mtiles += (p->h_counts[we.expert] + kBM - 1) / kBM;
+      wave_rows += p->h_counts[we.expert];
     }
     st = wait_ready(p, used, f.cs);
     if (st != MSI_OK) return st;
@@ -1053,7 +1080,8 @@ msi_status msi_moe_forward_streamed(msi_plan* p, int layer, const void* x, int T
     LAUNCH(p, MSI_K_SETUP, f.cs, launch_setup_wave(sa, wp, f.cs));
     const int g1 = std::max(1, std::min(p->sms, mtiles * (d.inter / 128)));
     const int g2 = std::max(1, std::min(p->sms, mtiles * (d.hidden / kBN)));
-    st = routed_ffn(p, f, wp.n, g1, g2);
+    st = routed_ffn(p, f, wp.n, g1, g2,
+                    d.wdtype == MSI_W_BF16 && pair_tiles(f, wave_rows, wp.n));
     if (st != MSI_OK) return st;
     st = consumer_record(p, used, f.cs);
     if (st != MSI_OK) return st;

@@ -30,6 +30,7 @@ MSI_W_Q4G32 = 1
 MSI_TRACE_HIT, MSI_TRACE_STAGE, MSI_TRACE_EVICT = 0, 1, 2
 MSI_SLOT_VACANT, MSI_SLOT_LOADING, MSI_SLOT_DEVICE_READY, MSI_SLOT_IN_USE, MSI_SLOT_RECYCLABLE = range(5)
 MSI_FWD_RESIDUAL = 1
+MSI_FWD_SINGLE_CTA = 2
 KERNEL_KINDS = ["upload", "router", "scan", "scatter", "setup", "gateup", "down", "shared_gateup",
                 "shared_down", "combine", "publish"]
 

@@ -1,0 +1,91 @@
+"""CTA-pair expert GEMMs (256-row tiles, tcgen05 cta_group::2): the forwards
+pick them when a launch's groups average at least 1,024 rows.  Each case runs
+the same inputs through the pair kernels (default) and through the single-CTA
+kernels (MSI_FWD_SINGLE_CTA); both must match the fp64 oracle within the
+output tolerance, with route events exact, and agree with each other."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+from gpu_case import Case, bf16_bits, bf16_tensor, compare_out, compare_routes
+from paper_2608_23805_gb300 import native as N
+
+pytestmark = pytest.mark.gpu
+
+
+def _both(case, x_bits, table, gens, **kw):
+    outs = []
+    for single in (False, True):
+        out, ev = case.plan.forward(0, bf16_tensor(x_bits), case.router[0], table, gens,
+                                    single_cta=single, **kw)
+        torch.cuda.synchronize()
+        assert case.plan.status() == N.MSI_OK
+        outs.append((bf16_bits(out), ev.ids.cpu().numpy(), ev.weights.cpu().numpy()))
+    return outs
+
+
+def _agree(a, b):
+    fa, fb = oracle.bf16_to_f64(a), oracle.bf16_to_f64(b)
+    assert np.abs(fa - fb).max() <= 2e-2
+    assert np.linalg.norm(fa - fb) <= 5e-3 * max(np.linalg.norm(fa), 1e-30)
+
+
+@pytest.mark.parametrize("tokens", [4100, 6000])
+def test_pair_resident_small_shape_full_oracle(tokens):
+    """H 512, I 256, 16 experts, top-4, shared expert: ~1,025-1,500 rows per
+    expert (ragged pair tiles, several 256-row tiles per expert, partial halves)."""
+    cfg = synth.config("tiny", hidden=512, inter=256, n_experts=16, top_k=4, tokens=tokens,
+                       n_slots=16, has_shared=True, lru=False)
+    case = Case(cfg)
+    table, gens = case.stage_all()
+    x_bits = synth.hidden(cfg, 0, 11)
+    (op, ip, wp), (os_, is_, ws_) = _both(case, x_bits, table, gens)
+    ref = case.oracle_layer(x_bits)
+    compare_routes(ip, wp, oracle.router(x_bits, case.router_np[0], cfg.top_k))
+    assert np.array_equal(ip, is_)
+    compare_out(op, ref["out"])
+    compare_out(os_, ref["out"])
+    _agree(op, os_)
+    case.close()
+
+
+def test_pair_qwen_shape_sampled_tokens():
+    """H 2048, I 512, 64 experts, top-10, 8,192 tokens: ~1,280 rows per
+    expert, five 256-row tiles each; outputs checked on sampled tokens."""
+    cfg = synth.config("qwen3next_4k", n_experts=64, tokens=8192, n_slots=64)
+    case = Case(cfg)
+    table, gens = case.stage_all()
+    x_bits = synth.hidden(cfg, 0, 12)
+    (op, ip, wp), (os_, is_, ws_) = _both(case, x_bits, table, gens)
+    rng = np.random.default_rng(5)
+    toks = np.sort(rng.choice(cfg.tokens, 48, replace=False))
+    ref = case.oracle_layer(x_bits, tokens=toks)
+    compare_out(op[toks], ref["out"])
+    compare_out(os_[toks], ref["out"])
+    assert np.array_equal(ip, is_)
+    _agree(op, os_)
+    case.close()
+
+
+def test_pair_streamed_waves_full_oracle():
+    """Streamed LRU waves large enough for pair tiles (32 experts, 16 slots,
+    waves of 8, ~2,048 rows per expert): matches the oracle, with pair and
+    single-CTA tiles."""
+    cfg = synth.config("tiny", hidden=512, inter=256, n_experts=32, top_k=8, tokens=8192,
+                       n_slots=16, has_shared=False)
+    case = Case(cfg)
+    x_bits = synth.hidden(cfg, 0, 13)
+    out, ev = case.plan.forward_streamed(0, bf16_tensor(x_bits), case.router[0])
+    torch.cuda.synchronize()
+    assert case.plan.status() == N.MSI_OK
+    ref = case.oracle_layer(x_bits)
+    compare_routes(ev.ids.cpu().numpy(), ev.weights.cpu().numpy(),
+                   oracle.router(x_bits, case.router_np[0], cfg.top_k))
+    compare_out(bf16_bits(out), ref["out"])
+    out1, _ = case.plan.forward_streamed(0, bf16_tensor(x_bits), case.router[0], single_cta=True)
+    torch.cuda.synchronize()
+    assert case.plan.status() == N.MSI_OK
+    compare_out(bf16_bits(out1), ref["out"])
+    case.close()
