@@ -60,7 +60,11 @@ struct Cfg {
   // gather threads arrive one by one as their copies land (cp.async ... arrive.noinc)
   static constexpr int kFullCount = (kTmaAny ? 1 : 0) + (kGather ? kGatherWarps * 32 : 0) + (kQ4 ? kDqWarps : 0);
   static constexpr int kRawBytes = kQ4 ? kRaw * kBN * (kRawRowBytes + 4) : 0;
-  static constexpr int kSmem = 1024 + kStages * (kABytes + kBBytes) + kRawBytes + 256;
+  // bf16 modes stage each epilogue warp's rows in shared memory (4 KB per
+  // warp) for row-coalesced stores; the q4 raw ring leaves no room for it
+  static constexpr bool kStagedEpi = !kQ4;
+  static constexpr int kSmem = 1024 + kStages * (kABytes + kBBytes) + kRawBytes + 256 +
+                               (kStagedEpi ? kEpiWarps * 4096 : 0);
 };
 
 struct TileCoord {
@@ -104,6 +108,7 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
   uint64_t* drain = tempty + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  uint8_t* epi_stage = reinterpret_cast<uint8_t*>(full) + 256;  // kEpiWarps x 4 KB (bf16 modes)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -225,7 +230,15 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
       if (!mbar_wait(&tfull[acc], aph, abort_flag, lim)) break;
       tc_fence_after();
       const uint32_t tb = tmem_base + ((uint32_t)(warp * 32) << 16) + acc * kBN;
-      epilogue_tile<C::kGateUp>(tb, a.out + orow * a.out_ld + tc.n * (C::kGateUp ? 128 : kBN), valid);
+      const int ncol0 = tc.n * (C::kGateUp ? 128 : kBN);
+      if (C::kStagedEpi) {
+        const int row_w = tc.m * kBM + warp * 32;  // the warp's first row inside the group
+        epilogue_tile_staged<C::kGateUp>(
+            tb, a.out + ((size_t)__ldg(&G->row_begin) + row_w) * a.out_ld + ncol0, a.out_ld,
+            cnt - row_w, epi_stage + warp * 4096, lane);
+      } else {
+        epilogue_tile<C::kGateUp>(tb, a.out + orow * a.out_ld + ncol0, valid);
+      }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&tempty[acc]);

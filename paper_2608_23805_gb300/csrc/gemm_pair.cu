@@ -64,7 +64,7 @@ struct PCfg {
   static constexpr uint32_t kTx = kPB + (kGather ? 0 : kPA);
   // own producer (expect_tx) + own gather threads (one arrival each as their copies land)
   static constexpr int kFullLocal = 1 + (kGather ? kPGatherWarps * 32 : 0);
-  static constexpr int kSmem = 1024 + kPStages * (kPA + kPB) + 256;
+  static constexpr int kSmem = 1024 + kPStages * (kPA + kPB) + 256 + kPEpiWarps * 4096;
 };
 
 struct PairTile {
@@ -108,6 +108,7 @@ __global__ void __launch_bounds__(PCfg<MODE>::kThreads, 1)
   uint64_t* drain = tempty + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  uint8_t* epi_stage = reinterpret_cast<uint8_t*>(full) + 256;  // 4 KB per epilogue warp
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -231,21 +232,20 @@ __global__ void __launch_bounds__(PCfg<MODE>::kThreads, 1)
   } else if (warp < kPEpiWarps) {
     // ------------------------------------------------------------- epilogue
     uint32_t jt = 0;
-    const int r = warp * 32 + lane;
     const uint32_t lead_tempty[2] = {mapa_shared(smem_u32(&tempty[0]), 0),
                                      mapa_shared(smem_u32(&tempty[1]), 0)};
     for (int t = pair; t < total; t += npairs, ++jt) {
       const PairTile tc = decode_pair(a, t);
       const Group* G = &a.groups[tc.g];
       const int cnt = __ldg(&G->row_count);
-      const int grow = tc.m2 * kPairRows + (int)rank * kBM + r;  // row inside the group
-      const bool valid = grow < cnt;
-      const size_t orow = (size_t)__ldg(&G->row_begin) + (size_t)grow;
       const uint32_t acc = jt & 1, aph = (jt >> 1) & 1;
       if (!mbar_wait(&tfull[acc], aph, abort_flag, lim)) break;
       tc_fence_after();
       const uint32_t tb = tmem_base + ((uint32_t)(warp * 32) << 16) + acc * kBN;
-      epilogue_tile<C::kGateUp>(tb, a.out + orow * a.out_ld + tc.n * (C::kGateUp ? 128 : kBN), valid);
+      const int row_w = tc.m2 * kPairRows + (int)rank * kBM + warp * 32;  // warp's first row in the group
+      epilogue_tile_staged<C::kGateUp>(
+          tb, a.out + ((size_t)__ldg(&G->row_begin) + row_w) * a.out_ld + tc.n * (C::kGateUp ? 128 : kBN),
+          a.out_ld, cnt - row_w, epi_stage + warp * 4096, lane);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive_remote(lead_tempty[acc]);

@@ -554,6 +554,77 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tb, __nv_bfloat16* dst, b
   epilogue_cols<GATEUP>(tb, dst, valid, 0, GATEUP ? 128 : 256);
 }
 
+// Store 32 rows of RB bytes each, held one row per lane (16-byte words in p),
+// through the warp's shared-memory staging buffer (32 x RB bytes, chunks
+// XOR-swizzled by row): read back eight lanes per 128 bytes of a row, so each
+// global store instruction covers whole rows (RB = 128: four rows of 128 B;
+// RB = 64: eight rows of 64 B) instead of one 16-32 B piece of 32 rows.
+// Rows >= nvalid (past the expert's segment) are not stored.
+template <int RB>
+__device__ __forceinline__ void store_rows_staged(const uint32_t* p, uint8_t* stg,
+                                                  __nv_bfloat16* row0, size_t ld, int nvalid,
+                                                  int lane) {
+  constexpr int Q = RB / 16;  // 16-byte chunks per row
+#pragma unroll
+  for (int q = 0; q < Q; ++q)
+    *reinterpret_cast<uint4*>(stg + lane * RB + ((q ^ (lane & (Q - 1))) << 4)) =
+        make_uint4(p[4 * q], p[4 * q + 1], p[4 * q + 2], p[4 * q + 3]);
+  __syncwarp();
+#pragma unroll
+  for (int it = 0; it < Q; ++it) {
+    const int idx = it * 32 + lane;
+    const int row = idx / Q, q = idx % Q;
+    const uint4 v = *reinterpret_cast<const uint4*>(stg + row * RB + ((q ^ (row & (Q - 1))) << 4));
+    if (row < nvalid)
+      *reinterpret_cast<uint4*>(reinterpret_cast<uint8_t*>(row0 + (size_t)row * ld) + q * 16) = v;
+  }
+  __syncwarp();
+}
+
+// Whole-tile epilogue of one warp (32 token rows, TMEM lanes of the warp's
+// quarter) with staged, row-coalesced stores.  row0: output of the warp's
+// first row at the tile's first column; nvalid: rows of the 32 inside the
+// expert's segment; stg: the warp's 4 KB staging buffer.
+template <bool GATEUP>
+__device__ __forceinline__ void epilogue_tile_staged(uint32_t tb, __nv_bfloat16* row0, size_t ld,
+                                                     int nvalid, uint8_t* stg, int lane) {
+  if (GATEUP) {
+#pragma unroll 1
+    for (int c = 0; c < 128; c += 32) {
+      uint32_t g[32], u[32];
+      tmem_ld32(tb + c, g);
+      tmem_ld32(tb + 128 + c, u);
+      tmem_wait_regs(g);
+      tmem_wait_regs(u);
+      uint32_t p[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const float g0 = __uint_as_float(g[2 * i]), g1 = __uint_as_float(g[2 * i + 1]);
+        const float u0 = __uint_as_float(u[2 * i]), u1 = __uint_as_float(u[2 * i + 1]);
+        p[i] = pack_bf16x2(__fdividef(g0 * u0, 1.0f + __expf(-g0)),
+                           __fdividef(g1 * u1, 1.0f + __expf(-g1)));
+      }
+      store_rows_staged<64>(p, stg, row0 + c, ld, nvalid, lane);
+    }
+  } else {
+#pragma unroll 1
+    for (int c = 0; c < 256; c += 64) {
+      uint32_t v[32], w[32];
+      tmem_ld32(tb + c, v);
+      tmem_ld32(tb + c + 32, w);
+      tmem_wait_regs(v);
+      tmem_wait_regs(w);
+      uint32_t p[32];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        p[i] = pack_bf16x2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1]));
+        p[16 + i] = pack_bf16x2(__uint_as_float(w[2 * i]), __uint_as_float(w[2 * i + 1]));
+      }
+      store_rows_staged<128>(p, stg, row0 + c, ld, nvalid, lane);
+    }
+  }
+}
+
 #endif  // __CUDACC__
 
 }  // namespace msi
