@@ -20,21 +20,20 @@
 //     of all three planes, by TMA, feeding 12 MMAs), then each token's
 //     top-(k+1) candidates within the chunk by warp-shuffle argmax (logit
 //     desc, id asc) from shared memory, four rows at a time per warp.
-//  2. router_merge_kernel, one warp per 8 tokens (four at a time): the
-//     top-(k+1) of the union of the chunks' candidates (it contains the global
-//     top-(k+1)), weights, gap, and the per-32-token expert histogram for the
-//     permutation; then shared_gate_kernel, one warp per token, computes the
-//     shared-expert gate sigmoid(x . w_sg).
-// Warps 0-3 epilogue, warp 4 MMA + TMEM, warp 5 TMA producer (one lane each
-// for the single-thread roles; every role claims its whole warp).  All waits
-// are bounded.
+//  2. router_merge_kernel, one CTA per 32 tokens (eight warps, four tokens
+//     each): the top-(k+1) of the union of the chunks' candidates (it contains
+//     the global top-(k+1)), weights, gap, the block's expert histogram for
+//     the permutation and the shared-expert gate sigmoid(x . w_sg).
+// Warps 0-3 move the logits from TMEM to shared memory, warp 4 MMA + TMEM,
+// warp 5 TMA producer (one lane each for the single-thread roles; every role
+// claims its whole warp); then all eight warps select.  All waits are bounded.
 #include "internal.cuh"
 
 namespace msi {
 
 namespace {
 
-constexpr int NTH = 192;
+constexpr int NTH = 256;  // 8 warps: all of them select top-k once the logits are in smem
 constexpr int RT_STAGES = 3;
 constexpr int RT_A = 128 * 64 * 2;                   // x tile (64 K)
 constexpr int RT_B = kRouterChunk * 64 * 2;          // one plane's chunk weight rows (64 K)
@@ -54,19 +53,6 @@ __global__ void split3_kernel(const float* __restrict__ w, long long n, __nv_bfl
     out[i] = hi;
     out[n + i] = mid;
     out[2 * n + i] = __float2bfloat16_rn(r2);
-  }
-}
-
-// Warp-wide argmax over per-lane candidates (value desc, id asc).
-__device__ __forceinline__ void warp_best(float& bv, int& bi) {
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1) {
-    const float ov = __shfl_xor_sync(0xffffffffu, bv, off);
-    const int oi = __shfl_xor_sync(0xffffffffu, bi, off);
-    if (ov > bv || (ov == bv && oi < bi)) {
-      bv = ov;
-      bi = oi;
-    }
   }
 }
 
@@ -103,9 +89,10 @@ __global__ void __launch_bounds__(NTH, 1)
   uint64_t* drain = tfull + 1;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  int* ready_flag = const_cast<int*>(abort_flag) + 1;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int E = a.E, k = a.k;
+  const int E = a.E;
   const int ch = a.chunk;                 // experts per chunk
   const int c = blockIdx.y;               // chunk index
   const int kblocks = a.H / 64;
@@ -188,11 +175,11 @@ __global__ void __launch_bounds__(NTH, 1)
       while (!mbar_try_wait(drain, 0) && clock64() - t0 < lim) {
       }
     }
-  } else {
+  } else if (warp < 4) {
     // ------------------------------------------------------------- epilogue
     // Chunk logits TMEM -> shared memory (the stage buffers are free once the
     // MMA loop is done; rows padded so the 32 lanes' column writes fall into
-    // distinct banks), then one warp per token picks its top k+1 in the chunk.
+    // distinct banks).
     const bool ready = __all_sync(0xffffffffu, mbar_wait(tfull, 0, abort_flag, lim));
     tc_fence_after();
     float* L = reinterpret_cast<float*>(smem);
@@ -207,61 +194,66 @@ __global__ void __launch_bounds__(NTH, 1)
         for (int j = 0; j < 16; ++j) row[e0 + j] = __uint_as_float(v[j]);
       }
     }
-    tc_fence_before();
-    asm volatile("bar.sync 1, 128;" ::: "memory");
+    if (threadIdx.x == 0) *ready_flag = ready ? 1 : 0;
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (*ready_flag) {
+    // ------------------------------------------------------------- top-k
+    // every warp: its 16 tokens' top k+1 in the chunk, four tokens at a time
+    const float* L = reinterpret_cast<const float*>(smem);
     const int kp = a.kp;  // candidates per chunk: min(k + 1, chunk)
-    if (ready) {
-      for (int q0 = 0; q0 < 32; q0 += 4) {  // four of this warp's rows at a time
-        float v[4][4];
-        uint32_t removed[4] = {0, 0, 0, 0};
-        float my_v[4];
-        int my_i[4];
+    for (int q0 = warp * 16; q0 < warp * 16 + 16; q0 += 4) {
+      float v[4][4];
+      uint32_t removed[4] = {0, 0, 0, 0};
+      float my_v[4];
+      int my_i[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const float* row = L + (size_t)(q0 + u) * RT_LLD;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const int e = lane + 32 * i;
+          v[u][i] = e < ch ? row[e] : -INFINITY;
+        }
+        my_v[u] = -INFINITY;
+        my_i[u] = 0x7fffffff;
+      }
+      for (int rr = 0; rr < kp; ++rr) {
+        float bv[4];
+        int bi[4];
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
-          const float* row = L + (size_t)(warp * 32 + q0 + u) * RT_LLD;
+          bv[u] = -INFINITY;
+          bi[u] = 0x7fffffff;
 #pragma unroll
           for (int i = 0; i < 4; ++i) {
             const int e = lane + 32 * i;
-            v[u][i] = e < ch ? row[e] : -INFINITY;
-          }
-          my_v[u] = -INFINITY;
-          my_i[u] = 0x7fffffff;
-        }
-        for (int rr = 0; rr < kp; ++rr) {
-          float bv[4];
-          int bi[4];
-#pragma unroll
-          for (int u = 0; u < 4; ++u) {
-            bv[u] = -INFINITY;
-            bi[u] = 0x7fffffff;
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-              const int e = lane + 32 * i;
-              if (e < ch && !((removed[u] >> i) & 1u) &&
-                  (v[u][i] > bv[u] || (v[u][i] == bv[u] && e < bi[u]))) {
-                bv[u] = v[u][i];
-                bi[u] = e;
-              }
-            }
-          }
-          warp_best4(bv, bi);
-#pragma unroll
-          for (int u = 0; u < 4; ++u) {
-            if ((bi[u] & 31) == lane) removed[u] |= 1u << (bi[u] >> 5);
-            if (rr == lane) {
-              my_v[u] = bv[u];
-              my_i[u] = c * ch + bi[u];  // global expert id
+            if (e < ch && !((removed[u] >> i) & 1u) &&
+                (v[u][i] > bv[u] || (v[u][i] == bv[u] && e < bi[u]))) {
+              bv[u] = v[u][i];
+              bi[u] = e;
             }
           }
         }
+        warp_best4(bv, bi);
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
-          const int t = m0 + warp * 32 + q0 + u;
-          if (lane < kp && t < a.T) {
-            const size_t o = ((size_t)t * a.nchunk + c) * kp + lane;
-            a.cand_v[o] = my_v[u];
-            a.cand_i[o] = my_i[u];
+          if ((bi[u] & 31) == lane) removed[u] |= 1u << (bi[u] >> 5);
+          if (rr == lane) {
+            my_v[u] = bv[u];
+            my_i[u] = c * ch + bi[u];  // global expert id
           }
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int t = m0 + q0 + u;
+        if (lane < kp && t < a.T) {
+          const size_t o = ((size_t)t * a.nchunk + c) * kp + lane;
+          a.cand_v[o] = my_v[u];
+          a.cand_i[o] = my_i[u];
         }
       }
     }
@@ -277,23 +269,25 @@ __global__ void __launch_bounds__(NTH, 1)
   if (threadIdx.x == 0 && *abort_flag) atomicCAS(a.status, 0, (int)MSI_ERR_TIMEOUT);
 }
 
-// One warp per token: top-(k+1) of the union of the chunks' candidates, the
-// route event (ids, weights, gap) and the block's expert histogram.
-__global__ void __launch_bounds__(512) router_merge_kernel(const RouterTcArgs a) {
-  __shared__ int hist[4][kMaxExperts];  // one histogram per 32-token sub-block
+// One CTA per 32-token block (eight warps, four tokens each, selected
+// together): top-(k+1) of the union of the chunks' candidates, the route
+// event (ids, weights, gap), the block's expert histogram (one row of bcount
+// for the permutation) and, when the layer has a shared expert, its gate
+// sigmoid(x . w_sg).
+__global__ void __launch_bounds__(256) router_merge_kernel(const RouterTcArgs a) {
+  __shared__ int hist[kMaxExperts];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int E = a.E, k = a.k;
   const int ncand = a.nchunk * a.kp;  // <= 160
-  for (int e = threadIdx.x; e < 4 * kMaxExperts; e += blockDim.x) (&hist[0][0])[e] = 0;
+  for (int e = threadIdx.x; e < E; e += blockDim.x) hist[e] = 0;
   __syncthreads();
-  const int m0 = blockIdx.x * 128;
-  const int sb = warp >> 2;  // this warp's 8 tokens lie in sub-block sb
-  for (int q0 = 0; q0 < 8; q0 += 4) {
+  const int tw = blockIdx.x * 32 + warp * 4;  // this warp's first token
+  {
     float v[4][5];
     int id[4][5];
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
-      const int t = m0 + warp * 8 + q0 + u;
+      const int t = tw + u;
 #pragma unroll
       for (int i = 0; i < 5; ++i) {
         const int j = lane + 32 * i;
@@ -346,7 +340,7 @@ __global__ void __launch_bounds__(512) router_merge_kernel(const RouterTcArgs a)
     }
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
-      const int t = m0 + warp * 8 + q0 + u;
+      const int t = tw + u;
       const float l0 = __shfl_sync(0xffffffffu, my_v[u], 0);
       const float ex = (lane < k) ? expf(my_v[u] - l0) : 0.f;
       float sum = ex;
@@ -358,47 +352,44 @@ __global__ void __launch_bounds__(512) router_merge_kernel(const RouterTcArgs a)
           const bool real = my_i[u] >= 0 && my_i[u] < E;
           a.ids[(size_t)t * k + lane] = real ? my_i[u] : 0;
           a.weights[(size_t)t * k + lane] = ex / sum;
-          if (real) atomicAdd(&hist[sb][my_i[u]], 1);
+          if (real) atomicAdd(&hist[my_i[u]], 1);
         }
         if (a.gap != nullptr && lane == 0) a.gap[t] = (k < E) ? (lk1 - next_v[u]) : INFINITY;
       }
     }
   }
-  __syncthreads();
-  const int nsub = (a.T + 31) / 32;  // rows of bcount (32-token sub-blocks)
-  for (int i = threadIdx.x; i < 4 * E; i += blockDim.x) {
-    const int s = i / E, e = i - s * E;
-    const int row = blockIdx.x * 4 + s;
-    if (row < nsub) a.bcount[(size_t)row * E + e] = hist[s][e];
-  }
-}
-
-// Shared-expert gate sigmoid(x . w_sg), one warp per token.
-__global__ void __launch_bounds__(256) shared_gate_kernel(const __nv_bfloat16* __restrict__ x,
-                                                          const float* __restrict__ wsg, int T, int H,
-                                                          float* __restrict__ sg) {
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int t = blockIdx.x * 8 + warp;
-  if (t >= T) return;
-  const __nv_bfloat16* xr = x + (size_t)t * H;
-  float s = 0.f;
-#pragma unroll 8
-  for (int h = lane * 8; h < H; h += 256) {
-    const uint4 xv = __ldg(reinterpret_cast<const uint4*>(xr + h));
-    const float4 w0 = __ldg(reinterpret_cast<const float4*>(wsg + h));
-    const float4 w1 = __ldg(reinterpret_cast<const float4*>(wsg + h + 4));
-    s = fmaf(bf16_lo(xv.x), w0.x, s);
-    s = fmaf(bf16_hi(xv.x), w0.y, s);
-    s = fmaf(bf16_lo(xv.y), w0.z, s);
-    s = fmaf(bf16_hi(xv.y), w0.w, s);
-    s = fmaf(bf16_lo(xv.z), w1.x, s);
-    s = fmaf(bf16_hi(xv.z), w1.y, s);
-    s = fmaf(bf16_lo(xv.w), w1.z, s);
-    s = fmaf(bf16_hi(xv.w), w1.w, s);
-  }
+  if (a.wsg != nullptr) {
+    // shared-expert gate of the warp's four tokens, dot products interleaved
+    float sum[4] = {0.f, 0.f, 0.f, 0.f};
+    for (int h = lane * 8; h < a.H; h += 256) {
+      const float4 w0 = __ldg(reinterpret_cast<const float4*>(a.wsg + h));
+      const float4 w1 = __ldg(reinterpret_cast<const float4*>(a.wsg + h + 4));
 #pragma unroll
-  for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
-  if (lane == 0) sg[t] = 1.0f / (1.0f + expf(-s));
+      for (int u = 0; u < 4; ++u) {
+        if (tw + u >= a.T) continue;
+        const uint4 xv = __ldg(reinterpret_cast<const uint4*>(a.x + (size_t)(tw + u) * a.H + h));
+        float s = sum[u];
+        s = fmaf(bf16_lo(xv.x), w0.x, s);
+        s = fmaf(bf16_hi(xv.x), w0.y, s);
+        s = fmaf(bf16_lo(xv.y), w0.z, s);
+        s = fmaf(bf16_hi(xv.y), w0.w, s);
+        s = fmaf(bf16_lo(xv.z), w1.x, s);
+        s = fmaf(bf16_hi(xv.z), w1.y, s);
+        s = fmaf(bf16_lo(xv.w), w1.z, s);
+        s = fmaf(bf16_hi(xv.w), w1.w, s);
+        sum[u] = s;
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      float s = sum[u];
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+      if (lane == 0 && tw + u < a.T) a.sg[tw + u] = 1.0f / (1.0f + expf(-s));
+    }
+  }
+  __syncthreads();
+  for (int e = threadIdx.x; e < E; e += blockDim.x) a.bcount[(size_t)blockIdx.x * E + e] = hist[e];
 }
 
 }  // namespace
@@ -422,10 +413,7 @@ cudaError_t launch_router_tc(const CUtensorMap& tmX, const CUtensorMap& tmW, con
   router_tc_kernel<<<dim3(nb, a.nchunk), NTH, RT_SMEM, s>>>(tmX, tmW, a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  router_merge_kernel<<<nb, 512, 0, s>>>(a);
-  e = cudaGetLastError();
-  if (e != cudaSuccess || a.wsg == nullptr) return e;
-  shared_gate_kernel<<<(a.T + 7) / 8, 256, 0, s>>>(a.x, a.wsg, a.T, a.H, a.sg);
+  router_merge_kernel<<<(a.T + 31) / 32, 256, 0, s>>>(a);
   return cudaGetLastError();
 }
 
