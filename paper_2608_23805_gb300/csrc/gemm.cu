@@ -12,8 +12,9 @@
 // from the slot and dequantise them to bf16 in shared memory inside the
 // producer: eight warps prefetch codes and scales with cp.async into a
 // three-stage raw ring and each thread converts its own B row
-// (w = scale * (q - 8), rounded once to bf16) into the swizzled layout the
-// MMA reads, so the weights cross HBM at 0.5625 bytes each.
+// (w = scale * (q - 8), exact in fp32 and rounded once to bf16, two values
+// per packed f32x2 instruction) into the swizzled layout the MMA reads, so the
+// weights cross HBM at 0.5625 bytes each.
 // Tile: 128 token rows x 256 weight rows x 64 K per stage, 4-stage smem ring,
 // fp32 accumulators double-buffered in TMEM (2 x 256 columns).  Weights (B)
 // come by TMA from the slot pool viewed as one 2-D tensor per operand; the
@@ -42,7 +43,6 @@ constexpr int kGatherWarps = 4;
 constexpr uint32_t kIdesc = idesc_bf16(kBM, kBN);
 
 constexpr int kDqWarps = 8;   // one thread per B row (256 rows)
-constexpr int kRaw = 3;       // raw (packed) stages in flight ahead of conversion
 constexpr int kRawRowBytes = 32;  // 64 codes of one B row per stage
 
 template <int MODE>
@@ -59,11 +59,16 @@ struct Cfg {
   static constexpr uint32_t kTxBytes = (kTmaB ? kBBytes : 0) + (kTmaA ? kABytes : 0);
   // gather threads arrive one by one as their copies land (cp.async ... arrive.noinc)
   static constexpr int kFullCount = (kTmaAny ? 1 : 0) + (kGather ? kGatherWarps * 32 : 0) + (kQ4 ? kDqWarps : 0);
+  // operand ring depth and, in the q4 modes, the raw (packed) stages in flight
+  // ahead of the conversion (eight raw stages in a three-stage operand ring
+  // measured no faster)
+  static constexpr int kStg = kStages;
+  static constexpr int kRaw = kQ4 ? 3 : 1;
   static constexpr int kRawBytes = kQ4 ? kRaw * kBN * (kRawRowBytes + 4) : 0;
   // bf16 modes stage each epilogue warp's rows in shared memory (4 KB per
   // warp) for row-coalesced stores; the q4 raw ring leaves no room for it
   static constexpr bool kStagedEpi = !kQ4;
-  static constexpr int kSmem = 1024 + kStages * (kABytes + kBBytes) + kRawBytes + 256 +
+  static constexpr int kSmem = 1024 + kStg * (kABytes + kBBytes) + kRawBytes + 256 +
                                (kStagedEpi ? kEpiWarps * 4096 : 0);
 };
 
@@ -87,6 +92,40 @@ __device__ __forceinline__ TileCoord decode_tile(const GemmArgs& a, int t) {
   return c;
 }
 
+__device__ __forceinline__ uint64_t f32x2(float lo, float hi) {
+  uint64_t v;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(v) : "r"(__float_as_uint(lo)), "r"(__float_as_uint(hi)));
+  return v;
+}
+
+// Eight 4-bit codes of one 32-bit word (code 2i in the low nibble of byte i,
+// code 2i+1 in its high nibble) -> eight bf16 weights scale * (q - 8), the
+// 16-byte chunk of one K-major row.  Each code becomes the float 2^23 + q by
+// placing its byte under the exponent byte 0x4B (one byte permute); then
+// (2^23 + q) - (2^23 + 8) = q - 8 and the product with the fp16-exact scale
+// are exact in fp32, two values per instruction, and each weight is rounded
+// once to bf16.
+__device__ __forceinline__ uint4 dequant8(uint32_t w, uint64_t scale2) {
+  const uint32_t lo = w & 0x0F0F0F0Fu, hi = (w >> 4) & 0x0F0F0F0Fu;
+  const uint64_t bias2 = 0x4B0000084B000008ull;  // (2^23 + 8, 2^23 + 8)
+  uint32_t o[4];
+#pragma unroll
+  for (int b = 0; b < 4; ++b) {
+    uint32_t el, eh;
+    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(el) : "r"(lo), "r"(0x4B000000u), "r"(0x7440u + b));
+    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(eh) : "r"(hi), "r"(0x4B000000u), "r"(0x7440u + b));
+    uint64_t v;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(v) : "r"(el), "r"(eh));
+    asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(v) : "l"(v), "l"(bias2));
+    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(v) : "l"(v), "l"(scale2));
+    uint32_t vl, vh;
+    asm("mov.b64 {%0, %1}, %2;" : "=r"(vl), "=r"(vh) : "l"(v));
+    // the first operand lands in the upper half: (odd column, even column)
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(o[b]) : "r"(vh), "r"(vl));
+  }
+  return make_uint4(o[0], o[1], o[2], o[3]);
+}
+
 }  // namespace
 
 template <int MODE>
@@ -98,12 +137,12 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   uint8_t* sA = smem;
-  uint8_t* sB = smem + kStages * kABytes;
-  uint8_t* raw_codes = sB + kStages * kBBytes;                    // q4: [kRaw][256][32]
-  uint32_t* raw_scales = reinterpret_cast<uint32_t*>(raw_codes + (C::kQ4 ? kRaw * kBN * kRawRowBytes : 0));
+  uint8_t* sB = smem + C::kStg * kABytes;
+  uint8_t* raw_codes = sB + C::kStg * kBBytes;                    // q4: [C::kRaw][256][32]
+  uint32_t* raw_scales = reinterpret_cast<uint32_t*>(raw_codes + (C::kQ4 ? C::kRaw * kBN * kRawRowBytes : 0));
   uint64_t* full = reinterpret_cast<uint64_t*>(raw_codes + C::kRawBytes);
-  uint64_t* empty = full + kStages;
-  uint64_t* tfull = empty + kStages;
+  uint64_t* empty = full + C::kStg;
+  uint64_t* tfull = empty + C::kStg;
   uint64_t* tempty = tfull + 2;
   uint64_t* drain = tempty + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
@@ -114,7 +153,7 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
   const int lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) {
+    for (int s = 0; s < C::kStg; ++s) {
       mbar_init(&full[s], C::kFullCount);
       mbar_init(&empty[s], 1);
     }
@@ -152,8 +191,8 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
         const int arow = __ldg(&G->row_begin) + tc.m * kBM;
         bool ok = true;
         for (int kb = 0; kb < a.kblocks; ++kb, ++it) {
-          const int s = it % kStages;
-          const uint32_t ph = (it / kStages) & 1;
+          const int s = it % C::kStg;
+          const uint32_t ph = (it / C::kStg) & 1;
           if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, lim)) { ok = false; break; }
           mbar_arrive_expect_tx(&full[s], C::kTxBytes);
           uint8_t* b = sB + s * kBBytes;
@@ -171,11 +210,11 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
       // On abort, wait (bounded) for the copies this thread armed to land
       // before the CTA's shared memory is released.
       if (*abort_flag) {
-        for (int d = 0; d < kStages && it > 0; ++d) {
+        for (int d = 0; d < C::kStg && it > 0; ++d) {
           const uint32_t j = it - 1 - d;
           if ((int)j < 0) break;
           const long long t0 = clock64();
-          while (!mbar_try_wait(&full[j % kStages], (j / kStages) & 1) && clock64() - t0 < lim) {
+          while (!mbar_try_wait(&full[j % C::kStg], (j / C::kStg) & 1) && clock64() - t0 < lim) {
           }
         }
       }
@@ -191,8 +230,8 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
         const uint32_t d = tmem_base + acc * kBN;
         bool ok = true;
         for (int kb = 0; kb < a.kblocks; ++kb, ++it) {
-          const int s = it % kStages;
-          const uint32_t ph = (it / kStages) & 1;
+          const int s = it % C::kStg;
+          const uint32_t ph = (it / C::kStg) & 1;
           if (!mbar_wait(&full[s], ph, abort_flag, lim)) { ok = false; break; }
           // cp.async (generic proxy) wrote A in the gather modes: order those
           // writes before this thread's tensor-core (async proxy) reads
@@ -270,8 +309,8 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
         }
       }
       for (int kb = 0; kb < a.kblocks; ++kb, ++it) {
-        const int s = it % kStages;
-        const uint32_t ph = (it / kStages) & 1;
+        const int s = it % C::kStg;
+        const uint32_t ph = (it / C::kStg) & 1;
         if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, lim)) { ok = false; break; }
         uint8_t* dstA = sA + s * kABytes;
 #pragma unroll
@@ -308,13 +347,13 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
         code_row = base + a.q4_code_off + (size_t)row * a.q4_code_ld;
         scale_row = base + a.q4_scale_off + (size_t)row * a.q4_scale_ld;
       }
-      const int r = j % kRaw;
+      const int r = j % C::kRaw;
       uint8_t* dst = raw_codes + (r * kBN + d) * kRawRowBytes;
       cp_async16(dst, code_row + kb * 32, 16u);
       cp_async16(dst + 16, code_row + kb * 32 + 16, 16u);
       cp_async4(&raw_scales[r * kBN + d], scale_row + kb * 4);
     };
-    for (int i = 0; i < kRaw - 1; ++i, ++jp) {
+    for (int i = 0; i < C::kRaw - 1; ++i, ++jp) {
       if (jp < nstages) issue(jp);
       cp_async_commit();
     }
@@ -322,11 +361,11 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
     for (uint32_t it = 0; it < nstages; ++it, ++jp) {
       if (jp < nstages) issue(jp);
       cp_async_commit();
-      cp_async_wait<kRaw - 1>();  // this thread's raw stage `it` has landed
-      const int s = it % kStages;
-      const uint32_t ph = (it / kStages) & 1;
+      cp_async_wait<C::kRaw - 1>();  // this thread's raw stage `it` has landed
+      const int s = it % C::kStg;
+      const uint32_t ph = (it / C::kStg) & 1;
       if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, lim)) { ok = false; break; }
-      const int r = it % kRaw;
+      const int r = it % C::kRaw;
       const uint4* rc = reinterpret_cast<const uint4*>(raw_codes + (r * kBN + d) * kRawRowBytes);
       const uint4 c0 = rc[0], c1 = rc[1];
       const uint32_t sc = raw_scales[r * kBN + d];
@@ -334,21 +373,11 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
       const float s1 = __half2float(__ushort_as_half((unsigned short)(sc >> 16)));
       uint8_t* dst_row = sB + s * kBBytes + d * 128;
       const uint32_t words[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
+      const uint64_t s0x2 = f32x2(s0, s0), s1x2 = f32x2(s1, s1);
 #pragma unroll
-      for (int c = 0; c < 8; ++c) {
-        const float sc_f = c < 4 ? s0 : s1;
-        const uint32_t w = words[c];
-        uint32_t o[4];
-#pragma unroll
-        for (int b = 0; b < 4; ++b) {
-          const uint32_t lo = (w >> (8 * b)) & 0xFu, hi = (w >> (8 * b + 4)) & 0xFu;
-          // exact small integers: 2^23 + q - (2^23 + 8) = q - 8
-          const float ql = __uint_as_float(0x4B000000u | lo) - 8388616.0f;
-          const float qh = __uint_as_float(0x4B000000u | hi) - 8388616.0f;
-          o[b] = pack_bf16x2(ql * sc_f, qh * sc_f);
-        }
-        *reinterpret_cast<uint4*>(dst_row + ((c ^ (d & 7)) << 4)) = make_uint4(o[0], o[1], o[2], o[3]);
-      }
+      for (int c = 0; c < 8; ++c)
+        *reinterpret_cast<uint4*>(dst_row + ((c ^ (d & 7)) << 4)) =
+            dequant8(words[c], c < 4 ? s0x2 : s1x2);
       fence_proxy_async_smem();
       __syncwarp();
       if (lane == 0) mbar_arrive(&full[s]);
