@@ -114,6 +114,15 @@ struct ScatterArgs {
   int* perm;          // [T*k]
   int* inv;           // [T*k]
   int* offsets;       // [E+1]
+  // block 0 also writes the shared-expert group (when sh_group) and, for a
+  // resident call (table entries in the kernel's TableParams), re-checks the
+  // named slots' generations and builds the GEMM groups
+  const GenWord* genwords;
+  Group* groups;
+  int* total_mtiles;   // [0]: 128-row tiles, [1]: 256-row pair tiles
+  int* status;
+  Group* sh_group;     // or nullptr
+  int* sh_total;
 };
 
 // Per-call tables uploaded by value (kernel parameters, < 32 KB).
@@ -145,8 +154,6 @@ struct SetupArgs {
   const int* counts;
   const int* offsets;
   const GenWord* genwords;
-  const int* table;                       // resident mode
-  const unsigned long long* expected;     // resident mode
   int E, layer;
   Group* groups;
   int* total_mtiles;   // [0]: 128-row tiles, [1]: 256-row pair tiles
@@ -197,14 +204,15 @@ enum GemmMode { kGateUpGather = 0, kGateUpTma = 1, kDown = 2, kGateUpGatherQ4 = 
 // Launchers (return cudaError_t of the launch)
 // ---------------------------------------------------------------------------
 cudaError_t launch_router(const RouterArgs& a, cudaStream_t s);
-cudaError_t launch_split3(const float* w, long long n, __nv_bfloat16* out, cudaStream_t s);
+// Also clears the forward's status word (the first kernel of a forward).
+cudaError_t launch_split3(const float* w, long long n, __nv_bfloat16* out, int* status,
+                          cudaStream_t s);
 cudaError_t launch_router_tc(const CUtensorMap& tmX, const CUtensorMap& tmW, const RouterTcArgs& a,
                              cudaStream_t s);
 cudaError_t launch_colscan(const ScanArgs& a, cudaStream_t s);
-cudaError_t launch_scatter(const ScatterArgs& a, cudaStream_t s);
+cudaError_t launch_scatter(const ScatterArgs& a, const TableParams& tp, cudaStream_t s);
 cudaError_t launch_upload(const TableParams& p, int* table, unsigned long long* expected,
                           int* status, Group* shared_group, int* shared_total, cudaStream_t s);
-cudaError_t launch_setup_resident(const SetupArgs& a, cudaStream_t s);
 cudaError_t launch_setup_wave(const SetupArgs& a, const WaveParams& w, cudaStream_t s);
 cudaError_t launch_publish(const PublishParams& p, GenWord* genwords, cudaStream_t s);
 cudaError_t launch_gemm(int mode, const CUtensorMap& tmA, const CUtensorMap& tmB,

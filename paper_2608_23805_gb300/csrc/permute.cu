@@ -41,10 +41,116 @@ __global__ void __launch_bounds__(1024) colscan_kernel(const ScanArgs a) {
   }
 }
 
+__device__ __forceinline__ int check_code(const GenWord* gw, int slot, int layer, int e,
+                                          unsigned long long expected) {
+  if (slot < 0) return MSI_ERR_NOT_RESIDENT;
+  const unsigned long long obj = gw[slot].obj;
+  const unsigned long long gen = gw[slot].gen;
+  if (obj != obj_key(layer, e)) return MSI_ERR_WRONG_OBJECT;
+  if (gen != expected) return MSI_ERR_STALE_GENERATION;
+  return 0;
+}
+
 // ---- scatter: one warp per router block ----
 constexpr int kScatterWarps = 4;
 
-__global__ void __launch_bounds__(kScatterWarps * 32) scatter_kernel(const ScatterArgs a) {
+// Exclusive scan over the block of four values per thread (128 threads);
+// returns the thread's base and leaves the block total in *total.
+__device__ __forceinline__ int scan4(const int (&v)[4], int* wsum, int* total) {
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int s = v[0] + v[1] + v[2] + v[3];
+  int incl = s;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const int o = __shfl_up_sync(0xffffffffu, incl, off);
+    if (lane >= off) incl += o;
+  }
+  if (lane == 31) wsum[warp] = incl;
+  __syncthreads();
+  int base = incl - s, tot = 0;
+  for (int w = 0; w < kScatterWarps; ++w) {
+    if (w < warp) base += wsum[w];
+    tot += wsum[w];
+  }
+  *total = tot;
+  __syncthreads();
+  return base;
+}
+
+// Block 0 of the scatter: the shared-expert group, and for a resident call
+// the generation re-check of every routed expert's slot (fail closed) and the
+// GEMM groups with their 128- and 256-row tile prefixes.
+__device__ void scatter_setup(const ScatterArgs& a, const TableParams& tp, const int* offs) {
+  __shared__ int wsum[kScatterWarps];
+  __shared__ int kmin[kScatterWarps];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  if (a.sh_group != nullptr && tid == 0) {
+    Group g;
+    g.row_begin = 0;
+    g.row_count = tp.T;
+    g.slot = tp.shared_slot;
+    g.mt_begin = 0;
+    g.ok = 1;
+    g.expert = -1;
+    g.pt_begin = g.pad1 = 0;
+    *a.sh_group = g;
+    a.sh_total[0] = (tp.T + kBM - 1) / kBM;
+    a.sh_total[1] = (tp.T + 2 * kBM - 1) / (2 * kBM);
+  }
+  if (tp.E == 0) return;  // streamed call: the groups are built per wave
+  int cnt[4], code[4], mt[4], pt[4];
+  int key = 0x7fffffff;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int e = tid * 4 + i;
+    cnt[i] = code[i] = mt[i] = pt[i] = 0;
+    if (e < a.E) {
+      cnt[i] = a.counts[e];
+      if (cnt[i] > 0) code[i] = check_code(a.genwords, tp.slot[e], tp.layer, e, tp.expected[e]);
+      if (code[i] == 0) {
+        mt[i] = (cnt[i] + kBM - 1) / kBM;
+        pt[i] = (cnt[i] + 2 * kBM - 1) / (2 * kBM);
+      } else {
+        key = min(key, (e << 4) | code[i]);
+      }
+    }
+  }
+  int mtot = 0, ptot = 0;
+  int mb = scan4(mt, wsum, &mtot);
+  int pb = scan4(pt, wsum, &ptot);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int e = tid * 4 + i;
+    if (e < a.E) {
+      Group g;
+      g.row_begin = offs[e];
+      g.row_count = cnt[i];
+      g.slot = tp.slot[e] < 0 ? 0 : tp.slot[e];
+      g.mt_begin = mb;
+      g.ok = code[i] == 0;
+      g.expert = e;
+      g.pt_begin = pb;
+      g.pad1 = 0;
+      a.groups[e] = g;
+    }
+    mb += mt[i];
+    pb += pt[i];
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) key = min(key, __shfl_xor_sync(0xffffffffu, key, off));
+  if (lane == 0) kmin[warp] = key;
+  __syncthreads();
+  if (tid == 0) {
+    int m = kmin[0];
+    for (int w = 1; w < kScatterWarps; ++w) m = min(m, kmin[w]);
+    a.total_mtiles[0] = mtot;
+    a.total_mtiles[1] = ptot;
+    if (m != 0x7fffffff) atomicCAS(a.status, 0, m & 15);
+  }
+}
+
+__global__ void __launch_bounds__(kScatterWarps * 32) scatter_kernel(const ScatterArgs a,
+                                                                     const TableParams tp) {
   __shared__ int offs[kMaxExperts + 1];
   __shared__ int run[kScatterWarps][kMaxExperts];
   __shared__ int wsum[kScatterWarps];
@@ -76,8 +182,10 @@ __global__ void __launch_bounds__(kScatterWarps * 32) scatter_kernel(const Scatt
   }
   if (tid == kScatterWarps * 32 - 1 && a.E == kMaxExperts) offs[kMaxExperts] = base;
   __syncthreads();
-  if (blockIdx.x == 0)
+  if (blockIdx.x == 0) {
     for (int e = tid; e <= a.E; e += blockDim.x) a.offsets[e] = offs[e];
+    scatter_setup(a, tp, offs);
+  }
 
   const int b = blockIdx.x * kScatterWarps + warp;
   if (b >= a.nb) return;
@@ -161,28 +269,18 @@ __device__ __forceinline__ int block_min(int v, int* tmp) {
   return m;
 }
 
-__device__ __forceinline__ int check_code(const GenWord* gw, int slot, int layer, int e,
-                                          unsigned long long expected) {
-  if (slot < 0) return MSI_ERR_NOT_RESIDENT;
-  const unsigned long long obj = gw[slot].obj;
-  const unsigned long long gen = gw[slot].gen;
-  if (obj != obj_key(layer, e)) return MSI_ERR_WRONG_OBJECT;
-  if (gen != expected) return MSI_ERR_STALE_GENERATION;
-  return 0;
-}
-
-template <bool WAVE>
+// One LRU wave of a streamed call: re-check the wave's slots and build its
+// GEMM groups (the resident call does this in the scatter kernel).
 __global__ void __launch_bounds__(kMaxExperts) setup_kernel(const SetupArgs a, const WaveParams w) {
   __shared__ int tmp[32];
   const int i = threadIdx.x;
-  const int n = WAVE ? w.n : a.E;
+  const int n = w.n;
   int e = -1, cnt = 0, slot = -1, code = 0;
   if (i < n) {
-    e = WAVE ? w.expert[i] : i;
+    e = w.expert[i];
     cnt = a.counts[e];
-    slot = WAVE ? w.slot[i] : a.table[e];
-    const unsigned long long exp = WAVE ? w.expected[i] : a.expected[e];
-    if (cnt > 0) code = check_code(a.genwords, slot, a.layer, e, exp);
+    slot = w.slot[i];
+    if (cnt > 0) code = check_code(a.genwords, slot, a.layer, e, w.expected[i]);
   }
   const int mt = (i < n && code == 0) ? (cnt + kBM - 1) / kBM : 0;
   const int pt = (i < n && code == 0) ? (cnt + 2 * kBM - 1) / (2 * kBM) : 0;
@@ -222,39 +320,48 @@ __global__ void publish_kernel(const PublishParams p, GenWord* gw) {
 }
 
 // ---- combine: out[t] = sum_j w[t,j] yp[inv[t*k+j]] (+ sg[t] ys[t]) (+ x[t]) ----
+__device__ __forceinline__ void fma8(float (&acc)[8], float w, const uint4& y) {
+  acc[0] = fmaf(w, bf16_lo(y.x), acc[0]);
+  acc[1] = fmaf(w, bf16_hi(y.x), acc[1]);
+  acc[2] = fmaf(w, bf16_lo(y.y), acc[2]);
+  acc[3] = fmaf(w, bf16_hi(y.y), acc[3]);
+  acc[4] = fmaf(w, bf16_lo(y.z), acc[4]);
+  acc[5] = fmaf(w, bf16_hi(y.z), acc[5]);
+  acc[6] = fmaf(w, bf16_lo(y.w), acc[6]);
+  acc[7] = fmaf(w, bf16_hi(y.w), acc[7]);
+}
+
+// One block per token; the token's k row indices and weights are read once
+// into shared memory, and four expert rows are loaded before they are summed
+// (still in j order, fp32).
 __global__ void __launch_bounds__(256) combine_kernel(const CombineArgs a) {
   if (*a.status != 0) return;  // fail closed: nothing stale becomes visible
+  __shared__ int s_row[kMaxTopK];
+  __shared__ float s_w[kMaxTopK];
   const int t = blockIdx.x;
+  if (threadIdx.x < a.k) {
+    s_row[threadIdx.x] = __ldg(&a.inv[(size_t)t * a.k + threadIdx.x]);
+    s_w[threadIdx.x] = __ldg(&a.weights[(size_t)t * a.k + threadIdx.x]);
+  }
+  __syncthreads();
   const int nchunk = a.H >> 3;
   for (int c = threadIdx.x; c < nchunk; c += blockDim.x) {
     float acc[8];
 #pragma unroll
     for (int i = 0; i < 8; ++i) acc[i] = 0.f;
-    for (int j = 0; j < a.k; ++j) {
-      const int r = __ldg(&a.inv[(size_t)t * a.k + j]);
-      const float w = __ldg(&a.weights[(size_t)t * a.k + j]);
-      const uint4 y = __ldg(reinterpret_cast<const uint4*>(a.yp + (size_t)r * a.H) + c);
-      acc[0] = fmaf(w, bf16_lo(y.x), acc[0]);
-      acc[1] = fmaf(w, bf16_hi(y.x), acc[1]);
-      acc[2] = fmaf(w, bf16_lo(y.y), acc[2]);
-      acc[3] = fmaf(w, bf16_hi(y.y), acc[3]);
-      acc[4] = fmaf(w, bf16_lo(y.z), acc[4]);
-      acc[5] = fmaf(w, bf16_hi(y.z), acc[5]);
-      acc[6] = fmaf(w, bf16_lo(y.w), acc[6]);
-      acc[7] = fmaf(w, bf16_hi(y.w), acc[7]);
+    int j = 0;
+    for (; j + 4 <= a.k; j += 4) {
+      uint4 y[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+        y[u] = __ldg(reinterpret_cast<const uint4*>(a.yp + (size_t)s_row[j + u] * a.H) + c);
+#pragma unroll
+      for (int u = 0; u < 4; ++u) fma8(acc, s_w[j + u], y[u]);
     }
-    if (a.ys != nullptr) {
-      const float g = a.sg[t];
-      const uint4 y = __ldg(reinterpret_cast<const uint4*>(a.ys + (size_t)t * a.H) + c);
-      acc[0] = fmaf(g, bf16_lo(y.x), acc[0]);
-      acc[1] = fmaf(g, bf16_hi(y.x), acc[1]);
-      acc[2] = fmaf(g, bf16_lo(y.y), acc[2]);
-      acc[3] = fmaf(g, bf16_hi(y.y), acc[3]);
-      acc[4] = fmaf(g, bf16_lo(y.z), acc[4]);
-      acc[5] = fmaf(g, bf16_hi(y.z), acc[5]);
-      acc[6] = fmaf(g, bf16_lo(y.w), acc[6]);
-      acc[7] = fmaf(g, bf16_hi(y.w), acc[7]);
-    }
+    for (; j < a.k; ++j)
+      fma8(acc, s_w[j], __ldg(reinterpret_cast<const uint4*>(a.yp + (size_t)s_row[j] * a.H) + c));
+    if (a.ys != nullptr)
+      fma8(acc, a.sg[t], __ldg(reinterpret_cast<const uint4*>(a.ys + (size_t)t * a.H) + c));
     if (a.x != nullptr) {
       const uint4 y = __ldg(reinterpret_cast<const uint4*>(a.x + (size_t)t * a.H) + c);
       acc[0] += bf16_lo(y.x);
@@ -286,9 +393,9 @@ cudaError_t launch_colscan(const ScanArgs& a, cudaStream_t s) {
   return cudaGetLastError();
 }
 
-cudaError_t launch_scatter(const ScatterArgs& a, cudaStream_t s) {
+cudaError_t launch_scatter(const ScatterArgs& a, const TableParams& tp, cudaStream_t s) {
   const int grid = (a.nb + kScatterWarps - 1) / kScatterWarps;
-  scatter_kernel<<<grid, kScatterWarps * 32, 0, s>>>(a);
+  scatter_kernel<<<grid, kScatterWarps * 32, 0, s>>>(a, tp);
   return cudaGetLastError();
 }
 
@@ -298,16 +405,9 @@ cudaError_t launch_upload(const TableParams& p, int* table, unsigned long long* 
   return cudaGetLastError();
 }
 
-cudaError_t launch_setup_resident(const SetupArgs& a, cudaStream_t s) {
-  WaveParams none;
-  none.n = 0;
-  none.layer = a.layer;
-  setup_kernel<false><<<1, kMaxExperts, 0, s>>>(a, none);
-  return cudaGetLastError();
-}
 
 cudaError_t launch_setup_wave(const SetupArgs& a, const WaveParams& w, cudaStream_t s) {
-  setup_kernel<true><<<1, kMaxExperts, 0, s>>>(a, w);
+  setup_kernel<<<1, kMaxExperts, 0, s>>>(a, w);
   return cudaGetLastError();
 }
 

@@ -452,9 +452,13 @@ msi_status front(msi_plan* p, FwdCtx& f, const TableParams& tp) {
   const int E = d.n_experts, k = d.top_k, H = d.hidden, I = d.inter;
   void* ws = f.ws;
   const WsLayout& L = f.L;
-  LAUNCH(p, MSI_K_UPLOAD, f.cs, launch_upload(tp, at<int>(ws, L.table), at<unsigned long long>(ws, L.expected),
-                          at<int>(ws, L.status), d.has_shared ? at<Group>(ws, L.sh_group) : nullptr,
-                          at<int>(ws, L.sh_total), f.cs));
+  // The tensor-router path clears the status word in its first kernel and
+  // the scatter kernel writes the shared group and (resident calls) the GEMM
+  // groups, so only the other paths need the upload kernel.
+  if (f.T == 0 || !tensor_router(d))
+    LAUNCH(p, MSI_K_UPLOAD, f.cs, launch_upload(tp, at<int>(ws, L.table), at<unsigned long long>(ws, L.expected),
+                            at<int>(ws, L.status), d.has_shared ? at<Group>(ws, L.sh_group) : nullptr,
+                            at<int>(ws, L.sh_total), f.cs));
   if (f.T == 0) {
     LAUNCH(p, MSI_K_UPLOAD, f.cs, launch_zero_counts(f.ev->counts, E, f.cs));
     return MSI_OK;
@@ -463,7 +467,8 @@ msi_status front(msi_plan* p, FwdCtx& f, const TableParams& tp) {
   if (!make_tmap(&f.tm_x, f.x, H, f.T, 128)) return MSI_ERR_CUDA;
   if (tensor_router(d)) {
     __nv_bfloat16* w3 = at<__nv_bfloat16>(ws, L.w3);
-    LAUNCH(p, MSI_K_ROUTER, f.cs, launch_split3(f.router_w, (long long)E * H, w3, f.cs));
+    LAUNCH(p, MSI_K_ROUTER, f.cs,
+           launch_split3(f.router_w, (long long)E * H, w3, at<int>(ws, L.status), f.cs));
     const int ch = std::min(E, kRouterChunk);
     CUtensorMap tm_w3;
     if (!make_tmap(&tm_w3, w3, H, (uint64_t)3 * E, (uint32_t)ch)) return MSI_ERR_CUDA;
@@ -508,9 +513,25 @@ msi_status front(msi_plan* p, FwdCtx& f, const TableParams& tp) {
   }
   ScanArgs sa{at<int>(ws, L.bcount), nb, E, at<int>(ws, L.bbase), f.ev->counts};
   LAUNCH(p, MSI_K_SCAN, f.cs, launch_colscan(sa, f.cs));
-  ScatterArgs xa{f.ev->ids, f.ev->counts, at<int>(ws, L.bbase), f.T, k, E, nb, L.tm,
-                 at<int>(ws, L.perm), at<int>(ws, L.inv), at<int>(ws, L.offsets)};
-  LAUNCH(p, MSI_K_SCATTER, f.cs, launch_scatter(xa, f.cs));
+  ScatterArgs xa{};
+  xa.ids = f.ev->ids;
+  xa.counts = f.ev->counts;
+  xa.bbase = at<int>(ws, L.bbase);
+  xa.T = f.T;
+  xa.k = k;
+  xa.E = E;
+  xa.nb = nb;
+  xa.tm = L.tm;
+  xa.perm = at<int>(ws, L.perm);
+  xa.inv = at<int>(ws, L.inv);
+  xa.offsets = at<int>(ws, L.offsets);
+  xa.genwords = p->d_gen;
+  xa.groups = at<Group>(ws, L.groups);
+  xa.total_mtiles = at<int>(ws, L.total);
+  xa.status = at<int>(ws, L.status);
+  xa.sh_group = d.has_shared ? at<Group>(ws, L.sh_group) : nullptr;
+  xa.sh_total = at<int>(ws, L.sh_total);
+  LAUNCH(p, MSI_K_SCATTER, f.cs, launch_scatter(xa, tp, f.cs));
   const size_t Tk = (size_t)f.T * k;
   if (!make_tmap(&f.tm_h, at<char>(ws, L.h), I, Tk, 128)) return MSI_ERR_CUDA;
   if (d.has_shared) {
@@ -898,18 +919,8 @@ msi_status msi_moe_forward(msi_plan* p, int layer, const void* x, int T, const f
   st = front(p, f, tp);
   if (st != MSI_OK) return st;
   if (T > 0) {
-    SetupArgs sa{};
-    sa.counts = ev->counts;
-    sa.offsets = at<int>(ws, f.L.offsets);
-    sa.genwords = p->d_gen;
-    sa.table = at<int>(ws, f.L.table);
-    sa.expected = at<unsigned long long>(ws, f.L.expected);
-    sa.E = E;
-    sa.layer = layer;
-    sa.groups = at<Group>(ws, f.L.groups);
-    sa.total_mtiles = at<int>(ws, f.L.total);
-    sa.status = at<int>(ws, f.L.status);
-    LAUNCH(p, MSI_K_SETUP, f.cs, launch_setup_resident(sa, f.cs));
+    // the scatter kernel has re-checked the slots' generations and built the
+    // GEMM groups (`tp` carries the table)
     const long long mt_max = ((long long)T * d.top_k + kBM - 1) / kBM + E;
     const int g1 = (int)std::min<long long>(p->sms, mt_max * (d.inter / 128));
     const int g2 = (int)std::min<long long>(p->sms, mt_max * (d.hidden / kBN));

@@ -42,7 +42,9 @@ constexpr int RT_LLD = kRouterChunk + 1;             // padded logits row (float
 constexpr int RT_SMEM = 1024 + RT_STAGES * RT_STAGE + 256;
 static_assert(128 * RT_LLD * 4 <= RT_STAGES * RT_STAGE, "logits tile does not fit");
 
-__global__ void split3_kernel(const float* __restrict__ w, long long n, __nv_bfloat16* __restrict__ out) {
+__global__ void split3_kernel(const float* __restrict__ w, long long n, __nv_bfloat16* __restrict__ out,
+                              int* status) {
+  if (blockIdx.x == 0 && threadIdx.x == 0) *status = 0;  // the forward's first kernel
   for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < n;
        i += (long long)gridDim.x * blockDim.x) {
     const float v = w[i];
@@ -394,10 +396,11 @@ __global__ void __launch_bounds__(256) router_merge_kernel(const RouterTcArgs a)
 
 }  // namespace
 
-cudaError_t launch_split3(const float* w, long long n, __nv_bfloat16* out, cudaStream_t s) {
+cudaError_t launch_split3(const float* w, long long n, __nv_bfloat16* out, int* status,
+                          cudaStream_t s) {
   const long long want = (n + 255) / 256;
   const int grid = (int)(want < 152 * 8 ? want : 152 * 8);
-  split3_kernel<<<grid, 256, 0, s>>>(w, n, out);
+  split3_kernel<<<grid, 256, 0, s>>>(w, n, out, status);
   return cudaGetLastError();
 }
 
