@@ -114,15 +114,13 @@ struct ScatterArgs {
   int* perm;          // [T*k]
   int* inv;           // [T*k]
   int* offsets;       // [E+1]
-  // block 0 also writes the shared-expert group (when sh_group) and, for a
-  // resident call (table entries in the kernel's TableParams), re-checks the
-  // named slots' generations and builds the GEMM groups
+  // block 0 also, for a resident call (table entries in the kernel's
+  // TableParams), re-checks the named slots' generations and builds the GEMM
+  // groups
   const GenWord* genwords;
   Group* groups;
   int* total_mtiles;   // [0]: 128-row tiles, [1]: 256-row pair tiles
   int* status;
-  Group* sh_group;     // or nullptr
-  int* sh_total;
 };
 
 // Per-call tables uploaded by value (kernel parameters, < 32 KB).
@@ -204,9 +202,11 @@ enum GemmMode { kGateUpGather = 0, kGateUpTma = 1, kDown = 2, kGateUpGatherQ4 = 
 // Launchers (return cudaError_t of the launch)
 // ---------------------------------------------------------------------------
 cudaError_t launch_router(const RouterArgs& a, cudaStream_t s);
-// Also clears the forward's status word (the first kernel of a forward).
-cudaError_t launch_split3(const float* w, long long n, __nv_bfloat16* out, int* status,
-                          cudaStream_t s);
+// Also begins the forward (its first kernel): clears the status word and,
+// when sh is not null, writes the shared-expert group of T rows in block
+// `shared_slot` and its tile counts.
+cudaError_t launch_split3(const float* w, long long n, __nv_bfloat16* out, int* status, Group* sh,
+                          int* sh_total, int T, int shared_slot, cudaStream_t s);
 cudaError_t launch_router_tc(const CUtensorMap& tmX, const CUtensorMap& tmW, const RouterTcArgs& a,
                              cudaStream_t s);
 cudaError_t launch_colscan(const ScanArgs& a, cudaStream_t s);

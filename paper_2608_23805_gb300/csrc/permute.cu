@@ -77,26 +77,13 @@ __device__ __forceinline__ int scan4(const int (&v)[4], int* wsum, int* total) {
   return base;
 }
 
-// Block 0 of the scatter: the shared-expert group, and for a resident call
-// the generation re-check of every routed expert's slot (fail closed) and the
-// GEMM groups with their 128- and 256-row tile prefixes.
+// Block 0 of the scatter, resident call: the generation re-check of every
+// routed expert's slot (fail closed) and the GEMM groups with their 128- and
+// 256-row tile prefixes.
 __device__ void scatter_setup(const ScatterArgs& a, const TableParams& tp, const int* offs) {
   __shared__ int wsum[kScatterWarps];
   __shared__ int kmin[kScatterWarps];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  if (a.sh_group != nullptr && tid == 0) {
-    Group g;
-    g.row_begin = 0;
-    g.row_count = tp.T;
-    g.slot = tp.shared_slot;
-    g.mt_begin = 0;
-    g.ok = 1;
-    g.expert = -1;
-    g.pt_begin = g.pad1 = 0;
-    *a.sh_group = g;
-    a.sh_total[0] = (tp.T + kBM - 1) / kBM;
-    a.sh_total[1] = (tp.T + 2 * kBM - 1) / (2 * kBM);
-  }
   if (tp.E == 0) return;  // streamed call: the groups are built per wave
   int cnt[4], code[4], mt[4], pt[4];
   int key = 0x7fffffff;

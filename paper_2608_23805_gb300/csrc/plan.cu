@@ -217,6 +217,11 @@ struct msi_plan {
   uint64_t epoch = 0;
   std::map<uint64_t, int> faults;  // one-shot host-side fault hooks by object key
   KernelTimer timer;
+  // the shared expert of a resident forward runs on `side`, forked after the
+  // forward's first kernel and joined before the combine (plans with a shared
+  // expert only)
+  cudaStream_t side = nullptr;
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
   std::mutex mu;
 
   explicit msi_plan(int S) : holds(S) {
@@ -465,10 +470,21 @@ msi_status front(msi_plan* p, FwdCtx& f, const TableParams& tp) {
   }
   const int nb = (f.T + L.tm - 1) / L.tm;
   if (!make_tmap(&f.tm_x, f.x, H, f.T, 128)) return MSI_ERR_CUDA;
+  if (d.has_shared) {
+    if (!make_tmap(&f.tm_hs, at<char>(ws, L.hs), I, f.T, 128)) return MSI_ERR_CUDA;
+  }
   if (tensor_router(d)) {
     __nv_bfloat16* w3 = at<__nv_bfloat16>(ws, L.w3);
     LAUNCH(p, MSI_K_ROUTER, f.cs,
-           launch_split3(f.router_w, (long long)E * H, w3, at<int>(ws, L.status), f.cs));
+           launch_split3(f.router_w, (long long)E * H, w3, at<int>(ws, L.status),
+                         d.has_shared ? at<Group>(ws, L.sh_group) : nullptr, at<int>(ws, L.sh_total),
+                         f.T, tp.shared_slot, f.cs));
+  }
+  // the forward has begun (status cleared, shared group written): the shared
+  // expert may start on the side stream from here
+  if (d.has_shared) CK(cudaEventRecord(p->ev_fork, f.cs));
+  if (tensor_router(d)) {
+    __nv_bfloat16* w3 = at<__nv_bfloat16>(ws, L.w3);
     const int ch = std::min(E, kRouterChunk);
     CUtensorMap tm_w3;
     if (!make_tmap(&tm_w3, w3, H, (uint64_t)3 * E, (uint32_t)ch)) return MSI_ERR_CUDA;
@@ -529,14 +545,9 @@ msi_status front(msi_plan* p, FwdCtx& f, const TableParams& tp) {
   xa.groups = at<Group>(ws, L.groups);
   xa.total_mtiles = at<int>(ws, L.total);
   xa.status = at<int>(ws, L.status);
-  xa.sh_group = d.has_shared ? at<Group>(ws, L.sh_group) : nullptr;
-  xa.sh_total = at<int>(ws, L.sh_total);
   LAUNCH(p, MSI_K_SCATTER, f.cs, launch_scatter(xa, tp, f.cs));
   const size_t Tk = (size_t)f.T * k;
   if (!make_tmap(&f.tm_h, at<char>(ws, L.h), I, Tk, 128)) return MSI_ERR_CUDA;
-  if (d.has_shared) {
-    if (!make_tmap(&f.tm_hs, at<char>(ws, L.hs), I, f.T, 128)) return MSI_ERR_CUDA;
-  }
   return MSI_OK;
 }
 
@@ -622,7 +633,7 @@ msi_status routed_ffn(msi_plan* p, FwdCtx& f, int ng, int grid1, int grid2, bool
   return MSI_OK;
 }
 
-msi_status shared_ffn(msi_plan* p, FwdCtx& f) {
+msi_status shared_ffn(msi_plan* p, FwdCtx& f, cudaStream_t stream) {
   if (!p->d.has_shared || f.T == 0) return MSI_OK;
   const Group* g = at<Group>(f.ws, f.L.sh_group);
   const int* total = at<int>(f.ws, f.L.sh_total);
@@ -631,14 +642,14 @@ msi_status shared_ffn(msi_plan* p, FwdCtx& f) {
   GemmArgs s2 = down_args(p, f, g, 1, total, at<__nv_bfloat16>(f.ws, f.L.ys));
   if (p->d.wdtype == MSI_W_BF16 && pair_tiles(f, f.T, 1)) {
     const int pt = (f.T + 2 * kBM - 1) / (2 * kBM);
-    LAUNCH(p, MSI_K_SHARED_GATEUP, f.cs,
-           launch_gemm_pair(kGateUpTma, f.tm_x, p->tm_sh13, s1, pt * s1.nt, f.cs));
-    LAUNCH(p, MSI_K_SHARED_DOWN, f.cs,
-           launch_gemm_pair(kDown, f.tm_hs, p->tm_sh2, s2, pt * s2.nt, f.cs));
+    LAUNCH(p, MSI_K_SHARED_GATEUP, stream,
+           launch_gemm_pair(kGateUpTma, f.tm_x, p->tm_sh13, s1, pt * s1.nt, stream));
+    LAUNCH(p, MSI_K_SHARED_DOWN, stream,
+           launch_gemm_pair(kDown, f.tm_hs, p->tm_sh2, s2, pt * s2.nt, stream));
     return MSI_OK;
   }
-  LAUNCH(p, MSI_K_SHARED_GATEUP, f.cs, launch_gemm(kGateUpTma, f.tm_x, p->tm_sh13, s1, std::min(p->sms, mt * s1.nt), f.cs));
-  LAUNCH(p, MSI_K_SHARED_DOWN, f.cs, launch_gemm(kDown, f.tm_hs, p->tm_sh2, s2, std::min(p->sms, mt * s2.nt), f.cs));
+  LAUNCH(p, MSI_K_SHARED_GATEUP, stream, launch_gemm(kGateUpTma, f.tm_x, p->tm_sh13, s1, std::min(p->sms, mt * s1.nt), stream));
+  LAUNCH(p, MSI_K_SHARED_DOWN, stream, launch_gemm(kDown, f.tm_hs, p->tm_sh2, s2, std::min(p->sms, mt * s2.nt), stream));
   return MSI_OK;
 }
 
@@ -747,6 +758,9 @@ msi_status msi_plan_create(const msi_plan_desc* desc, msi_plan** out) {
     if (p->d_gen) cudaFree(p->d_gen);
     if (p->h_status) cudaFreeHost(p->h_status);
     if (p->h_counts) cudaFreeHost(p->h_counts);
+    if (p->side) cudaStreamDestroy(p->side);
+    if (p->ev_fork) cudaEventDestroy(p->ev_fork);
+    if (p->ev_join) cudaEventDestroy(p->ev_join);
     delete p;
     return s;
   };
@@ -757,6 +771,9 @@ msi_status msi_plan_create(const msi_plan_desc* desc, msi_plan** out) {
   if (e == cudaSuccess) e = cudaMemset(p->d_gen, 0, sizeof(GenWord) * d.n_slots);
   if (e == cudaSuccess) e = cudaMallocHost(&p->h_status, sizeof(int));
   if (e == cudaSuccess) e = cudaMallocHost(&p->h_counts, sizeof(int) * d.n_experts);
+  if (e == cudaSuccess && d.has_shared) e = cudaStreamCreateWithFlags(&p->side, cudaStreamNonBlocking);
+  if (e == cudaSuccess && d.has_shared) e = cudaEventCreateWithFlags(&p->ev_fork, cudaEventDisableTiming);
+  if (e == cudaSuccess && d.has_shared) e = cudaEventCreateWithFlags(&p->ev_join, cudaEventDisableTiming);
   if (e != cudaSuccess) return fail(cuda_fail(e, "msi_plan_create"));
   *p->h_status = 0;
   const uint64_t H = d.hidden, I = d.inter, S = d.n_slots;
@@ -787,11 +804,15 @@ msi_status msi_plan_destroy(msi_plan* p) {
       if (s.consumer >= 0) cudaEventSynchronize(p->pool.ev[s.consumer]);
     }
     if (p->fwd_ev >= 0) cudaEventSynchronize(p->pool.ev[p->fwd_ev]);
+    if (p->side) cudaStreamSynchronize(p->side);
     p->timer.destroy();
     for (auto ev : p->pool.ev) cudaEventDestroy(ev);
     cudaFree(p->d_gen);
     cudaFreeHost(p->h_status);
     cudaFreeHost(p->h_counts);
+    if (p->side) cudaStreamDestroy(p->side);
+    if (p->ev_fork) cudaEventDestroy(p->ev_fork);
+    if (p->ev_join) cudaEventDestroy(p->ev_join);
   }
   delete p;
   return MSI_OK;
@@ -918,6 +939,16 @@ msi_status msi_moe_forward(msi_plan* p, int layer, const void* x, int T, const f
   }
   st = front(p, f, tp);
   if (st != MSI_OK) return st;
+  const bool fork = d.has_shared && T > 0;
+  if (fork) {
+    // the shared expert needs no routing: it runs on the side stream while
+    // the router, scan and scatter leave most SMs idle, and joins before the
+    // combine
+    CK(cudaStreamWaitEvent(p->side, p->ev_fork, 0));
+    st = shared_ffn(p, f, p->side);
+    if (st != MSI_OK) return st;
+    CK(cudaEventRecord(p->ev_join, p->side));
+  }
   if (T > 0) {
     // the scatter kernel has re-checked the slots' generations and built the
     // GEMM groups (`tp` carries the table)
@@ -929,9 +960,8 @@ msi_status msi_moe_forward(msi_plan* p, int layer, const void* x, int T, const f
     if (st != MSI_OK) return st;
     st = consumer_record(p, used, f.cs);
     if (st != MSI_OK) return st;
-    st = shared_ffn(p, f);
-    if (st != MSI_OK) return st;
   }
+  if (fork) CK(cudaStreamWaitEvent(f.cs, p->ev_join, 0));
   st = finish(p, f);
   if (st != MSI_OK) return st;
   p->ctr.forwards++;
@@ -972,7 +1002,7 @@ msi_status msi_moe_forward_streamed(msi_plan* p, int layer, const void* x, int T
   st = p->pool.acquire(&cev);
   if (st != MSI_OK) return st;
   CK(cudaEventRecord(p->pool.ev[cev], f.cs));
-  st = shared_ffn(p, f);  // overlaps the host planning and the first wave's copies
+  st = shared_ffn(p, f, f.cs);  // overlaps the host planning and the first wave's copies
   if (st != MSI_OK) return st;
   const cudaError_t se = cudaEventSynchronize(p->pool.ev[cev]);
   p->pool.unref(cev);

@@ -43,8 +43,23 @@ constexpr int RT_SMEM = 1024 + RT_STAGES * RT_STAGE + 256;
 static_assert(128 * RT_LLD * 4 <= RT_STAGES * RT_STAGE, "logits tile does not fit");
 
 __global__ void split3_kernel(const float* __restrict__ w, long long n, __nv_bfloat16* __restrict__ out,
-                              int* status) {
-  if (blockIdx.x == 0 && threadIdx.x == 0) *status = 0;  // the forward's first kernel
+                              int* status, Group* sh, int* sh_total, int T, int shared_slot) {
+  if (blockIdx.x == 0 && threadIdx.x == 0) {  // the forward's first kernel
+    *status = 0;
+    if (sh != nullptr) {
+      Group g;
+      g.row_begin = 0;
+      g.row_count = T;
+      g.slot = shared_slot;
+      g.mt_begin = 0;
+      g.ok = 1;
+      g.expert = -1;
+      g.pt_begin = g.pad1 = 0;
+      *sh = g;
+      sh_total[0] = (T + kBM - 1) / kBM;
+      sh_total[1] = (T + 2 * kBM - 1) / (2 * kBM);
+    }
+  }
   for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < n;
        i += (long long)gridDim.x * blockDim.x) {
     const float v = w[i];
@@ -396,11 +411,11 @@ __global__ void __launch_bounds__(256) router_merge_kernel(const RouterTcArgs a)
 
 }  // namespace
 
-cudaError_t launch_split3(const float* w, long long n, __nv_bfloat16* out, int* status,
-                          cudaStream_t s) {
+cudaError_t launch_split3(const float* w, long long n, __nv_bfloat16* out, int* status, Group* sh,
+                          int* sh_total, int T, int shared_slot, cudaStream_t s) {
   const long long want = (n + 255) / 256;
   const int grid = (int)(want < 152 * 8 ? want : 152 * 8);
-  split3_kernel<<<grid, 256, 0, s>>>(w, n, out, status);
+  split3_kernel<<<grid, 256, 0, s>>>(w, n, out, status, sh, sh_total, T, shared_slot);
   return cudaGetLastError();
 }
 
