@@ -387,11 +387,27 @@ msi_status stage_enqueue(msi_plan* p, int layer, const std::vector<WaveEntry>& m
   }
   LAUNCH(p, MSI_K_PUBLISH, stage, launch_publish(inv, p->d_gen, stage));
   const uint64_t eb = p->d.extent_bytes;
-  for (const auto& m : misses) {
-    const char* src = static_cast<const char*>(p->d.host_windows) +
-                      p->off[(size_t)layer * p->d.n_experts + m.expert];
-    char* dst = static_cast<char*>(p->d.slot_pool) + (size_t)m.slot * eb;
-    CK(cudaMemcpyAsync(dst, src, eb, cudaMemcpyHostToDevice, stage));
+  auto src_of = [&](const WaveEntry& m) {
+    return static_cast<const char*>(p->d.host_windows) +
+           p->off[(size_t)layer * p->d.n_experts + m.expert];
+  };
+  auto dst_of = [&](const WaveEntry& m) {
+    return static_cast<char*>(p->d.slot_pool) + (size_t)m.slot * eb;
+  };
+  // one copy per run of extents that continue each other in both the host
+  // window and the slot pool (consecutive experts into consecutive slots):
+  // large copies reach the host link's rate, per-extent copies fall short
+  for (size_t i = 0; i < misses.size();) {
+    const char* src = src_of(misses[i]);
+    char* dst = dst_of(misses[i]);
+    uint64_t bytes = eb;
+    size_t j = i + 1;
+    while (j < misses.size() && src_of(misses[j]) == src + bytes && dst_of(misses[j]) == dst + bytes) {
+      bytes += eb;
+      ++j;
+    }
+    CK(cudaMemcpyAsync(dst, src, bytes, cudaMemcpyHostToDevice, stage));
+    i = j;
   }
   LAUNCH(p, MSI_K_PUBLISH, stage, launch_publish(pub, p->d_gen, stage));
   int ev;

@@ -148,3 +148,27 @@ def test_balanced_counters_after_streamed_calls():
     occupied = sum(1 for s in range(cfg.n_slots) if case.plan.slot_state(s) != N.MSI_SLOT_VACANT)
     assert occupied == c["stages"] - c["evicts"]
     case.close()
+
+
+def test_back_to_back_forwards_with_shared_expert_match_sequential():
+    """The shared expert of a resident forward runs on the plan's side stream
+    (forked after the forward's first kernel, joined before the combine).
+    Three forwards enqueued back to back with different inputs, no host sync
+    between them, equal the same forwards run one at a time, bit for bit."""
+    cfg = synth.config("qwen3next_4k", n_experts=64, tokens=2048, n_slots=64)
+    case = Case(cfg)
+    table, gens = case.stage_all()
+    xs = [bf16_tensor(synth.hidden(cfg, 0, 40 + i)) for i in range(3)]
+    seq = []
+    for x in xs:
+        out, _ = case.plan.forward(0, x, case.router[0], table, gens)
+        torch.cuda.synchronize()
+        seq.append(out.clone())
+    outs = [case.plan.forward(0, x, case.router[0], table, gens)[0] for x in xs]
+    torch.cuda.synchronize()
+    assert case.plan.status() == N.MSI_OK
+    for a, b in zip(seq, outs):
+        assert torch.equal(a.view(torch.int16), b.view(torch.int16))
+    toks = np.arange(0, 2048, 64)
+    compare_out(bf16_bits(outs[2])[toks], case.oracle_layer(synth.hidden(cfg, 0, 42), tokens=toks)["out"])
+    case.close()
