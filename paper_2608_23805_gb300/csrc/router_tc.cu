@@ -73,24 +73,51 @@ __global__ void split3_kernel(const float* __restrict__ w, long long n, __nv_bfl
   }
 }
 
-// Four independent warp-wide argmaxes interleaved (hides shuffle latency).
-__device__ __forceinline__ void warp_best4(float (&bv)[4], int (&bi)[4]) {
+// Selection order of the route event: logit descending, then expert id
+// ascending.  A logit maps to a 32-bit key with the same order (-0 counted as
+// +0), so a warp finds the best head of its lanes with one redux.sync max and
+// breaks a tie with one redux.sync min over the ids holding that key.
+__device__ __forceinline__ uint32_t logit_key(float v) {
+  uint32_t b = __float_as_uint(v);
+  if (b == 0x80000000u) b = 0u;
+  return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+}
+__device__ __forceinline__ float key_logit(uint32_t k) {
+  return __uint_as_float((k & 0x80000000u) ? (k & 0x7FFFFFFFu) : ~k);
+}
+
+// Sort one lane's N (key, id) pairs: key descending, id ascending.
+template <int N>
+__device__ __forceinline__ void sort_desc(uint32_t (&k)[N], int (&id)[N]) {
 #pragma unroll
-  for (int off = 16; off > 0; off >>= 1) {
-    float ov[4];
-    int oi[4];
+  for (int i = 1; i < N; ++i) {
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      ov[u] = __shfl_xor_sync(0xffffffffu, bv[u], off);
-      oi[u] = __shfl_xor_sync(0xffffffffu, bi[u], off);
+    for (int j = i; j > 0; --j) {
+      const bool sw = k[j] > k[j - 1] || (k[j] == k[j - 1] && id[j] < id[j - 1]);
+      const uint32_t tk = sw ? k[j - 1] : k[j];
+      const int ti = sw ? id[j - 1] : id[j];
+      k[j - 1] = sw ? k[j] : k[j - 1];
+      id[j - 1] = sw ? id[j] : id[j - 1];
+      k[j] = tk;
+      id[j] = ti;
     }
+  }
+}
+
+// One selection round over the lanes' sorted heads: returns the winning key
+// and id (same in every lane); the lane that held it drops its head.
+template <int N>
+__device__ __forceinline__ void take_best(uint32_t (&k)[N], int (&id)[N], uint32_t& bk, int& bi) {
+  bk = __reduce_max_sync(0xffffffffu, k[0]);
+  bi = __reduce_min_sync(0xffffffffu, k[0] == bk ? id[0] : 0x7fffffff);
+  if (id[0] == bi && k[0] == bk) {
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      if (ov[u] > bv[u] || (ov[u] == bv[u] && oi[u] < bi[u])) {
-        bv[u] = ov[u];
-        bi[u] = oi[u];
-      }
+    for (int i = 0; i + 1 < N; ++i) {
+      k[i] = k[i + 1];
+      id[i] = id[i + 1];
     }
+    k[N - 1] = 0u;  // below every logit's key
+    id[N - 1] = 0x7fffffff;
   }
 }
 
@@ -222,8 +249,8 @@ __global__ void __launch_bounds__(NTH, 1)
     const float* L = reinterpret_cast<const float*>(smem);
     const int kp = a.kp;  // candidates per chunk: min(k + 1, chunk)
     for (int q0 = warp * 16; q0 < warp * 16 + 16; q0 += 4) {
-      float v[4][4];
-      uint32_t removed[4] = {0, 0, 0, 0};
+      uint32_t kk[4][4];
+      int id[4][4];
       float my_v[4];
       int my_i[4];
 #pragma unroll
@@ -232,35 +259,22 @@ __global__ void __launch_bounds__(NTH, 1)
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
           const int e = lane + 32 * i;
-          v[u][i] = e < ch ? row[e] : -INFINITY;
+          kk[u][i] = e < ch ? logit_key(row[e]) : 0u;
+          id[u][i] = e < ch ? e : 0x7fffffff;
         }
+        sort_desc(kk[u], id[u]);
         my_v[u] = -INFINITY;
         my_i[u] = 0x7fffffff;
       }
       for (int rr = 0; rr < kp; ++rr) {
-        float bv[4];
-        int bi[4];
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
-          bv[u] = -INFINITY;
-          bi[u] = 0x7fffffff;
-#pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            const int e = lane + 32 * i;
-            if (e < ch && !((removed[u] >> i) & 1u) &&
-                (v[u][i] > bv[u] || (v[u][i] == bv[u] && e < bi[u]))) {
-              bv[u] = v[u][i];
-              bi[u] = e;
-            }
-          }
-        }
-        warp_best4(bv, bi);
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          if ((bi[u] & 31) == lane) removed[u] |= 1u << (bi[u] >> 5);
+          uint32_t bk;
+          int bi;
+          take_best(kk[u], id[u], bk, bi);
           if (rr == lane) {
-            my_v[u] = bv[u];
-            my_i[u] = c * ch + bi[u];  // global expert id
+            my_v[u] = key_logit(bk);
+            my_i[u] = c * ch + bi;  // global expert id
           }
         }
       }
@@ -300,7 +314,7 @@ __global__ void __launch_bounds__(256) router_merge_kernel(const RouterTcArgs a)
   __syncthreads();
   const int tw = blockIdx.x * 32 + warp * 4;  // this warp's first token
   {
-    float v[4][5];
+    uint32_t kk[4][5];
     int id[4][5];
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
@@ -311,11 +325,11 @@ __global__ void __launch_bounds__(256) router_merge_kernel(const RouterTcArgs a)
         const bool in = t < a.T && j < ncand;
         const int cid = in ? a.cand_i[(size_t)t * ncand + j] : -1;
         const bool real = cid >= 0 && cid < E;  // an aborted router leaves no valid candidate
-        v[u][i] = real ? a.cand_v[(size_t)t * ncand + j] : -INFINITY;
+        kk[u][i] = real ? logit_key(a.cand_v[(size_t)t * ncand + j]) : 0u;
         id[u][i] = real ? cid : 0x7fffffff;
       }
+      sort_desc(kk[u], id[u]);
     }
-    uint32_t removed[4] = {0, 0, 0, 0};
     float my_v[4], next_v[4];
     int my_i[4];
 #pragma unroll
@@ -326,33 +340,17 @@ __global__ void __launch_bounds__(256) router_merge_kernel(const RouterTcArgs a)
     }
     const int rounds = min(k + 1, E);
     for (int rr = 0; rr < rounds; ++rr) {
-      float bv[4];
-      int bi[4], bslot[4], mine[4];
 #pragma unroll
       for (int u = 0; u < 4; ++u) {
-        bv[u] = -INFINITY;
-        bi[u] = 0x7fffffff;
-        bslot[u] = -1;
-#pragma unroll
-        for (int i = 0; i < 5; ++i) {
-          if (!((removed[u] >> i) & 1u) &&
-              (v[u][i] > bv[u] || (v[u][i] == bv[u] && id[u][i] < bi[u]))) {
-            bv[u] = v[u][i];
-            bi[u] = id[u][i];
-            bslot[u] = i;
-          }
-        }
-        mine[u] = bi[u];
-      }
-      warp_best4(bv, bi);
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        if (bslot[u] >= 0 && mine[u] == bi[u]) removed[u] |= 1u << bslot[u];  // ids are unique
+        uint32_t bk;
+        int bi;
+        take_best(kk[u], id[u], bk, bi);
+        const float bv = bk == 0u ? -INFINITY : key_logit(bk);
         if (rr == lane) {
-          my_v[u] = bv[u];
-          my_i[u] = bi[u];
+          my_v[u] = bv;
+          my_i[u] = bi;
         }
-        if (rr == k) next_v[u] = bv[u];
+        if (rr == k) next_v[u] = bv;
       }
     }
 #pragma unroll
