@@ -279,3 +279,39 @@ def test_router_limits_and_chunks(E, k):
     np.testing.assert_allclose(g[ok], ref["gap_k"][ok], rtol=0, atol=2e-5)
     compare_out(bf16_bits(out), ref["out"], ~oracle.near_tie_tokens(ref["gap_k"]))
     case.close()
+
+
+@pytest.mark.parametrize("E", [64, 256])
+def test_exact_logit_ties_rank_lower_id_first(E):
+    """Duplicated (and amplified) router rows give exactly equal logits; the
+    route event must rank the lower expert id first (the oracle's order), the
+    pair adjacent with equal weights, within one 128-expert chunk (E = 64)
+    and across chunks through the candidate merge (E = 256)."""
+    cfg = synth.config("tiny", n_experts=E, n_slots=E, top_k=6, tokens=512, lru=False)
+    case = Case(cfg)
+    table, gens = case.stage_all()
+    w = case.router_np[0].copy()
+    pairs = [(3, 40), (10, 11), (0, 63)] if E == 64 else [(5, 133), (120, 200), (7, 8)]
+    for lo, hi in pairs:
+        w[lo] *= 4.0
+        w[hi] = w[lo]
+    case.router[0] = torch.from_numpy(w).cuda()
+    case.router_np[0] = w
+    x_bits = synth.hidden(cfg, 0, 21)
+    out, ev = case.plan.forward(0, bf16_tensor(x_bits), case.router[0], table, gens)
+    torch.cuda.synchronize()
+    assert case.plan.status() == N.MSI_OK
+    ids = ev.ids.cpu().numpy()
+    wts = ev.weights.cpu().numpy()
+    seen = 0
+    for t in range(cfg.tokens):
+        row = ids[t].tolist()
+        for lo, hi in pairs:
+            if hi in row:
+                seen += 1
+                j = row.index(hi)
+                assert j > 0 and row[j - 1] == lo, f"token {t}: {row}"
+                assert wts[t, j] == wts[t, j - 1]
+    assert seen > 50  # the amplified pairs are routed often
+    compare_routes(ids, wts, oracle.router(x_bits, w, cfg.top_k))
+    case.close()
