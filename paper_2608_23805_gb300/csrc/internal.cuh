@@ -114,9 +114,9 @@ struct ScatterArgs {
   int* perm;          // [T*k]
   int* inv;           // [T*k]
   int* offsets;       // [E+1]
-  // block 0 also, for a resident call (table entries in the kernel's
-  // TableParams), re-checks the named slots' generations and builds the GEMM
-  // groups
+  // an extra last block writes the offsets and, for a resident call (table
+  // entries in the kernel's TableParams), re-checks the named slots'
+  // generations and builds the GEMM groups
   const GenWord* genwords;
   Group* groups;
   int* total_mtiles;   // [0]: 128-row tiles, [1]: 256-row pair tiles

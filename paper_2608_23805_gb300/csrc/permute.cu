@@ -77,7 +77,7 @@ __device__ __forceinline__ int scan4(const int (&v)[4], int* wsum, int* total) {
   return base;
 }
 
-// Block 0 of the scatter, resident call: the generation re-check of every
+// Setup block of the scatter, resident call: the generation re-check of every
 // routed expert's slot (fail closed) and the GEMM groups with their 128- and
 // 256-row tile prefixes.
 __device__ void scatter_setup(const ScatterArgs& a, const TableParams& tp, const int* offs) {
@@ -169,9 +169,12 @@ __global__ void __launch_bounds__(kScatterWarps * 32) scatter_kernel(const Scatt
   }
   if (tid == kScatterWarps * 32 - 1 && a.E == kMaxExperts) offs[kMaxExperts] = base;
   __syncthreads();
-  if (blockIdx.x == 0) {
+  // the last block (one past the scatter blocks) writes the offsets and runs
+  // the resident setup, in parallel with the scatter
+  if (blockIdx.x == gridDim.x - 1) {
     for (int e = tid; e <= a.E; e += blockDim.x) a.offsets[e] = offs[e];
     scatter_setup(a, tp, offs);
+    return;
   }
 
   const int b = blockIdx.x * kScatterWarps + warp;
@@ -381,7 +384,7 @@ cudaError_t launch_colscan(const ScanArgs& a, cudaStream_t s) {
 }
 
 cudaError_t launch_scatter(const ScatterArgs& a, const TableParams& tp, cudaStream_t s) {
-  const int grid = (a.nb + kScatterWarps - 1) / kScatterWarps;
+  const int grid = (a.nb + kScatterWarps - 1) / kScatterWarps + 1;  // + the setup block
   scatter_kernel<<<grid, kScatterWarps * 32, 0, s>>>(a, tp);
   return cudaGetLastError();
 }
