@@ -608,11 +608,17 @@ GemmArgs down_args(msi_plan* p, FwdCtx& f, const Group* groups, int ng, const in
 // below that their coarser row padding and tile rounds lose (measured at
 // ~680 rows per group: 90 us against 80 us).
 constexpr long long kPairMinRows = 1024;
-bool pair_tiles(const FwdCtx& f, long long rows, int groups) {
-  return !(f.flags & MSI_FWD_SINGLE_CTA) && groups > 0 && rows >= kPairMinRows * groups;
+// The down projection (K = 512, output-stream heavy) gains from pair tiles
+// already at ~640 rows per group (measured 4 %), the gate-up does not.
+constexpr long long kPairMinRowsDown = 512;
+bool pair_tiles(const FwdCtx& f, long long rows, int groups, long long min_rows = kPairMinRows) {
+  return !(f.flags & MSI_FWD_SINGLE_CTA) && groups > 0 && rows >= min_rows * groups;
 }
 
-msi_status routed_ffn(msi_plan* p, FwdCtx& f, int ng, int grid1, int grid2, bool pair) {
+msi_status routed_ffn(msi_plan* p, FwdCtx& f, int ng, int grid1, int grid2, long long rows) {
+  const bool bf16 = p->d.wdtype == MSI_W_BF16;
+  const bool pair_up = bf16 && pair_tiles(f, rows, ng);
+  const bool pair_down = bf16 && pair_tiles(f, rows, ng, kPairMinRowsDown);
   const auto& d = p->d;
   const Group* groups = at<Group>(f.ws, f.L.groups);
   const int* total = at<int>(f.ws, f.L.total);
@@ -637,15 +643,16 @@ msi_status routed_ffn(msi_plan* p, FwdCtx& f, int ng, int grid1, int grid2, bool
     LAUNCH(p, MSI_K_DOWN, f.cs, launch_gemm(kDownQ4, f.tm_h, f.tm_h, g2, grid2, f.cs));
     return MSI_OK;
   }
-  if (pair) {
+  if (pair_up)
     LAUNCH(p, MSI_K_GATEUP, f.cs,
            launch_gemm_pair(kGateUpGather, p->tm_w13, p->tm_w13, g1, std::max(1, grid1 / 2), f.cs));
+  else
+    LAUNCH(p, MSI_K_GATEUP, f.cs, launch_gemm(kGateUpGather, p->tm_w13, p->tm_w13, g1, grid1, f.cs));
+  if (pair_down)
     LAUNCH(p, MSI_K_DOWN, f.cs,
            launch_gemm_pair(kDown, f.tm_h, p->tm_w2, g2, std::max(1, grid2 / 2), f.cs));
-    return MSI_OK;
-  }
-  LAUNCH(p, MSI_K_GATEUP, f.cs, launch_gemm(kGateUpGather, p->tm_w13, p->tm_w13, g1, grid1, f.cs));
-  LAUNCH(p, MSI_K_DOWN, f.cs, launch_gemm(kDown, f.tm_h, p->tm_w2, g2, grid2, f.cs));
+  else
+    LAUNCH(p, MSI_K_DOWN, f.cs, launch_gemm(kDown, f.tm_h, p->tm_w2, g2, grid2, f.cs));
   return MSI_OK;
 }
 
@@ -971,8 +978,7 @@ msi_status msi_moe_forward(msi_plan* p, int layer, const void* x, int T, const f
     const long long mt_max = ((long long)T * d.top_k + kBM - 1) / kBM + E;
     const int g1 = (int)std::min<long long>(p->sms, mt_max * (d.inter / 128));
     const int g2 = (int)std::min<long long>(p->sms, mt_max * (d.hidden / kBN));
-    st = routed_ffn(p, f, E, g1, g2,
-                    d.wdtype == MSI_W_BF16 && pair_tiles(f, (long long)T * d.top_k, E));
+    st = routed_ffn(p, f, E, g1, g2, (long long)T * d.top_k);
     if (st != MSI_OK) return st;
     st = consumer_record(p, used, f.cs);
     if (st != MSI_OK) return st;
@@ -1137,8 +1143,7 @@ msi_status msi_moe_forward_streamed(msi_plan* p, int layer, const void* x, int T
     LAUNCH(p, MSI_K_SETUP, f.cs, launch_setup_wave(sa, wp, f.cs));
     const int g1 = std::max(1, std::min(p->sms, mtiles * (d.inter / 128)));
     const int g2 = std::max(1, std::min(p->sms, mtiles * (d.hidden / kBN)));
-    st = routed_ffn(p, f, wp.n, g1, g2,
-                    d.wdtype == MSI_W_BF16 && pair_tiles(f, wave_rows, wp.n));
+    st = routed_ffn(p, f, wp.n, g1, g2, wave_rows);
     if (st != MSI_OK) return st;
     st = consumer_record(p, used, f.cs);
     if (st != MSI_OK) return st;

@@ -69,11 +69,13 @@ def test_pair_qwen_shape_sampled_tokens():
     case.close()
 
 
-def test_pair_streamed_waves_full_oracle():
-    """Streamed LRU waves large enough for pair tiles (32 experts, 16 slots,
-    waves of 8, ~2,048 rows per expert): matches the oracle, with pair and
-    single-CTA tiles."""
-    cfg = synth.config("tiny", hidden=512, inter=256, n_experts=32, top_k=8, tokens=8192,
+@pytest.mark.parametrize("tokens,top_k", [(8192, 8), (4096, 5)])
+def test_pair_streamed_waves_full_oracle(tokens, top_k):
+    """Streamed LRU waves (32 experts, 16 slots, waves of 8): ~2,048 rows per
+    expert (pair tiles for both projections) and ~640 rows per expert (pair
+    tiles for the down projection only); matches the oracle, with the default
+    tiles and with single-CTA tiles."""
+    cfg = synth.config("tiny", hidden=512, inter=256, n_experts=32, top_k=top_k, tokens=tokens,
                        n_slots=16, has_shared=False)
     case = Case(cfg)
     x_bits = synth.hidden(cfg, 0, 13)
