@@ -68,23 +68,27 @@ struct Cfg {
   // bf16 modes stage each epilogue warp's rows in shared memory (4 KB per
   // warp) for row-coalesced stores; the q4 raw ring leaves no room for it
   static constexpr bool kStagedEpi = !kQ4;
+  // the groups' 128-row tile prefix and slot, read once per launch so that
+  // tile lookups (every role, every tile) stay in shared memory
+  static constexpr int kGroupTableBytes = (2 * kMaxExperts + 2) * 4;
   static constexpr int kSmem = 1024 + kStg * (kABytes + kBBytes) + kRawBytes + 256 +
-                               (kStagedEpi ? kEpiWarps * 4096 : 0);
+                               (kStagedEpi ? kEpiWarps * 4096 : 0) + kGroupTableBytes;
 };
 
 struct TileCoord {
   int g, m, n;
 };
 
-__device__ __forceinline__ TileCoord decode_tile(const GemmArgs& a, int t) {
+// Tile t -> (group, 128-row tile, column tile) from the shared-memory table
+// of the groups' tile prefix (s_mt[num_groups] = total tiles).
+__device__ __forceinline__ TileCoord decode_tile(const GemmArgs& a, const int* s_mt, int t) {
   int lo = 0, hi = a.num_groups - 1;
   while (lo < hi) {
     const int mid = (lo + hi + 1) >> 1;
-    if (__ldg(&a.groups[mid].mt_begin) * a.nt <= t) lo = mid; else hi = mid - 1;
+    if (s_mt[mid] * a.nt <= t) lo = mid; else hi = mid - 1;
   }
-  const int cnt = __ldg(&a.groups[lo].row_count);
-  const int mt = (cnt + kBM - 1) / kBM;
-  const int local = t - __ldg(&a.groups[lo].mt_begin) * a.nt;
+  const int mt = s_mt[lo + 1] - s_mt[lo];
+  const int local = t - s_mt[lo] * a.nt;
   TileCoord c;
   c.g = lo;
   c.n = local / mt;
@@ -148,6 +152,10 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   uint8_t* epi_stage = reinterpret_cast<uint8_t*>(full) + 256;  // kEpiWarps x 4 KB (bf16 modes)
+  // group table after the epilogue staging (bf16 modes) or the barriers (q4)
+  int* s_mt = reinterpret_cast<int*>(reinterpret_cast<uint8_t*>(full) + 256 +
+                                     (C::kStagedEpi ? kEpiWarps * 4096 : 0));  // [num_groups + 1]
+  int* s_slot = s_mt + kMaxExperts + 1;                                       // [num_groups]
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -173,11 +181,16 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
     if (C::kTmaB) tma_prefetch(&tmB);
     if (C::kTmaA) tma_prefetch(&tmA);
   }
+  for (int g = threadIdx.x; g < a.num_groups; g += blockDim.x) {
+    s_mt[g] = __ldg(&a.groups[g].mt_begin);
+    s_slot[g] = __ldg(&a.groups[g].slot);
+  }
+  if (threadIdx.x == 0) s_mt[a.num_groups] = __ldg(a.total_mtiles);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  const int total = __ldg(a.total_mtiles) * a.nt;
+  const int total = s_mt[a.num_groups] * a.nt;
   const long long lim = a.wait_limit;
 
   if (warp == 5) {
@@ -185,9 +198,9 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
     if (lane == 0 && C::kTmaAny) {
       uint32_t it = 0;
       for (int t = blockIdx.x; t < total; t += gridDim.x) {
-        const TileCoord tc = decode_tile(a, t);
+        const TileCoord tc = decode_tile(a, s_mt, t);
         const Group* G = &a.groups[tc.g];
-        const int brow = __ldg(&G->slot) * a.b_rows_per_slot + a.b_row_off;
+        const int brow = s_slot[tc.g] * a.b_rows_per_slot + a.b_row_off;
         const int arow = __ldg(&G->row_begin) + tc.m * kBM;
         bool ok = true;
         for (int kb = 0; kb < a.kblocks; ++kb, ++it) {
@@ -260,7 +273,7 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
     uint32_t jt = 0;
     const int r = warp * 32 + lane;
     for (int t = blockIdx.x; t < total; t += gridDim.x, ++jt) {
-      const TileCoord tc = decode_tile(a, t);
+      const TileCoord tc = decode_tile(a, s_mt, t);
       const Group* G = &a.groups[tc.g];
       const int cnt = __ldg(&G->row_count);
       const bool valid = tc.m * kBM + r < cnt;
@@ -290,7 +303,7 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
     uint32_t it = 0;
     bool ok = true;
     for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
-      const TileCoord tc = decode_tile(a, t);
+      const TileCoord tc = decode_tile(a, s_mt, t);
       const Group* G = &a.groups[tc.g];
       const int cnt = __ldg(&G->row_count);
       const int rb = __ldg(&G->row_begin);
@@ -328,30 +341,39 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
     const uint32_t my_tiles =
         (uint32_t)blockIdx.x < (uint32_t)total ? (total - 1 - blockIdx.x) / gridDim.x + 1 : 0;
     const uint32_t nstages = my_tiles * a.kblocks;
-    // prefetch cursor: (tile, kb) of the next raw stage, with this row's sources
-    uint32_t jp = 0;
-    int cur_tile = -1;
+    // tile lookups from the shared-memory group table: a search in global
+    // memory here would stall this row's whole pipeline once per tile
     const uint8_t* code_row = nullptr;
     const uint8_t* scale_row = nullptr;
-    auto issue = [&](uint32_t j) {
-      const int tile_idx = (int)(j / a.kblocks);
-      const int kb = (int)(j % a.kblocks);
-      if (tile_idx != cur_tile) {
-        cur_tile = tile_idx;
-        const TileCoord tc = decode_tile(a, blockIdx.x + tile_idx * gridDim.x);
-        const uint8_t* base =
-            a.q4_pool + (unsigned long long)__ldg(&a.groups[tc.g].slot) * a.q4_extent;
-        int row;
-        if (C::kGateUp) row = d < 128 ? tc.n * 128 + d : a.up_off + tc.n * 128 + (d - 128);
-        else row = tc.n * kBN + d;
-        code_row = base + a.q4_code_off + (size_t)row * a.q4_code_ld;
-        scale_row = base + a.q4_scale_off + (size_t)row * a.q4_scale_ld;
+    auto rows_of = [&](int t) {  // this thread's code and scale rows of tile t
+      int lo = 0, hi = a.num_groups - 1;
+      while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (s_mt[mid] * a.nt <= t) lo = mid; else hi = mid - 1;
       }
+      const int mt = s_mt[lo + 1] - s_mt[lo];
+      const int n = (t - s_mt[lo] * a.nt) / mt;
+      const uint8_t* base = a.q4_pool + (unsigned long long)s_slot[lo] * a.q4_extent;
+      int row;
+      if (C::kGateUp) row = d < 128 ? n * 128 + d : a.up_off + n * 128 + (d - 128);
+      else row = n * kBN + d;
+      code_row = base + a.q4_code_off + (size_t)row * a.q4_code_ld;
+      scale_row = base + a.q4_scale_off + (size_t)row * a.q4_scale_ld;
+    };
+    // prefetch cursor (tile ordinal, k block) of the next raw stage
+    uint32_t jp = 0, p_tile = 0;
+    int p_kb = 0;
+    if (my_tiles > 0) rows_of(blockIdx.x);
+    auto issue = [&](uint32_t j) {
       const int r = j % C::kRaw;
       uint8_t* dst = raw_codes + (r * kBN + d) * kRawRowBytes;
-      cp_async16(dst, code_row + kb * 32, 16u);
-      cp_async16(dst + 16, code_row + kb * 32 + 16, 16u);
-      cp_async4(&raw_scales[r * kBN + d], scale_row + kb * 4);
+      cp_async16(dst, code_row + p_kb * 32, 16u);
+      cp_async16(dst + 16, code_row + p_kb * 32 + 16, 16u);
+      cp_async4(&raw_scales[r * kBN + d], scale_row + p_kb * 4);
+      if (++p_kb == a.kblocks) {
+        p_kb = 0;
+        if (++p_tile < my_tiles) rows_of(blockIdx.x + p_tile * gridDim.x);
+      }
     };
     for (int i = 0; i < C::kRaw - 1; ++i, ++jp) {
       if (jp < nstages) issue(jp);

@@ -64,22 +64,25 @@ struct PCfg {
   static constexpr uint32_t kTx = kPB + (kGather ? 0 : kPA);
   // own producer (expect_tx) + own gather threads (one arrival each as their copies land)
   static constexpr int kFullLocal = 1 + (kGather ? kPGatherWarps * 32 : 0);
-  static constexpr int kSmem = 1024 + kPStages * (kPA + kPB) + 256 + kPEpiWarps * 4096;
+  // + the groups' 256-row tile prefix and slot (shared-memory tile lookups)
+  static constexpr int kSmem = 1024 + kPStages * (kPA + kPB) + 256 + kPEpiWarps * 4096 +
+                               (2 * kMaxExperts + 2) * 4;
 };
 
 struct PairTile {
   int g, m2, n;
 };
 
-__device__ __forceinline__ PairTile decode_pair(const GemmArgs& a, int t) {
+// Pair tile t -> (group, 256-row tile, column tile) from the shared-memory
+// table of the groups' pair-tile prefix (s_pt[num_groups] = total).
+__device__ __forceinline__ PairTile decode_pair(const GemmArgs& a, const int* s_pt, int t) {
   int lo = 0, hi = a.num_groups - 1;
   while (lo < hi) {
     const int mid = (lo + hi + 1) >> 1;
-    if (__ldg(&a.groups[mid].pt_begin) * a.nt <= t) lo = mid; else hi = mid - 1;
+    if (s_pt[mid] * a.nt <= t) lo = mid; else hi = mid - 1;
   }
-  const int cnt = __ldg(&a.groups[lo].row_count);
-  const int mt2 = (cnt + kPairRows - 1) / kPairRows;
-  const int local = t - __ldg(&a.groups[lo].pt_begin) * a.nt;
+  const int mt2 = s_pt[lo + 1] - s_pt[lo];
+  const int local = t - s_pt[lo] * a.nt;
   PairTile c;
   c.g = lo;
   c.n = local / mt2;
@@ -109,6 +112,8 @@ __global__ void __launch_bounds__(PCfg<MODE>::kThreads, 1)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   uint8_t* epi_stage = reinterpret_cast<uint8_t*>(full) + 256;  // 4 KB per epilogue warp
+  int* s_pt = reinterpret_cast<int*>(epi_stage + kPEpiWarps * 4096);  // [num_groups + 1]
+  int* s_slot = s_pt + kMaxExperts + 1;                               // [num_groups]
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -136,11 +141,16 @@ __global__ void __launch_bounds__(PCfg<MODE>::kThreads, 1)
     tma_prefetch(&tmB);
     if (!C::kGather) tma_prefetch(&tmA);
   }
+  for (int g = threadIdx.x; g < a.num_groups; g += blockDim.x) {
+    s_pt[g] = __ldg(&a.groups[g].pt_begin);
+    s_slot[g] = __ldg(&a.groups[g].slot);
+  }
+  if (threadIdx.x == 0) s_pt[a.num_groups] = __ldg(a.total_mtiles + 1);
   tc_fence_before();
   cluster_sync_all();  // both CTAs' barriers initialised before any cross-CTA arrival
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  const int total = __ldg(a.total_mtiles + 1) * a.nt;
+  const int total = s_pt[a.num_groups] * a.nt;
   const int pair = blockIdx.x >> 1;
   const int npairs = gridDim.x >> 1;
   const long long lim = a.wait_limit;
@@ -150,9 +160,9 @@ __global__ void __launch_bounds__(PCfg<MODE>::kThreads, 1)
     if (lane == 0) {
       uint32_t it = 0;
       for (int t = pair; t < total; t += npairs) {
-        const PairTile tc = decode_pair(a, t);
+        const PairTile tc = decode_pair(a, s_pt, t);
         const Group* G = &a.groups[tc.g];
-        const int brow0 = __ldg(&G->slot) * a.b_rows_per_slot + a.b_row_off;
+        const int brow0 = s_slot[tc.g] * a.b_rows_per_slot + a.b_row_off;
         // gate-up: the even CTA holds 128 gate rows, the odd CTA the matching up rows
         const int brow = C::kGateUp ? brow0 + (rank ? a.up_off : 0) + tc.n * 128
                                     : brow0 + tc.n * kBN + (int)rank * 128;
@@ -235,7 +245,7 @@ __global__ void __launch_bounds__(PCfg<MODE>::kThreads, 1)
     const uint32_t lead_tempty[2] = {mapa_shared(smem_u32(&tempty[0]), 0),
                                      mapa_shared(smem_u32(&tempty[1]), 0)};
     for (int t = pair; t < total; t += npairs, ++jt) {
-      const PairTile tc = decode_pair(a, t);
+      const PairTile tc = decode_pair(a, s_pt, t);
       const Group* G = &a.groups[tc.g];
       const int cnt = __ldg(&G->row_count);
       const uint32_t acc = jt & 1, aph = (jt >> 1) & 1;
@@ -258,7 +268,7 @@ __global__ void __launch_bounds__(PCfg<MODE>::kThreads, 1)
     uint32_t it = 0;
     bool ok = true;
     for (int t = pair; t < total && ok; t += npairs) {
-      const PairTile tc = decode_pair(a, t);
+      const PairTile tc = decode_pair(a, s_pt, t);
       const Group* G = &a.groups[tc.g];
       const int cnt = __ldg(&G->row_count);
       const int rb = __ldg(&G->row_begin);
