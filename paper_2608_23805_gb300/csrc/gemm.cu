@@ -197,11 +197,15 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
     // ------------------------------------------------------------- TMA producer
     if (lane == 0 && C::kTmaAny) {
       uint32_t it = 0;
+      // the next tile's first A row is loaded one tile ahead (its latency
+      // hides behind this tile's stages instead of stalling the ring)
+      int rb_next = blockIdx.x < total ? __ldg(&a.groups[decode_tile(a, s_mt, blockIdx.x).g].row_begin) : 0;
       for (int t = blockIdx.x; t < total; t += gridDim.x) {
         const TileCoord tc = decode_tile(a, s_mt, t);
-        const Group* G = &a.groups[tc.g];
         const int brow = s_slot[tc.g] * a.b_rows_per_slot + a.b_row_off;
-        const int arow = __ldg(&G->row_begin) + tc.m * kBM;
+        const int arow = rb_next + tc.m * kBM;
+        if (t + (int)gridDim.x < total)
+          rb_next = __ldg(&a.groups[decode_tile(a, s_mt, t + gridDim.x).g].row_begin);
         bool ok = true;
         for (int kb = 0; kb < a.kblocks; ++kb, ++it) {
           const int s = it % C::kStg;
@@ -302,19 +306,31 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
     const int r0 = gt >> 3;               // rows r0 + 16 i
     uint32_t it = 0;
     bool ok = true;
-    for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+    // permuted-row entries (t*k + j, or -1 past the expert's segment) of this
+    // thread's eight rows, loaded one tile ahead so that the next tile's first
+    // copies do not wait on the group and permutation loads
+    auto tile_rows = [&](int t, int (&pr)[8]) {
       const TileCoord tc = decode_tile(a, s_mt, t);
       const Group* G = &a.groups[tc.g];
       const int cnt = __ldg(&G->row_count);
       const int rb = __ldg(&G->row_begin);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const int rr = tc.m * kBM + r0 + 16 * i;
+        pr[i] = rr < cnt ? __ldg(&a.perm[rb + rr]) : -1;
+      }
+    };
+    int pr[8], pr_next[8];
+    if (blockIdx.x < total) tile_rows(blockIdx.x, pr);
+    for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+      const bool has_next = t + (int)gridDim.x < total;
+      if (has_next) tile_rows(t + gridDim.x, pr_next);
       const __nv_bfloat16* src[8];
       uint32_t nbytes[8];
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
-        const int rr = tc.m * kBM + r0 + 16 * i;
-        if (rr < cnt) {
-          const int tok = __ldg(&a.perm[rb + rr]) / a.top_k;
-          src[i] = a.x + (size_t)tok * a.x_ld + chunk * 8;
+        if (pr[i] >= 0) {
+          src[i] = a.x + (size_t)(pr[i] / a.top_k) * a.x_ld + chunk * 8;
           nbytes[i] = 16;
         } else {
           src[i] = a.x;
@@ -332,6 +348,10 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
           cp_async16(dstA + rr * 128 + ((chunk ^ (rr & 7)) << 4), src[i] + kb * kBK, nbytes[i]);
         }
         cp_async_arrive_noinc(&full[s]);  // arrives when this thread's copies land
+      }
+      if (has_next) {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) pr[i] = pr_next[i];
       }
     }
     cp_async_wait<0>();
