@@ -159,14 +159,17 @@ __global__ void __launch_bounds__(PCfg<MODE>::kThreads, 1)
     // ------------------------------------------------------------- TMA producer
     if (lane == 0) {
       uint32_t it = 0;
+      // the next tile's first A row is loaded one tile ahead
+      int rb_next = pair < total ? __ldg(&a.groups[decode_pair(a, s_pt, pair).g].row_begin) : 0;
       for (int t = pair; t < total; t += npairs) {
         const PairTile tc = decode_pair(a, s_pt, t);
-        const Group* G = &a.groups[tc.g];
+        const int rb = rb_next;
+        if (t + npairs < total) rb_next = __ldg(&a.groups[decode_pair(a, s_pt, t + npairs).g].row_begin);
         const int brow0 = s_slot[tc.g] * a.b_rows_per_slot + a.b_row_off;
         // gate-up: the even CTA holds 128 gate rows, the odd CTA the matching up rows
         const int brow = C::kGateUp ? brow0 + (rank ? a.up_off : 0) + tc.n * 128
                                     : brow0 + tc.n * kBN + (int)rank * 128;
-        const int arow = __ldg(&G->row_begin) + tc.m2 * kPairRows + (int)rank * kBM;
+        const int arow = rb + tc.m2 * kPairRows + (int)rank * kBM;
         bool ok = true;
         for (int kb = 0; kb < a.kblocks; ++kb, ++it) {
           const int s = it % kPStages;
@@ -267,19 +270,29 @@ __global__ void __launch_bounds__(PCfg<MODE>::kThreads, 1)
     const int r0 = gt >> 3;               // rows r0 + 16 i of this CTA's 128
     uint32_t it = 0;
     bool ok = true;
-    for (int t = pair; t < total && ok; t += npairs) {
+    // permuted-row entries of this thread's eight rows, one tile ahead
+    auto tile_rows = [&](int t, int (&pr)[8]) {
       const PairTile tc = decode_pair(a, s_pt, t);
       const Group* G = &a.groups[tc.g];
       const int cnt = __ldg(&G->row_count);
       const int rb = __ldg(&G->row_begin);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const int rr = tc.m2 * kPairRows + (int)rank * kBM + r0 + 16 * i;
+        pr[i] = rr < cnt ? __ldg(&a.perm[rb + rr]) : -1;
+      }
+    };
+    int pr[8], pr_next[8];
+    if (pair < total) tile_rows(pair, pr);
+    for (int t = pair; t < total && ok; t += npairs) {
+      const bool has_next = t + npairs < total;
+      if (has_next) tile_rows(t + npairs, pr_next);
       const __nv_bfloat16* src[8];
       uint32_t nbytes[8];
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
-        const int rr = tc.m2 * kPairRows + (int)rank * kBM + r0 + 16 * i;
-        if (rr < cnt) {
-          const int tok = __ldg(&a.perm[rb + rr]) / a.top_k;
-          src[i] = a.x + (size_t)tok * a.x_ld + chunk * 8;
+        if (pr[i] >= 0) {
+          src[i] = a.x + (size_t)(pr[i] / a.top_k) * a.x_ld + chunk * 8;
           nbytes[i] = 16;
         } else {
           src[i] = a.x;
@@ -297,6 +310,10 @@ __global__ void __launch_bounds__(PCfg<MODE>::kThreads, 1)
           cp_async16(dstA + rr * 128 + ((chunk ^ (rr & 7)) << 4), src[i] + kb * kBK, nbytes[i]);
         }
         cp_async_arrive_noinc(&full[s]);  // arrives when this thread's copies land
+      }
+      if (has_next) {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) pr[i] = pr_next[i];
       }
     }
     cp_async_wait<0>();
