@@ -81,7 +81,9 @@ enum {
                                       (alone or inside a bundle) fails with MSI_ERR_SOURCE */
   MSI_FAULT_STALE_COMPLETION = 2,  /* the object's next publication carries the previous
                                       generation (a late stale completion) */
-  MSI_FAULT_WRONG_OBJECT = 3       /* the object's next publication names another object */
+  MSI_FAULT_WRONG_OBJECT = 3,      /* the object's next publication names another object */
+  MSI_FAULT_IO_ERROR = 4           /* with a source attached: the object's next read completes
+                                      with an I/O error (EIO); its bundle is not published */
 };
 
 /* Forward flags. */
@@ -256,6 +258,73 @@ msi_status msi_fault_inject(msi_plan* plan, int kind, int layer, int expert);
 
 /* Host-side consumer tickets: a caller that reads slots outside a forward
  * holds the slot while reading.  Staging into a held slot waits, bounded. */
+/* ---------------------------------------------------------------------------
+ * Bounded source service (paper, Sec. "Bounded Source Service"; window
+ * lifecycle Free -> Reading -> HostReady -> Copying -> Free, Sec. "Separate
+ * Window and GPU-Slot Lifecycles").  Expert extents are read from a file into
+ * a fixed set of aligned host windows: at most n_windows reads are in flight
+ * and the streamed weights occupy at most n_windows * window_bytes of host
+ * memory (the paper's M_source bound).  With direct = 1 the file is opened
+ * with O_DIRECT and each extent is read by a covering read (the range rounded
+ * out to `align`), so no copy of the payload accumulates in the page cache;
+ * direct = 0 reads through the page cache.  A read is rejected, and nothing
+ * of it is copied or published, on an I/O error, a short read (fewer bytes
+ * than cover the extent), an extent past the end of the file, or a
+ * completion that does not match its request (object, epoch, generation).
+ * ------------------------------------------------------------------------- */
+#define MSI_MAX_WINDOWS 64
+
+typedef struct msi_source msi_source; /* opaque, owned by the library */
+
+typedef struct {
+  const char* path;      /* file holding the extents (read-only) */
+  int direct;            /* 1: O_DIRECT covering reads; 0: buffered reads */
+  uint32_t align;        /* covering-read alignment, a power of two; 0 means 4096 */
+  int n_windows;         /* fixed window count = in-flight read limit, 1..MSI_MAX_WINDOWS */
+  void* windows;         /* caller-owned host memory, n_windows * window_bytes; pinned for
+                            asynchronous H2D copies; with direct = 1 aligned to `align` */
+  uint64_t window_bytes; /* W; >= an extent's covering read (extent + 2 * align rounded
+                            up to align for direct reads); with direct = 1 a multiple of align */
+} msi_source_desc;
+
+typedef struct {
+  uint64_t reads;          /* completed reads */
+  uint64_t rejected;       /* reads or submissions rejected */
+  uint64_t logical_bytes;  /* extent bytes of accepted reads */
+  uint64_t physical_bytes; /* covering-read bytes of accepted reads */
+  uint64_t padding_bytes;  /* physical - logical */
+  double read_seconds;     /* summed completion latency of completed reads */
+  int max_in_flight;       /* peak reads in flight */
+} msi_source_stats;
+
+/* Open: the file is opened (O_RDONLY, plus O_DIRECT when direct = 1) and one
+ * reader thread is started per window.  Errors: MSI_ERR_INVALID_ARG (null
+ * pointers, alignment, sizes), MSI_ERR_UNSUPPORTED (the file system refuses
+ * O_DIRECT), MSI_ERR_SOURCE (the file cannot be opened).  Close waits for
+ * every read in flight and every window's copy. */
+msi_status msi_source_open(const msi_source_desc* desc, msi_source** out);
+msi_status msi_source_close(msi_source* src);
+msi_status msi_source_stats_read(msi_source* src, msi_source_stats* out);
+
+/* Synchronous read of one extent [file_off, file_off + bytes) into a free
+ * window: on MSI_OK *data points at the extent's first byte inside window
+ * *window, which stays HostReady (reserved) until msi_source_release.
+ * MSI_ERR_SOURCE on a rejected read (nothing is left reserved). */
+msi_status msi_source_read(msi_source* src, uint64_t file_off, uint64_t bytes, const void** data,
+                           int* window);
+msi_status msi_source_release(msi_source* src, int window);
+
+/* Attach a source to a plan: from then on msi_slot_stage and the LRU waves of
+ * msi_moe_forward_streamed read each missing extent (layer l, expert e) from
+ * the file at file_off[l * n_experts + e] (extent_bytes long) through the
+ * source's windows instead of the plan's host windows, submitting up to
+ * n_windows reads ahead of the H2D copies.  A rejected read fails the call
+ * with MSI_ERR_SOURCE: the failing bundle (the wave, and every later wave of
+ * the call) is neither copied nor published, its slots are left Vacant, and
+ * no output row of the call is written.  src = NULL detaches.  The source
+ * must outlive the plan or be detached first.  file_off is copied. */
+msi_status msi_plan_set_source(msi_plan* plan, msi_source* src, const uint64_t* file_off);
+
 msi_status msi_consumer_hold(msi_plan* plan, int slot);
 msi_status msi_consumer_release(msi_plan* plan, int slot);
 

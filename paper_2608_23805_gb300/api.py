@@ -100,6 +100,16 @@ class Plan:
     def inject(self, kind: int, layer: int, expert: int):
         N.check(N.lib().msi_fault_inject(self.h, kind, layer, expert), "msi_fault_inject")
 
+    def set_source(self, src: "Source | None", file_off=None):
+        """Stage missing extents from `src` (file offsets [L*E]); None detaches."""
+        if src is None:
+            N.check(N.lib().msi_plan_set_source(self.h, None, None), "msi_plan_set_source")
+            self._src = None
+            return
+        off = np.ascontiguousarray(file_off, dtype=np.uint64)
+        N.check(N.lib().msi_plan_set_source(self.h, src.h, off.ctypes.data), "msi_plan_set_source")
+        self._src = src  # keep the source alive while attached
+
     def hold(self, slot: int):
         N.check(N.lib().msi_consumer_hold(self.h, slot), "msi_consumer_hold")
 
@@ -194,5 +204,61 @@ class Plan:
         try:
             if getattr(self, "h", None) is not None and self.h.value:
                 N.lib().msi_plan_destroy(self.h)
+        except Exception:
+            pass
+
+
+class Source:
+    """Bounded source service: extents read from `path` into `n_windows`
+    fixed, aligned host windows (O_DIRECT covering reads when direct=True).
+    The windows are pinned (page-locked) host memory when CUDA is available,
+    so that the H2D copies out of them are asynchronous; otherwise aligned
+    ordinary host memory (synchronous reads only)."""
+
+    def __init__(self, path: str, window_bytes: int, n_windows: int = 8, direct: bool = True,
+                 align: int = 4096):
+        wb = (int(window_bytes) + align - 1) // align * align
+        nbytes = wb * n_windows + align
+        if torch.cuda.is_available():
+            self._buf = torch.empty(nbytes, dtype=torch.uint8, pin_memory=True)
+            base = self._buf.data_ptr()
+        else:
+            self._buf = np.empty(nbytes, dtype=np.uint8)
+            base = self._buf.ctypes.data
+        self._off = (-base) % align
+        self.window_bytes = wb
+        self.n_windows = n_windows
+        self.direct = direct
+        self._path = path.encode()
+        d = N.msi_source_desc(self._path, 1 if direct else 0, align, n_windows,
+                              base + self._off, wb)
+        self.h = ctypes.c_void_p()
+        N.check(N.lib().msi_source_open(ctypes.byref(d), ctypes.byref(self.h)), "msi_source_open")
+
+    def read(self, file_off: int, nbytes: int):
+        """Synchronous read: (window, bytes of the extent as a numpy copy)."""
+        data = ctypes.c_void_p()
+        w = ctypes.c_int()
+        N.check(N.lib().msi_source_read(self.h, file_off, nbytes, ctypes.byref(data), ctypes.byref(w)),
+                "msi_source_read")
+        out = np.ctypeslib.as_array((ctypes.c_uint8 * nbytes).from_address(data.value)).copy()
+        return w.value, out
+
+    def release(self, window: int):
+        N.check(N.lib().msi_source_release(self.h, window), "msi_source_release")
+
+    def stats(self) -> dict:
+        st = N.msi_source_stats()
+        N.check(N.lib().msi_source_stats_read(self.h, ctypes.byref(st)), "msi_source_stats_read")
+        return {n: getattr(st, n) for n, _ in N.msi_source_stats._fields_}
+
+    def close(self):
+        if getattr(self, "h", None) is not None and self.h.value:
+            N.check(N.lib().msi_source_close(self.h), "msi_source_close")
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
         except Exception:
             pass

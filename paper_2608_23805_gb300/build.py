@@ -1,6 +1,7 @@
 """Build the CUDA library libmsi.so in-tree for sm_103a (GB300).
 
-Each translation unit under csrc/ is compiled in parallel with nvcc
+Each translation unit under csrc/ (CUDA, and the host-only source service in
+source.cpp) is compiled in parallel with nvcc
 (-gencode arch=compute_103a,code=sm_103a), then linked with the static CUDA
 runtime into paper_2608_23805_gb300/libmsi.so.  No GPU is needed to build.
 """
@@ -17,7 +18,8 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libmsi.so")
-SOURCES = ["plan.cu", "router.cu", "router_tc.cu", "permute.cu", "gemm.cu", "gemm_pair.cu", "noalloc.cu"]
+SOURCES = ["plan.cu", "router.cu", "router_tc.cu", "permute.cu", "gemm.cu", "gemm_pair.cu", "noalloc.cu",
+           "source.cpp"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 
@@ -39,7 +41,8 @@ def _flags(verbose_ptxas: bool) -> list[str]:
 def _stale(obj: str, src: str) -> bool:
     if not os.path.exists(obj):
         return True
-    deps = [src, os.path.join(CSRC, "internal.cuh"), os.path.join(ROOT, "include", "msi.h")]
+    deps = [src, os.path.join(CSRC, "internal.cuh"), os.path.join(CSRC, "source.h"),
+            os.path.join(ROOT, "include", "msi.h")]
     return any(os.path.getmtime(d) > os.path.getmtime(obj) for d in deps)
 
 
@@ -49,7 +52,7 @@ def build(force: bool = False, verbose_ptxas: bool = False, jobs: int = 0) -> st
     work = []
     for s in SOURCES:
         src = os.path.join(CSRC, s)
-        obj = os.path.join(BUILD, s.replace(".cu", ".o"))
+        obj = os.path.join(BUILD, os.path.splitext(s)[0] + ".o")
         if force or _stale(obj, src):
             work.append((src, obj))
 
@@ -66,10 +69,10 @@ def build(force: bool = False, verbose_ptxas: bool = False, jobs: int = 0) -> st
     if verbose_ptxas:
         for l in logs:
             sys.stderr.write(l)
-    objs = [os.path.join(BUILD, s.replace(".cu", ".o")) for s in SOURCES]
+    objs = [os.path.join(BUILD, os.path.splitext(s)[0] + ".o") for s in SOURCES]
     if work or force or not os.path.exists(LIB):
         tmp = LIB + ".%d.tmp" % os.getpid()
-        cmd = [cc] + ARCH + ["-shared", "-cudart", "static", "-o", tmp] + objs
+        cmd = [cc] + ARCH + ["-shared", "-cudart", "static", "-o", tmp] + objs + ["-lpthread"]
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
             raise RuntimeError("link failed:\n%s\n%s" % (r.stdout, r.stderr))

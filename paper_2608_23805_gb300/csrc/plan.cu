@@ -33,6 +33,7 @@
 #include <vector>
 
 #include "internal.cuh"
+#include "source.h"
 
 using namespace msi;
 
@@ -222,6 +223,10 @@ struct msi_plan {
   // expert only)
   cudaStream_t side = nullptr;
   cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
+  // bounded source service: when attached, missing extents are read from its
+  // file (src_off[l * E + e]) through its windows instead of host_windows
+  msi_source* src = nullptr;
+  std::vector<uint64_t> src_off;
   std::mutex mu;
 
   explicit msi_plan(int S) : holds(S) {
@@ -324,6 +329,17 @@ void ledger_stage(msi_plan* p, int s, int layer, int e, int call, int wave) {
   p->ctr.h2d_bytes += p->d.extent_bytes;
 }
 
+// A slot whose content is no longer its ledger object (a staging call that
+// failed after invalidating it): the object is evicted and the slot Vacant.
+void ledger_vacate(msi_plan* p, int s, int call, int wave) {
+  Slot& sl = p->slots[s];
+  if (sl.layer < 0) return;
+  add_trace(p, call, sl.layer, sl.expert, s, sl.gen, MSI_TRACE_EVICT, wave);
+  p->where[(size_t)sl.layer * p->d.n_experts + sl.expert] = -1;
+  p->ctr.evicts++;
+  sl.layer = sl.expert = -1;
+}
+
 // Wait on `stream` for every not-yet-complete event in ids (deduplicated).
 msi_status wait_events(msi_plan* p, std::vector<int>& ids, cudaStream_t stream) {
   std::sort(ids.begin(), ids.end());
@@ -394,6 +410,52 @@ msi_status stage_enqueue(msi_plan* p, int layer, const std::vector<WaveEntry>& m
   auto dst_of = [&](const WaveEntry& m) {
     return static_cast<char*>(p->d.slot_pool) + (size_t)m.slot * eb;
   };
+  if (p->src != nullptr) {
+    // source path: up to n_windows reads ahead of the copies, each read
+    // checked (identity, length, completion status) before its copy
+    const int nw = source_windows(p->src);
+    std::vector<int> win(misses.size(), -1);
+    std::vector<SourceRequest> rq(misses.size());
+    for (size_t i = 0; i < misses.size(); ++i) {
+      SourceRequest& r = rq[i];
+      r.object = obj_key(layer, misses[i].expert);
+      r.epoch = p->epoch;
+      r.generation = misses[i].gen;
+      r.file_off = p->src_off[(size_t)layer * p->d.n_experts + misses[i].expert];
+      r.bytes = eb;
+      r.inject = kInjectNone;
+      auto f = p->faults.find(r.object);
+      if (f != p->faults.end() && (f->second == MSI_FAULT_IO_ERROR || f->second == MSI_FAULT_SHORT_READ)) {
+        r.inject = f->second == MSI_FAULT_IO_ERROR ? kInjectIoError : kInjectShortRead;
+        p->faults.erase(f);
+      }
+    }
+    size_t next = 0;
+    msi_status fail = MSI_OK;
+    for (size_t i = 0; i < misses.size() && fail == MSI_OK; ++i) {
+      while (next < misses.size() && next < i + (size_t)nw && fail == MSI_OK) {
+        fail = source_submit(p->src, rq[next], &win[next]);
+        ++next;
+      }
+      if (fail != MSI_OK) break;
+      const void* data = nullptr;
+      fail = source_wait(p->src, win[i], rq[i], &data);
+      win[i] = fail == MSI_OK ? win[i] : -1;
+      if (fail != MSI_OK) break;
+      CK(cudaMemcpyAsync(dst_of(misses[i]), data, eb, cudaMemcpyHostToDevice, stage));
+      st = source_copying(p->src, win[i], stage);
+      if (st != MSI_OK) return st;
+      win[i] = -1;
+    }
+    if (fail != MSI_OK) {
+      // nothing more is copied and the bundle is not published: reads still
+      // in flight land and their windows return to Free
+      for (size_t i = 0; i < next; ++i)
+        if (win[i] >= 0) source_release(p->src, win[i]);
+      p->ctr.rejections++;
+      return fail == MSI_ERR_SOURCE ? MSI_ERR_SOURCE : fail;
+    }
+  } else {
   // one copy per run of extents that continue each other in both the host
   // window and the slot pool (consecutive experts into consecutive slots):
   // large copies reach the host link's rate, per-extent copies fall short
@@ -408,6 +470,7 @@ msi_status stage_enqueue(msi_plan* p, int layer, const std::vector<WaveEntry>& m
     }
     CK(cudaMemcpyAsync(dst, src, bytes, cudaMemcpyHostToDevice, stage));
     i = j;
+  }
   }
   LAUNCH(p, MSI_K_PUBLISH, stage, launch_publish(pub, p->d_gen, stage));
   int ev;
@@ -858,7 +921,7 @@ msi_status msi_slot_stage(msi_plan* p, int slot, int layer, int expert, msi_stre
     return MSI_ERR_INVALID_ARG;
   const int cur = p->where[(size_t)layer * d.n_experts + expert];
   if (cur >= 0 && cur != slot) return MSI_ERR_INVALID_ARG;  // one slot per object
-  {
+  if (p->src == nullptr) {
     auto f = p->faults.find(obj_key(layer, expert));
     if (f != p->faults.end() && f->second == MSI_FAULT_SHORT_READ) {
       p->faults.erase(f);  // the source delivered less than the extent: nothing is staged
@@ -874,6 +937,12 @@ msi_status msi_slot_stage(msi_plan* p, int slot, int layer, int expert, msi_stre
   const uint64_t gen = sl.gen + 1;
   std::vector<WaveEntry> m{{expert, slot, true, gen}};
   msi_status st = stage_enqueue(p, layer, m, reinterpret_cast<cudaStream_t>(stage));
+  if (st == MSI_ERR_SOURCE) {
+    // the slot's published word was invalidated before the read failed: the
+    // object it held is gone
+    ledger_vacate(p, slot, -1, -1);
+    return st;
+  }
   if (st != MSI_OK) return st;
   ledger_stage(p, slot, layer, expert, -1, -1);
   if (new_generation) *new_generation = sl.gen;
@@ -1037,8 +1106,10 @@ msi_status msi_moe_forward_streamed(msi_plan* p, int layer, const void* x, int T
       return MSI_ERR_TIMEOUT;
     }
 
-  // every miss's source must be whole before any bundle is planned or published
-  for (int e = 0; e < E; ++e) {
+  // host windows: every miss's source must be whole before any bundle is
+  // planned or published (with a source attached, reads are checked as they
+  // complete and a failure unwinds the call's remaining bundles)
+  for (int e = 0; e < E && p->src == nullptr; ++e) {
     if (p->h_counts[e] <= 0 || p->where[(size_t)layer * E + e] >= 0) continue;
     auto f = p->faults.find(obj_key(layer, e));
     if (f != p->faults.end() && f->second == MSI_FAULT_SHORT_READ) {
@@ -1057,11 +1128,16 @@ msi_status msi_moe_forward_streamed(msi_plan* p, int layer, const void* x, int T
   }
   std::vector<int> order(hits);
   order.insert(order.end(), misses.begin(), misses.end());
+  // Waves are planned one at a time, just before they are staged: the rules
+  // (and so the trace) are those of planning them all up front, and a bundle
+  // whose read is rejected leaves no later wave planned.
+  const size_t n_waves = (order.size() + p->C - 1) / p->C;
   std::vector<std::vector<WaveEntry>> waves;
   std::vector<char> pinned(d.n_slots, 0);
   std::vector<int> prev;
-  for (size_t w0 = 0; w0 < order.size(); w0 += p->C) {
+  auto plan_wave = [&]() {
     const int w = (int)waves.size();
+    const size_t w0 = (size_t)w * p->C;
     std::vector<WaveEntry> wave;
     std::fill(pinned.begin(), pinned.end(), 0);
     for (int s : prev) pinned[s] = 1;
@@ -1096,22 +1172,31 @@ msi_status msi_moe_forward_streamed(msi_plan* p, int layer, const void* x, int T
       prev.push_back(we.slot);
     }
     waves.push_back(std::move(wave));
-  }
+  };
 
-  // ---- issue: stage(w + 1) overlaps compute(w) ----
+  // ---- issue: plan + stage(w + 1) overlaps compute(w) ----
   auto stage_wave = [&](size_t w) -> msi_status {
+    plan_wave();
     std::vector<WaveEntry> m;
     for (const auto& we : waves[w])
       if (we.miss) m.push_back(we);
-    return stage_enqueue(p, layer, m, ss);
+    msi_status r = stage_enqueue(p, layer, m, ss);
+    if (r == MSI_ERR_SOURCE) {
+      // a rejected read: this bundle is not published and no later one is
+      // planned; the bundle's slots hold nothing (each was invalidated before
+      // its copies) and become Vacant in the ledger
+      for (const auto& we : waves[w])
+        if (we.miss) ledger_vacate(p, we.slot, call, (int)w);
+    }
+    return r;
   };
-  if (!waves.empty()) {
+  if (n_waves > 0) {
     st = stage_wave(0);
     if (st != MSI_OK) return st;
   }
   static thread_local WaveParams wp;
-  for (size_t w = 0; w < waves.size(); ++w) {
-    if (w + 1 < waves.size()) {
+  for (size_t w = 0; w < n_waves; ++w) {
+    if (w + 1 < n_waves) {
       st = stage_wave(w + 1);
       if (st != MSI_OK) return st;
     }
@@ -1202,12 +1287,23 @@ msi_status msi_plan_reset(msi_plan* p, uint64_t* new_epoch) {
   return MSI_OK;
 }
 
+msi_status msi_plan_set_source(msi_plan* p, msi_source* src, const uint64_t* file_off) {
+  if (p == nullptr || (src != nullptr && file_off == nullptr)) return MSI_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> g(p->mu);
+  if (p->dying) return MSI_ERR_SHUT_DOWN;
+  p->src = src;
+  p->src_off.clear();
+  if (src != nullptr)
+    p->src_off.assign(file_off, file_off + (size_t)p->d.n_layers * p->d.n_experts);
+  return MSI_OK;
+}
+
 msi_status msi_fault_inject(msi_plan* p, int kind, int layer, int expert) {
   if (p == nullptr || layer < 0 || layer >= p->d.n_layers || expert < 0 ||
       expert >= p->d.n_experts)
     return MSI_ERR_INVALID_ARG;
   if (kind != MSI_FAULT_SHORT_READ && kind != MSI_FAULT_STALE_COMPLETION &&
-      kind != MSI_FAULT_WRONG_OBJECT)
+      kind != MSI_FAULT_WRONG_OBJECT && kind != MSI_FAULT_IO_ERROR)
     return MSI_ERR_INVALID_ARG;
   std::lock_guard<std::mutex> g(p->mu);
   p->faults[obj_key(layer, expert)] = kind;

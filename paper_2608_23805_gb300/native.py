@@ -23,7 +23,8 @@ MSI_ERR_SHUT_DOWN = 8
 MSI_ERR_UNSUPPORTED = 9
 MSI_ERR_WORKSPACE = 10
 MSI_ERR_SOURCE = 11
-MSI_FAULT_SHORT_READ, MSI_FAULT_STALE_COMPLETION, MSI_FAULT_WRONG_OBJECT = 1, 2, 3
+MSI_FAULT_SHORT_READ, MSI_FAULT_STALE_COMPLETION, MSI_FAULT_WRONG_OBJECT, MSI_FAULT_IO_ERROR = 1, 2, 3, 4
+MSI_MAX_WINDOWS = 64
 
 MSI_W_BF16 = 0
 MSI_W_Q4G32 = 1
@@ -64,6 +65,19 @@ class msi_counters(ctypes.Structure):
                  "rejections")]
 
 
+class msi_source_desc(ctypes.Structure):
+    _fields_ = [("path", ctypes.c_char_p), ("direct", ctypes.c_int), ("align", ctypes.c_uint32),
+                ("n_windows", ctypes.c_int), ("windows", ctypes.c_void_p),
+                ("window_bytes", ctypes.c_uint64)]
+
+
+class msi_source_stats(ctypes.Structure):
+    _fields_ = [("reads", ctypes.c_uint64), ("rejected", ctypes.c_uint64),
+                ("logical_bytes", ctypes.c_uint64), ("physical_bytes", ctypes.c_uint64),
+                ("padding_bytes", ctypes.c_uint64), ("read_seconds", ctypes.c_double),
+                ("max_in_flight", ctypes.c_int)]
+
+
 _P = ctypes.c_void_p
 _SIGS = {
     "msi_extent_bytes": (ctypes.c_uint64, [ctypes.c_int, ctypes.c_int, ctypes.c_int]),
@@ -85,6 +99,13 @@ _SIGS = {
     "msi_forward_status": (ctypes.c_int, [_P, ctypes.POINTER(ctypes.c_int)]),
     "msi_plan_reset": (ctypes.c_int, [_P, ctypes.POINTER(ctypes.c_uint64)]),
     "msi_fault_inject": (ctypes.c_int, [_P, ctypes.c_int, ctypes.c_int, ctypes.c_int]),
+    "msi_source_open": (ctypes.c_int, [ctypes.POINTER(msi_source_desc), ctypes.POINTER(_P)]),
+    "msi_source_close": (ctypes.c_int, [_P]),
+    "msi_source_stats_read": (ctypes.c_int, [_P, ctypes.POINTER(msi_source_stats)]),
+    "msi_source_read": (ctypes.c_int, [_P, ctypes.c_uint64, ctypes.c_uint64, ctypes.POINTER(_P),
+                                       ctypes.POINTER(ctypes.c_int)]),
+    "msi_source_release": (ctypes.c_int, [_P, ctypes.c_int]),
+    "msi_plan_set_source": (ctypes.c_int, [_P, _P, _P]),
     "msi_consumer_hold": (ctypes.c_int, [_P, ctypes.c_int]),
     "msi_consumer_release": (ctypes.c_int, [_P, ctypes.c_int]),
     "msi_trace_read": (ctypes.c_int, [_P, ctypes.POINTER(msi_trace_rec), ctypes.c_size_t,
