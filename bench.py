@@ -325,6 +325,17 @@ def run_ours(args):
     __graft_entry__.build()
     w = Workload(args.workload)
     cfg = w.cfg
+    src = None
+    if args.source != "none":
+        if not cfg.lru:
+            raise SystemExit("--source applies to the staged (LRU) workloads")
+        from paper_2608_23805_gb300 import api
+        path = os.path.join(os.environ.get("MSI_SOURCE_DIR", "/tmp"), "msi_extents_%d.bin" % os.getpid())
+        with open(path, "wb") as f:
+            f.write(w.windows.numpy().tobytes())
+        src = api.Source(path, cfg.extent_bytes + 2 * 4096, n_windows=8, direct=args.source == "direct")
+        os.unlink(path)  # the open file stays readable
+        w.plan.set_source(src, np.arange(cfg.n_experts, dtype=np.uint64) * cfg.extent_bytes)
     peaks, peak_kind = load_peaks()
 
     flush = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device="cuda")
@@ -428,6 +439,15 @@ def run_ours(args):
         "step_ms": [round(a.elapsed_time(b), 3) for a, b in evs],
         "peaks": peak_kind,
     }
+    if src is not None:
+        ss = src.stats()
+        line["config"]["source"] = {
+            "kind": args.source, "windows": 8, "reads": ss["reads"], "rejected": ss["rejected"],
+            "logical_gb": ss["logical_bytes"] / 1e9, "padding_mb": ss["padding_bytes"] / 1e6,
+            "read_gbs_per_window": ss["logical_bytes"] / max(ss["read_seconds"], 1e-9) / 1e9,
+            "max_in_flight": ss["max_in_flight"]}
+        line["config"]["residency"] = "LRU waves of %d, staged from a file through the bounded " \
+            "source service (%s reads)" % (cfg.n_slots // 2, args.source)
     if world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(w, SAMPLE_TOKENS.get(args.workload, 256))
     print(json.dumps(line), flush=True)
@@ -498,6 +518,9 @@ def main():
                     choices=["qwen3next_4k", "prefill32k_lru64", "prefill32k_q4_lru64", "tiny"])
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--source", default="none", choices=["none", "buffered", "direct"],
+                    help="staged workloads: read every missing extent from a file through the "
+                         "bounded source service (8 windows) instead of pinned host windows")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
