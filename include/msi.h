@@ -82,8 +82,11 @@ enum {
   MSI_FAULT_STALE_COMPLETION = 2,  /* the object's next publication carries the previous
                                       generation (a late stale completion) */
   MSI_FAULT_WRONG_OBJECT = 3,      /* the object's next publication names another object */
-  MSI_FAULT_IO_ERROR = 4           /* with a source attached: the object's next read completes
+  MSI_FAULT_IO_ERROR = 4,          /* with a source attached: the object's next read completes
                                       with an I/O error (EIO); its bundle is not published */
+  MSI_FAULT_STALE_EPOCH = 5        /* with a source attached: the object's next read carries the
+                                      previous request epoch (a completion from before a reset);
+                                      it is rejected at completion, its bundle not published */
 };
 
 /* Forward flags. */
@@ -295,13 +298,18 @@ typedef struct {
   uint64_t padding_bytes;  /* physical - logical */
   double read_seconds;     /* summed completion latency of completed reads */
   int max_in_flight;       /* peak reads in flight */
+  int windows_busy;        /* windows not Free at the query (a copy still in flight counts) */
 } msi_source_stats;
 
 /* Open: the file is opened (O_RDONLY, plus O_DIRECT when direct = 1) and one
  * reader thread is started per window.  Errors: MSI_ERR_INVALID_ARG (null
  * pointers, alignment, sizes), MSI_ERR_UNSUPPORTED (the file system refuses
- * O_DIRECT), MSI_ERR_SOURCE (the file cannot be opened).  Close waits for
- * every read in flight and every window's copy. */
+ * O_DIRECT), MSI_ERR_SOURCE (the file cannot be opened).
+ * Close is the source's shutdown check: it refuses with MSI_ERR_SLOT_BUSY,
+ * changing nothing, while a plan still has the source attached
+ * (msi_plan_set_source; msi_plan_destroy detaches) or a caller still holds a
+ * window from msi_source_read; otherwise it waits for every read in flight and
+ * every window's copy, then frees the source. */
 msi_status msi_source_open(const msi_source_desc* desc, msi_source** out);
 msi_status msi_source_close(msi_source* src);
 msi_status msi_source_stats_read(msi_source* src, msi_source_stats* out);
@@ -322,7 +330,8 @@ msi_status msi_source_release(msi_source* src, int window);
  * with MSI_ERR_SOURCE: the failing bundle (the wave, and every later wave of
  * the call) is neither copied nor published, its slots are left Vacant, and
  * no output row of the call is written.  src = NULL detaches.  The source
- * must outlive the plan or be detached first.  file_off is copied. */
+ * stays attached until detached or until msi_plan_destroy, and refuses to
+ * close meanwhile.  file_off is copied. */
 msi_status msi_plan_set_source(msi_plan* plan, msi_source* src, const uint64_t* file_off);
 
 msi_status msi_consumer_hold(msi_plan* plan, int slot);

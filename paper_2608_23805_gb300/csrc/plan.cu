@@ -430,6 +430,16 @@ msi_status stage_enqueue(msi_plan* p, int layer, const std::vector<WaveEntry>& m
         p->faults.erase(f);
       }
     }
+    // the identity each completion must carry; a hooked read is submitted
+    // with the previous epoch, as a read from before a reset would be
+    std::vector<SourceRequest> expect(rq);
+    for (size_t i = 0; i < misses.size(); ++i) {
+      auto f = p->faults.find(rq[i].object);
+      if (f != p->faults.end() && f->second == MSI_FAULT_STALE_EPOCH) {
+        rq[i].epoch = p->epoch - 1;
+        p->faults.erase(f);
+      }
+    }
     size_t next = 0;
     msi_status fail = MSI_OK;
     for (size_t i = 0; i < misses.size() && fail == MSI_OK; ++i) {
@@ -439,7 +449,7 @@ msi_status stage_enqueue(msi_plan* p, int layer, const std::vector<WaveEntry>& m
       }
       if (fail != MSI_OK) break;
       const void* data = nullptr;
-      fail = source_wait(p->src, win[i], rq[i], &data);
+      fail = source_wait(p->src, win[i], expect[i], &data);
       win[i] = fail == MSI_OK ? win[i] : -1;
       if (fail != MSI_OK) break;
       CK(cudaMemcpyAsync(dst_of(misses[i]), data, eb, cudaMemcpyHostToDevice, stage));
@@ -891,6 +901,8 @@ msi_status msi_plan_destroy(msi_plan* p) {
     }
     if (p->fwd_ev >= 0) cudaEventSynchronize(p->pool.ev[p->fwd_ev]);
     if (p->side) cudaStreamSynchronize(p->side);
+    source_attach(p->src, -1);  // every window copy of this plan has completed
+    p->src = nullptr;
     p->timer.destroy();
     for (auto ev : p->pool.ev) cudaEventDestroy(ev);
     cudaFree(p->d_gen);
@@ -1291,6 +1303,10 @@ msi_status msi_plan_set_source(msi_plan* p, msi_source* src, const uint64_t* fil
   if (p == nullptr || (src != nullptr && file_off == nullptr)) return MSI_ERR_INVALID_ARG;
   std::lock_guard<std::mutex> g(p->mu);
   if (p->dying) return MSI_ERR_SHUT_DOWN;
+  if (p->src != src) {
+    source_attach(p->src, -1);
+    source_attach(src, +1);
+  }
   p->src = src;
   p->src_off.clear();
   if (src != nullptr)
@@ -1303,7 +1319,7 @@ msi_status msi_fault_inject(msi_plan* p, int kind, int layer, int expert) {
       expert >= p->d.n_experts)
     return MSI_ERR_INVALID_ARG;
   if (kind != MSI_FAULT_SHORT_READ && kind != MSI_FAULT_STALE_COMPLETION &&
-      kind != MSI_FAULT_WRONG_OBJECT && kind != MSI_FAULT_IO_ERROR)
+      kind != MSI_FAULT_WRONG_OBJECT && kind != MSI_FAULT_IO_ERROR && kind != MSI_FAULT_STALE_EPOCH)
     return MSI_ERR_INVALID_ARG;
   std::lock_guard<std::mutex> g(p->mu);
   p->faults[obj_key(layer, expert)] = kind;

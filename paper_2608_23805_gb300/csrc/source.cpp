@@ -58,6 +58,7 @@ struct msi_source {
   bool stop = false;
   msi_source_stats st{};
   int in_flight = 0;
+  int attached = 0;  // plans staging through this source
 
   void worker() {
     for (;;) {
@@ -220,6 +221,12 @@ msi_status source_release(msi_source* s, int i) {
 
 int source_windows(const msi_source* s) { return s ? (int)s->w.size() : 0; }
 
+void source_attach(msi_source* s, int delta) {
+  if (s == nullptr) return;
+  std::lock_guard<std::mutex> l(s->mu);
+  s->attached += delta;
+}
+
 }  // namespace msi
 
 extern "C" {
@@ -255,7 +262,17 @@ msi_status msi_source_open(const msi_source_desc* d, msi_source** out) {
 msi_status msi_source_close(msi_source* s) {
   if (s == nullptr) return MSI_ERR_INVALID_ARG;
   {
-    std::lock_guard<std::mutex> l(s->mu);
+    std::unique_lock<std::mutex> l(s->mu);
+    // shutdown check: no plan may still stage through the source and no
+    // caller may still hold a window it read
+    if (s->attached > 0) return MSI_ERR_SLOT_BUSY;
+    s->cv_done.wait(l, [&] {
+      for (const auto& x : s->w)
+        if (x.st == msi_source::kReading) return false;
+      return true;
+    });
+    for (const auto& x : s->w)
+      if (x.st == msi_source::kHostReady) return MSI_ERR_SLOT_BUSY;
     s->stop = true;
   }
   s->cv_job.notify_all();
@@ -275,6 +292,9 @@ msi_status msi_source_stats_read(msi_source* s, msi_source_stats* out) {
   if (s == nullptr || out == nullptr) return MSI_ERR_INVALID_ARG;
   std::lock_guard<std::mutex> l(s->mu);
   *out = s->st;
+  out->windows_busy = 0;
+  for (int i = 0; i < (int)s->w.size(); ++i)
+    if (!s->reclaim(i)) out->windows_busy++;
   return MSI_OK;
 }
 

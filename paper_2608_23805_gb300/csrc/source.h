@@ -38,5 +38,7 @@ msi_status source_copying(msi_source* s, int window, cudaStream_t stream);
 // Return a window (its read, if in flight, lands first) without copying it.
 msi_status source_release(msi_source* s, int window);
 int source_windows(const msi_source* s);
+// A plan attaches (+1) or detaches (-1); an attached source refuses to close.
+void source_attach(msi_source* s, int delta);
 
 }  // namespace msi

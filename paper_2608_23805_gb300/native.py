@@ -23,7 +23,8 @@ MSI_ERR_SHUT_DOWN = 8
 MSI_ERR_UNSUPPORTED = 9
 MSI_ERR_WORKSPACE = 10
 MSI_ERR_SOURCE = 11
-MSI_FAULT_SHORT_READ, MSI_FAULT_STALE_COMPLETION, MSI_FAULT_WRONG_OBJECT, MSI_FAULT_IO_ERROR = 1, 2, 3, 4
+(MSI_FAULT_SHORT_READ, MSI_FAULT_STALE_COMPLETION, MSI_FAULT_WRONG_OBJECT, MSI_FAULT_IO_ERROR,
+ MSI_FAULT_STALE_EPOCH) = 1, 2, 3, 4, 5
 MSI_MAX_WINDOWS = 64
 
 MSI_W_BF16 = 0
@@ -75,7 +76,7 @@ class msi_source_stats(ctypes.Structure):
     _fields_ = [("reads", ctypes.c_uint64), ("rejected", ctypes.c_uint64),
                 ("logical_bytes", ctypes.c_uint64), ("physical_bytes", ctypes.c_uint64),
                 ("padding_bytes", ctypes.c_uint64), ("read_seconds", ctypes.c_double),
-                ("max_in_flight", ctypes.c_int)]
+                ("max_in_flight", ctypes.c_int), ("windows_busy", ctypes.c_int)]
 
 
 _P = ctypes.c_void_p

@@ -55,6 +55,7 @@ def test_streamed_from_file_equals_host_windows(tmp_path, direct):
     assert st["reads"] == c["stages"] and st["rejected"] == 0
     assert st["logical_bytes"] == c["stages"] * cfg.extent_bytes
     assert 1 <= st["max_in_flight"] <= 4
+    assert st["windows_busy"] == 0  # balanced terminal state: every window Free
     if direct:
         assert st["padding_bytes"] > 0 and st["physical_bytes"] % 4096 == 0
     b.plan.set_source(None)
@@ -80,10 +81,12 @@ def test_slot_stage_from_file_matches_oracle(tmp_path):
     case.close()
 
 
-@pytest.mark.parametrize("kind", [N.MSI_FAULT_IO_ERROR, N.MSI_FAULT_SHORT_READ])
+@pytest.mark.parametrize("kind", [N.MSI_FAULT_IO_ERROR, N.MSI_FAULT_SHORT_READ,
+                                  N.MSI_FAULT_STALE_EPOCH])
 def test_rejected_read_mid_call_unwinds_the_remaining_bundles(tmp_path, kind):
     """Qwen-shaped layer with 64 experts, 16 slots (waves of 8): the read of
-    an expert in the third wave fails.  The call returns MSI_ERR_SOURCE; the
+    an expert in the third wave fails (I/O error, short read, or a completion
+    carrying the previous request epoch).  The call returns MSI_ERR_SOURCE; the
     third bundle is not published, its slots are Vacant, no later wave is
     planned; the output buffer keeps its contents; the next call matches the
     oracle."""
@@ -113,10 +116,46 @@ def test_rejected_read_mid_call_unwinds_the_remaining_bundles(tmp_path, kind):
     busy = sum(1 for s in range(cfg.n_slots) if case.plan.slot_state(s) != N.MSI_SLOT_VACANT)
     assert busy == 8
     assert src.stats()["rejected"] == 1
+    assert src.stats()["windows_busy"] == 0  # the executor drained: every window Free
     out2, _ = case.plan.forward_streamed(0, bf16_tensor(x_bits), case.router[0])
     torch.cuda.synchronize()
     assert case.plan.status() == N.MSI_OK
     compare_out(bf16_bits(out2), case.oracle_layer(x_bits)["out"])
+    assert src.stats()["windows_busy"] == 0
     case.plan.set_source(None)
     src.close()
     case.close()
+
+
+def test_reset_and_shutdown_with_source_work(tmp_path):
+    """Reset with source work, shutdown with a live consumer (paper, Table 6).
+    A streamed call stages through the source, then the plan is reset: the
+    reset drains every window copy (all windows Free), advances the epoch and
+    evicts every slot; the next call restages everything from the file and
+    matches the oracle.  Closing the source while the plan has it attached is
+    refused and changes nothing; destroying the plan detaches it, after which
+    the source closes."""
+    cfg = synth.config("tiny", n_slots=8, lru=True)
+    case = Case(cfg)
+    src, off = _source(case, tmp_path, False, n_windows=3)
+    case.plan.set_source(src, off)
+    x_bits = synth.hidden(cfg, 0, 62)
+    expect = case.oracle_layer(x_bits)["out"]
+    out, _ = case.plan.forward_streamed(0, bf16_tensor(x_bits), case.router[0])
+    reads = src.stats()["reads"]
+    epoch = case.plan.reset()
+    assert src.stats()["windows_busy"] == 0
+    assert all(case.plan.slot_state(s) == N.MSI_SLOT_VACANT for s in range(cfg.n_slots))
+    compare_out(bf16_bits(out), expect)
+    out2, _ = case.plan.forward_streamed(0, bf16_tensor(x_bits), case.router[0])
+    torch.cuda.synchronize()
+    assert case.plan.status() == N.MSI_OK
+    compare_out(bf16_bits(out2), expect)
+    assert src.stats()["reads"] == 2 * reads and src.stats()["rejected"] == 0
+    assert case.plan.reset() == epoch + 1
+    with pytest.raises(N.MsiError) as ei:
+        src.close()  # still attached
+    assert ei.value.status == N.MSI_ERR_SLOT_BUSY
+    case.close()  # destroy drains and detaches
+    assert src.stats()["windows_busy"] == 0
+    src.close()

@@ -4,7 +4,7 @@ bytes delivered equal the file's extent bytes; covering reads under O_DIRECT
 add exactly the padding that rounds each extent out to the alignment, and
 padding is counted apart from logical bytes; extent overflow, short reads and
 an exhausted window set are rejected; reads in flight never exceed the
-window count."""
+window count; a source with a window still held refuses to close."""
 import ctypes
 import os
 
@@ -114,3 +114,22 @@ def test_open_rejects_bad_descriptors(tmp_path):
         assert N.lib().msi_source_open(ctypes.byref(d), ctypes.byref(h)) == N.MSI_ERR_INVALID_ARG
     d = N.msi_source_desc(str(tmp_path / "missing").encode(), 0, 4096, 2, base, 8192)
     assert N.lib().msi_source_open(ctypes.byref(d), ctypes.byref(h)) == N.MSI_ERR_SOURCE
+
+
+def test_close_refuses_while_a_window_is_held(tmp_path):
+    """Shutdown with a live consumer (paper, Table 6): a caller still holds a
+    HostReady window, so close refuses and changes nothing; once the window is
+    released every window is Free and close succeeds."""
+    cfg = synth.config("tiny")
+    eb = cfg.extent_bytes
+    path, win, off = _file(tmp_path, cfg)
+    src = _open(path, eb, False, n=2)
+    w, got = src.read(off[1], eb)
+    with pytest.raises(N.MsiError) as ei:
+        src.close()
+    assert ei.value.status == N.MSI_ERR_SLOT_BUSY
+    assert src.stats()["windows_busy"] == 1
+    assert np.array_equal(got, win[eb:2 * eb])  # the held bytes are untouched
+    src.release(w)
+    assert src.stats()["windows_busy"] == 0
+    src.close()
