@@ -19,7 +19,7 @@ bijection, a textbook OrderedDict LRU, hand-worked 3-slot LRU traces in
 """
 from .moe import (  # noqa: F401
     STATUS_OK, STATUS_STALE_GENERATION, STATUS_WRONG_OBJECT, STATUS_NOT_RESIDENT,
-    TRACE_HIT, TRACE_STAGE, TRACE_EVICT,
+    TRACE_HIT, TRACE_STAGE, TRACE_EVICT, TRACE_PREFETCH,
     bf16_to_f64, f16_to_f64, decode_extent, dequant_q4g32,
     router, permutation, swiglu_expert, moe_layer, moe_tokens, dense_masked_moe,
     combine, generation_check, LRUWaveSim, near_tie_tokens,

@@ -25,7 +25,9 @@ computation runs inside its pinned native runtime):
   R7  LRU-wave slot policy made exact (see LRUWaveSim);
   R9  4-bit weights: symmetric offset 8, low nibble = even column, one fp16
       scale per 32 consecutive weights of a row;
-  R10 decode stack: x_{l+1} = x_l + moe_l(x_l) (residual passed to combine).
+  R10 decode stack: x_{l+1} = x_l + moe_l(x_l) (residual passed to combine);
+  R13 next-layer prediction, two-bank prefetch and pins made exact (see
+      LRUWaveSim).
 """
 from __future__ import annotations
 
@@ -39,6 +41,7 @@ STATUS_NOT_RESIDENT = "not_resident"
 TRACE_HIT = "hit"
 TRACE_STAGE = "stage"
 TRACE_EVICT = "evict"
+TRACE_PREFETCH = "prefetch"
 
 _W_BF16 = 0
 _W_Q4G32 = 1
@@ -306,6 +309,36 @@ class LRUWaveSim:
       * trace records (call, layer, expert, slot, generation, kind, wave) for
         each hit, each eviction (with the evicted object and its generation)
         and each stage (with the new generation).
+
+    Prediction, two-bank prefetch and pinning (reading R13).  The paper runs a
+    protected LRU64 together with a two-bank next-layer prefetch (Sec.
+    "Evaluation", "Cache and storage state"; Sec. "Qwen-Specific Natural
+    Utility") and states that demand loading, LRU, prediction and pinning pick
+    different future objects through one lifecycle (Sec. "A Shared
+    Cross-Adapter Plan Core").  It specifies neither the predictor nor the
+    banks; made exact here:
+
+      * a call may carry a prediction for another layer: the number of token
+        choices predicted per expert of that layer (the forward predicts layer
+        l + 1 by routing the call's input through layer l + 1's router);
+      * after the call's last wave, one prefetch bundle: the predicted experts
+        that are not resident, ranked by predicted count descending (ties ->
+        lower id), the first `wave_capacity` of them, assigned in ascending
+        expert order;
+      * two banks: the slots of the call's last wave (computed on), of the
+        prefetch bundle being assigned, and of every predicted object already
+        resident are pinned; victims by the same rule; the bundle ends early
+        when no unpinned slot is left;
+      * a prefetched object's last-use tick is the current tick (prefetching
+        is not consumption: the tick does not advance);
+      * trace: eviction records and "prefetch" records, wave index = the
+        number of waves of the call;
+      * caller pins: a pinned object is never a victim; at most
+        S - 2 * wave_capacity objects may be pinned (S - wave_capacity
+        without previous-wave pinning), so every wave and bundle finds
+        victims;
+      * counters: objects prefetched, and hits on a prefetched object before
+        its first consumption.
     """
 
     def __init__(self, n_slots: int, wave_capacity: int | None = None, pin_previous: bool = True):
@@ -321,16 +354,46 @@ class LRUWaveSim:
         self.calls = 0
         self.trace = []
         self.where = {}
+        self.pins = set()
+        self.prefetched = set()   # slots holding a prefetched, unconsumed object
+        self.prefetches = 0
+        self.prefetch_hits = 0
+
+    def pin(self, layer: int, e: int):
+        """Pin object (layer, e): once resident it is never a victim."""
+        limit = self.S - self.C * (2 if self.pin_previous else 1)
+        if (layer, e) not in self.pins and len(self.pins) + 1 > limit:
+            raise ValueError("too many pinned objects")
+        self.pins.add((layer, e))
+
+    def unpin(self, layer: int, e: int):
+        self.pins.discard((layer, e))
 
     def _victim(self, pinned):
-        cands = [s for s in range(self.S) if s not in pinned]
+        cands = [s for s in range(self.S) if s not in pinned and self.obj[s] not in self.pins]
+        if not cands:
+            return None
         vacant = [s for s in cands if self.obj[s] is None]
         if vacant:
             return vacant[0]
         return min(cands, key=lambda s: (self.last_use[s], s))
 
-    def call(self, layer: int, needed) -> list:
-        """Process one layer call; returns the waves as lists of (expert, slot)."""
+    def _load(self, call, layer, e, s, kind, w):
+        if self.obj[s] is not None:
+            ol, oe = self.obj[s]
+            self.trace.append((call, ol, oe, s, self.gen[s], TRACE_EVICT, w))
+            del self.where[self.obj[s]]
+        self.prefetched.discard(s)
+        self.gen[s] += 1
+        self.obj[s] = (layer, e)
+        self.where[(layer, e)] = s
+        self.trace.append((call, layer, e, s, self.gen[s], kind, w))
+
+    def call(self, layer: int, needed, predict=None) -> list:
+        """Process one layer call; returns the waves as lists of (expert, slot).
+
+        predict: None, or (next_layer, counts) with counts[e] the predicted
+        number of token choices of expert e in next_layer."""
         call = self.calls
         self.calls += 1
         needed = sorted(set(int(e) for e in needed))
@@ -346,22 +409,35 @@ class LRUWaveSim:
                 if (layer, e) in self.where:
                     s = self.where[(layer, e)]
                     self.trace.append((call, layer, e, s, self.gen[s], TRACE_HIT, w))
+                    if s in self.prefetched:
+                        self.prefetch_hits += 1
+                        self.prefetched.discard(s)
                 else:
                     s = self._victim((prev if self.pin_previous else set()) | set(cur))
-                    if self.obj[s] is not None:
-                        ol, oe = self.obj[s]
-                        self.trace.append((call, ol, oe, s, self.gen[s], TRACE_EVICT, w))
-                        del self.where[self.obj[s]]
-                    self.gen[s] += 1
-                    self.obj[s] = (layer, e)
-                    self.where[(layer, e)] = s
-                    self.trace.append((call, layer, e, s, self.gen[s], TRACE_STAGE, w))
+                    self._load(call, layer, e, s, TRACE_STAGE, w)
                 cur.append(s)
             for s in cur:                                   # the wave is consumed
                 self.tick += 1
                 self.last_use[s] = self.tick
             out.append(list(zip(wave, cur)))
             prev = set(cur)
+        if predict is not None:                             # the prefetch bank
+            nl, counts = predict
+            cand = [e for e in range(len(counts)) if counts[e] > 0 and (nl, e) not in self.where]
+            cand.sort(key=lambda e: (-int(counts[e]), e))
+            bank = sorted(cand[:self.C])
+            kept = {self.where[(nl, e)] for e in range(len(counts))
+                    if counts[e] > 0 and (nl, e) in self.where}
+            cur = []
+            for e in bank:
+                s = self._victim((prev if self.pin_previous else set()) | kept | set(cur))
+                if s is None:
+                    break
+                self._load(call, nl, e, s, TRACE_PREFETCH, len(waves))
+                self.last_use[s] = self.tick
+                self.prefetched.add(s)
+                cur.append(s)
+            self.prefetches += len(cur)
         return out
 
     def slot_table(self, layer: int, E: int):

@@ -1,6 +1,7 @@
 """Pins of the oracle's slot simulator and generation check: hand-worked
-traces (tests/golden), a textbook OrderedDict LRU in the special case that
-reduces to it, and the reuse / generation invariants."""
+traces (tests/golden, including prediction, two-bank prefetch and pins), a
+textbook OrderedDict LRU in the special case that reduces to it, and the
+reuse / generation / prefetch / pin invariants."""
 import os
 from collections import OrderedDict
 
@@ -20,11 +21,25 @@ def _cases():
             continue
         tok = line.split()
         if tok[0] == "case":
-            cur = {"name": tok[1], "slots": int(tok[2].split("=")[1]), "calls": [], "trace": []}
+            kv = dict(t.split("=") for t in tok[2:])
+            cur = {"name": tok[1], "slots": int(kv["slots"]),
+                   "wave": int(kv["wave"]) if "wave" in kv else None,
+                   "pins": [], "calls": [], "trace": []}
+        elif tok[0] == "pin":
+            kv = dict(t.split("=") for t in tok[1:])
+            cur["pins"].append((int(kv["layer"]), int(kv["expert"])))
         elif tok[0] == "call":
-            layer = int(tok[1].split("=")[1])
-            needed = [int(v) for v in tok[2].split("=")[1].split(",")]
-            cur["calls"].append((layer, needed))
+            kv = dict(t.split("=") for t in tok[1:])
+            needed = [int(v) for v in kv["needed"].split(",")]
+            predict = None
+            if "predict" in kv:
+                nl, items = kv["predict"].split(":")
+                counts = np.zeros(16, dtype=np.int64)
+                for it in items.split(","):
+                    e, n = it.split("*")
+                    counts[int(e)] = int(n)
+                predict = (int(nl), counts)
+            cur["calls"].append((int(kv["layer"]), needed, predict))
         elif tok[0] == "trace":
             pass
         elif tok[0] == "end":
@@ -37,9 +52,11 @@ def _cases():
 
 @pytest.mark.parametrize("case", _cases(), ids=lambda c: c["name"])
 def test_hand_worked_traces(case):
-    sim = oracle.LRUWaveSim(case["slots"])
-    for layer, needed in case["calls"]:
-        sim.call(layer, needed)
+    sim = oracle.LRUWaveSim(case["slots"], case["wave"])
+    for layer, e in case["pins"]:
+        sim.pin(layer, e)
+    for layer, needed, predict in case["calls"]:
+        sim.call(layer, needed, predict)
     assert sim.trace == case["trace"]
 
 
@@ -131,3 +148,81 @@ def test_generation_check_fail_closed():
     assert oracle.generation_check(0, [2, 5, 6], table, exp, obj, gen) == ("not_resident", 6)
     # the lowest failing expert decides
     assert oracle.generation_check(0, [2, 5, 6], t2, exp2, obj, gen) == ("wrong_object", 2)
+
+
+def _decode_like(rng, sim, L, E, steps, k_max, exact):
+    """Calls over layers 0..L-1 per step; each call may predict the next
+    layer (the exact next needed set, or a random one)."""
+    seq = [(l, sorted(set(rng.integers(0, E, size=rng.integers(1, k_max + 1)).tolist())))
+           for _ in range(steps) for l in range(L)]
+    misses_after_exact = 0
+    for i, (layer, needed) in enumerate(seq):
+        predict = None
+        if i + 1 < len(seq) and seq[i + 1][0] == layer + 1:
+            nl, nxt = seq[i + 1]
+            counts = np.zeros(E, dtype=np.int64)
+            pool = nxt if exact else rng.integers(0, E, size=len(nxt)).tolist()
+            for e in pool:
+                counts[e] += 1
+            predict = (nl, counts)
+        n0 = len(sim.trace)
+        sim.call(layer, needed, predict)
+        if i > 0 and seq[i - 1][0] == layer - 1 and exact:
+            misses_after_exact += sum(1 for r in sim.trace[n0:]
+                                      if r[1] == layer and r[5] == oracle.TRACE_STAGE)
+    return seq, misses_after_exact
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_exact_prediction_leaves_no_miss(seed):
+    """With the next call's needed set predicted exactly and at most one wave
+    of it, every need of that call is a hit: the bundle always finds victims
+    (S >= 2C) and never evicts a predicted object already resident."""
+    rng = np.random.default_rng(seed)
+    sim = oracle.LRUWaveSim(8)
+    seq, misses = _decode_like(rng, sim, L=6, E=12, steps=5, k_max=4, exact=True)
+    assert misses == 0
+    n_pref_hits = sum(1 for r in sim.trace if r[5] == oracle.TRACE_PREFETCH)
+    assert sim.prefetches == n_pref_hits == sim.prefetch_hits > 0
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_prefetch_and_pin_invariants(seed):
+    """Random predictions and pins: no pinned object is ever evicted; no
+    prefetch evicts a slot of the call's last wave; prefetching never advances
+    the tick (tick = number of consumptions); a prediction of zero counts
+    leaves the trace of a call without prediction."""
+    rng = np.random.default_rng(100 + seed)
+    S, E, L = 8, 10, 4
+    sim = oracle.LRUWaveSim(S, 2)
+    pins = {(int(rng.integers(0, L)), int(rng.integers(0, E))) for _ in range(3)}
+    for p in pins:
+        sim.pin(*p)
+    with pytest.raises(ValueError):
+        for e in range(E):
+            sim.pin(L, e)  # beyond S - 2C
+    for e in range(E):
+        sim.unpin(L, e)
+    consumed = 0
+    for step in range(6):
+        for layer in range(L):
+            needed = sorted(set(rng.integers(0, E, size=rng.integers(1, 7)).tolist()))
+            counts = np.zeros(E, dtype=np.int64)
+            for e in rng.integers(0, E, size=rng.integers(0, 6)):
+                counts[e] += 1
+            n0 = len(sim.trace)
+            waves = sim.call(layer, needed, ((layer + 1) % L, counts))
+            consumed += len(needed)
+            assert sim.tick == consumed
+            last = {s for _, s in waves[-1]}
+            recs = sim.trace[n0:]
+            for r in recs:
+                if r[5] == oracle.TRACE_EVICT:
+                    assert (r[1], r[2]) not in pins
+                if r[6] == len(waves):
+                    assert r[3] not in last
+    a, b = oracle.LRUWaveSim(S), oracle.LRUWaveSim(S)
+    for layer, needed in [(0, [1, 2, 3]), (1, [2, 5]), (0, [1, 7, 8, 9]), (1, [0])]:
+        a.call(layer, needed)
+        b.call(layer, needed, (layer + 1, np.zeros(E, dtype=np.int64)))
+    assert a.trace == b.trace
