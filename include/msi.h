@@ -64,7 +64,8 @@ typedef enum {
 
 enum { MSI_W_BF16 = 0, MSI_W_Q4G32 = 1 };
 
-enum { MSI_TRACE_HIT = 0, MSI_TRACE_STAGE = 1, MSI_TRACE_EVICT = 2 };
+enum { MSI_TRACE_HIT = 0, MSI_TRACE_STAGE = 1, MSI_TRACE_EVICT = 2,
+       MSI_TRACE_PREFETCH = 3 /* a stage of a predicted object (next-layer prefetch) */ };
 
 /* GPU slot lifecycle states (Sec. "Separate Window and GPU-Slot Lifecycles"). */
 enum {
@@ -147,6 +148,8 @@ typedef struct {
   uint64_t forwards, streamed_forwards, stages, hits, evicts;
   uint64_t h2d_bytes;            /* extent bytes copied window -> slot */
   uint64_t rejections;           /* host prechecks and device checks that failed closed */
+  uint64_t prefetches;           /* objects staged by next-layer prediction (also in stages) */
+  uint64_t prefetch_hits;        /* hits on a prefetched object before its first consumption */
 } msi_counters;
 
 /* Bytes of one expert extent for the given shape and weight type (0 on bad input). */
@@ -233,6 +236,46 @@ msi_status msi_moe_forward_streamed(msi_plan* plan, int layer, const void* hidde
                                     const float* router_w, void* out, const msi_route_event* ev,
                                     void* workspace, size_t workspace_bytes, unsigned flags,
                                     msi_stream compute, msi_stream stage);
+
+/* msi_moe_forward_streamed plus next-layer prediction and a two-bank prefetch
+ * (the paper's protected LRU with two-bank next-layer prefetch, Sec.
+ * "Evaluation", "Cache and storage state"; prediction and pinning share the
+ * slot lifecycle, Sec. "A Shared Cross-Adapter Plan Core").  The call's rows
+ * are also routed through layer + 1's router (`next_router_w`, fp32 [E, H],
+ * device) on a plan-owned side stream while the call's own waves run; the
+ * predicted route event (top-k ids, weights, gap and per-expert counts of
+ * layer + 1 for these rows; same layouts as `ev`, caller-owned device
+ * buffers) is written to `next_ev`.  After the call's last wave is enqueued,
+ * the predicted objects of layer + 1 that are not resident, ranked by
+ * predicted count (descending; ties: lower expert id) and capped at
+ * wave_capacity, are staged on `stage` as one bundle in ascending expert
+ * order: victims by the wave rule, with the slots of the last wave, of the
+ * bundle itself and of every predicted object already resident pinned; the
+ * bundle ends early when no slot is left.  A prefetched object's last-use
+ * tick is the current tick; its stage is traced as MSI_TRACE_PREFETCH with
+ * wave = the call's number of waves.  The prediction changes residency only:
+ * the call's outputs and route event are those of msi_moe_forward_streamed.
+ * A rejected source read in the bundle unwinds that bundle (its slots become
+ * Vacant) and the call still returns MSI_OK: prediction is advisory.
+ * Errors: as msi_moe_forward_streamed, plus MSI_ERR_INVALID_ARG when
+ * layer + 1 >= n_layers, next_router_w or next_ev is NULL, or (T > 0)
+ * next_ev's ids / weights / gap are NULL. */
+msi_status msi_moe_forward_streamed_next(msi_plan* plan, int layer, const void* hidden, int T,
+                                         const float* router_w, void* out,
+                                         const msi_route_event* ev, const float* next_router_w,
+                                         const msi_route_event* next_ev, void* workspace,
+                                         size_t workspace_bytes, unsigned flags,
+                                         msi_stream compute, msi_stream stage);
+
+/* Pin (pinned = 1) or unpin (0) object (layer, expert): once resident, a
+ * pinned object is never chosen as a victim by the plan's waves or prefetch
+ * bundles (msi_slot_stage, where the caller names the slot, is not
+ * affected).  At most n_slots - 2 * wave_capacity objects may be pinned at
+ * once, so every wave and bundle finds victims; the default wave capacity
+ * (n_slots / 2) leaves no room for pins.  Pins survive msi_plan_reset.
+ * Errors: MSI_ERR_INVALID_ARG for a null plan or an index out of range,
+ * MSI_ERR_SLOT_BUSY when the pin limit is reached (nothing changes). */
+msi_status msi_plan_pin(msi_plan* plan, int layer, int expert, int pinned);
 
 /* Wait for the most recent forward of the plan and return its device-side
  * status (an msi_status value; MSI_OK when every needed expert passed the

@@ -143,19 +143,37 @@ class Plan:
         return rc, out, ev
 
     def forward_streamed(self, layer, x, router_w, out=None, ev=None, residual=False, stream=None,
-                         stage_stream=None, check=True, single_cta=False):
+                         stage_stream=None, check=True, single_cta=False, next_router_w=None,
+                         next_ev=None):
+        """Streamed layer forward.  With next_router_w (layer + 1's router), the
+        rows are also routed through it and layer + 1's predicted objects are
+        prefetched after the last wave; the predicted route event is written to
+        next_ev (allocated when None) and returned as ev.next."""
         T = x.shape[0]
         out = torch.empty_like(x) if out is None else out
         ev = RouteEvent(T, self.k, self.E) if ev is None else ev
         ws = self.workspace(T)
-        rc = N.lib().msi_moe_forward_streamed(self.h, layer, _ptr(x), T, _ptr(router_w), _ptr(out),
-                                              ctypes.byref(ev.c), _ptr(ws), ws.numel(),
-                                              _flags(residual, single_cta), _stream(stream),
-                                              _stream(stage_stream))
+        if next_router_w is None:
+            rc = N.lib().msi_moe_forward_streamed(self.h, layer, _ptr(x), T, _ptr(router_w), _ptr(out),
+                                                  ctypes.byref(ev.c), _ptr(ws), ws.numel(),
+                                                  _flags(residual, single_cta), _stream(stream),
+                                                  _stream(stage_stream))
+            where = "msi_moe_forward_streamed"
+        else:
+            next_ev = RouteEvent(T, self.k, self.E) if next_ev is None else next_ev
+            ev.next = next_ev
+            rc = N.lib().msi_moe_forward_streamed_next(
+                self.h, layer, _ptr(x), T, _ptr(router_w), _ptr(out), ctypes.byref(ev.c),
+                _ptr(next_router_w), ctypes.byref(next_ev.c), _ptr(ws), ws.numel(),
+                _flags(residual, single_cta), _stream(stream), _stream(stage_stream))
+            where = "msi_moe_forward_streamed_next"
         if check:
-            N.check(rc, "msi_moe_forward_streamed")
+            N.check(rc, where)
             return out, ev
         return rc, out, ev
+
+    def pin(self, layer: int, expert: int, pinned: bool = True):
+        N.check(N.lib().msi_plan_pin(self.h, layer, expert, int(pinned)), "msi_plan_pin")
 
     def status(self) -> int:
         s = ctypes.c_int()
@@ -169,7 +187,8 @@ class Plan:
         buf = (N.msi_trace_rec * cap)()
         n = ctypes.c_size_t()
         N.check(N.lib().msi_trace_read(self.h, buf, cap, ctypes.byref(n)), "msi_trace_read")
-        kinds = {N.MSI_TRACE_HIT: "hit", N.MSI_TRACE_STAGE: "stage", N.MSI_TRACE_EVICT: "evict"}
+        kinds = {N.MSI_TRACE_HIT: "hit", N.MSI_TRACE_STAGE: "stage", N.MSI_TRACE_EVICT: "evict",
+                 N.MSI_TRACE_PREFETCH: "prefetch"}
         out = [(r.call, r.layer, r.expert, r.slot, int(r.generation), kinds[r.kind], r.wave)
                for r in buf[:n.value]]
         if clear:

@@ -139,6 +139,7 @@ struct Slot {
   int ready = -1;               // event publishing the last stage
   int consumer = -1;            // event of the last consumer
   int64_t last_use = -1;        // LRU tick of the last consumption
+  bool prefetched = false;      // staged by prediction, not yet consumed
 };
 
 struct WaveEntry {
@@ -227,6 +228,14 @@ struct msi_plan {
   // file (src_off[l * E + e]) through its windows instead of host_windows
   msi_source* src = nullptr;
   std::vector<uint64_t> src_off;
+  // next-layer prediction: a plan-owned stream and events (created on first
+  // use) and the predicted counts read back to the host
+  cudaStream_t pred = nullptr;
+  cudaEvent_t ev_pfork = nullptr, ev_pjoin = nullptr;
+  int* h_pred = nullptr;
+  // caller pins by object [L * E]: never a victim of the plan's waves/bundles
+  std::vector<char> pinned_obj;
+  int n_pins = 0;
   std::mutex mu;
 
   explicit msi_plan(int S) : holds(S) {
@@ -312,7 +321,8 @@ void add_trace(msi_plan* p, int call, int layer, int expert, int slot, uint64_t 
 }
 
 // Occupy `s` with (layer, e): records the eviction, bumps the generation.
-void ledger_stage(msi_plan* p, int s, int layer, int e, int call, int wave) {
+void ledger_stage(msi_plan* p, int s, int layer, int e, int call, int wave,
+                  int kind = MSI_TRACE_STAGE) {
   Slot& sl = p->slots[s];
   const int E = p->d.n_experts;
   if (sl.layer >= 0) {
@@ -323,8 +333,9 @@ void ledger_stage(msi_plan* p, int s, int layer, int e, int call, int wave) {
   sl.gen += 1;
   sl.layer = layer;
   sl.expert = e;
+  sl.prefetched = false;
   p->where[(size_t)layer * E + e] = s;
-  add_trace(p, call, layer, e, s, sl.gen, MSI_TRACE_STAGE, wave);
+  add_trace(p, call, layer, e, s, sl.gen, kind, wave);
   p->ctr.stages++;
   p->ctr.h2d_bytes += p->d.extent_bytes;
 }
@@ -338,6 +349,23 @@ void ledger_vacate(msi_plan* p, int s, int call, int wave) {
   p->where[(size_t)sl.layer * p->d.n_experts + sl.expert] = -1;
   p->ctr.evicts++;
   sl.layer = sl.expert = -1;
+  sl.prefetched = false;
+}
+
+// Victim for a miss: the lowest-index vacant slot, else the least-recently
+// used slot (ties: lowest index), among the slots not pinned by the current
+// wave or bundle and not holding a caller-pinned object; -1 when none is left.
+int pick_victim(const msi_plan* p, const std::vector<char>& pinned) {
+  const int S = p->d.n_slots, E = p->d.n_experts;
+  for (int c = 0; c < S; ++c)
+    if (!pinned[c] && p->slots[c].layer < 0) return c;
+  int victim = -1;
+  for (int c = 0; c < S; ++c) {
+    const Slot& sl = p->slots[c];
+    if (pinned[c] || p->pinned_obj[(size_t)sl.layer * E + sl.expert]) continue;
+    if (victim < 0 || sl.last_use < p->slots[victim].last_use) victim = c;
+  }
+  return victim;
 }
 
 // Wait on `stream` for every not-yet-complete event in ids (deduplicated).
@@ -540,6 +568,80 @@ msi_status validate_fwd(msi_plan* p, int layer, const void* x, int T, const floa
   return MSI_OK;
 }
 
+// Router + histogram over the call's rows for router weight `rw`: the route
+// event (ids, weights, gap) and per-expert counts go to `ev`.  first: the
+// forward's own routing (its first kernel clears the status word and writes
+// the shared group; the shared gate is computed, and the side stream may fork
+// after it).  Otherwise a prediction pass: no status reset, no shared group,
+// no gate; it reuses the router scratch of the workspace, so it must be
+// ordered after the forward's own routing and scatter.
+msi_status route_rows(msi_plan* p, FwdCtx& f, const float* rw, const msi_route_event* ev, bool first,
+                      const TableParams& tp, cudaStream_t s) {
+  const auto& d = p->d;
+  const int E = d.n_experts, k = d.top_k, H = d.hidden;
+  void* ws = f.ws;
+  const WsLayout& L = f.L;
+  const int nb = (f.T + L.tm - 1) / L.tm;
+  const float* wsg = first && d.has_shared ? d.shared_gate_w + (size_t)f.layer * H : nullptr;
+  if (tensor_router(d)) {
+    __nv_bfloat16* w3 = at<__nv_bfloat16>(ws, L.w3);
+    LAUNCH(p, MSI_K_ROUTER, s,
+           launch_split3(rw, (long long)E * H, w3, first ? at<int>(ws, L.status) : nullptr,
+                         first && d.has_shared ? at<Group>(ws, L.sh_group) : nullptr,
+                         at<int>(ws, L.sh_total), f.T, tp.shared_slot, s));
+  }
+  // the forward has begun (status cleared, shared group written): the shared
+  // expert may start on the side stream from here
+  if (first && d.has_shared) CK(cudaEventRecord(p->ev_fork, s));
+  if (tensor_router(d)) {
+    __nv_bfloat16* w3 = at<__nv_bfloat16>(ws, L.w3);
+    const int ch = std::min(E, kRouterChunk);
+    CUtensorMap tm_w3;
+    if (!make_tmap(&tm_w3, w3, H, (uint64_t)3 * E, (uint32_t)ch)) return MSI_ERR_CUDA;
+    RouterTcArgs ra{};
+    ra.x = static_cast<const __nv_bfloat16*>(f.x);
+    ra.wsg = wsg;
+    ra.T = f.T;
+    ra.H = H;
+    ra.E = E;
+    ra.k = k;
+    ra.chunk = ch;
+    ra.nchunk = E / ch;
+    ra.kp = std::min(k + 1, ch);
+    int cols = 32;
+    while (cols < ch) cols <<= 1;
+    ra.tmem_cols = cols;
+    ra.cand_v = at<float>(ws, L.cand_v);
+    ra.cand_i = at<int>(ws, L.cand_i);
+    ra.ids = ev->ids;
+    ra.weights = ev->weights;
+    ra.gap = ev->gap;
+    ra.sg = at<float>(ws, L.sg);
+    ra.bcount = at<int>(ws, L.bcount);
+    ra.status = at<int>(ws, L.status);
+    ra.wait_limit = kDeviceWaitCycles;
+    LAUNCH(p, MSI_K_ROUTER, s, launch_router_tc(f.tm_x, tm_w3, ra, s));
+  } else {
+    RouterArgs ra{};
+    ra.x = static_cast<const __nv_bfloat16*>(f.x);
+    ra.wr = rw;
+    ra.wsg = wsg;
+    ra.T = f.T;
+    ra.H = H;
+    ra.E = E;
+    ra.k = k;
+    ra.ids = ev->ids;
+    ra.weights = ev->weights;
+    ra.gap = ev->gap;
+    ra.sg = at<float>(ws, L.sg);
+    ra.bcount = at<int>(ws, L.bcount);
+    LAUNCH(p, MSI_K_ROUTER, s, launch_router(ra, s));
+  }
+  ScanArgs sa{at<int>(ws, L.bcount), nb, E, at<int>(ws, L.bbase), ev->counts};
+  LAUNCH(p, MSI_K_SCAN, s, launch_colscan(sa, s));
+  return MSI_OK;
+}
+
 // Forward begin + router + histogram + permutation.
 msi_status front(msi_plan* p, FwdCtx& f, const TableParams& tp) {
   const auto& d = p->d;
@@ -562,62 +664,8 @@ msi_status front(msi_plan* p, FwdCtx& f, const TableParams& tp) {
   if (d.has_shared) {
     if (!make_tmap(&f.tm_hs, at<char>(ws, L.hs), I, f.T, 128)) return MSI_ERR_CUDA;
   }
-  if (tensor_router(d)) {
-    __nv_bfloat16* w3 = at<__nv_bfloat16>(ws, L.w3);
-    LAUNCH(p, MSI_K_ROUTER, f.cs,
-           launch_split3(f.router_w, (long long)E * H, w3, at<int>(ws, L.status),
-                         d.has_shared ? at<Group>(ws, L.sh_group) : nullptr, at<int>(ws, L.sh_total),
-                         f.T, tp.shared_slot, f.cs));
-  }
-  // the forward has begun (status cleared, shared group written): the shared
-  // expert may start on the side stream from here
-  if (d.has_shared) CK(cudaEventRecord(p->ev_fork, f.cs));
-  if (tensor_router(d)) {
-    __nv_bfloat16* w3 = at<__nv_bfloat16>(ws, L.w3);
-    const int ch = std::min(E, kRouterChunk);
-    CUtensorMap tm_w3;
-    if (!make_tmap(&tm_w3, w3, H, (uint64_t)3 * E, (uint32_t)ch)) return MSI_ERR_CUDA;
-    RouterTcArgs ra{};
-    ra.x = static_cast<const __nv_bfloat16*>(f.x);
-    ra.wsg = d.has_shared ? d.shared_gate_w + (size_t)f.layer * H : nullptr;
-    ra.T = f.T;
-    ra.H = H;
-    ra.E = E;
-    ra.k = k;
-    ra.chunk = ch;
-    ra.nchunk = E / ch;
-    ra.kp = std::min(k + 1, ch);
-    int cols = 32;
-    while (cols < ch) cols <<= 1;
-    ra.tmem_cols = cols;
-    ra.cand_v = at<float>(ws, L.cand_v);
-    ra.cand_i = at<int>(ws, L.cand_i);
-    ra.ids = f.ev->ids;
-    ra.weights = f.ev->weights;
-    ra.gap = f.ev->gap;
-    ra.sg = at<float>(ws, L.sg);
-    ra.bcount = at<int>(ws, L.bcount);
-    ra.status = at<int>(ws, L.status);
-    ra.wait_limit = kDeviceWaitCycles;
-    LAUNCH(p, MSI_K_ROUTER, f.cs, launch_router_tc(f.tm_x, tm_w3, ra, f.cs));
-  } else {
-    RouterArgs ra{};
-    ra.x = static_cast<const __nv_bfloat16*>(f.x);
-    ra.wr = f.router_w;
-    ra.wsg = d.has_shared ? d.shared_gate_w + (size_t)f.layer * H : nullptr;
-    ra.T = f.T;
-    ra.H = H;
-    ra.E = E;
-    ra.k = k;
-    ra.ids = f.ev->ids;
-    ra.weights = f.ev->weights;
-    ra.gap = f.ev->gap;
-    ra.sg = at<float>(ws, L.sg);
-    ra.bcount = at<int>(ws, L.bcount);
-    LAUNCH(p, MSI_K_ROUTER, f.cs, launch_router(ra, f.cs));
-  }
-  ScanArgs sa{at<int>(ws, L.bcount), nb, E, at<int>(ws, L.bbase), f.ev->counts};
-  LAUNCH(p, MSI_K_SCAN, f.cs, launch_colscan(sa, f.cs));
+  msi_status st = route_rows(p, f, f.router_w, f.ev, true, tp, f.cs);
+  if (st != MSI_OK) return st;
   ScatterArgs xa{};
   xa.ids = f.ev->ids;
   xa.counts = f.ev->counts;
@@ -850,6 +898,7 @@ msi_status msi_plan_create(const msi_plan_desc* desc, msi_plan** out) {
   for (size_t i = 0; i < nobj; ++i) p->off[i] = d.extent_off ? d.extent_off[i] : i * d.extent_bytes;
   p->slots.resize(d.n_slots);
   p->where.assign(nobj, -1);
+  p->pinned_obj.assign(nobj, 0);
   auto fail = [&](msi_status s) {
     if (p->d_gen) cudaFree(p->d_gen);
     if (p->h_status) cudaFreeHost(p->h_status);
@@ -901,6 +950,7 @@ msi_status msi_plan_destroy(msi_plan* p) {
     }
     if (p->fwd_ev >= 0) cudaEventSynchronize(p->pool.ev[p->fwd_ev]);
     if (p->side) cudaStreamSynchronize(p->side);
+    if (p->pred) cudaStreamSynchronize(p->pred);
     source_attach(p->src, -1);  // every window copy of this plan has completed
     p->src = nullptr;
     p->timer.destroy();
@@ -911,6 +961,10 @@ msi_status msi_plan_destroy(msi_plan* p) {
     if (p->side) cudaStreamDestroy(p->side);
     if (p->ev_fork) cudaEventDestroy(p->ev_fork);
     if (p->ev_join) cudaEventDestroy(p->ev_join);
+    if (p->pred) cudaStreamDestroy(p->pred);
+    if (p->ev_pfork) cudaEventDestroy(p->ev_pfork);
+    if (p->ev_pjoin) cudaEventDestroy(p->ev_pjoin);
+    if (p->h_pred) cudaFreeHost(p->h_pred);
   }
   delete p;
   return MSI_OK;
@@ -1071,13 +1125,87 @@ msi_status msi_moe_forward(msi_plan* p, int layer, const void* x, int T, const f
   return MSI_OK;
 }
 
-msi_status msi_moe_forward_streamed(msi_plan* p, int layer, const void* x, int T, const float* rw,
-                                    void* out, const msi_route_event* ev, void* ws, size_t ws_bytes,
-                                    unsigned flags, msi_stream compute, msi_stream stage) {
-  if (p == nullptr) return MSI_ERR_INVALID_ARG;
-  std::lock_guard<std::mutex> g(p->mu);
+namespace {
+
+// Plan-owned prediction stream, its fork/join events and the host copy of
+// the predicted counts (created on the first predicting call).
+msi_status prediction_resources(msi_plan* p) {
+  if (p->pred != nullptr) return MSI_OK;
+  cudaError_t e = cudaMallocHost(&p->h_pred, sizeof(int) * p->d.n_experts);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&p->ev_pfork, cudaEventDisableTiming);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&p->ev_pjoin, cudaEventDisableTiming);
+  if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&p->pred, cudaStreamNonBlocking);
+  return e == cudaSuccess ? MSI_OK : cuda_fail(e, "prediction stream");
+}
+
+// The prefetch bundle for layer `nl` after call `call`'s last wave (slots
+// `last`): predicted objects not resident, ranked by predicted count
+// (descending; ties: lower id), at most C, staged in ascending expert order;
+// the last wave's slots, the bundle's own and those of predicted objects
+// already resident are pinned.  A rejected read unwinds the bundle only.
+msi_status prefetch_bundle(msi_plan* p, int nl, int call, int wave, const std::vector<int>& last,
+                           cudaStream_t ss) {
+  const int E = p->d.n_experts;
+  const int* cnt = p->h_pred;
+  std::vector<char> pinned(p->d.n_slots, 0);
+  for (int sl : last) pinned[sl] = 1;
+  std::vector<int> cand;
+  for (int e = 0; e < E; ++e) {
+    if (cnt[e] <= 0) continue;
+    const int r = p->where[(size_t)nl * E + e];
+    if (r >= 0)
+      pinned[r] = 1;
+    else
+      cand.push_back(e);
+  }
+  std::stable_sort(cand.begin(), cand.end(), [&](int a, int b) { return cnt[a] > cnt[b]; });
+  if ((int)cand.size() > p->C) cand.resize(p->C);
+  std::sort(cand.begin(), cand.end());
+  // host windows: a source known to be short is refused before anything is
+  // planned (the bundle is dropped; the call itself is unaffected)
+  for (int e : cand) {
+    if (p->src != nullptr) break;
+    auto f = p->faults.find(obj_key(nl, e));
+    if (f != p->faults.end() && f->second == MSI_FAULT_SHORT_READ) {
+      p->faults.erase(f);
+      p->ctr.rejections++;
+      return MSI_OK;
+    }
+  }
+  std::vector<WaveEntry> bundle;
+  for (int e : cand) {
+    const int sl = pick_victim(p, pinned);
+    if (sl < 0) break;
+    ledger_stage(p, sl, nl, e, call, wave, MSI_TRACE_PREFETCH);
+    p->slots[sl].last_use = p->tick;  // prefetching is not consumption
+    p->slots[sl].prefetched = true;
+    pinned[sl] = 1;
+    p->ctr.prefetches++;
+    bundle.push_back({e, sl, true, p->slots[sl].gen});
+  }
+  if (bundle.empty()) return MSI_OK;
+  const msi_status r = stage_enqueue(p, nl, bundle, ss);
+  if (r == MSI_ERR_SOURCE) {
+    for (const auto& we : bundle) ledger_vacate(p, we.slot, call, wave);
+    return MSI_OK;
+  }
+  return r;
+}
+
+msi_status forward_streamed(msi_plan* p, int layer, const void* x, int T, const float* rw, void* out,
+                            const msi_route_event* ev, const float* next_rw,
+                            const msi_route_event* next_ev, void* ws, size_t ws_bytes,
+                            unsigned flags, msi_stream compute, msi_stream stage) {
   msi_status st = validate_fwd(p, layer, x, T, rw, out, ev, ws, ws_bytes);
   if (st != MSI_OK) return st;
+  const bool predict = next_rw != nullptr;
+  if (predict) {
+    if (layer + 1 >= p->d.n_layers || next_ev == nullptr || next_ev->counts == nullptr ||
+        (T > 0 && (next_ev->ids == nullptr || next_ev->weights == nullptr || next_ev->gap == nullptr)))
+      return MSI_ERR_INVALID_ARG;
+    st = prediction_resources(p);
+    if (st != MSI_OK) return st;
+  }
   const auto& d = p->d;
   const int E = d.n_experts;
   FwdCtx f{};
@@ -1105,6 +1233,21 @@ msi_status msi_moe_forward_streamed(msi_plan* p, int layer, const void* x, int T
   st = p->pool.acquire(&cev);
   if (st != MSI_OK) return st;
   CK(cudaEventRecord(p->pool.ev[cev], f.cs));
+  if (predict) {
+    // layer + 1's router over the same rows, on the prediction stream while
+    // this call's waves run; it reuses the router scratch, so it forks after
+    // the scatter, and the compute stream joins it before the call ends
+    CK(cudaEventRecord(p->ev_pfork, f.cs));
+    CK(cudaStreamWaitEvent(p->pred, p->ev_pfork, 0));
+    if (T == 0) {
+      LAUNCH(p, MSI_K_UPLOAD, p->pred, launch_zero_counts(next_ev->counts, E, p->pred));
+    } else {
+      st = route_rows(p, f, next_rw, next_ev, false, tp, p->pred);
+      if (st != MSI_OK) return st;
+    }
+    CK(cudaMemcpyAsync(p->h_pred, next_ev->counts, sizeof(int) * E, cudaMemcpyDeviceToHost, p->pred));
+    CK(cudaEventRecord(p->ev_pjoin, p->pred));
+  }
   st = shared_ffn(p, f, f.cs);  // overlaps the host planning and the first wave's copies
   if (st != MSI_OK) return st;
   const cudaError_t se = cudaEventSynchronize(p->pool.ev[cev]);
@@ -1147,7 +1290,7 @@ msi_status msi_moe_forward_streamed(msi_plan* p, int layer, const void* x, int T
   std::vector<std::vector<WaveEntry>> waves;
   std::vector<char> pinned(d.n_slots, 0);
   std::vector<int> prev;
-  auto plan_wave = [&]() {
+  auto plan_wave = [&]() -> msi_status {
     const int w = (int)waves.size();
     const size_t w0 = (size_t)w * p->C;
     std::vector<WaveEntry> wave;
@@ -1160,17 +1303,13 @@ msi_status msi_moe_forward_streamed(msi_plan* p, int layer, const void* x, int T
       if (s >= 0) {
         add_trace(p, call, layer, e, s, p->slots[s].gen, MSI_TRACE_HIT, w);
         p->ctr.hits++;
-      } else {
-        int victim = -1;
-        for (int c = 0; c < d.n_slots && victim < 0; ++c)
-          if (!pinned[c] && p->slots[c].layer < 0) victim = c;
-        if (victim < 0) {
-          for (int c = 0; c < d.n_slots; ++c) {
-            if (pinned[c]) continue;
-            if (victim < 0 || p->slots[c].last_use < p->slots[victim].last_use) victim = c;
-          }
+        if (p->slots[s].prefetched) {
+          p->ctr.prefetch_hits++;
+          p->slots[s].prefetched = false;
         }
-        s = victim;
+      } else {
+        s = pick_victim(p, pinned);
+        if (s < 0) return MSI_ERR_SLOT_BUSY;  // excluded by the pin limit
         ledger_stage(p, s, layer, e, call, w);
         miss = true;
       }
@@ -1184,11 +1323,13 @@ msi_status msi_moe_forward_streamed(msi_plan* p, int layer, const void* x, int T
       prev.push_back(we.slot);
     }
     waves.push_back(std::move(wave));
+    return MSI_OK;
   };
 
   // ---- issue: plan + stage(w + 1) overlaps compute(w) ----
   auto stage_wave = [&](size_t w) -> msi_status {
-    plan_wave();
+    const msi_status pw = plan_wave();
+    if (pw != MSI_OK) return pw;
     std::vector<WaveEntry> m;
     for (const auto& we : waves[w])
       if (we.miss) m.push_back(we);
@@ -1245,10 +1386,53 @@ msi_status msi_moe_forward_streamed(msi_plan* p, int layer, const void* x, int T
     st = consumer_record(p, used, f.cs);
     if (st != MSI_OK) return st;
   }
+  if (predict) {
+    // the predicted counts (the prediction ran beside the waves' GEMMs), then
+    // the prefetch bundle on the stage stream, overlapping those GEMMs
+    const cudaError_t pe = cudaEventSynchronize(p->ev_pjoin);
+    if (pe != cudaSuccess) return cuda_fail(pe, "predicted counts readback");
+    st = prefetch_bundle(p, layer + 1, call, (int)n_waves, prev, ss);
+    if (st != MSI_OK) return st;
+    CK(cudaStreamWaitEvent(f.cs, p->ev_pjoin, 0));
+  }
   st = finish(p, f);
   if (st != MSI_OK) return st;
   p->ctr.forwards++;
   p->ctr.streamed_forwards++;
+  return MSI_OK;
+}
+
+}  // namespace
+
+msi_status msi_moe_forward_streamed(msi_plan* p, int layer, const void* x, int T, const float* rw,
+                                    void* out, const msi_route_event* ev, void* ws, size_t ws_bytes,
+                                    unsigned flags, msi_stream compute, msi_stream stage) {
+  if (p == nullptr) return MSI_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> g(p->mu);
+  return forward_streamed(p, layer, x, T, rw, out, ev, nullptr, nullptr, ws, ws_bytes, flags, compute,
+                          stage);
+}
+
+msi_status msi_moe_forward_streamed_next(msi_plan* p, int layer, const void* x, int T, const float* rw,
+                                         void* out, const msi_route_event* ev, const float* next_rw,
+                                         const msi_route_event* next_ev, void* ws, size_t ws_bytes,
+                                         unsigned flags, msi_stream compute, msi_stream stage) {
+  if (p == nullptr || next_rw == nullptr) return MSI_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> g(p->mu);
+  return forward_streamed(p, layer, x, T, rw, out, ev, next_rw, next_ev, ws, ws_bytes, flags, compute,
+                          stage);
+}
+
+msi_status msi_plan_pin(msi_plan* p, int layer, int expert, int pinned) {
+  if (p == nullptr || layer < 0 || expert < 0) return MSI_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> g(p->mu);
+  if (layer >= p->d.n_layers || expert >= p->d.n_experts) return MSI_ERR_INVALID_ARG;
+  char& o = p->pinned_obj[(size_t)layer * p->d.n_experts + expert];
+  const bool on = pinned != 0;
+  if (on == (o != 0)) return MSI_OK;
+  if (on && p->n_pins + 1 > p->d.n_slots - 2 * p->C) return MSI_ERR_SLOT_BUSY;
+  o = on ? 1 : 0;
+  p->n_pins += on ? 1 : -1;
   return MSI_OK;
 }
 
@@ -1289,6 +1473,7 @@ msi_status msi_plan_reset(msi_plan* p, uint64_t* new_epoch) {
     }
     sl.layer = sl.expert = -1;
     sl.last_use = -1;
+    sl.prefetched = false;
     p->pool.unref(sl.ready);
     p->pool.unref(sl.consumer);
     sl.ready = sl.consumer = -1;

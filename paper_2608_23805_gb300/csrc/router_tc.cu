@@ -45,7 +45,7 @@ static_assert(128 * RT_LLD * 4 <= RT_STAGES * RT_STAGE, "logits tile does not fi
 __global__ void split3_kernel(const float* __restrict__ w, long long n, __nv_bfloat16* __restrict__ out,
                               int* status, Group* sh, int* sh_total, int T, int shared_slot) {
   if (blockIdx.x == 0 && threadIdx.x == 0) {  // the forward's first kernel
-    *status = 0;
+    if (status != nullptr) *status = 0;         // (null: a prediction pass)
     if (sh != nullptr) {
       Group g;
       g.row_begin = 0;

@@ -29,7 +29,7 @@ MSI_MAX_WINDOWS = 64
 
 MSI_W_BF16 = 0
 MSI_W_Q4G32 = 1
-MSI_TRACE_HIT, MSI_TRACE_STAGE, MSI_TRACE_EVICT = 0, 1, 2
+MSI_TRACE_HIT, MSI_TRACE_STAGE, MSI_TRACE_EVICT, MSI_TRACE_PREFETCH = 0, 1, 2, 3
 MSI_SLOT_VACANT, MSI_SLOT_LOADING, MSI_SLOT_DEVICE_READY, MSI_SLOT_IN_USE, MSI_SLOT_RECYCLABLE = range(5)
 MSI_FWD_RESIDUAL = 1
 MSI_FWD_SINGLE_CTA = 2
@@ -63,7 +63,7 @@ class msi_trace_rec(ctypes.Structure):
 class msi_counters(ctypes.Structure):
     _fields_ = [(n, ctypes.c_uint64) for n in
                 ("forwards", "streamed_forwards", "stages", "hits", "evicts", "h2d_bytes",
-                 "rejections")]
+                 "rejections", "prefetches", "prefetch_hits")]
 
 
 class msi_source_desc(ctypes.Structure):
@@ -95,6 +95,11 @@ _SIGS = {
     "msi_moe_forward_streamed": (ctypes.c_int, [_P, ctypes.c_int, _P, ctypes.c_int, _P, _P,
                                                 ctypes.POINTER(msi_route_event), _P, ctypes.c_size_t,
                                                 ctypes.c_uint, _P, _P]),
+    "msi_moe_forward_streamed_next": (ctypes.c_int, [_P, ctypes.c_int, _P, ctypes.c_int, _P, _P,
+                                                     ctypes.POINTER(msi_route_event), _P,
+                                                     ctypes.POINTER(msi_route_event), _P,
+                                                     ctypes.c_size_t, ctypes.c_uint, _P, _P]),
+    "msi_plan_pin": (ctypes.c_int, [_P, ctypes.c_int, ctypes.c_int, ctypes.c_int]),
     "msi_moe_forward_static": (ctypes.c_int, [_P, ctypes.c_int, _P, ctypes.c_int, _P, _P, _P, _P,
                                               ctypes.POINTER(msi_route_event), ctypes.c_uint, _P]),
     "msi_forward_status": (ctypes.c_int, [_P, ctypes.POINTER(ctypes.c_int)]),

@@ -44,7 +44,29 @@ def test_host_only_entry_points(lib):
     assert l.msi_kernel_launches(None) == 0
 
 
-def test_struct_layouts_match_header():
-    assert ctypes.sizeof(N.msi_trace_rec) == 40
-    assert ctypes.sizeof(N.msi_route_event) == 32
-    assert ctypes.sizeof(N.msi_counters) == 56
+STRUCTS = ["msi_plan_desc", "msi_route_event", "msi_trace_rec", "msi_counters", "msi_source_desc",
+           "msi_source_stats"]
+
+
+def test_struct_layouts_match_header(tmp_path):
+    """Sizes and field offsets of the binding's structures equal those the C
+    compiler gives the header's."""
+    src = tmp_path / "layout.c"
+    lines = ['#include <stdio.h>', '#include <stddef.h>', '#include "msi.h"', "int main(void) {"]
+    for name in STRUCTS:
+        lines.append('printf("%s %%zu\\n", sizeof(%s));' % (name, name))
+        for f, _ in getattr(N, name)._fields_:
+            lines.append('printf("%s.%s %%zu\\n", offsetof(%s, %s));' % (name, f, name, f))
+    lines.append("return 0; }")
+    src.write_text("\n".join(lines))
+    exe = tmp_path / "layout"
+    import subprocess
+    subprocess.run(["gcc", "-std=c11", "-I", os.path.dirname(HEADER), str(src), "-o", str(exe)],
+                   check=True)
+    got = dict(l.split() for l in subprocess.run([str(exe)], capture_output=True, text=True,
+                                                 check=True).stdout.splitlines())
+    for name in STRUCTS:
+        st = getattr(N, name)
+        assert ctypes.sizeof(st) == int(got[name]), name
+        for f, _ in st._fields_:
+            assert getattr(st, f).offset == int(got[name + "." + f]), (name, f)
