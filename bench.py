@@ -10,7 +10,12 @@ Default workload: the Qwen3-Next-shaped layer (hidden 2048, 512 experts,
 top-10, intermediate 512, shared expert) over 4,096 tokens with all 512
 experts resident in slots.  --workload prefill32k_lru64 runs the same layer
 at 32,768 tokens with a 64-slot pool: 448 of the 512 experts are staged from
-pinned host windows per call in LRU waves.
+pinned host windows per call in LRU waves.  --workload decode48 runs one
+decode step through a stack of 48 layers of the tiny shape (hidden 256, 16
+experts, top-2, intermediate 128) over --batch rows, one 64-slot LRU pool
+shared by the 768 objects; --predict adds next-layer prediction with the
+two-bank prefetch (each call routes its rows through the next layer's router
+and stages the predicted objects after its last wave).
 
 Prints one JSON line (rank 0).  `value` is whole-job tokens/s over the timed
 steps (device time, CUDA events on the compute stream); `e2e` repeats the
@@ -37,6 +42,7 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "MoE-layer prefill tokens/s"
+METRIC_DECODE = "MoE decode tokens/s through a 48-layer stack"
 PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
                   "sm_max_mhz": 2070.0}
 N_SMS = 152
@@ -168,18 +174,26 @@ class ClockSampler:
 # ---------------------------------------------------------------------------
 
 class Workload:
-    def __init__(self, name: str):
+    def __init__(self, name: str, batch: int | None = None, predict: bool = False):
         import torch
 
         import synth
         from paper_2608_23805_gb300 import api
-        self.cfg = cfg = synth.config(name)
+        cfg = synth.config(name)
+        if batch is not None and cfg.n_layers > 1:
+            cfg = synth.config(name, tokens=batch)
+        self.cfg = cfg
         self.name = name
+        self.L = L = cfg.n_layers
+        self.predict = predict and L > 1
         E, H, I, eb = cfg.n_experts, cfg.hidden, cfg.inter, cfg.extent_bytes
-        self.windows = torch.empty(E * eb, dtype=torch.uint8, pin_memory=True)
-        synth.fill_extents(cfg, 0, self.windows.numpy())
-        self.router_np = synth.router_weight(cfg)
-        self.router = torch.from_numpy(self.router_np).cuda()
+        self.windows = torch.empty(L * E * eb, dtype=torch.uint8, pin_memory=True)
+        wnp = self.windows.numpy()
+        for l in range(L):
+            synth.fill_extents(cfg, l, wnp[l * E * eb:(l + 1) * E * eb])
+        self.routers_np = [synth.router_weight(cfg, l) for l in range(L)]
+        self.routers = [torch.from_numpy(w).cuda() for w in self.routers_np]
+        self.router_np, self.router = self.routers_np[0], self.routers[0]
         self.x_bits = synth.hidden(cfg)
         self.x_host = torch.from_numpy(self.x_bits.view(np.int16)).view(torch.bfloat16).pin_memory()
         self.x = self.x_host.cuda()
@@ -190,7 +204,7 @@ class Workload:
             self.gate_np = synth.shared_gate_weight(cfg)
             shared_w = torch.from_numpy(self.shared_np).cuda()
             gate_w = torch.from_numpy(self.gate_np[None, :].copy()).cuda()
-        self.plan = api.Plan(n_layers=1, n_experts=E, top_k=cfg.top_k, hidden=H, inter=I,
+        self.plan = api.Plan(n_layers=L, n_experts=E, top_k=cfg.top_k, hidden=H, inter=I,
                              n_slots=cfg.n_slots, host_windows=self.windows,
                              has_shared=cfg.has_shared, shared_w=shared_w, shared_gate_w=gate_w,
                              wdtype=cfg.wdtype)
@@ -198,6 +212,11 @@ class Workload:
         self.ss = torch.cuda.Stream()
         self.out = torch.empty_like(self.x)
         self.ev = api.RouteEvent(cfg.tokens, cfg.top_k, E)
+        if L > 1:  # a layer stack: outputs alternate between two buffers
+            self.outs = [self.out, torch.empty_like(self.x)]
+            self.evs = [api.RouteEvent(cfg.tokens, cfg.top_k, E) for _ in range(L)]
+            self.nevs = [api.RouteEvent(cfg.tokens, cfg.top_k, E) for _ in range(L)]
+            self.out, self.ev = self.outs[(L - 1) % 2], self.evs[L - 1]
         self.table = self.gens = None
         if not cfg.lru:
             for e in range(E):
@@ -207,6 +226,16 @@ class Workload:
 
     def step(self, x=None):
         x = self.x if x is None else x
+        if self.L > 1:
+            for l in range(self.L):
+                nxt = self.routers[l + 1] if self.predict and l + 1 < self.L else None
+                out = self.outs[l % 2]
+                self.plan.forward_streamed(l, x, self.routers[l], out=out, ev=self.evs[l],
+                                           residual=True, stream=self.cs, stage_stream=self.ss,
+                                           next_router_w=nxt, next_ev=self.nevs[l] if nxt is not None
+                                           else None)
+                x = out
+            return
         if self.cfg.lru:
             self.plan.forward_streamed(0, x, self.router, out=self.out, ev=self.ev, stream=self.cs,
                                        stage_stream=self.ss)
@@ -288,6 +317,14 @@ def cpu_baseline(w: "Workload", tokens: int):
     kw = {}
     if cfg.has_shared:
         kw = dict(shared_extent=w.shared_np, w_sg=w.gate_np)
+    if w.L > 1:
+        dt = oracle_stack(cfg, w.x_bits[:tokens], w.routers_np, wnp)
+        cores = int(os.environ.get("OMP_NUM_THREADS", os.environ.get("OPENBLAS_NUM_THREADS",
+                                                                     os.cpu_count() or 1)))
+        return {"value": tokens / dt, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                "sample": "fp64 oracle of one decode step of %d rows through all %d layers (router, "
+                          "expert FFNs, combine with residual, LRU-wave plan of the shared pool), "
+                          "%.2f s" % (tokens, w.L, dt)}
     t0 = time.perf_counter()
     oracle.moe_layer(w.x_bits[:tokens], w.router_np, cfg.top_k, lambda e: wnp[e * eb:(e + 1) * eb],
                      cfg.hidden, cfg.inter, cfg.wdtype, **kw)
@@ -300,6 +337,26 @@ def cpu_baseline(w: "Workload", tokens: int):
             "sample": "fp64 oracle forward of the first %d of %d tokens (router over all %d experts, "
                       "expert FFNs, shared expert, combine, LRU-wave plan), %.1f s" %
                       (tokens, cfg.tokens, cfg.n_experts, dt)}
+
+
+def oracle_stack(cfg, x_bits, routers_np, wnp) -> float:
+    """Seconds the fp64 oracle takes for one decode step through the layer
+    stack (each layer's output rounded to bf16 for the next, as the GPU
+    stack does; the LRU-wave plan of the shared pool alongside)."""
+    import torch
+
+    import oracle
+    E, eb = cfg.n_experts, cfg.extent_bytes
+    sim = oracle.LRUWaveSim(cfg.n_slots)
+    t0 = time.perf_counter()
+    x = x_bits
+    for l, wr in enumerate(routers_np):
+        r = oracle.moe_layer(x, wr, cfg.top_k,
+                             lambda e, l=l: wnp[(l * E + e) * eb:(l * E + e + 1) * eb],
+                             cfg.hidden, cfg.inter, cfg.wdtype, residual=True)
+        sim.call(l, sorted(set(r["ids"].reshape(-1).tolist())))
+        x = torch.from_numpy(r["out"]).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    return time.perf_counter() - t0
 
 
 SAMPLE_TOKENS = {"prefill32k_lru64": 4096, "prefill32k_q4_lru64": 4096, "qwen3next_4k": 4096,
@@ -323,7 +380,7 @@ def run_ours(args):
         torch.cuda.set_device(0)
     import __graft_entry__
     __graft_entry__.build()
-    w = Workload(args.workload)
+    w = Workload(args.workload, args.batch, args.predict)
     cfg = w.cfg
     src = None
     if args.source != "none":
@@ -335,7 +392,7 @@ def run_ours(args):
             f.write(w.windows.numpy().tobytes())
         src = api.Source(path, cfg.extent_bytes + 2 * 4096, n_windows=8, direct=args.source == "direct")
         os.unlink(path)  # the open file stays readable
-        w.plan.set_source(src, np.arange(cfg.n_experts, dtype=np.uint64) * cfg.extent_bytes)
+        w.plan.set_source(src, np.arange(w.L * cfg.n_experts, dtype=np.uint64) * cfg.extent_bytes)
     peaks, peak_kind = load_peaks()
 
     flush = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device="cuda")
@@ -411,10 +468,11 @@ def run_ours(args):
     e2e_value, _ = aggregate(units, e2e_s, world, backend)
     if rank != 0:
         return
-    rl = roofline(cfg, {k: v for k, v in kt.items() if v[1] > 0}, args.steps, peaks, clocks,
+    rl = roofline(cfg, {k: v for k, v in kt.items() if v[1] > 0}, args.steps * w.L, peaks, clocks,
                   args.workload)
     line = {
-        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+        "metric": METRIC if w.L == 1 else METRIC_DECODE, "value": value, "unit": "tokens/s",
+        "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": tmax / args.steps * 1e3, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic: seeded N(0,1) bf16 hidden rows, N(0,0.02) bf16 expert weights, "
@@ -424,6 +482,7 @@ def run_ours(args):
                    "shared_expert": cfg.has_shared, "slots": cfg.n_slots,
                    "residency": "LRU waves of %d, staged from pinned host windows" % (cfg.n_slots // 2)
                    if cfg.lru else "all experts resident",
+                   "layers": w.L,
                    "weights": "bf16" if cfg.wdtype == 0 else "q4g32",
                    "parallelism": "replicas" if world > 1 else "single GPU",
                    "l2": "flushed between timed steps (2x L2 write, untimed)"},
@@ -448,8 +507,17 @@ def run_ours(args):
             "max_in_flight": ss["max_in_flight"]}
         line["config"]["residency"] = "LRU waves of %d, staged from a file through the bounded " \
             "source service (%s reads)" % (cfg.n_slots // 2, args.source)
+    if w.L > 1:
+        c = w.plan.counters()
+        line["config"]["residency"] = (
+            "one %d-slot LRU pool shared by %d layers (%d objects), waves of %d, staged from pinned "
+            "host windows%s" % (cfg.n_slots, w.L, w.L * cfg.n_experts, cfg.n_slots // 2,
+                                "; next-layer prediction with two-bank prefetch" if w.predict else ""))
+        line["config"]["prediction"] = {"on": w.predict, "prefetches": c["prefetches"],
+                                        "prefetch_hits": c["prefetch_hits"], "stages": c["stages"],
+                                        "hits": c["hits"]}
     if world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(w, SAMPLE_TOKENS.get(args.workload, 256))
+        line["cpu_baseline"] = cpu_baseline(w, SAMPLE_TOKENS.get(args.workload, cfg.tokens))
     print(json.dumps(line), flush=True)
 
 
@@ -462,6 +530,32 @@ def run_reference(args):
     import oracle
     import synth
     cfg = synth.config(args.workload)
+    if cfg.n_layers > 1:
+        cfg = synth.config(args.workload, tokens=args.batch)
+        E, eb = cfg.n_experts, cfg.extent_bytes
+        wnp = np.empty(cfg.n_layers * E * eb, dtype=np.uint8)
+        for l in range(cfg.n_layers):
+            synth.fill_extents(cfg, l, wnp[l * E * eb:(l + 1) * E * eb])
+        routers = [synth.router_weight(cfg, l) for l in range(cfg.n_layers)]
+        x = synth.hidden(cfg)
+        for _ in range(args.warmup):
+            oracle_stack(cfg, x, routers, wnp)
+        dt = sum(oracle_stack(cfg, x, routers, wnp) for _ in range(args.steps))
+        value = cfg.tokens * args.steps / dt
+        sample = ("fp64 oracle of one decode step of %d rows through all %d layers per step"
+                  % (cfg.tokens, cfg.n_layers))
+        print(json.dumps({
+            "impl": "reference", "metric": METRIC_DECODE, "value": value, "unit": "tokens/s",
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": dt / args.steps * 1e3, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic (same seeded inputs)",
+            "config": {"workload": args.workload, "tokens": cfg.tokens, "layers": cfg.n_layers},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": os.cpu_count() or 1,
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0},
+        }), flush=True)
+        return
     ntok = REF_TOKENS.get(args.workload, 128)
     eb = cfg.extent_bytes
     x = synth.hidden(cfg, tokens=ntok)
@@ -515,7 +609,11 @@ def main():
     ap.add_argument("--steps", type=int, default=10)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--workload", default="qwen3next_4k",
-                    choices=["qwen3next_4k", "prefill32k_lru64", "prefill32k_q4_lru64", "tiny"])
+                    choices=["qwen3next_4k", "prefill32k_lru64", "prefill32k_q4_lru64", "tiny",
+                             "decode48"])
+    ap.add_argument("--batch", type=int, default=64, help="decode48: rows per decode step")
+    ap.add_argument("--predict", action="store_true",
+                    help="decode48: next-layer prediction with the two-bank prefetch")
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--source", default="none", choices=["none", "buffered", "direct"],
