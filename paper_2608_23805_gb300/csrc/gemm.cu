@@ -43,7 +43,7 @@ constexpr int kGatherWarps = 4;
 constexpr uint32_t kIdesc = idesc_bf16(kBM, kBN);
 
 constexpr int kDqWarps = 8;   // one thread per B row (256 rows)
-constexpr int kRawRowBytes = 32;  // 64 codes of one B row per stage
+constexpr int kRawRowBytes = 32;  // 64 codes of one B row per stage (one TMA box row)
 
 template <int MODE>
 struct Cfg {
@@ -59,12 +59,12 @@ struct Cfg {
   static constexpr uint32_t kTxBytes = (kTmaB ? kBBytes : 0) + (kTmaA ? kABytes : 0);
   // gather threads arrive one by one as their copies land (cp.async ... arrive.noinc)
   static constexpr int kFullCount = (kTmaAny ? 1 : 0) + (kGather ? kGatherWarps * 32 : 0) + (kQ4 ? kDqWarps : 0);
-  // operand ring depth and, in the q4 modes, the raw (packed) stages in flight
-  // ahead of the conversion (eight raw stages in a three-stage operand ring
-  // measured no faster)
+  // operand ring depth and, in the q4 modes, the ring of packed code stages
+  // that the producer fills by TMA ahead of the conversion
   static constexpr int kStg = kStages;
   static constexpr int kRaw = kQ4 ? 3 : 1;
-  static constexpr int kRawBytes = kQ4 ? kRaw * kBN * (kRawRowBytes + 4) : 0;
+  static constexpr int kRawBytes = kQ4 ? kRaw * kBN * kRawRowBytes : 0;
+  static constexpr uint32_t kRawTx = kBN * kRawRowBytes;
   // bf16 modes stage each epilogue warp's rows in shared memory (4 KB per
   // warp) for row-coalesced stores; the q4 raw ring leaves no room for it
   static constexpr bool kStagedEpi = !kQ4;
@@ -104,24 +104,23 @@ __device__ __forceinline__ uint64_t f32x2(float lo, float hi) {
 
 // Eight 4-bit codes of one 32-bit word (code 2i in the low nibble of byte i,
 // code 2i+1 in its high nibble) -> eight bf16 weights scale * (q - 8), the
-// 16-byte chunk of one K-major row.  Each code becomes the float 2^23 + q by
-// placing its byte under the exponent byte 0x4B (one byte permute); then
-// (2^23 + q) - (2^23 + 8) = q - 8 and the product with the fp16-exact scale
-// are exact in fp32, two values per instruction, and each weight is rounded
-// once to bf16.
-__device__ __forceinline__ uint4 dequant8(uint32_t w, uint64_t scale2) {
+// 16-byte chunk of one K-major row.  Each code becomes the float 128 + q by
+// placing its byte under the exponent byte 0x43 (one byte permute; q < 16
+// fills the top mantissa bits); one fused multiply-add per two values then
+// gives (128 + q) * s - 136 * s = (q - 8) * s exactly (the product needs at
+// most 8 + 11 bits and the fp16-exact scale times 136 is exact in fp32), and
+// each weight is rounded once to bf16.  nbias2 holds -136 * s twice.
+__device__ __forceinline__ uint4 dequant8(uint32_t w, uint64_t scale2, uint64_t nbias2) {
   const uint32_t lo = w & 0x0F0F0F0Fu, hi = (w >> 4) & 0x0F0F0F0Fu;
-  const uint64_t bias2 = 0x4B0000084B000008ull;  // (2^23 + 8, 2^23 + 8)
   uint32_t o[4];
 #pragma unroll
   for (int b = 0; b < 4; ++b) {
     uint32_t el, eh;
-    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(el) : "r"(lo), "r"(0x4B000000u), "r"(0x7440u + b));
-    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(eh) : "r"(hi), "r"(0x4B000000u), "r"(0x7440u + b));
+    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(el) : "r"(lo), "r"(0x43000000u), "r"(0x7044u + (b << 8)));
+    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(eh) : "r"(hi), "r"(0x43000000u), "r"(0x7044u + (b << 8)));
     uint64_t v;
     asm("mov.b64 %0, {%1, %2};" : "=l"(v) : "r"(el), "r"(eh));
-    asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(v) : "l"(v), "l"(bias2));
-    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(v) : "l"(v), "l"(scale2));
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(v) : "l"(v), "l"(scale2), "l"(nbias2));
     uint32_t vl, vh;
     asm("mov.b64 {%0, %1}, %2;" : "=r"(vl), "=r"(vh) : "l"(v));
     // the first operand lands in the upper half: (odd column, even column)
@@ -143,13 +142,14 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
   uint8_t* sA = smem;
   uint8_t* sB = smem + C::kStg * kABytes;
   uint8_t* raw_codes = sB + C::kStg * kBBytes;                    // q4: [C::kRaw][256][32]
-  uint32_t* raw_scales = reinterpret_cast<uint32_t*>(raw_codes + (C::kQ4 ? C::kRaw * kBN * kRawRowBytes : 0));
   uint64_t* full = reinterpret_cast<uint64_t*>(raw_codes + C::kRawBytes);
   uint64_t* empty = full + C::kStg;
   uint64_t* tfull = empty + C::kStg;
   uint64_t* tempty = tfull + 2;
   uint64_t* drain = tempty + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  uint64_t* raw_full = drain + 1;           // q4: code stage landed (TMA bytes)
+  uint64_t* raw_empty = raw_full + C::kRaw;  // q4: code stage converted by every dequant warp
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(raw_empty + C::kRaw);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   uint8_t* epi_stage = reinterpret_cast<uint8_t*>(full) + 256;  // kEpiWarps x 4 KB (bf16 modes)
   // group table after the epilogue staging (bf16 modes) or the barriers (q4)
@@ -170,6 +170,10 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
       mbar_init(&tempty[b], kEpiWarps);
     }
     mbar_init(drain, 1);
+    for (int r = 0; r < C::kRaw && C::kQ4; ++r) {
+      mbar_init(&raw_full[r], 1);
+      mbar_init(&raw_empty[r], kDqWarps);
+    }
     *abort_flag = 0;
     mbar_fence_init();
   }
@@ -178,7 +182,7 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
     tmem_relinquish();
   }
   if (warp == 5 && lane == 0) {
-    if (C::kTmaB) tma_prefetch(&tmB);
+    if (C::kTmaB || C::kQ4) tma_prefetch(&tmB);
     if (C::kTmaA) tma_prefetch(&tmA);
   }
   for (int g = threadIdx.x; g < a.num_groups; g += blockDim.x) {
@@ -195,8 +199,8 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
 
   if (warp == 5) {
     // ------------------------------------------------------------- TMA producer
-    if (lane == 0 && C::kTmaAny) {
-      uint32_t it = 0;
+    if (lane == 0 && (C::kTmaAny || C::kQ4)) {
+      uint32_t it = 0, raw_issued = 0;
       // the next tile's first A row is loaded one tile ahead (its latency
       // hides behind this tile's stages instead of stalling the ring)
       int rb_next = blockIdx.x < total ? __ldg(&a.groups[decode_tile(a, s_mt, blockIdx.x).g].row_begin) : 0;
@@ -204,10 +208,25 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
         const TileCoord tc = decode_tile(a, s_mt, t);
         const int brow = s_slot[tc.g] * a.b_rows_per_slot + a.b_row_off;
         const int arow = rb_next + tc.m * kBM;
+        // q4: the tile's two 128-row blocks of packed codes (gate: n * 128 and
+        // up: up_off + n * 128; down: n * 256 and n * 256 + 128)
+        const int qbase = s_slot[tc.g] * a.q4_rows_per_slot + a.q4_row_off;
+        const int qrow0 = qbase + (C::kGateUp ? tc.n * 128 : tc.n * kBN);
+        const int qrow1 = C::kGateUp ? qbase + a.up_off + tc.n * 128 : qrow0 + 128;
         if (t + (int)gridDim.x < total)
           rb_next = __ldg(&a.groups[decode_tile(a, s_mt, t + gridDim.x).g].row_begin);
         bool ok = true;
         for (int kb = 0; kb < a.kblocks; ++kb, ++it) {
+          if (C::kQ4) {
+            const int r = it % C::kRaw;
+            if (!mbar_wait(&raw_empty[r], ((it / C::kRaw) & 1) ^ 1, abort_flag, lim)) { ok = false; break; }
+            mbar_arrive_expect_tx(&raw_full[r], C::kRawTx);
+            uint8_t* q = raw_codes + r * (kBN * kRawRowBytes);
+            tma_load_2d(q, &tmB, &raw_full[r], kb * kRawRowBytes, qrow0);
+            tma_load_2d(q + 128 * kRawRowBytes, &tmB, &raw_full[r], kb * kRawRowBytes, qrow1);
+            ++raw_issued;
+            if (!C::kTmaAny) continue;
+          }
           const int s = it % C::kStg;
           const uint32_t ph = (it / C::kStg) & 1;
           if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, lim)) { ok = false; break; }
@@ -227,11 +246,18 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
       // On abort, wait (bounded) for the copies this thread armed to land
       // before the CTA's shared memory is released.
       if (*abort_flag) {
-        for (int d = 0; d < C::kStg && it > 0; ++d) {
+        for (int d = 0; d < C::kStg && it > 0 && C::kTmaAny; ++d) {
           const uint32_t j = it - 1 - d;
           if ((int)j < 0) break;
           const long long t0 = clock64();
           while (!mbar_try_wait(&full[j % C::kStg], (j / C::kStg) & 1) && clock64() - t0 < lim) {
+          }
+        }
+        for (int d = 0; d < C::kRaw && C::kQ4; ++d) {
+          if ((int)raw_issued - 1 - d < 0) break;
+          const uint32_t j = raw_issued - 1 - d;
+          const long long t0 = clock64();
+          while (!mbar_try_wait(&raw_full[j % C::kRaw], (j / C::kRaw) & 1) && clock64() - t0 < lim) {
           }
         }
       }
@@ -361,70 +387,65 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
     const uint32_t my_tiles =
         (uint32_t)blockIdx.x < (uint32_t)total ? (total - 1 - blockIdx.x) / gridDim.x + 1 : 0;
     const uint32_t nstages = my_tiles * a.kblocks;
-    // tile lookups from the shared-memory group table: a search in global
-    // memory here would stall this row's whole pipeline once per tile
-    const uint8_t* code_row = nullptr;
-    const uint8_t* scale_row = nullptr;
-    auto rows_of = [&](int t) {  // this thread's code and scale rows of tile t
-      int lo = 0, hi = a.num_groups - 1;
-      while (lo < hi) {
-        const int mid = (lo + hi + 1) >> 1;
-        if (s_mt[mid] * a.nt <= t) lo = mid; else hi = mid - 1;
+    // this thread's scale row for tile ordinal j, from the shared-memory group
+    // table (a search in global memory would stall the row's pipeline)
+    uint32_t srow_tile = 0xFFFFFFFFu;
+    const uint8_t* srow = nullptr;
+    auto scales_of = [&](uint32_t st) -> uint2 {  // the two stages st, st + 1 (st even)
+      const uint32_t j = st / a.kblocks;
+      if (j != srow_tile) {
+        const int t = blockIdx.x + j * gridDim.x;
+        int lo = 0, hi = a.num_groups - 1;
+        while (lo < hi) {
+          const int mid = (lo + hi + 1) >> 1;
+          if (s_mt[mid] * a.nt <= t) lo = mid; else hi = mid - 1;
+        }
+        const int mt = s_mt[lo + 1] - s_mt[lo];
+        const int n = (t - s_mt[lo] * a.nt) / mt;
+        int row;
+        if (C::kGateUp) row = d < 128 ? n * 128 + d : a.up_off + n * 128 + (d - 128);
+        else row = n * kBN + d;
+        srow = a.q4_pool + (unsigned long long)s_slot[lo] * a.q4_extent + a.q4_scale_off +
+               (size_t)row * a.q4_scale_ld;
+        srow_tile = j;
       }
-      const int mt = s_mt[lo + 1] - s_mt[lo];
-      const int n = (t - s_mt[lo] * a.nt) / mt;
-      const uint8_t* base = a.q4_pool + (unsigned long long)s_slot[lo] * a.q4_extent;
-      int row;
-      if (C::kGateUp) row = d < 128 ? n * 128 + d : a.up_off + n * 128 + (d - 128);
-      else row = n * kBN + d;
-      code_row = base + a.q4_code_off + (size_t)row * a.q4_code_ld;
-      scale_row = base + a.q4_scale_off + (size_t)row * a.q4_scale_ld;
+      // 4 fp16 scales, 8-byte aligned (row stride K / 16 bytes, K a multiple of 128)
+      return __ldg(reinterpret_cast<const uint2*>(srow + (st % a.kblocks) * 4));
     };
-    // prefetch cursor (tile ordinal, k block) of the next raw stage
-    uint32_t jp = 0, p_tile = 0;
-    int p_kb = 0;
-    if (my_tiles > 0) rows_of(blockIdx.x);
-    auto issue = [&](uint32_t j) {
-      const int r = j % C::kRaw;
-      uint8_t* dst = raw_codes + (r * kBN + d) * kRawRowBytes;
-      cp_async16(dst, code_row + p_kb * 32, 16u);
-      cp_async16(dst + 16, code_row + p_kb * 32 + 16, 16u);
-      cp_async4(&raw_scales[r * kBN + d], scale_row + p_kb * 4);
-      if (++p_kb == a.kblocks) {
-        p_kb = 0;
-        if (++p_tile < my_tiles) rows_of(blockIdx.x + p_tile * gridDim.x);
-      }
-    };
-    for (int i = 0; i < C::kRaw - 1; ++i, ++jp) {
-      if (jp < nstages) issue(jp);
-      cp_async_commit();
-    }
+    // scales of a stage pair are loaded one pair ahead (kblocks is even)
+    uint2 sc_cur = nstages > 0 ? scales_of(0) : make_uint2(0, 0);
+    uint2 sc_nxt = nstages > 2 ? scales_of(2) : make_uint2(0, 0);
     bool ok = true;
-    for (uint32_t it = 0; it < nstages; ++it, ++jp) {
-      if (jp < nstages) issue(jp);
-      cp_async_commit();
-      cp_async_wait<C::kRaw - 1>();  // this thread's raw stage `it` has landed
+    for (uint32_t it = 0; it < nstages; ++it) {
+      if (it > 0 && (it & 1) == 0) {
+        sc_cur = sc_nxt;
+        if (it + 2 < nstages) sc_nxt = scales_of(it + 2);
+      }
+      const int r = it % C::kRaw;
+      if (!mbar_wait(&raw_full[r], (it / C::kRaw) & 1, abort_flag, lim)) { ok = false; break; }
       const int s = it % C::kStg;
       const uint32_t ph = (it / C::kStg) & 1;
       if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, lim)) { ok = false; break; }
-      const int r = it % C::kRaw;
-      const uint4* rc = reinterpret_cast<const uint4*>(raw_codes + (r * kBN + d) * kRawRowBytes);
+      const uint4* rc = reinterpret_cast<const uint4*>(raw_codes + r * (kBN * kRawRowBytes) + d * kRawRowBytes);
       const uint4 c0 = rc[0], c1 = rc[1];
-      const uint32_t sc = raw_scales[r * kBN + d];
+      const uint32_t sc = (it & 1) ? sc_cur.y : sc_cur.x;
       const float s0 = __half2float(__ushort_as_half((unsigned short)(sc & 0xFFFFu)));
       const float s1 = __half2float(__ushort_as_half((unsigned short)(sc >> 16)));
       uint8_t* dst_row = sB + s * kBBytes + d * 128;
       const uint32_t words[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
       const uint64_t s0x2 = f32x2(s0, s0), s1x2 = f32x2(s1, s1);
+      const uint64_t n0x2 = f32x2(-136.0f * s0, -136.0f * s0), n1x2 = f32x2(-136.0f * s1, -136.0f * s1);
 #pragma unroll
       for (int c = 0; c < 8; ++c)
         *reinterpret_cast<uint4*>(dst_row + ((c ^ (d & 7)) << 4)) =
-            dequant8(words[c], c < 4 ? s0x2 : s1x2);
+            dequant8(words[c], c < 4 ? s0x2 : s1x2, c < 4 ? n0x2 : n1x2);
       fence_proxy_async_smem();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&full[s]);
+      if (lane == 0) {
+        mbar_arrive(&full[s]);
+        mbar_arrive(&raw_empty[r]);  // the warp's rows of this code stage are consumed
+      }
     }
-    cp_async_wait<0>();
     (void)ok;
   }
 

@@ -178,8 +178,8 @@ struct GemmArgs {
   // 4-bit weights (q4 modes): codes and fp16 scales read from the slot pool
   const uint8_t* q4_pool;
   unsigned long long q4_extent;  // bytes per slot
-  long long q4_code_off;         // byte offset of this operand's codes in an extent
-  int q4_code_ld;                // bytes per weight row of codes (K / 2)
+  int q4_rows_per_slot;          // rows of the code tensor map per slot (extent / row bytes)
+  int q4_row_off;                // first code row of this operand inside a slot
   long long q4_scale_off;        // byte offset of this operand's scales in an extent
   int q4_scale_ld;               // bytes per weight row of scales (K / 16)
 };

@@ -96,6 +96,20 @@ bool make_tmap(CUtensorMap* m, const void* base, uint64_t inner, uint64_t rows, 
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Byte-granular 2-D map over rows of `row_bytes` (4-bit codes): boxes of 32
+// bytes (64 codes, one K block) x 128 rows, no swizzle.
+bool make_tmap_codes(CUtensorMap* m, const void* base, uint64_t row_bytes, uint64_t rows) {
+  auto fn = encode_fn();
+  if (fn == nullptr || rows == 0) return false;
+  cuuint64_t dims[2] = {row_bytes, rows};
+  cuuint64_t strides[1] = {row_bytes};
+  cuuint32_t box[2] = {32, 128};
+  cuuint32_t es[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void*>(base), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // Reference-counted pool of CUDA events (readiness and consumer fences).
 struct EventPool {
   std::vector<cudaEvent_t> ev;
@@ -208,6 +222,7 @@ struct msi_plan {
   EventPool pool;
   int fwd_ev = -1;
   CUtensorMap tm_w13{}, tm_w2{}, tm_sh13{}, tm_sh2{};
+  CUtensorMap tm_q13{}, tm_q2{};  // 4-bit plans: packed codes of W13 / W2 over the pool
   std::vector<msi_trace_rec> trace;
   uint64_t seq = 0;
   msi_counters ctr{};
@@ -752,16 +767,18 @@ msi_status routed_ffn(msi_plan* p, FwdCtx& f, int ng, int grid1, int grid2, long
       g->q4_pool = static_cast<const uint8_t*>(d.slot_pool);
       g->q4_extent = d.extent_bytes;
     }
-    g1.q4_code_off = 0;
-    g1.q4_code_ld = d.hidden / 2;
+    // code rows through the byte maps: W13 rows of H/2 bytes, W2 rows of I/2
+    // bytes; an extent is a whole number of either (27 I / 8 and 27 H / 8)
+    g1.q4_rows_per_slot = (int)(d.extent_bytes / (d.hidden / 2));
+    g1.q4_row_off = 0;
     g1.q4_scale_off = 3 * HI / 2;
     g1.q4_scale_ld = d.hidden / 16;
-    g2.q4_code_off = HI;
-    g2.q4_code_ld = d.inter / 2;
+    g2.q4_rows_per_slot = (int)(d.extent_bytes / (d.inter / 2));
+    g2.q4_row_off = (int)(HI / (d.inter / 2));
     g2.q4_scale_off = 3 * HI / 2 + HI / 8;
     g2.q4_scale_ld = d.inter / 16;
-    LAUNCH(p, MSI_K_GATEUP, f.cs, launch_gemm(kGateUpGatherQ4, f.tm_h, f.tm_h, g1, grid1, f.cs));
-    LAUNCH(p, MSI_K_DOWN, f.cs, launch_gemm(kDownQ4, f.tm_h, f.tm_h, g2, grid2, f.cs));
+    LAUNCH(p, MSI_K_GATEUP, f.cs, launch_gemm(kGateUpGatherQ4, f.tm_h, p->tm_q13, g1, grid1, f.cs));
+    LAUNCH(p, MSI_K_DOWN, f.cs, launch_gemm(kDownQ4, f.tm_h, p->tm_q2, g2, grid2, f.cs));
     return MSI_OK;
   }
   if (pair_up)
@@ -925,6 +942,12 @@ msi_status msi_plan_create(const msi_plan_desc* desc, msi_plan** out) {
   if (d.wdtype == MSI_W_BF16) {
     if (!make_tmap(&p->tm_w13, d.slot_pool, H, S * 3 * I, 128) ||
         !make_tmap(&p->tm_w2, d.slot_pool, I, S * 3 * H, 128))
+      return fail(MSI_ERR_CUDA);
+  }
+  if (d.wdtype == MSI_W_Q4G32) {
+    if (d.extent_bytes % (H / 2) || d.extent_bytes % (I / 2) ||
+        !make_tmap_codes(&p->tm_q13, d.slot_pool, H / 2, S * (d.extent_bytes / (H / 2))) ||
+        !make_tmap_codes(&p->tm_q2, d.slot_pool, I / 2, S * (d.extent_bytes / (I / 2))))
       return fail(MSI_ERR_CUDA);
   }
   if (d.has_shared) {
