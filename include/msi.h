@@ -277,6 +277,35 @@ msi_status msi_moe_forward_streamed_next(msi_plan* plan, int layer, const void* 
  * MSI_ERR_SLOT_BUSY when the pin limit is reached (nothing changes). */
 msi_status msi_plan_pin(msi_plan* plan, int layer, int expert, int pinned);
 
+/* ---------------------------------------------------------------------------
+ * End-to-end calls from and to host memory.  The same forwards as
+ * msi_moe_forward / msi_moe_forward_streamed, with the token rows read from
+ * and the outputs written to host buffers: hidden_host [T, H] bf16 in,
+ * out_host [T, H] bf16 out, and (nullable) ids_host [T, k] int32 receiving the
+ * route ids.  Pinned host memory gives the full host-link rate; pageable
+ * memory is staged by the driver.  The route event still goes to the device
+ * buffers of `ev`.  The rows are copied into the workspace on a plan-owned
+ * copy stream forked from `compute` (the router waits for them), the route
+ * ids are copied back beside the expert GEMMs, and the combine runs in row
+ * chunks whose outputs are copied back while the next chunk is combined.  The
+ * copy stream joins `compute` before the call returns, so out_host and
+ * ids_host hold the results once `compute` has reached the point after the
+ * call (synchronise it, or an event recorded on it).  The host buffers must
+ * stay valid until then.  Workspace: msi_workspace_size_host (the device
+ * workspace plus two [T, H] bf16 row buffers).  Errors: as the device-buffer
+ * forwards; MSI_ERR_INVALID_ARG for a null hidden_host or out_host with T > 0. */
+msi_status msi_workspace_size_host(const msi_plan* plan, int T, size_t* bytes);
+msi_status msi_moe_forward_host(msi_plan* plan, int layer, const void* hidden_host, int T,
+                                const float* router_w, const int32_t* slot_table,
+                                const uint64_t* expected_generations, void* out_host,
+                                int32_t* ids_host, const msi_route_event* ev, void* workspace,
+                                size_t workspace_bytes, unsigned flags, msi_stream compute);
+msi_status msi_moe_forward_streamed_host(msi_plan* plan, int layer, const void* hidden_host, int T,
+                                         const float* router_w, void* out_host, int32_t* ids_host,
+                                         const msi_route_event* ev, void* workspace,
+                                         size_t workspace_bytes, unsigned flags,
+                                         msi_stream compute, msi_stream stage);
+
 /* Wait for the most recent forward of the plan and return its device-side
  * status (an msi_status value; MSI_OK when every needed expert passed the
  * generation re-check and every bounded device wait completed). */

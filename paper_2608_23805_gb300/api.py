@@ -172,6 +172,49 @@ class Plan:
             return out, ev
         return rc, out, ev
 
+    def workspace_host(self, T: int) -> torch.Tensor:
+        n = ctypes.c_size_t()
+        N.check(N.lib().msi_workspace_size_host(self.h, T, ctypes.byref(n)), "msi_workspace_size_host")
+        ws = self._ws.get("host")
+        if ws is None or ws.numel() < n.value:
+            ws = torch.empty(max(n.value, 256), dtype=torch.uint8, device="cuda")
+            self._ws["host"] = ws
+        return ws
+
+    def forward_host(self, layer, x_host, router_w, slot_table=None, expected=None, out_host=None,
+                     ids_host=None, ev=None, residual=False, stream=None, stage_stream=None,
+                     check=True, single_cta=False):
+        """End-to-end call from and to host memory: x_host and out_host are CPU
+        bf16 tensors [T, H] (pinned for the full link rate), ids_host an
+        optional CPU int32 [T, k].  With a slot table the resident forward runs,
+        without one the streamed forward.  The results are in out_host once the
+        compute stream has passed this call."""
+        T = x_host.shape[0]
+        assert x_host.device.type == "cpu" and x_host.is_contiguous()
+        out_host = torch.empty_like(x_host) if out_host is None else out_host
+        ev = RouteEvent(T, self.k, self.E) if ev is None else ev
+        ws = self.workspace_host(T)
+        fl = _flags(residual, single_cta)
+        if slot_table is not None:
+            st = np.ascontiguousarray(slot_table, dtype=np.int32)
+            ex = np.ascontiguousarray(expected, dtype=np.uint64)
+            rc = N.lib().msi_moe_forward_host(self.h, layer, x_host.data_ptr(), T, _ptr(router_w),
+                                              st.ctypes.data, ex.ctypes.data, out_host.data_ptr(),
+                                              _ptr(ids_host), ctypes.byref(ev.c), _ptr(ws), ws.numel(),
+                                              fl, _stream(stream))
+            where = "msi_moe_forward_host"
+        else:
+            rc = N.lib().msi_moe_forward_streamed_host(self.h, layer, x_host.data_ptr(), T,
+                                                       _ptr(router_w), out_host.data_ptr(),
+                                                       _ptr(ids_host), ctypes.byref(ev.c), _ptr(ws),
+                                                       ws.numel(), fl, _stream(stream),
+                                                       _stream(stage_stream))
+            where = "msi_moe_forward_streamed_host"
+        if check:
+            N.check(rc, where)
+            return out_host, ev
+        return rc, out_host, ev
+
     def pin(self, layer: int, expert: int, pinned: bool = True):
         N.check(N.lib().msi_plan_pin(self.h, layer, expert, int(pinned)), "msi_plan_pin")
 

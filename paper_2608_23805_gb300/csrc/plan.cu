@@ -248,6 +248,10 @@ struct msi_plan {
   cudaStream_t pred = nullptr;
   cudaEvent_t ev_pfork = nullptr, ev_pjoin = nullptr;
   int* h_pred = nullptr;
+  // host-buffer calls: a plan-owned copy stream and two events (compute ->
+  // copy, copy -> compute), created on first use
+  cudaStream_t io = nullptr;
+  cudaEvent_t ev_io_a = nullptr, ev_io_b = nullptr;
   // caller pins by object [L * E]: never a victim of the plan's waves/bundles
   std::vector<char> pinned_obj;
   int n_pins = 0;
@@ -566,7 +570,28 @@ struct FwdCtx {
   unsigned flags;
   cudaStream_t cs;
   CUtensorMap tm_h, tm_x, tm_hs;
+  // host-buffer calls: the rows land on the copy stream (x_ready, recorded
+  // there); the route ids and the output rows go back on it
+  cudaStream_t io = nullptr;
+  cudaEvent_t x_ready = nullptr;
+  void* out_host = nullptr;
+  int32_t* ids_host = nullptr;
 };
+
+struct HostIO {
+  cudaStream_t io;
+  cudaEvent_t x_ready;  // null when there are no rows (T = 0)
+  void* out_host;
+  int32_t* ids_host;
+};
+
+void apply_io(FwdCtx& f, const HostIO* h) {
+  if (h == nullptr) return;
+  f.io = h->io;
+  f.x_ready = h->x_ready;
+  f.out_host = h->out_host;
+  f.ids_host = h->ids_host;
+}
 
 msi_status validate_fwd(msi_plan* p, int layer, const void* x, int T, const float* rw, void* out,
                         const msi_route_event* ev, void* ws, size_t ws_bytes) {
@@ -605,6 +630,9 @@ msi_status route_rows(msi_plan* p, FwdCtx& f, const float* rw, const msi_route_e
                          first && d.has_shared ? at<Group>(ws, L.sh_group) : nullptr,
                          at<int>(ws, L.sh_total), f.T, tp.shared_slot, s));
   }
+  // host-buffer calls: every reader of the rows (router, shared expert) comes
+  // after they have landed
+  if (f.x_ready != nullptr) CK(cudaStreamWaitEvent(s, f.x_ready, 0));
   // the forward has begun (status cleared, shared group written): the shared
   // expert may start on the side stream from here
   if (first && d.has_shared) CK(cudaEventRecord(p->ev_fork, s));
@@ -699,6 +727,12 @@ msi_status front(msi_plan* p, FwdCtx& f, const TableParams& tp) {
   xa.status = at<int>(ws, L.status);
   LAUNCH(p, MSI_K_SCATTER, f.cs, launch_scatter(xa, tp, f.cs));
   const size_t Tk = (size_t)f.T * k;
+  if (f.ids_host != nullptr) {
+    // the route ids go back beside the expert GEMMs
+    CK(cudaEventRecord(p->ev_io_a, f.cs));
+    CK(cudaStreamWaitEvent(f.io, p->ev_io_a, 0));
+    CK(cudaMemcpyAsync(f.ids_host, f.ev->ids, Tk * sizeof(int32_t), cudaMemcpyDeviceToHost, f.io));
+  }
   if (!make_tmap(&f.tm_h, at<char>(ws, L.h), I, Tk, 128)) return MSI_ERR_CUDA;
   return MSI_OK;
 }
@@ -817,19 +851,32 @@ msi_status shared_ffn(msi_plan* p, FwdCtx& f, cudaStream_t stream) {
 msi_status finish(msi_plan* p, FwdCtx& f) {
   const auto& d = p->d;
   if (f.T > 0) {
-    CombineArgs c{};
-    c.yp = at<__nv_bfloat16>(f.ws, f.L.yp);
-    c.weights = f.ev->weights;
-    c.inv = at<int>(f.ws, f.L.inv);
-    c.sg = d.has_shared ? at<float>(f.ws, f.L.sg) : nullptr;
-    c.ys = d.has_shared ? at<__nv_bfloat16>(f.ws, f.L.ys) : nullptr;
-    c.x = (f.flags & MSI_FWD_RESIDUAL) ? static_cast<const __nv_bfloat16*>(f.x) : nullptr;
-    c.out = static_cast<__nv_bfloat16*>(f.out);
-    c.T = f.T;
-    c.H = d.hidden;
-    c.k = d.top_k;
-    c.status = at<int>(f.ws, f.L.status);
-    LAUNCH(p, MSI_K_COMBINE, f.cs, launch_combine(c, f.cs));
+    // host-buffer calls combine in row chunks; each chunk's rows go back
+    // while the next chunk is combined
+    const int H = d.hidden, k = d.top_k;
+    const int nc = (f.out_host != nullptr && f.T >= 1024) ? 4 : 1;
+    for (int ci = 0; ci < nc; ++ci) {
+      const long long t0 = (long long)f.T * ci / nc, t1 = (long long)f.T * (ci + 1) / nc;
+      CombineArgs c{};
+      c.yp = at<__nv_bfloat16>(f.ws, f.L.yp);
+      c.weights = f.ev->weights + t0 * k;
+      c.inv = at<int>(f.ws, f.L.inv) + t0 * k;
+      c.sg = d.has_shared ? at<float>(f.ws, f.L.sg) + t0 : nullptr;
+      c.ys = d.has_shared ? at<__nv_bfloat16>(f.ws, f.L.ys) + t0 * H : nullptr;
+      c.x = (f.flags & MSI_FWD_RESIDUAL) ? static_cast<const __nv_bfloat16*>(f.x) + t0 * H : nullptr;
+      c.out = static_cast<__nv_bfloat16*>(f.out) + t0 * H;
+      c.T = (int)(t1 - t0);
+      c.H = H;
+      c.k = k;
+      c.status = at<int>(f.ws, f.L.status);
+      LAUNCH(p, MSI_K_COMBINE, f.cs, launch_combine(c, f.cs));
+      if (f.out_host != nullptr) {
+        CK(cudaEventRecord(p->ev_io_a, f.cs));
+        CK(cudaStreamWaitEvent(f.io, p->ev_io_a, 0));
+        CK(cudaMemcpyAsync(static_cast<char*>(f.out_host) + t0 * H * 2, c.out, (t1 - t0) * H * 2,
+                           cudaMemcpyDeviceToHost, f.io));
+      }
+    }
   }
   CK(cudaMemcpyAsync(p->h_status, at<int>(f.ws, f.L.status), sizeof(int), cudaMemcpyDeviceToHost,
                      f.cs));
@@ -988,6 +1035,12 @@ msi_status msi_plan_destroy(msi_plan* p) {
     if (p->ev_pfork) cudaEventDestroy(p->ev_pfork);
     if (p->ev_pjoin) cudaEventDestroy(p->ev_pjoin);
     if (p->h_pred) cudaFreeHost(p->h_pred);
+    if (p->io) {
+      cudaStreamSynchronize(p->io);
+      cudaStreamDestroy(p->io);
+    }
+    if (p->ev_io_a) cudaEventDestroy(p->ev_io_a);
+    if (p->ev_io_b) cudaEventDestroy(p->ev_io_b);
   }
   delete p;
   return MSI_OK;
@@ -1066,12 +1119,12 @@ msi_status msi_slot_state(const msi_plan* cp, int slot, int* state) {
   return MSI_OK;
 }
 
-msi_status msi_moe_forward(msi_plan* p, int layer, const void* x, int T, const float* rw,
-                           const int32_t* table, const uint64_t* expected, void* out,
-                           const msi_route_event* ev, void* ws, size_t ws_bytes, unsigned flags,
-                           msi_stream compute) {
-  if (p == nullptr) return MSI_ERR_INVALID_ARG;
-  std::lock_guard<std::mutex> g(p->mu);
+namespace {
+
+msi_status forward_resident(msi_plan* p, int layer, const void* x, int T, const float* rw,
+                            const int32_t* table, const uint64_t* expected, void* out,
+                            const msi_route_event* ev, void* ws, size_t ws_bytes, unsigned flags,
+                            msi_stream compute, const HostIO* hio) {
   msi_status st = validate_fwd(p, layer, x, T, rw, out, ev, ws, ws_bytes);
   if (st != MSI_OK) return st;
   if (table == nullptr || expected == nullptr) return MSI_ERR_INVALID_ARG;
@@ -1106,6 +1159,7 @@ msi_status msi_moe_forward(msi_plan* p, int layer, const void* x, int T, const f
   f.L = layout(p, T);
   f.flags = flags;
   f.cs = reinterpret_cast<cudaStream_t>(compute);
+  apply_io(f, hio);
   // readiness: the compute stream waits for every pending publication it reads
   st = wait_ready(p, used, f.cs);
   if (st != MSI_OK) return st;
@@ -1146,6 +1200,18 @@ msi_status msi_moe_forward(msi_plan* p, int layer, const void* x, int T, const f
   if (st != MSI_OK) return st;
   p->ctr.forwards++;
   return MSI_OK;
+}
+
+}  // namespace
+
+msi_status msi_moe_forward(msi_plan* p, int layer, const void* x, int T, const float* rw,
+                           const int32_t* table, const uint64_t* expected, void* out,
+                           const msi_route_event* ev, void* ws, size_t ws_bytes, unsigned flags,
+                           msi_stream compute) {
+  if (p == nullptr) return MSI_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> g(p->mu);
+  return forward_resident(p, layer, x, T, rw, table, expected, out, ev, ws, ws_bytes, flags, compute,
+                          nullptr);
 }
 
 namespace {
@@ -1218,7 +1284,8 @@ msi_status prefetch_bundle(msi_plan* p, int nl, int call, int wave, const std::v
 msi_status forward_streamed(msi_plan* p, int layer, const void* x, int T, const float* rw, void* out,
                             const msi_route_event* ev, const float* next_rw,
                             const msi_route_event* next_ev, void* ws, size_t ws_bytes,
-                            unsigned flags, msi_stream compute, msi_stream stage) {
+                            unsigned flags, msi_stream compute, msi_stream stage,
+                            const HostIO* hio = nullptr) {
   msi_status st = validate_fwd(p, layer, x, T, rw, out, ev, ws, ws_bytes);
   if (st != MSI_OK) return st;
   const bool predict = next_rw != nullptr;
@@ -1242,6 +1309,7 @@ msi_status forward_streamed(msi_plan* p, int layer, const void* x, int T, const 
   f.L = layout(p, T);
   f.flags = flags;
   f.cs = reinterpret_cast<cudaStream_t>(compute);
+  apply_io(f, hio);
   cudaStream_t ss = reinterpret_cast<cudaStream_t>(stage);
   static thread_local TableParams tp;
   tp.E = 0;
@@ -1444,6 +1512,89 @@ msi_status msi_moe_forward_streamed_next(msi_plan* p, int layer, const void* x, 
   std::lock_guard<std::mutex> g(p->mu);
   return forward_streamed(p, layer, x, T, rw, out, ev, next_rw, next_ev, ws, ws_bytes, flags, compute,
                           stage);
+}
+
+namespace {
+
+size_t rows_bytes(const msi_plan* p, int T) {
+  return ((size_t)T * p->d.hidden * 2 + 255) / 256 * 256;
+}
+
+// Host-buffer call, first half: the rows go into the workspace tail on the
+// copy stream (forked from `compute`); x_dev / out_dev are the device row
+// buffers the forward then uses with h (x_ready, out_host) set.
+msi_status host_begin(msi_plan* p, int T, const void* hidden_host, void* out_host, void* ws,
+                      size_t ws_bytes, cudaStream_t cs, HostIO* h, void** x_dev, void** out_dev) {
+  if (T < 0 || (T > 0 && (hidden_host == nullptr || out_host == nullptr))) return MSI_ERR_INVALID_ARG;
+  if (p->dying) return MSI_ERR_SHUT_DOWN;
+  const size_t base = layout(p, T).bytes, rb = rows_bytes(p, T);
+  if (ws == nullptr || (uintptr_t)ws % 256 || ws_bytes < base + 2 * rb) return MSI_ERR_WORKSPACE;
+  if (p->io == nullptr) {
+    cudaError_t e = cudaStreamCreateWithFlags(&p->io, cudaStreamNonBlocking);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&p->ev_io_a, cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&p->ev_io_b, cudaEventDisableTiming);
+    if (e != cudaSuccess) return cuda_fail(e, "copy stream");
+  }
+  *x_dev = static_cast<char*>(ws) + base;
+  *out_dev = static_cast<char*>(ws) + base + rb;
+  *h = HostIO{p->io, nullptr, T > 0 ? out_host : nullptr, nullptr};
+  CK(cudaEventRecord(p->ev_io_a, cs));
+  CK(cudaStreamWaitEvent(p->io, p->ev_io_a, 0));
+  if (T > 0) {
+    CK(cudaMemcpyAsync(*x_dev, hidden_host, (size_t)T * p->d.hidden * 2, cudaMemcpyHostToDevice, p->io));
+    CK(cudaEventRecord(p->ev_io_b, p->io));
+    h->x_ready = p->ev_io_b;
+  }
+  return MSI_OK;
+}
+
+// Second half: the copy stream joins `compute` (also after a failed forward,
+// so that no copy outlives the call's place in the compute stream).
+msi_status host_end(msi_plan* p, cudaStream_t cs, msi_status st) {
+  CK(cudaEventRecord(p->ev_io_b, p->io));
+  CK(cudaStreamWaitEvent(cs, p->ev_io_b, 0));
+  return st;
+}
+
+}  // namespace
+
+msi_status msi_workspace_size_host(const msi_plan* p, int T, size_t* bytes) {
+  if (p == nullptr || bytes == nullptr || T < 0) return MSI_ERR_INVALID_ARG;
+  *bytes = layout(p, T).bytes + 2 * rows_bytes(p, T);
+  return MSI_OK;
+}
+
+msi_status msi_moe_forward_host(msi_plan* p, int layer, const void* hidden_host, int T,
+                                const float* rw, const int32_t* table, const uint64_t* expected,
+                                void* out_host, int32_t* ids_host, const msi_route_event* ev,
+                                void* ws, size_t ws_bytes, unsigned flags, msi_stream compute) {
+  if (p == nullptr) return MSI_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> g(p->mu);
+  cudaStream_t cs = reinterpret_cast<cudaStream_t>(compute);
+  HostIO h{};
+  void *x = nullptr, *out = nullptr;
+  msi_status st = host_begin(p, T, hidden_host, out_host, ws, ws_bytes, cs, &h, &x, &out);
+  if (st != MSI_OK) return st;
+  h.ids_host = T > 0 ? ids_host : nullptr;
+  st = forward_resident(p, layer, x, T, rw, table, expected, out, ev, ws, ws_bytes, flags, compute, &h);
+  return host_end(p, cs, st);
+}
+
+msi_status msi_moe_forward_streamed_host(msi_plan* p, int layer, const void* hidden_host, int T,
+                                         const float* rw, void* out_host, int32_t* ids_host,
+                                         const msi_route_event* ev, void* ws, size_t ws_bytes,
+                                         unsigned flags, msi_stream compute, msi_stream stage) {
+  if (p == nullptr) return MSI_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> g(p->mu);
+  cudaStream_t cs = reinterpret_cast<cudaStream_t>(compute);
+  HostIO h{};
+  void *x = nullptr, *out = nullptr;
+  msi_status st = host_begin(p, T, hidden_host, out_host, ws, ws_bytes, cs, &h, &x, &out);
+  if (st != MSI_OK) return st;
+  h.ids_host = T > 0 ? ids_host : nullptr;
+  st = forward_streamed(p, layer, x, T, rw, out, ev, nullptr, nullptr, ws, ws_bytes, flags, compute,
+                        stage, &h);
+  return host_end(p, cs, st);
 }
 
 msi_status msi_plan_pin(msi_plan* p, int layer, int expert, int pinned) {

@@ -100,6 +100,13 @@ _SIGS = {
                                                      ctypes.POINTER(msi_route_event), _P,
                                                      ctypes.c_size_t, ctypes.c_uint, _P, _P]),
     "msi_plan_pin": (ctypes.c_int, [_P, ctypes.c_int, ctypes.c_int, ctypes.c_int]),
+    "msi_workspace_size_host": (ctypes.c_int, [_P, ctypes.c_int, ctypes.POINTER(ctypes.c_size_t)]),
+    "msi_moe_forward_host": (ctypes.c_int, [_P, ctypes.c_int, _P, ctypes.c_int, _P, _P, _P, _P, _P,
+                                            ctypes.POINTER(msi_route_event), _P, ctypes.c_size_t,
+                                            ctypes.c_uint, _P]),
+    "msi_moe_forward_streamed_host": (ctypes.c_int, [_P, ctypes.c_int, _P, ctypes.c_int, _P, _P, _P,
+                                                     ctypes.POINTER(msi_route_event), _P,
+                                                     ctypes.c_size_t, ctypes.c_uint, _P, _P]),
     "msi_moe_forward_static": (ctypes.c_int, [_P, ctypes.c_int, _P, ctypes.c_int, _P, _P, _P, _P,
                                               ctypes.POINTER(msi_route_event), ctypes.c_uint, _P]),
     "msi_forward_status": (ctypes.c_int, [_P, ctypes.POINTER(ctypes.c_int)]),
