@@ -204,13 +204,15 @@ def combine(weights, inv, Y, sg=None, ys=None, residual=None):
 # ---------------------------------------------------------------------------
 
 def moe_layer(x_bf16, router_w, k, extent_of, H, I, wdtype=_W_BF16,
-              shared_extent=None, w_sg=None, residual=False):
+              shared_extent=None, w_sg=None, residual=False, shared_gated=True):
     """The MoE layer forward of one call.
 
     extent_of(e) returns expert e's canonical extent (uint8).  Returns the
     router dict plus counts, offsets, perm, inv, Y (expert outputs in permuted
-    row order) and out [T, H] (float64)."""
-    r = router(x_bf16, router_w, k, w_sg if shared_extent is not None else None)
+    row order) and out [T, H] (float64).  shared_gated=False takes the other
+    reading of the shared expert (R4): its output is added with gate 1."""
+    r = router(x_bf16, router_w, k,
+               w_sg if shared_extent is not None and shared_gated else None)
     E = np.asarray(router_w).shape[0]
     counts, offsets, perm, inv = permutation(r["ids"], E)
     x = bf16_to_f64(x_bf16)
@@ -227,7 +229,8 @@ def moe_layer(x_bf16, router_w, k, extent_of, H, I, wdtype=_W_BF16,
     if shared_extent is not None:
         Sg, Su, S2 = decode_extent(shared_extent, H, I, _W_BF16)
         ys = swiglu_expert(x, Sg, Su, S2)
-    out = combine(r["weights"], inv, Y, r["sg"], ys, x if residual else None)
+    sg = r["sg"] if shared_gated or ys is None else np.ones(T, dtype=np.float64)
+    out = combine(r["weights"], inv, Y, sg, ys, x if residual else None)
     r.update(counts=counts, offsets=offsets, perm=perm, inv=inv, Y=Y, ys=ys, out=out)
     return r
 

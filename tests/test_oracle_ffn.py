@@ -83,6 +83,10 @@ def test_shared_expert_and_residual_terms():
     gate = torch.sigmoid(xt @ torch.from_numpy(wsg.astype(np.float64))).numpy()
     np.testing.assert_allclose(full["out"], base["out"] + gate[:, None] * ys + xf, rtol=1e-12,
                                atol=1e-14)
+    # the ungated reading adds the library MLP's output with weight 1
+    ungated = oracle.moe_layer(x, Wr, 2, ext.__getitem__, cfg.hidden, cfg.inter,
+                               shared_extent=sh, w_sg=wsg, shared_gated=False)
+    np.testing.assert_allclose(ungated["out"], base["out"] + ys, rtol=1e-12, atol=1e-14)
 
 
 @pytest.mark.parametrize("seed", range(4))
