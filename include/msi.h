@@ -93,10 +93,13 @@ enum {
 /* Forward flags. */
 enum {
   MSI_FWD_RESIDUAL = 1,   /* out = x + moe(x), rounded once to bf16 (decode stacks) */
-  MSI_FWD_SINGLE_CTA = 2  /* run every expert GEMM on single-CTA 128-row tiles; by default
+  MSI_FWD_SINGLE_CTA = 2, /* run every expert GEMM on single-CTA 128-row tiles; by default
                              bf16 launches whose groups average >= 1,024 rows use CTA-pair
                              256-row tiles (both accumulate in fp32 over the same K order
                              and meet the same output tolerance) */
+  MSI_FWD_SHARED_UNGATED = 4 /* the shared expert's output is added with gate 1 instead of
+                                sigmoid(x . w_sg) (the other reading of its gate; no effect
+                                without a shared expert) */
 };
 
 /* Plan description (copied by msi_plan_create; pointers must outlive the plan). */

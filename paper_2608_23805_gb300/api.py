@@ -18,8 +18,9 @@ def _ptr(t) -> int | None:
     return None if t is None else t.data_ptr()
 
 
-def _flags(residual: bool, single_cta: bool) -> int:
-    return (N.MSI_FWD_RESIDUAL if residual else 0) | (N.MSI_FWD_SINGLE_CTA if single_cta else 0)
+def _flags(residual: bool, single_cta: bool, shared_gate: bool = True) -> int:
+    return ((N.MSI_FWD_RESIDUAL if residual else 0) | (N.MSI_FWD_SINGLE_CTA if single_cta else 0)
+            | (0 if shared_gate else N.MSI_FWD_SHARED_UNGATED))
 
 
 def _stream(s) -> int | None:
@@ -127,7 +128,7 @@ class Plan:
         return ws
 
     def forward(self, layer, x, router_w, slot_table, expected, out=None, ev=None, residual=False,
-                stream=None, check=True, single_cta=False):
+                stream=None, check=True, single_cta=False, shared_gate=True):
         T = x.shape[0]
         out = torch.empty_like(x) if out is None else out
         ev = RouteEvent(T, self.k, self.E) if ev is None else ev
@@ -136,7 +137,8 @@ class Plan:
         ex = np.ascontiguousarray(expected, dtype=np.uint64)
         rc = N.lib().msi_moe_forward(self.h, layer, _ptr(x), T, _ptr(router_w), st.ctypes.data,
                                      ex.ctypes.data, _ptr(out), ctypes.byref(ev.c), _ptr(ws),
-                                     ws.numel(), _flags(residual, single_cta), _stream(stream))
+                                     ws.numel(), _flags(residual, single_cta, shared_gate),
+                                     _stream(stream))
         if check:
             N.check(rc, "msi_moe_forward")
             return out, ev

@@ -188,7 +188,7 @@ struct CombineArgs {
   const __nv_bfloat16* yp;   // [T*k, H]
   const float* weights;      // [T, k]
   const int* inv;            // [T*k]
-  const float* sg;           // [T] or nullptr
+  const float* sg;           // [T]; nullptr: gate 1 (with ys)
   const __nv_bfloat16* ys;   // [T, H] or nullptr
   const __nv_bfloat16* x;    // residual or nullptr
   __nv_bfloat16* out;        // [T, H]

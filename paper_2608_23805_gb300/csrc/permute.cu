@@ -350,8 +350,9 @@ __global__ void __launch_bounds__(256) combine_kernel(const CombineArgs a) {
     }
     for (; j < a.k; ++j)
       fma8(acc, s_w[j], __ldg(reinterpret_cast<const uint4*>(a.yp + (size_t)s_row[j] * a.H) + c));
-    if (a.ys != nullptr)
-      fma8(acc, a.sg[t], __ldg(reinterpret_cast<const uint4*>(a.ys + (size_t)t * a.H) + c));
+    if (a.ys != nullptr)  // gate sigmoid(x . w_sg), or 1 for an ungated shared expert
+      fma8(acc, a.sg != nullptr ? a.sg[t] : 1.0f,
+           __ldg(reinterpret_cast<const uint4*>(a.ys + (size_t)t * a.H) + c));
     if (a.x != nullptr) {
       const uint4 y = __ldg(reinterpret_cast<const uint4*>(a.x + (size_t)t * a.H) + c);
       acc[0] += bf16_lo(y.x);

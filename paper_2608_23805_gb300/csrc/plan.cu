@@ -622,7 +622,9 @@ msi_status route_rows(msi_plan* p, FwdCtx& f, const float* rw, const msi_route_e
   void* ws = f.ws;
   const WsLayout& L = f.L;
   const int nb = (f.T + L.tm - 1) / L.tm;
-  const float* wsg = first && d.has_shared ? d.shared_gate_w + (size_t)f.layer * H : nullptr;
+  const float* wsg = first && d.has_shared && !(f.flags & MSI_FWD_SHARED_UNGATED)
+                         ? d.shared_gate_w + (size_t)f.layer * H
+                         : nullptr;
   if (tensor_router(d)) {
     __nv_bfloat16* w3 = at<__nv_bfloat16>(ws, L.w3);
     LAUNCH(p, MSI_K_ROUTER, s,
@@ -861,7 +863,8 @@ msi_status finish(msi_plan* p, FwdCtx& f) {
       c.yp = at<__nv_bfloat16>(f.ws, f.L.yp);
       c.weights = f.ev->weights + t0 * k;
       c.inv = at<int>(f.ws, f.L.inv) + t0 * k;
-      c.sg = d.has_shared ? at<float>(f.ws, f.L.sg) + t0 : nullptr;
+      c.sg = d.has_shared && !(f.flags & MSI_FWD_SHARED_UNGATED) ? at<float>(f.ws, f.L.sg) + t0
+                                                                 : nullptr;
       c.ys = d.has_shared ? at<__nv_bfloat16>(f.ws, f.L.ys) + t0 * H : nullptr;
       c.x = (f.flags & MSI_FWD_RESIDUAL) ? static_cast<const __nv_bfloat16*>(f.x) + t0 * H : nullptr;
       c.out = static_cast<__nv_bfloat16*>(f.out) + t0 * H;

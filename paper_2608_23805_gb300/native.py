@@ -33,6 +33,7 @@ MSI_TRACE_HIT, MSI_TRACE_STAGE, MSI_TRACE_EVICT, MSI_TRACE_PREFETCH = 0, 1, 2, 3
 MSI_SLOT_VACANT, MSI_SLOT_LOADING, MSI_SLOT_DEVICE_READY, MSI_SLOT_IN_USE, MSI_SLOT_RECYCLABLE = range(5)
 MSI_FWD_RESIDUAL = 1
 MSI_FWD_SINGLE_CTA = 2
+MSI_FWD_SHARED_UNGATED = 4
 KERNEL_KINDS = ["upload", "router", "scan", "scatter", "setup", "gateup", "down", "shared_gateup",
                 "shared_down", "combine", "publish"]
 

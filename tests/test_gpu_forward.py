@@ -315,3 +315,26 @@ def test_exact_logit_ties_rank_lower_id_first(E):
     assert seen > 50  # the amplified pairs are routed often
     compare_routes(ids, wts, oracle.router(x_bits, w, cfg.top_k))
     case.close()
+
+
+def test_ungated_shared_expert_flag():
+    """MSI_FWD_SHARED_UNGATED: the shared expert's output enters with gate 1
+    (the other reading of its gate) and matches the oracle taking that
+    reading; without the flag the gated output is unchanged."""
+    cfg = synth.config("qwen3next_4k", n_experts=64, n_slots=64, tokens=300)
+    case = Case(cfg)
+    table, gens = case.stage_all()
+    x_bits = synth.hidden(cfg, 0, 150)
+    out_u, _ = case.plan.forward(0, bf16_tensor(x_bits), case.router[0], table, gens,
+                                 shared_gate=False)
+    torch.cuda.synchronize()
+    assert case.plan.status() == N.MSI_OK
+    ref_u = oracle.moe_layer(x_bits, case.router_np[0], cfg.top_k, lambda e: case.extent(0, e),
+                             cfg.hidden, cfg.inter, shared_extent=case.shared_np[0],
+                             w_sg=case.gate_np[0], shared_gated=False)
+    compare_out(bf16_bits(out_u), ref_u["out"])
+    out_g, _ = case.plan.forward(0, bf16_tensor(x_bits), case.router[0], table, gens)
+    torch.cuda.synchronize()
+    compare_out(bf16_bits(out_g), case.oracle_layer(x_bits)["out"])
+    assert not torch.equal(out_u, out_g)
+    case.close()
