@@ -53,11 +53,11 @@ L2_BYTES = 129 * 1024 * 1024
 # (the summaries under profiles/), keyed by (workload, kernel kind); reported
 # only while the GEMM source still hashes to the value the capture was taken at.
 TRAFFIC = {
-    ("qwen3next_4k", "gateup"): {"bytes_per_launch": 2268160768 + 41969408, "src_hash": "428ac7b1d69c5e60",
+    ("qwen3next_4k", "gateup"): {"bytes_per_launch": 2268160768 + 41969408, "src_hash": "8439729f64f80b0f",
                                  "profile": "profiles/gemm_gateup_qwen3next_4k.md"},
-    ("prefill32k_lru64", "gateup"): {"bytes_per_launch": 205889024 + 14773504, "src_hash": "428ac7b1d69c5e60",
+    ("prefill32k_lru64", "gateup"): {"bytes_per_launch": 205889024 + 14773504, "src_hash": "8439729f64f80b0f",
                                      "profile": "profiles/gemm_gateup_prefill32k_lru64.md"},
-    ("prefill32k_q4_lru64", "gateup"): {"bytes_per_launch": 104654592 + 8550656, "src_hash": "428ac7b1d69c5e60",
+    ("prefill32k_q4_lru64", "gateup"): {"bytes_per_launch": 104654592 + 8550656, "src_hash": "8439729f64f80b0f",
                                         "profile": "profiles/gemm_gateup_q4_prefill32k_q4_lru64.md"},
 }
 
@@ -72,11 +72,17 @@ def load_peaks():
 
 
 def kernel_source_hash() -> str:
-    """Hash of the grouped-GEMM source (the dominant kernels' code)."""
+    """Hash of the grouped-GEMM source (the dominant kernels' code), comments
+    and blank lines left out: a capture stays valid until the code changes."""
+    import re
     h = hashlib.sha256()
     for name in ("gemm.cu", "internal.cuh"):
-        with open(os.path.join(ROOT, "paper_2608_23805_gb300", "csrc", name), "rb") as f:
-            h.update(f.read())
+        with open(os.path.join(ROOT, "paper_2608_23805_gb300", "csrc", name)) as f:
+            src = re.sub(r"/\*.*?\*/", "", f.read(), flags=re.S)
+        for line in src.splitlines():
+            code = re.sub(r"//.*", "", line).strip()
+            if code:
+                h.update(code.encode() + b"\n")
     return h.hexdigest()[:16]
 
 
@@ -127,7 +133,7 @@ class ClockSampler:
         try:
             self.f = open(self.path, "w")
             self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.idx), "--query-gpu=" + self.Q,
-                                          "--format=csv,noheader,nounits", "-lms", os.environ.get("MSI_CLOCK_MS", "100")],
+                                          "--format=csv,noheader,nounits", "-lms", os.environ.get("MSI_CLOCK_MS", "20")],
                                          stdout=self.f, stderr=subprocess.DEVNULL)
         except (OSError, FileNotFoundError):
             self.proc = None
@@ -510,6 +516,7 @@ def run_ours(args):
         "kernels_ms_per_step": {k: round(v[0] / args.steps, 4) for k, v in kt.items() if v[1] > 0},
         "wall_s_timed": wall,
         "step_ms": [round(a.elapsed_time(b), 3) for a, b in evs],
+        "e2e_step_ms": [round(a.elapsed_time(b), 3) for a, b in e2e_evs],
         "peaks": peak_kind,
     }
     if src is not None:
