@@ -621,7 +621,7 @@ def run_reference(args):
     }), flush=True)
 
 
-REF_TOKENS = {"prefill32k_lru64": 256, "prefill32k_q4_lru64": 256, "qwen3next_4k": 256, "tiny": 64}
+REF_TOKENS = {"prefill32k_lru64": 4096, "prefill32k_q4_lru64": 4096, "qwen3next_4k": 4096, "tiny": 64}
 
 
 def main():
