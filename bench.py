@@ -18,7 +18,10 @@ two-bank prefetch (each call routes its rows through the next layer's router
 and stages the predicted objects after its last wave).
 
 Prints one JSON line (rank 0).  `value` is whole-job tokens/s over the timed
-steps (device time, CUDA events on the compute stream); `e2e` repeats the
+steps (device time, CUDA events on the compute stream around each step, no
+per-kernel events inside it); a second timed pass of the same steps with an
+event pair around every kernel launch gives `kernels_ms_per_step` and the
+roofline kernel's launch duration; `e2e` repeats the
 metric with the hidden rows copied from pinned host memory and the outputs
 read back inside the timed region; `roofline` is the dominant kernel's
 algorithmic work per launch over its event-timed duration; `cpu_baseline` is
@@ -411,7 +414,6 @@ def run_ours(args):
     flush = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device="cuda")
     sampler = ClockSampler(local)
     sampler.start()
-    w.plan.timing(True)
     def flush_l2():
         # on the compute stream, so that it is ordered before the step's start
         # event and never overlaps a timed step
@@ -423,31 +425,40 @@ def run_ours(args):
         flush_l2()
         w.step()
     torch.cuda.synchronize()
-    w.plan.timing_read(reset=True)
     flush_l2()                                       # one more untimed step right before timing
     w.step()
     torch.cuda.synchronize()
-    w.plan.timing_read(reset=True)
+
+    def timed_steps():
+        evs = []
+        for _ in range(args.steps):
+            flush_l2()                               # L2 flushed between timed steps (untimed)
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            a.record(w.cs)
+            w.step()
+            b.record(w.cs)
+            evs.append((a, b))
+        torch.cuda.synchronize()
+        return evs
+
+    # (1) the step itself, no per-kernel events inside it: `value`
     if backend:
         torch.distributed.barrier()
     torch.cuda.synchronize()
     launches0 = w.plan.launches()
     staged0 = w.plan.counters()["h2d_bytes"]
-    evs = []
     wall0 = time.perf_counter()
-    for _ in range(args.steps):
-        flush_l2()                                   # L2 flushed between timed steps (untimed)
-        a = torch.cuda.Event(enable_timing=True)
-        b = torch.cuda.Event(enable_timing=True)
-        a.record(w.cs)
-        w.step()
-        b.record(w.cs)
-        evs.append((a, b))
-    torch.cuda.synchronize()
+    evs = timed_steps()
     wall = time.perf_counter() - wall0
     launches = w.plan.launches() - launches0
     staged = (w.plan.counters()["h2d_bytes"] - staged0) // args.steps
     dev_s = sum(a.elapsed_time(b) for a, b in evs) / 1e3
+    # (2) the same steps with an event pair around every kernel launch: the
+    # per-kernel times and the roofline kernel's launch duration
+    w.plan.timing(True)
+    w.plan.timing_read(reset=True)
+    evs_k = timed_steps()
     kt = w.plan.timing_read(reset=True)
     w.plan.timing(False)
     assert w.plan.status() == 0, "device status %d" % w.plan.status()
@@ -516,6 +527,7 @@ def run_ours(args):
         "kernels_ms_per_step": {k: round(v[0] / args.steps, 4) for k, v in kt.items() if v[1] > 0},
         "wall_s_timed": wall,
         "step_ms": [round(a.elapsed_time(b), 3) for a, b in evs],
+        "step_ms_kernel_timing": [round(a.elapsed_time(b), 3) for a, b in evs_k],
         "e2e_step_ms": [round(a.elapsed_time(b), 3) for a, b in e2e_evs],
         "peaks": peak_kind,
     }
