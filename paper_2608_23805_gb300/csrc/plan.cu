@@ -1223,11 +1223,27 @@ namespace {
 // the predicted counts (created on the first predicting call).
 msi_status prediction_resources(msi_plan* p) {
   if (p->pred != nullptr) return MSI_OK;
-  cudaError_t e = cudaMallocHost(&p->h_pred, sizeof(int) * p->d.n_experts);
-  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&p->ev_pfork, cudaEventDisableTiming);
-  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&p->ev_pjoin, cudaEventDisableTiming);
-  if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&p->pred, cudaStreamNonBlocking);
-  return e == cudaSuccess ? MSI_OK : cuda_fail(e, "prediction stream");
+  // created into locals and kept only all together, so that a failure
+  // leaves nothing half-made behind for the next call
+  int* h = nullptr;
+  cudaEvent_t fork = nullptr, join = nullptr;
+  cudaStream_t s = nullptr;
+  cudaError_t e = cudaMallocHost(&h, sizeof(int) * p->d.n_experts);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&fork, cudaEventDisableTiming);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&join, cudaEventDisableTiming);
+  if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&s, cudaStreamNonBlocking);
+  if (e != cudaSuccess) {
+    if (h) cudaFreeHost(h);
+    if (fork) cudaEventDestroy(fork);
+    if (join) cudaEventDestroy(join);
+    if (s) cudaStreamDestroy(s);
+    return cuda_fail(e, "prediction stream");
+  }
+  p->h_pred = h;
+  p->ev_pfork = fork;
+  p->ev_pjoin = join;
+  p->pred = s;
+  return MSI_OK;
 }
 
 // The prefetch bundle for layer `nl` after call `call`'s last wave (slots
@@ -1342,6 +1358,16 @@ msi_status forward_streamed(msi_plan* p, int layer, const void* x, int T, const 
     CK(cudaMemcpyAsync(p->h_pred, next_ev->counts, sizeof(int) * E, cudaMemcpyDeviceToHost, p->pred));
     CK(cudaEventRecord(p->ev_pjoin, p->pred));
   }
+  // every return from here on (an error included) leaves the compute stream
+  // joined to the prediction, which reads the router scratch the next call
+  // overwrites
+  struct PredJoin {
+    cudaStream_t cs;
+    cudaEvent_t ev;
+    ~PredJoin() {
+      if (ev != nullptr) cudaStreamWaitEvent(cs, ev, 0);
+    }
+  } pred_join{f.cs, predict ? p->ev_pjoin : nullptr};
   st = shared_ffn(p, f, f.cs);  // overlaps the host planning and the first wave's copies
   if (st != MSI_OK) return st;
   const cudaError_t se = cudaEventSynchronize(p->pool.ev[cev]);
@@ -1488,6 +1514,7 @@ msi_status forward_streamed(msi_plan* p, int layer, const void* x, int T, const 
     st = prefetch_bundle(p, layer + 1, call, (int)n_waves, prev, ss);
     if (st != MSI_OK) return st;
     CK(cudaStreamWaitEvent(f.cs, p->ev_pjoin, 0));
+    pred_join.ev = nullptr;
   }
   st = finish(p, f);
   if (st != MSI_OK) return st;
@@ -1533,10 +1560,21 @@ msi_status host_begin(msi_plan* p, int T, const void* hidden_host, void* out_hos
   const size_t base = layout(p, T).bytes, rb = rows_bytes(p, T);
   if (ws == nullptr || (uintptr_t)ws % 256 || ws_bytes < base + 2 * rb) return MSI_ERR_WORKSPACE;
   if (p->io == nullptr) {
-    cudaError_t e = cudaStreamCreateWithFlags(&p->io, cudaStreamNonBlocking);
-    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&p->ev_io_a, cudaEventDisableTiming);
-    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&p->ev_io_b, cudaEventDisableTiming);
-    if (e != cudaSuccess) return cuda_fail(e, "copy stream");
+    // created into locals and kept only all together (see prediction_resources)
+    cudaStream_t s = nullptr;
+    cudaEvent_t ea = nullptr, eb = nullptr;
+    cudaError_t e = cudaStreamCreateWithFlags(&s, cudaStreamNonBlocking);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ea, cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&eb, cudaEventDisableTiming);
+    if (e != cudaSuccess) {
+      if (s) cudaStreamDestroy(s);
+      if (ea) cudaEventDestroy(ea);
+      if (eb) cudaEventDestroy(eb);
+      return cuda_fail(e, "copy stream");
+    }
+    p->io = s;
+    p->ev_io_a = ea;
+    p->ev_io_b = eb;
   }
   *x_dev = static_cast<char*>(ws) + base;
   *out_dev = static_cast<char*>(ws) + base + rb;

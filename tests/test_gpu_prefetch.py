@@ -215,3 +215,30 @@ def test_rejected_prefetch_read_unwinds_only_its_bundle(tmp_path):
     case.plan.set_source(None)
     src.close()
     case.close()
+
+
+def test_failed_predicting_call_leaves_the_plan_usable():
+    """A predicting call that fails after its prediction was launched (a
+    caller-held slot times out before the waves are planned) still joins the
+    prediction before returning; once the slot is released, the next calls
+    (with and without prediction) match the oracle."""
+    cfg = synth.config("decode48", tokens=16, n_layers=2)
+    case = Case(cfg, wait_timeout_s=0.2)
+    x_bits = synth.hidden(cfg, 0, 97)
+    out, ev = case.plan.forward_streamed(0, bf16_tensor(x_bits), case.router[0],
+                                         next_router_w=case.router[1])
+    torch.cuda.synchronize()
+    held = int(case.plan.slot_table(0)[0].max())
+    case.plan.hold(held)
+    rc, _, _ = case.plan.forward_streamed(0, bf16_tensor(x_bits), case.router[0],
+                                          next_router_w=case.router[1], check=False)
+    assert rc == N.MSI_ERR_TIMEOUT
+    case.plan.release(held)
+    out1, _ = case.plan.forward_streamed(1, bf16_tensor(x_bits), case.router[1])
+    out0, _ = case.plan.forward_streamed(0, bf16_tensor(x_bits), case.router[0],
+                                         next_router_w=case.router[1])
+    torch.cuda.synchronize()
+    assert case.plan.status() == N.MSI_OK
+    compare_out(bf16_bits(out1), case.oracle_layer(x_bits, 1)["out"])
+    compare_out(bf16_bits(out0), case.oracle_layer(x_bits, 0)["out"])
+    case.close()
