@@ -30,7 +30,7 @@
  *    W13 codes [2I, H/2] | W2 codes [H, I/2] | W13 fp16 scales [2I, H/32] |
  *    W2 fp16 scales [H, I/32], code q -> scale * (q - 8), even column in the
  *    low nibble.
- *  - Shape limits of this build: E <= 512, 1 <= k <= min(E, 32), H a multiple
+ *  - Shape limits of the library: E <= 512, 1 <= k <= min(E, 32), H a multiple
  *    of 256, I a multiple of 128, T >= 0.  Other shapes return
  *    MSI_ERR_UNSUPPORTED.
  */
@@ -56,7 +56,7 @@ typedef enum {
   MSI_ERR_TIMEOUT = 6,           /* a bounded host or device wait ran out */
   MSI_ERR_CUDA = 7,              /* a CUDA runtime call failed (see msi_last_cuda_error) */
   MSI_ERR_SHUT_DOWN = 8,         /* the plan is being destroyed */
-  MSI_ERR_UNSUPPORTED = 9,       /* shape outside this build's limits */
+  MSI_ERR_UNSUPPORTED = 9,       /* shape outside the library's limits */
   MSI_ERR_WORKSPACE = 10,        /* workspace missing, misaligned or too small */
   MSI_ERR_SOURCE = 11            /* a source extent failed (short read / I/O error); its
                                     bundle was not staged and nothing was published */

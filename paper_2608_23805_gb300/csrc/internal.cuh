@@ -30,7 +30,7 @@ inline cudaError_t smem_attr_once(K* kernel, int bytes, std::atomic<unsigned lon
 
 
 // ---------------------------------------------------------------------------
-// Limits of this build
+// Limits of the kernels
 // ---------------------------------------------------------------------------
 constexpr int kMaxExperts = 512;
 constexpr int kMaxTopK = 32;

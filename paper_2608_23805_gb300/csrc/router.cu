@@ -22,7 +22,7 @@ namespace msi {
 namespace {
 constexpr int TM = kRouterTM;
 constexpr int BK = 32;
-constexpr int EP = 512;                      // experts per pass (this build: one pass)
+constexpr int EP = 512;                      // experts per pass (one pass covers every supported E)
 constexpr int NTH = 256;
 constexpr int XS_BYTES = TM * BK * 2;        // 2 KB
 constexpr int WS_BYTES = EP * BK * 4;        // 64 KB
