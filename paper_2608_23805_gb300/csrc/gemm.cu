@@ -42,7 +42,6 @@ constexpr int kEpiWarps = 4;
 constexpr int kGatherWarps = 4;
 constexpr uint32_t kIdesc = idesc_bf16(kBM, kBN);
 
-constexpr int kDqWarps = 8;   // one thread per B row (256 rows)
 constexpr int kRawRowBytes = 32;  // 64 codes of one B row per stage (one TMA box row)
 
 template <int MODE>
@@ -55,10 +54,12 @@ struct Cfg {
   static constexpr bool kTmaAny = kTmaA || kTmaB;
   static constexpr int kGatherWarp0 = 6;
   static constexpr int kDqWarp0 = 6 + (kGather ? kGatherWarps : 0);
-  static constexpr int kThreads = (kDqWarp0 + (kQ4 ? kDqWarps : 0)) * 32;
+  // q4: sixteen dequant warps, one thread per half B row (256 rows x 2)
+  static constexpr int kDq = kQ4 ? 16 : 0;
+  static constexpr int kThreads = (kDqWarp0 + kDq) * 32;
   static constexpr uint32_t kTxBytes = (kTmaB ? kBBytes : 0) + (kTmaA ? kABytes : 0);
   // gather threads arrive one by one as their copies land (cp.async ... arrive.noinc)
-  static constexpr int kFullCount = (kTmaAny ? 1 : 0) + (kGather ? kGatherWarps * 32 : 0) + (kQ4 ? kDqWarps : 0);
+  static constexpr int kFullCount = (kTmaAny ? 1 : 0) + (kGather ? kGatherWarps * 32 : 0) + kDq;
   // operand ring depth and, in the q4 modes, the ring of packed code stages
   // that the producer fills by TMA ahead of the conversion
   static constexpr int kStg = kStages;
@@ -129,6 +130,42 @@ __device__ __forceinline__ uint4 dequant8(uint32_t w, uint64_t scale2, uint64_t 
   return make_uint4(o[0], o[1], o[2], o[3]);
 }
 
+// q4 epilogue: TMEM read 16 columns at a time, so that the kernel's many
+// dequant threads fit the register file (one 32-byte store per chunk).
+template <bool GATEUP>
+__device__ __forceinline__ void epilogue_tile_lean(uint32_t tb, __nv_bfloat16* dst, bool valid) {
+  if (GATEUP) {
+#pragma unroll 1
+    for (int c = 0; c < 128; c += 16) {
+      uint32_t g[16], u[16];
+      tmem_ld16(tb + c, g);
+      tmem_ld16(tb + 128 + c, u);
+      tmem_ld_wait(g);
+      tmem_ld_wait(u);
+      uint32_t p[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const float g0 = __uint_as_float(g[2 * i]), g1 = __uint_as_float(g[2 * i + 1]);
+        const float u0 = __uint_as_float(u[2 * i]), u1 = __uint_as_float(u[2 * i + 1]);
+        p[i] = pack_bf16x2(__fdividef(g0 * u0, 1.0f + __expf(-g0)),
+                           __fdividef(g1 * u1, 1.0f + __expf(-g1)));
+      }
+      if (valid) st_global_v8(dst + c, p);
+    }
+  } else {
+#pragma unroll 1
+    for (int c = 0; c < kBN; c += 16) {
+      uint32_t v[16];
+      tmem_ld16(tb + c, v);
+      tmem_ld_wait(v);
+      uint32_t p[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) p[i] = pack_bf16x2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1]));
+      if (valid) st_global_v8(dst + c, p);
+    }
+  }
+}
+
 }  // namespace
 
 template <int MODE>
@@ -172,7 +209,7 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
     mbar_init(drain, 1);
     for (int r = 0; r < C::kRaw && C::kQ4; ++r) {
       mbar_init(&raw_full[r], 1);
-      mbar_init(&raw_empty[r], kDqWarps);
+      mbar_init(&raw_empty[r], C::kDq);
     }
     *abort_flag = 0;
     mbar_fence_init();
@@ -319,7 +356,7 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
             tb, a.out + ((size_t)__ldg(&G->row_begin) + row_w) * a.out_ld + ncol0, a.out_ld,
             cnt - row_w, epi_stage + warp * 4096, lane);
       } else {
-        epilogue_tile<C::kGateUp>(tb, a.out + orow * a.out_ld + ncol0, valid);
+        epilogue_tile_lean<C::kGateUp>(tb, a.out + orow * a.out_ld + ncol0, valid);
       }
       tc_fence_before();
       __syncwarp();
@@ -383,7 +420,9 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
     cp_async_wait<0>();
   } else if (C::kQ4) {
     // ------------------------------------------------------------- q4 dequant
-    const int d = threadIdx.x - C::kDqWarp0 * 32;  // B row of this thread, 0..255
+    const int dq = threadIdx.x - C::kDqWarp0 * 32;
+    const int d = dq & (kBN - 1);  // B row of this thread, 0..255
+    const int half = dq >> 8;      // codes 32 * half .. 32 * half + 31 of each stage
     const uint32_t my_tiles =
         (uint32_t)blockIdx.x < (uint32_t)total ? (total - 1 - blockIdx.x) / gridDim.x + 1 : 0;
     const uint32_t nstages = my_tiles * a.kblocks;
@@ -426,19 +465,19 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
       const int s = it % C::kStg;
       const uint32_t ph = (it / C::kStg) & 1;
       if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, lim)) { ok = false; break; }
-      const uint4* rc = reinterpret_cast<const uint4*>(raw_codes + r * (kBN * kRawRowBytes) + d * kRawRowBytes);
-      const uint4 c0 = rc[0], c1 = rc[1];
+      // this thread's half row: 32 codes (16 bytes) under one group scale
+      const uint4 cw = *reinterpret_cast<const uint4*>(raw_codes + r * (kBN * kRawRowBytes) +
+                                                        d * kRawRowBytes + half * 16);
       const uint32_t sc = (it & 1) ? sc_cur.y : sc_cur.x;
-      const float s0 = __half2float(__ushort_as_half((unsigned short)(sc & 0xFFFFu)));
-      const float s1 = __half2float(__ushort_as_half((unsigned short)(sc >> 16)));
+      const float sv = __half2float(__ushort_as_half((unsigned short)(half ? sc >> 16 : sc & 0xFFFFu)));
+      const uint64_t sx2 = f32x2(sv, sv), nx2 = f32x2(-136.0f * sv, -136.0f * sv);
       uint8_t* dst_row = sB + s * kBBytes + d * 128;
-      const uint32_t words[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
-      const uint64_t s0x2 = f32x2(s0, s0), s1x2 = f32x2(s1, s1);
-      const uint64_t n0x2 = f32x2(-136.0f * s0, -136.0f * s0), n1x2 = f32x2(-136.0f * s1, -136.0f * s1);
+      const uint32_t words[4] = {cw.x, cw.y, cw.z, cw.w};
 #pragma unroll
-      for (int c = 0; c < 8; ++c)
-        *reinterpret_cast<uint4*>(dst_row + ((c ^ (d & 7)) << 4)) =
-            dequant8(words[c], c < 4 ? s0x2 : s1x2, c < 4 ? n0x2 : n1x2);
+      for (int j = 0; j < 4; ++j) {
+        const int c = half * 4 + j;  // 16-byte chunk of the 128-byte row
+        *reinterpret_cast<uint4*>(dst_row + ((c ^ (d & 7)) << 4)) = dequant8(words[j], sx2, nx2);
+      }
       fence_proxy_async_smem();
       __syncwarp();
       if (lane == 0) {
