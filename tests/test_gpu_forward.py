@@ -338,3 +338,27 @@ def test_ungated_shared_expert_flag():
     compare_out(bf16_bits(out_g), case.oracle_layer(x_bits)["out"])
     assert not torch.equal(out_u, out_g)
     case.close()
+
+
+@pytest.mark.parametrize("E,k,H,I,T", [(512, 32, 256, 128, 200), (16, 16, 256, 128, 64),
+                                       (16, 1, 256, 128, 64), (512, 1, 2048, 512, 33)])
+def test_extreme_expert_counts_and_top_k(E, k, H, I, T):
+    """The library's limits and degenerate routings: E = 512 with k = 32 (the
+    largest of both), k = E (every token takes every expert: dense softmax
+    mixing, gap +inf), k = 1 at the tiny and the Qwen shape (ragged T)."""
+    cfg = synth.config("tiny", n_experts=E, top_k=k, hidden=H, inter=I, tokens=T, n_slots=E,
+                       lru=False)
+    case = Case(cfg)
+    table, gens = case.stage_all()
+    x_bits = synth.hidden(cfg, 0, 160)
+    out, ev = case.plan.forward(0, bf16_tensor(x_bits), case.router[0], table, gens)
+    torch.cuda.synchronize()
+    assert case.plan.status() == N.MSI_OK
+    ref = case.oracle_layer(x_bits)
+    ids = ev.ids.cpu().numpy()
+    compare_routes(ids, ev.weights.cpu().numpy(), ref)
+    assert np.array_equal(ev.counts.cpu().numpy(), np.bincount(ids.reshape(-1), minlength=E))
+    if k == E:
+        assert np.all(np.sort(ids, axis=1) == np.arange(E)) and np.all(np.isinf(ev.gap.cpu().numpy()))
+    compare_out(bf16_bits(out), ref["out"], ~oracle.near_tie_tokens(ref["gap_k"]))
+    case.close()
