@@ -266,8 +266,12 @@ namespace {
 
 // The tensor-core router splits E into chunks of min(E, 128) experts (MMA N,
 // a multiple of 16) and keeps k + 1 <= 32 candidates per chunk and token.
+// Small layers (E <= 64 and E * H <= 32,768) take the FFMA router instead:
+// sized for 64 experts, its blocks finish in a few microseconds, below the
+// fixed cost of the tensor path's three launches (decode sizes).
 bool tensor_router(const msi_plan_desc& d) {
   const int E = d.n_experts;
+  if (E <= 64 && (long long)E * d.hidden <= 32768) return false;
   return E % 16 == 0 && (E <= kRouterChunk || E % kRouterChunk == 0) && d.top_k <= 31 &&
          E / std::min(E, kRouterChunk) * std::min(d.top_k + 1, std::min(E, kRouterChunk)) <= 160;
 }

@@ -8,8 +8,10 @@
 // equal logits rank the lower expert id first.
 //
 // Block = 32 tokens x all E (<= 512) experts, 256 threads.  Each thread owns
-// an 8-token x 8-expert fp32 register tile (experts strided by 64 so a warp
-// reads 32 consecutive expert rows).  K is staged 32 at a time with cp.async:
+// an 8-token x (EP / 64)-expert fp32 register tile (experts strided by 64 so
+// a warp reads 32 consecutive expert rows); EP, the experts a block covers, is
+// 64 for E <= 64 (eight times less work and staging for small layers) and
+// 512 otherwise.  K is staged 32 at a time with cp.async:
 // x as bf16 [32 tok][32 k]; Wr as fp32 [512 e][32 k] with the eight 16-byte
 // chunks of each row XOR-swizzled by (e & 7), so a warp's 16-byte reads of
 // one k-quad hit all 32 banks once per 8 lanes.  Accumulation runs over h in
@@ -22,16 +24,23 @@ namespace msi {
 namespace {
 constexpr int TM = kRouterTM;
 constexpr int BK = 32;
-constexpr int EP = 512;                      // experts per pass (one pass covers every supported E)
 constexpr int NTH = 256;
 constexpr int XS_BYTES = TM * BK * 2;        // 2 KB
-constexpr int WS_BYTES = EP * BK * 4;        // 64 KB
-constexpr int STAGE_BYTES = XS_BYTES + WS_BYTES;
 constexpr int NSTAGE = 2;
-constexpr int LLD = EP + 4;                  // logits row stride (floats)
-constexpr int SMEM = NSTAGE * STAGE_BYTES;   // 132 KB (logits and ids reuse it)
-static_assert(TM * LLD * 4 + TM * kMaxTopK * 4 <= SMEM, "logits do not fit");
 
+// Shared-memory plan for EP experts per block (EP = 512: 132 KB; EP = 64: 20 KB;
+// the logits and ids reuse the stages).
+template <int EP>
+struct RCfg {
+  static constexpr int WS_BYTES = EP * BK * 4;
+  static constexpr int STAGE_BYTES = XS_BYTES + WS_BYTES;
+  static constexpr int LLD = EP + 4;         // logits row stride (floats)
+  static constexpr int SMEM = NSTAGE * STAGE_BYTES;
+  static constexpr int J = EP / 64;          // experts per thread
+  static_assert(TM * LLD * 4 + TM * kMaxTopK * 4 <= SMEM, "logits do not fit");
+};
+
+template <int EP>
 __device__ __forceinline__ void load_stage(const RouterArgs& a, uint8_t* st, int t0, int kb) {
   const int tid = threadIdx.x;
   uint8_t* xs = st;
@@ -52,23 +61,26 @@ __device__ __forceinline__ void load_stage(const RouterArgs& a, uint8_t* st, int
   }
 }
 
+template <int EP>
 __global__ void __launch_bounds__(NTH, 1) router_kernel(const RouterArgs a) {
+  using C = RCfg<EP>;
+  constexpr int STAGE_BYTES = C::STAGE_BYTES, LLD = C::LLD, J = C::J;
   extern __shared__ __align__(128) uint8_t smem[];
   const int tid = threadIdx.x;
   const int t0 = blockIdx.x * TM;
   const int tg = tid >> 6;   // token group: tokens tg*8 .. tg*8+7
   const int el = tid & 63;   // experts el + 64 j
-  float acc[8][8];
+  float acc[8][J];
 #pragma unroll
   for (int i = 0; i < 8; ++i)
 #pragma unroll
-    for (int j = 0; j < 8; ++j) acc[i][j] = 0.f;
+    for (int j = 0; j < J; ++j) acc[i][j] = 0.f;
 
   const int nk = a.H / BK;
-  load_stage(a, smem, t0, 0);
+  load_stage<EP>(a, smem, t0, 0);
   cp_async_commit();
   for (int kb = 0; kb < nk; ++kb) {
-    if (kb + 1 < nk) load_stage(a, smem + ((kb + 1) % NSTAGE) * STAGE_BYTES, t0, kb + 1);
+    if (kb + 1 < nk) load_stage<EP>(a, smem + ((kb + 1) % NSTAGE) * STAGE_BYTES, t0, kb + 1);
     cp_async_commit();
     cp_async_wait<1>();
     __syncthreads();
@@ -76,9 +88,9 @@ __global__ void __launch_bounds__(NTH, 1) router_kernel(const RouterArgs a) {
     const uint8_t* ws = xs + XS_BYTES;
 #pragma unroll
     for (int kq = 0; kq < BK / 4; ++kq) {
-      float4 w[8];
+      float4 w[J];
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
+      for (int j = 0; j < J; ++j) {
         const int e = el + 64 * j;
         w[j] = *reinterpret_cast<const float4*>(ws + e * 128 + ((kq ^ (e & 7)) << 4));
       }
@@ -87,7 +99,7 @@ __global__ void __launch_bounds__(NTH, 1) router_kernel(const RouterArgs a) {
         const uint2 xv = *reinterpret_cast<const uint2*>(xs + (tg * 8 + i) * 64 + kq * 8);
         const float x0 = bf16_lo(xv.x), x1 = bf16_hi(xv.x), x2 = bf16_lo(xv.y), x3 = bf16_hi(xv.y);
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
+        for (int j = 0; j < J; ++j) {
           float s = acc[i][j];
           s = fmaf(x0, w[j].x, s);
           s = fmaf(x1, w[j].y, s);
@@ -106,7 +118,7 @@ __global__ void __launch_bounds__(NTH, 1) router_kernel(const RouterArgs a) {
 #pragma unroll
   for (int i = 0; i < 8; ++i)
 #pragma unroll
-    for (int j = 0; j < 8; ++j) L[(tg * 8 + i) * LLD + el + 64 * j] = acc[i][j];
+    for (int j = 0; j < J; ++j) L[(tg * 8 + i) * LLD + el + 64 * j] = acc[i][j];
   __syncthreads();
 
   // top-k: warp w handles tokens w*4 .. w*4+3
@@ -196,16 +208,21 @@ __global__ void __launch_bounds__(NTH, 1) router_kernel(const RouterArgs a) {
 }
 }  // namespace
 
-cudaError_t launch_router(const RouterArgs& a, cudaStream_t s) {
+template <int EP>
+static cudaError_t launch_ep(const RouterArgs& a, cudaStream_t s) {
   static std::atomic<unsigned long long> attr_done{0};
   {
-    cudaError_t e = smem_attr_once(router_kernel, SMEM, attr_done);
+    cudaError_t e = smem_attr_once(router_kernel<EP>, RCfg<EP>::SMEM, attr_done);
     if (e != cudaSuccess) return e;
   }
   const int nb = (a.T + TM - 1) / TM;
   if (nb == 0) return cudaSuccess;
-  router_kernel<<<nb, NTH, SMEM, s>>>(a);
+  router_kernel<EP><<<nb, NTH, RCfg<EP>::SMEM, s>>>(a);
   return cudaGetLastError();
+}
+
+cudaError_t launch_router(const RouterArgs& a, cudaStream_t s) {
+  return a.E <= 64 ? launch_ep<64>(a, s) : launch_ep<512>(a, s);
 }
 
 }  // namespace msi

@@ -260,12 +260,13 @@ def test_simt_router_path_odd_expert_count():
     case.close()
 
 
-@pytest.mark.parametrize("E,k", [(64, 31), (64, 32), (256, 8)])
-def test_router_limits_and_chunks(E, k):
+@pytest.mark.parametrize("E,k,H", [(64, 31, 1024), (64, 32, 1024), (256, 8, 256), (64, 31, 256)])
+def test_router_limits_and_chunks(E, k, H):
     """k = 31 is the largest top-k of the tensor-core router (k + 1 candidates
     per chunk), k = 32 routes through the fp32 FFMA router, E = 256 merges two
-    128-expert chunks."""
-    cfg = synth.config("tiny", n_experts=E, top_k=k, n_slots=E, tokens=96)
+    128-expert chunks; small layers (E <= 64, E * H <= 32,768: the last case)
+    take the FFMA router sized for 64 experts."""
+    cfg = synth.config("tiny", n_experts=E, top_k=k, n_slots=E, tokens=96, hidden=H)
     case = Case(cfg)
     table, gens = case.stage_all()
     x_bits = synth.hidden(cfg, 0, 9)
@@ -281,13 +282,14 @@ def test_router_limits_and_chunks(E, k):
     case.close()
 
 
-@pytest.mark.parametrize("E", [64, 256])
-def test_exact_logit_ties_rank_lower_id_first(E):
+@pytest.mark.parametrize("E,H", [(64, 1024), (256, 256), (64, 256)])
+def test_exact_logit_ties_rank_lower_id_first(E, H):
     """Duplicated (and amplified) router rows give exactly equal logits; the
     route event must rank the lower expert id first (the oracle's order), the
-    pair adjacent with equal weights, within one 128-expert chunk (E = 64)
-    and across chunks through the candidate merge (E = 256)."""
-    cfg = synth.config("tiny", n_experts=E, n_slots=E, top_k=6, tokens=512, lru=False)
+    pair adjacent with equal weights: tensor router within one 128-expert
+    chunk (E = 64, H = 1024) and across chunks through the candidate merge
+    (E = 256); FFMA router sized for 64 experts (E = 64, H = 256)."""
+    cfg = synth.config("tiny", n_experts=E, n_slots=E, top_k=6, tokens=512, lru=False, hidden=H)
     case = Case(cfg)
     table, gens = case.stage_all()
     w = case.router_np[0].copy()
