@@ -63,6 +63,7 @@ struct Group {
   int pad1;
 };
 
+
 // ---------------------------------------------------------------------------
 // Kernel argument blocks
 // ---------------------------------------------------------------------------
@@ -77,6 +78,12 @@ struct RouterArgs {
   float* gap;              // [T] or nullptr
   float* sg;               // [T] (when wsg)
   int* bcount;             // [nb, E] routed ids per router block and expert
+  // the forward's first kernel: status cleared and the shared group written
+  // by block 0 (status null: a prediction pass, which begins nothing)
+  int* status;
+  Group* sh;               // or nullptr
+  int* sh_total;
+  int shared_slot;
 };
 
 struct RouterTcArgs {
@@ -234,6 +241,29 @@ constexpr int kBK = 64;
 constexpr int kStages = 4;
 constexpr int kABytes = kBM * kBK * 2;
 constexpr int kBBytes = kBN * kBK * 2;
+
+#ifdef __CUDACC__
+// The forward's start, written by its first kernel (one thread): the status
+// word cleared and, with a shared expert, its single group over all T rows
+// (slot = its weight block) with the 128-row and 256-row tile counts.
+__device__ __forceinline__ void forward_begin(int* status, Group* sh, int* sh_total, int T,
+                                              int shared_slot) {
+  *status = 0;
+  if (sh != nullptr) {
+    Group g;
+    g.row_begin = 0;
+    g.row_count = T;
+    g.slot = shared_slot;
+    g.mt_begin = 0;
+    g.ok = 1;
+    g.expert = -1;
+    g.pt_begin = g.pad1 = 0;
+    *sh = g;
+    sh_total[0] = (T + kBM - 1) / kBM;
+    sh_total[1] = (T + 2 * kBM - 1) / (2 * kBM);
+  }
+}
+#endif
 
 // ---------------------------------------------------------------------------
 // PTX wrappers (device)

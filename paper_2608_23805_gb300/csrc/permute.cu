@@ -208,22 +208,7 @@ __global__ void upload_kernel(const TableParams p, int* table, unsigned long lon
     table[e] = p.slot[e];
     expected[e] = p.expected[e];
   }
-  if (threadIdx.x == 0) {
-    *status = 0;
-    if (sh != nullptr) {
-      Group g;
-      g.row_begin = 0;
-      g.row_count = p.T;
-      g.slot = p.shared_slot;
-      g.mt_begin = 0;
-      g.ok = 1;
-      g.expert = -1;
-      g.pt_begin = g.pad1 = 0;
-      *sh = g;
-      sh_total[0] = (p.T + kBM - 1) / kBM;
-      sh_total[1] = (p.T + 2 * kBM - 1) / (2 * kBM);
-    }
-  }
+  if (threadIdx.x == 0) forward_begin(status, sh, sh_total, p.T, p.shared_slot);
 }
 
 // ---- generation re-check + GEMM groups (one block) ----

@@ -684,6 +684,10 @@ msi_status route_rows(msi_plan* p, FwdCtx& f, const float* rw, const msi_route_e
     ra.gap = ev->gap;
     ra.sg = at<float>(ws, L.sg);
     ra.bcount = at<int>(ws, L.bcount);
+    ra.status = first ? at<int>(ws, L.status) : nullptr;
+    ra.sh = first && d.has_shared ? at<Group>(ws, L.sh_group) : nullptr;
+    ra.sh_total = at<int>(ws, L.sh_total);
+    ra.shared_slot = tp.shared_slot;
     LAUNCH(p, MSI_K_ROUTER, s, launch_router(ra, s));
   }
   ScanArgs sa{at<int>(ws, L.bcount), nb, E, at<int>(ws, L.bbase), ev->counts};
@@ -697,10 +701,10 @@ msi_status front(msi_plan* p, FwdCtx& f, const TableParams& tp) {
   const int E = d.n_experts, k = d.top_k, H = d.hidden, I = d.inter;
   void* ws = f.ws;
   const WsLayout& L = f.L;
-  // The tensor-router path clears the status word in its first kernel and
-  // the scatter kernel writes the shared group and (resident calls) the GEMM
-  // groups, so only the other paths need the upload kernel.
-  if (f.T == 0 || !tensor_router(d))
+  // Both routers clear the status word and write the shared group in their
+  // first kernel, and the scatter kernel builds the GEMM groups (resident
+  // calls), so only a call without rows needs the upload kernel.
+  if (f.T == 0)
     LAUNCH(p, MSI_K_UPLOAD, f.cs, launch_upload(tp, at<int>(ws, L.table), at<unsigned long long>(ws, L.expected),
                             at<int>(ws, L.status), d.has_shared ? at<Group>(ws, L.sh_group) : nullptr,
                             at<int>(ws, L.sh_total), f.cs));

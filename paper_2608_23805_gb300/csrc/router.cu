@@ -65,6 +65,9 @@ template <int EP>
 __global__ void __launch_bounds__(NTH, 1) router_kernel(const RouterArgs a) {
   using C = RCfg<EP>;
   constexpr int STAGE_BYTES = C::STAGE_BYTES, LLD = C::LLD, J = C::J;
+  // the forward's first kernel (status null: a prediction pass)
+  if (blockIdx.x == 0 && threadIdx.x == 0 && a.status != nullptr)
+    forward_begin(a.status, a.sh, a.sh_total, a.T, a.shared_slot);
   extern __shared__ __align__(128) uint8_t smem[];
   const int tid = threadIdx.x;
   const int t0 = blockIdx.x * TM;

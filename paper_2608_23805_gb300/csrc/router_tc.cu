@@ -44,22 +44,9 @@ static_assert(128 * RT_LLD * 4 <= RT_STAGES * RT_STAGE, "logits tile does not fi
 
 __global__ void split3_kernel(const float* __restrict__ w, long long n, __nv_bfloat16* __restrict__ out,
                               int* status, Group* sh, int* sh_total, int T, int shared_slot) {
-  if (blockIdx.x == 0 && threadIdx.x == 0) {  // the forward's first kernel
-    if (status != nullptr) *status = 0;         // (null: a prediction pass)
-    if (sh != nullptr) {
-      Group g;
-      g.row_begin = 0;
-      g.row_count = T;
-      g.slot = shared_slot;
-      g.mt_begin = 0;
-      g.ok = 1;
-      g.expert = -1;
-      g.pt_begin = g.pad1 = 0;
-      *sh = g;
-      sh_total[0] = (T + kBM - 1) / kBM;
-      sh_total[1] = (T + 2 * kBM - 1) / (2 * kBM);
-    }
-  }
+  // the forward's first kernel (status null: a prediction pass)
+  if (blockIdx.x == 0 && threadIdx.x == 0 && status != nullptr)
+    forward_begin(status, sh, sh_total, T, shared_slot);
   for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < n;
        i += (long long)gridDim.x * blockDim.x) {
     const float v = w[i];
