@@ -41,7 +41,7 @@ def _flags(verbose_ptxas: bool) -> list[str]:
 def _stale(obj: str, src: str) -> bool:
     if not os.path.exists(obj):
         return True
-    deps = [src, os.path.join(CSRC, "internal.cuh"), os.path.join(CSRC, "source.h"),
+    deps = [src, os.path.join(CSRC, "internal.cuh"), os.path.join(CSRC, "kernels.cuh"), os.path.join(CSRC, "source.h"),
             os.path.join(ROOT, "include", "msi.h")]
     return any(os.path.getmtime(d) > os.path.getmtime(obj) for d in deps)
 

@@ -26,7 +26,7 @@
 //    library routine.
 #include <mutex>
 
-#include "internal.cuh"
+#include "kernels.cuh"
 
 namespace {
 

@@ -11,7 +11,7 @@
 // requested object and version, and a mismatch is rejected before any
 // consumer reads the slot (paper, Sec. "Lifetime Is Part of Correctness";
 // Sec. "Stable Slots and Bundle Publication").
-#include "internal.cuh"
+#include "kernels.cuh"
 
 namespace msi {
 

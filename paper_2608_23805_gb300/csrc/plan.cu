@@ -32,7 +32,7 @@
 #include <thread>
 #include <vector>
 
-#include "internal.cuh"
+#include "kernels.cuh"
 #include "source.h"
 
 using namespace msi;

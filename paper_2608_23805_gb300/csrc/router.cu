@@ -17,7 +17,7 @@
 // one k-quad hit all 32 banks once per 8 lanes.  Accumulation runs over h in
 // ascending order.  Top-k: one warp per token, k+1 rounds of a warp-shuffle
 // argmax over (logit desc, id asc).
-#include "internal.cuh"
+#include "kernels.cuh"
 
 namespace msi {
 

@@ -27,7 +27,7 @@
 // Warps 0-3 move the logits from TMEM to shared memory, warp 4 MMA + TMEM,
 // warp 5 TMA producer (one lane each for the single-thread roles; every role
 // claims its whole warp); then all eight warps select.  All waits are bounded.
-#include "internal.cuh"
+#include "kernels.cuh"
 
 namespace msi {
 
