@@ -10,6 +10,7 @@ namespace msi {
 
 constexpr int kRouterTM = 32;  // tokens per fp32 FFMA router block
 constexpr int kRouterChunk = 128;  // experts per tensor-core router CTA
+constexpr int kScatterWarps = 4;   // scatter warps per block, one per router block
 
 struct RouterArgs {
   const __nv_bfloat16* x;  // [T, H]
@@ -59,6 +60,12 @@ struct ScatterArgs {
   const int* ids;     // [T*k]
   const int* counts;  // [E]
   const int* bbase;   // [nb, E]
+  // fuse_scan (nb <= kScatterWarps: one block's warps cover every router
+  // block): counts and block prefixes are taken from bcount here, and the
+  // last block writes the counts to counts_out (no column-scan launch)
+  int fuse_scan;
+  const int* bcount;  // [nb, E]
+  int* counts_out;    // [E]
   int T, k, E, nb;
   int tm;             // tokens per router block
   int* perm;          // [T*k]

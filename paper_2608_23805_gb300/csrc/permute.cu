@@ -52,7 +52,6 @@ __device__ __forceinline__ int check_code(const GenWord* gw, int slot, int layer
 }
 
 // ---- scatter: one warp per router block ----
-constexpr int kScatterWarps = 4;
 
 // Exclusive scan over the block of four values per thread (128 threads);
 // returns the thread's base and leaves the block total in *total.
@@ -80,7 +79,8 @@ __device__ __forceinline__ int scan4(const int (&v)[4], int* wsum, int* total) {
 // Setup block of the scatter, resident call: the generation re-check of every
 // routed expert's slot (fail closed) and the GEMM groups with their 128- and
 // 256-row tile prefixes.
-__device__ void scatter_setup(const ScatterArgs& a, const TableParams& tp, const int* offs) {
+__device__ void scatter_setup(const ScatterArgs& a, const TableParams& tp, const int* offs,
+                              const int* s_cnt) {
   __shared__ int wsum[kScatterWarps];
   __shared__ int kmin[kScatterWarps];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -92,7 +92,7 @@ __device__ void scatter_setup(const ScatterArgs& a, const TableParams& tp, const
     const int e = tid * 4 + i;
     cnt[i] = code[i] = mt[i] = pt[i] = 0;
     if (e < a.E) {
-      cnt[i] = a.counts[e];
+      cnt[i] = s_cnt[e];
       if (cnt[i] > 0) code[i] = check_code(a.genwords, tp.slot[e], tp.layer, e, tp.expected[e]);
       if (code[i] == 0) {
         mt[i] = (cnt[i] + kBM - 1) / kBM;
@@ -139,16 +139,27 @@ __device__ void scatter_setup(const ScatterArgs& a, const TableParams& tp, const
 __global__ void __launch_bounds__(kScatterWarps * 32) scatter_kernel(const ScatterArgs a,
                                                                      const TableParams tp) {
   __shared__ int offs[kMaxExperts + 1];
+  __shared__ int s_cnt[kMaxExperts];
   __shared__ int run[kScatterWarps][kMaxExperts];
   __shared__ int wsum[kScatterWarps];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
-  // exclusive scan of counts (E <= 512, 128 threads x 4 values)
+  // exclusive scan of counts (E <= 512, 128 threads x 4 values); with
+  // fuse_scan the counts are the column sums of the router blocks' counts
   int v[4], s = 0;
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
     const int e = tid * 4 + i;
-    v[i] = (e < a.E) ? a.counts[e] : 0;
+    int c = 0;
+    if (e < a.E) {
+      if (a.fuse_scan) {
+        for (int b = 0; b < a.nb; ++b) c += a.bcount[(size_t)b * a.E + e];
+      } else {
+        c = a.counts[e];
+      }
+      s_cnt[e] = c;
+    }
+    v[i] = c;
     s += v[i];
   }
   int incl = s;
@@ -173,7 +184,9 @@ __global__ void __launch_bounds__(kScatterWarps * 32) scatter_kernel(const Scatt
   // the resident setup, in parallel with the scatter
   if (blockIdx.x == gridDim.x - 1) {
     for (int e = tid; e <= a.E; e += blockDim.x) a.offsets[e] = offs[e];
-    scatter_setup(a, tp, offs);
+    if (a.fuse_scan)
+      for (int e = tid; e < a.E; e += blockDim.x) a.counts_out[e] = s_cnt[e];
+    scatter_setup(a, tp, offs, s_cnt);
     return;
   }
 
@@ -191,7 +204,13 @@ __global__ void __launch_bounds__(kScatterWarps * 32) scatter_kernel(const Scatt
     int before = 0;
     if (valid) {
       before = run[warp][e];
-      const int pos = offs[e] + a.bbase[(size_t)b * a.E + e] + before + __popc(mask & lt);
+      int pre = 0;  // this expert's ids in the router blocks before b
+      if (a.fuse_scan) {
+        for (int bb = 0; bb < b; ++bb) pre += a.bcount[(size_t)bb * a.E + e];
+      } else {
+        pre = a.bbase[(size_t)b * a.E + e];
+      }
+      const int pos = offs[e] + pre + before + __popc(mask & lt);
       a.perm[pos] = f;
       a.inv[f] = pos;
     }

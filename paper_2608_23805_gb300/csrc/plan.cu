@@ -620,7 +620,7 @@ msi_status validate_fwd(msi_plan* p, int layer, const void* x, int T, const floa
 // no gate; it reuses the router scratch of the workspace, so it must be
 // ordered after the forward's own routing and scatter.
 msi_status route_rows(msi_plan* p, FwdCtx& f, const float* rw, const msi_route_event* ev, bool first,
-                      const TableParams& tp, cudaStream_t s) {
+                      const TableParams& tp, cudaStream_t s, bool scan = true) {
   const auto& d = p->d;
   const int E = d.n_experts, k = d.top_k, H = d.hidden;
   void* ws = f.ws;
@@ -690,8 +690,12 @@ msi_status route_rows(msi_plan* p, FwdCtx& f, const float* rw, const msi_route_e
     ra.shared_slot = tp.shared_slot;
     LAUNCH(p, MSI_K_ROUTER, s, launch_router(ra, s));
   }
-  ScanArgs sa{at<int>(ws, L.bcount), nb, E, at<int>(ws, L.bbase), ev->counts};
-  LAUNCH(p, MSI_K_SCAN, s, launch_colscan(sa, s));
+  // the column scan (per-block prefixes and counts); a small forward's
+  // scatter takes it over (scan = false)
+  if (scan) {
+    ScanArgs sa{at<int>(ws, L.bcount), nb, E, at<int>(ws, L.bbase), ev->counts};
+    LAUNCH(p, MSI_K_SCAN, s, launch_colscan(sa, s));
+  }
   return MSI_OK;
 }
 
@@ -717,11 +721,17 @@ msi_status front(msi_plan* p, FwdCtx& f, const TableParams& tp) {
   if (d.has_shared) {
     if (!make_tmap(&f.tm_hs, at<char>(ws, L.hs), I, f.T, 128)) return MSI_ERR_CUDA;
   }
-  msi_status st = route_rows(p, f, f.router_w, f.ev, true, tp, f.cs);
+  // up to kScatterWarps router blocks: one scatter block covers them all and
+  // takes over the column scan (one launch fewer for decode-sized calls)
+  const bool fuse_scan = nb <= kScatterWarps;
+  msi_status st = route_rows(p, f, f.router_w, f.ev, true, tp, f.cs, !fuse_scan);
   if (st != MSI_OK) return st;
   ScatterArgs xa{};
   xa.ids = f.ev->ids;
   xa.counts = f.ev->counts;
+  xa.fuse_scan = fuse_scan ? 1 : 0;
+  xa.bcount = at<int>(ws, L.bcount);
+  xa.counts_out = f.ev->counts;
   xa.bbase = at<int>(ws, L.bbase);
   xa.T = f.T;
   xa.k = k;
