@@ -26,14 +26,15 @@ constexpr int TM = kRouterTM;
 constexpr int BK = 32;
 constexpr int NTH = 256;
 constexpr int XS_BYTES = TM * BK * 2;        // 2 KB
-constexpr int NSTAGE = 2;
 
-// Shared-memory plan for EP experts per block (EP = 512: 132 KB; EP = 64: 20 KB;
-// the logits and ids reuse the stages).
+// Shared-memory plan for EP experts per block (the logits and ids reuse the
+// stages): EP = 512, two 66 KB stages; EP = 64, eight 10 KB stages, so that a
+// small layer's whole K (H <= 256) is in flight at once.
 template <int EP>
 struct RCfg {
   static constexpr int WS_BYTES = EP * BK * 4;
   static constexpr int STAGE_BYTES = XS_BYTES + WS_BYTES;
+  static constexpr int NSTAGE = EP <= 64 ? 8 : 2;
   static constexpr int LLD = EP + 4;         // logits row stride (floats)
   static constexpr int SMEM = NSTAGE * STAGE_BYTES;
   static constexpr int J = EP / 64;          // experts per thread
@@ -64,7 +65,7 @@ __device__ __forceinline__ void load_stage(const RouterArgs& a, uint8_t* st, int
 template <int EP>
 __global__ void __launch_bounds__(NTH, 1) router_kernel(const RouterArgs a) {
   using C = RCfg<EP>;
-  constexpr int STAGE_BYTES = C::STAGE_BYTES, LLD = C::LLD, J = C::J;
+  constexpr int STAGE_BYTES = C::STAGE_BYTES, LLD = C::LLD, J = C::J, NSTAGE = C::NSTAGE;
   // the forward's first kernel (status null: a prediction pass)
   if (blockIdx.x == 0 && threadIdx.x == 0 && a.status != nullptr)
     forward_begin(a.status, a.sh, a.sh_total, a.T, a.shared_slot);
@@ -80,12 +81,18 @@ __global__ void __launch_bounds__(NTH, 1) router_kernel(const RouterArgs a) {
     for (int j = 0; j < J; ++j) acc[i][j] = 0.f;
 
   const int nk = a.H / BK;
-  load_stage<EP>(a, smem, t0, 0);
-  cp_async_commit();
-  for (int kb = 0; kb < nk; ++kb) {
-    if (kb + 1 < nk) load_stage<EP>(a, smem + ((kb + 1) % NSTAGE) * STAGE_BYTES, t0, kb + 1);
+  // NSTAGE - 1 stages ahead; each iteration refills the slot the previous one
+  // consumed, then waits for its own stage
+#pragma unroll
+  for (int i = 0; i < NSTAGE - 1; ++i) {
+    if (i < nk) load_stage<EP>(a, smem + i * STAGE_BYTES, t0, i);
     cp_async_commit();
-    cp_async_wait<1>();
+  }
+  for (int kb = 0; kb < nk; ++kb) {
+    const int nx = kb + NSTAGE - 1;
+    if (nx < nk) load_stage<EP>(a, smem + (nx % NSTAGE) * STAGE_BYTES, t0, nx);
+    cp_async_commit();
+    cp_async_wait<NSTAGE - 1>();
     __syncthreads();
     const uint8_t* xs = smem + (kb % NSTAGE) * STAGE_BYTES;
     const uint8_t* ws = xs + XS_BYTES;
