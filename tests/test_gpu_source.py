@@ -37,9 +37,10 @@ def _source(case, tmp_path, direct, n_windows=8):
     return src, off
 
 
-@pytest.mark.parametrize("direct", [False, True])
-def test_streamed_from_file_equals_host_windows(tmp_path, direct):
-    cfg = synth.config("tiny")
+@pytest.mark.parametrize("direct,wdtype", [(False, N.MSI_W_BF16), (True, N.MSI_W_BF16),
+                                          (True, N.MSI_W_Q4G32)])
+def test_streamed_from_file_equals_host_windows(tmp_path, direct, wdtype):
+    cfg = synth.config("tiny", wdtype=wdtype)
     a, b = Case(cfg), Case(cfg)
     src, off = _source(b, tmp_path, direct, n_windows=4)
     b.plan.set_source(src, off)
