@@ -1,6 +1,9 @@
 // Host runtime of the C ABI: the Plan (immutable manifest + mutable slot
-// ledger), slot staging with generation publication, the LRU-wave residency
-// driver, and the two layer-forward entry points.
+// ledger), slot staging with generation publication (from host windows or
+// through the bounded source service), the LRU-wave residency driver with
+// next-layer prediction, the two-bank prefetch and caller pins, the layer
+// forwards (caller-managed residency, plan-managed waves, and their
+// host-buffer variants), reset, shutdown and the host-side fault hooks.
 //
 // Paper basis:
 //  - Plan = manifest (object -> extent, slot compatibility, stable device
@@ -16,10 +19,16 @@
 //    Sec. "Implementation", "Scheduling and copies").
 //  - Telemetry: stages, cache events, generations, H2D bytes, rejections
 //    (Sec. "Implementation", "Telemetry").
-//  - Per-layer LRU over 64 slots (Sec. "Evaluation", "Cache and storage
-//    state").  The wave policy (hits then misses, waves of half the pool, the
-//    previous wave pinned, least-recent victim, lowest index on ties) is the
-//    reading this library takes where the paper gives no rule.
+//  - Per-layer LRU over 64 slots, with a two-bank next-layer prefetch (Sec.
+//    "Evaluation", "Cache and storage state").  The wave policy (hits then
+//    misses, waves of half the pool, the previous wave pinned, least-recent
+//    victim, lowest index on ties) and the prefetch bundle (the predicted
+//    objects ranked by predicted count, placed after the last wave) are the
+//    readings this library takes where the paper gives no rule.
+//  - Reset advances the request epoch after the outstanding-work checks;
+//    shutdown also checks the source's outstanding work (Sec. "Separate
+//    Window and GPU-Slot Lifecycles"; the fault cells of the paper's fault
+//    table).
 #include <cudaTypedefs.h>
 
 #include <algorithm>
