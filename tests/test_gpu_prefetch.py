@@ -242,3 +242,39 @@ def test_failed_predicting_call_leaves_the_plan_usable():
     compare_out(bf16_bits(out1), case.oracle_layer(x_bits, 1)["out"])
     compare_out(bf16_bits(out0), case.oracle_layer(x_bits, 0)["out"])
     case.close()
+
+
+def test_pins_with_prediction_match_the_simulator():
+    """Pins and the prefetch bundle together (2 layers of the tiny shape, 16
+    slots in waves of 4, so four objects may be pinned): over alternating
+    layer calls with prediction, the trace equals the simulator's with the same
+    pins and predictions, and no pinned object is ever evicted."""
+    cfg = synth.config("decode48", tokens=24, n_layers=2, n_slots=16)
+    case = Case(cfg, wave_capacity=4)
+    sim = oracle.LRUWaveSim(cfg.n_slots, 4)
+    pins = [(0, 1), (0, 5), (1, 2), (1, 9)]
+    for l, e in pins:
+        case.plan.pin(l, e)
+        sim.pin(l, e)
+    stage = torch.cuda.Stream()
+    for step in range(5):
+        x_bits = synth.hidden(cfg, 0, 300 + step)
+        for l in range(2):
+            nxt = case.router[1] if l == 0 else None
+            out, ev = case.plan.forward_streamed(l, bf16_tensor(x_bits), case.router[l],
+                                                 residual=True, stage_stream=stage,
+                                                 next_router_w=nxt)
+            torch.cuda.synchronize()
+            assert case.plan.status() == N.MSI_OK
+            compare_out(bf16_bits(out), case.oracle_layer(x_bits, l, residual=True)["out"])
+            predict = None
+            if nxt is not None:
+                _, counts = _predicted_counts(ev.next, cfg.n_experts)
+                predict = (1, counts)
+            sim.call(l, sorted(set(ev.ids.cpu().numpy().reshape(-1).tolist())), predict)
+            x_bits = bf16_bits(out)
+    tr = case.plan.trace()
+    assert tr == sim.trace
+    assert not {(r[1], r[2]) for r in tr if r[5] == "evict"} & set(pins)
+    _check_counters(case, sim)
+    case.close()
