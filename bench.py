@@ -79,7 +79,7 @@ def kernel_source_hash() -> str:
     and blank lines left out: a capture stays valid until the code changes."""
     import re
     h = hashlib.sha256()
-    for name in ("gemm.cu", "internal.cuh"):
+    for name in ("gemm.cu", "gemm_pair.cu", "internal.cuh"):
         with open(os.path.join(ROOT, "paper_2608_23805_gb300", "csrc", name)) as f:
             src = re.sub(r"/\*.*?\*/", "", f.read(), flags=re.S)
         for line in src.splitlines():

@@ -38,7 +38,16 @@
 //
 // Roles per CTA: warps 0-3 epilogue, warp 4 MMA issue (even CTA) or stage
 // relay (odd CTA) and TMEM allocation, warp 5 TMA producer, warps 6-9 row
-// gather (gate-up over routed rows).
+// gather (gate-up over routed rows), and in the 4-bit modes sixteen dequant
+// warps.
+//
+// 4-bit modes: each CTA converts only its own 128 B rows (half of the pair
+// tile's 256), so per unit of tensor work a CTA dequantises half as many
+// weights as a single-CTA tile does.  The producer loads the CTA's 128 rows of
+// packed codes per stage by TMA into a three-stage raw ring; each dequant
+// thread converts a quarter row (16 codes under one group scale) into the
+// CTA's SW128 B stage and arrives on its own `full` barrier, which the relay
+// forwards as in the bf16 modes.
 #include <algorithm>
 
 #include "internal.cuh"
@@ -54,20 +63,68 @@ constexpr int kPB = 128 * kBK * 2;         // 16 KB: this CTA's 128 B rows of on
 constexpr uint32_t kPIdesc = idesc_bf16(kPairRows, kBN);
 constexpr int kPEpiWarps = 4;
 constexpr int kPGatherWarps = 4;
+constexpr int kPRawRow = 32;               // 64 codes of one B row per stage (one TMA box row)
 
 template <int MODE>
 struct PCfg {
-  static constexpr bool kGather = (MODE == kGateUpGather);
-  static constexpr bool kGateUp = (MODE == kGateUpGather || MODE == kGateUpTma);
+  static constexpr bool kQ4 = (MODE == kGateUpGatherQ4 || MODE == kDownQ4);
+  static constexpr bool kGather = (MODE == kGateUpGather || MODE == kGateUpGatherQ4);
+  static constexpr bool kGateUp = (MODE == kGateUpGather || MODE == kGateUpTma || MODE == kGateUpGatherQ4);
   static constexpr int kGatherWarp0 = 6;
-  static constexpr int kThreads = (kGatherWarp0 + (kGather ? kPGatherWarps : 0)) * 32;
-  static constexpr uint32_t kTx = kPB + (kGather ? 0 : kPA);
-  // own producer (expect_tx) + own gather threads (one arrival each as their copies land)
-  static constexpr int kFullLocal = 1 + (kGather ? kPGatherWarps * 32 : 0);
+  static constexpr int kDqWarp0 = kGatherWarp0 + (kGather ? kPGatherWarps : 0);
+  static constexpr int kDq = kQ4 ? 16 : 0;  // dequant warps (one thread per quarter B row)
+  static constexpr int kThreads = (kDqWarp0 + kDq) * 32;
+  // the producer arms `full` when it loads an operand by TMA (B in the bf16
+  // modes, A whenever the rows are not gathered)
+  static constexpr bool kProducerFull = !kQ4 || !kGather;
+  static constexpr uint32_t kTx = (kQ4 ? 0 : kPB) + (kGather ? 0 : kPA);
+  // own producer (expect_tx) + own gather threads (one arrival each as their
+  // copies land) + own dequant warps
+  static constexpr int kFullLocal = (kProducerFull ? 1 : 0) + (kGather ? kPGatherWarps * 32 : 0) + kDq;
+  static constexpr int kRaw = kQ4 ? 3 : 1;
+  static constexpr int kRawBytes = kQ4 ? kRaw * 128 * kPRawRow : 0;
+  static constexpr uint32_t kRawTx = 128 * kPRawRow;
   // + the groups' 256-row tile prefix and slot (shared-memory tile lookups)
-  static constexpr int kSmem = 1024 + kPStages * (kPA + kPB) + 256 + kPEpiWarps * 4096 +
+  static constexpr int kSmem = 1024 + kPStages * (kPA + kPB) + kRawBytes + 256 + kPEpiWarps * 4096 +
                                (2 * kMaxExperts + 2) * 4;
 };
+
+// The staged epilogue of one warp's 32 rows, TMEM read 16 columns at a time
+// (the 4-bit modes' thread count leaves 72 registers a thread).
+template <bool GATEUP>
+__device__ __forceinline__ void epilogue_tile_staged_lean(uint32_t tb, __nv_bfloat16* row0, size_t ld,
+                                                          int nvalid, uint8_t* stg, int lane) {
+  if (GATEUP) {
+#pragma unroll 1
+    for (int c = 0; c < 128; c += 16) {
+      uint32_t g[16], u[16];
+      tmem_ld16(tb + c, g);
+      tmem_ld16(tb + 128 + c, u);
+      tmem_ld_wait(g);
+      tmem_ld_wait(u);
+      uint32_t p[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const float g0 = __uint_as_float(g[2 * i]), g1 = __uint_as_float(g[2 * i + 1]);
+        const float u0 = __uint_as_float(u[2 * i]), u1 = __uint_as_float(u[2 * i + 1]);
+        p[i] = pack_bf16x2(__fdividef(g0 * u0, 1.0f + __expf(-g0)),
+                           __fdividef(g1 * u1, 1.0f + __expf(-g1)));
+      }
+      store_rows_staged<32>(p, stg, row0 + c, ld, nvalid, lane);
+    }
+  } else {
+#pragma unroll 1
+    for (int c = 0; c < kBN; c += 16) {
+      uint32_t v[16];
+      tmem_ld16(tb + c, v);
+      tmem_ld_wait(v);
+      uint32_t p[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) p[i] = pack_bf16x2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1]));
+      store_rows_staged<32>(p, stg, row0 + c, ld, nvalid, lane);
+    }
+  }
+}
 
 struct PairTile {
   int g, m2, n;
@@ -104,12 +161,15 @@ __global__ void __launch_bounds__(PCfg<MODE>::kThreads, 1)
                                              ~static_cast<uintptr_t>(1023));
   uint8_t* sA = smem;
   uint8_t* sB = smem + kPStages * kPA;
-  uint64_t* full = reinterpret_cast<uint64_t*>(sB + kPStages * kPB);
+  uint8_t* raw_codes = sB + kPStages * kPB;  // q4: [C::kRaw][128][32]
+  uint64_t* full = reinterpret_cast<uint64_t*>(raw_codes + C::kRawBytes);
   uint64_t* empty = full + kPStages;
   uint64_t* tfull = empty + kPStages;
   uint64_t* tempty = tfull + 2;
   uint64_t* drain = tempty + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  uint64_t* raw_full = drain + 1;            // q4: code stage landed (TMA bytes)
+  uint64_t* raw_empty = raw_full + C::kRaw;  // q4: code stage converted by every dequant warp
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(raw_empty + C::kRaw);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   uint8_t* epi_stage = reinterpret_cast<uint8_t*>(full) + 256;  // 4 KB per epilogue warp
   int* s_pt = reinterpret_cast<int*>(epi_stage + kPEpiWarps * 4096);  // [num_groups + 1]
@@ -130,6 +190,10 @@ __global__ void __launch_bounds__(PCfg<MODE>::kThreads, 1)
       mbar_init(&tempty[b], 2 * kPEpiWarps);  // the epilogue warps of both CTAs
     }
     mbar_init(drain, 1);
+    for (int r = 0; r < C::kRaw && C::kQ4; ++r) {
+      mbar_init(&raw_full[r], 1);
+      mbar_init(&raw_empty[r], C::kDq);
+    }
     *abort_flag = 0;
     mbar_fence_init();
   }
@@ -158,7 +222,7 @@ __global__ void __launch_bounds__(PCfg<MODE>::kThreads, 1)
   if (warp == 5) {
     // ------------------------------------------------------------- TMA producer
     if (lane == 0) {
-      uint32_t it = 0;
+      uint32_t it = 0, raw_issued = 0;
       // the next tile's first A row is loaded one tile ahead
       int rb_next = pair < total ? __ldg(&a.groups[decode_pair(a, s_pt, pair).g].row_begin) : 0;
       for (int t = pair; t < total; t += npairs) {
@@ -170,13 +234,26 @@ __global__ void __launch_bounds__(PCfg<MODE>::kThreads, 1)
         const int brow = C::kGateUp ? brow0 + (rank ? a.up_off : 0) + tc.n * 128
                                     : brow0 + tc.n * kBN + (int)rank * 128;
         const int arow = rb + tc.m2 * kPairRows + (int)rank * kBM;
+        // q4: this CTA's 128 rows of packed codes (gate-up: gate rows in the
+        // even CTA, up rows in the odd one, as for the bf16 rows)
+        const int qbase = s_slot[tc.g] * a.q4_rows_per_slot + a.q4_row_off;
+        const int qrow = C::kGateUp ? qbase + (rank ? a.up_off : 0) + tc.n * 128
+                                    : qbase + tc.n * kBN + (int)rank * 128;
         bool ok = true;
         for (int kb = 0; kb < a.kblocks; ++kb, ++it) {
+          if (C::kQ4) {
+            const int r = it % C::kRaw;
+            if (!mbar_wait(&raw_empty[r], ((it / C::kRaw) & 1) ^ 1, abort_flag, lim)) { ok = false; break; }
+            mbar_arrive_expect_tx(&raw_full[r], C::kRawTx);
+            tma_load_2d(raw_codes + r * (128 * kPRawRow), &tmB, &raw_full[r], kb * kPRawRow, qrow);
+            ++raw_issued;
+            if (!C::kProducerFull) continue;
+          }
           const int s = it % kPStages;
           const uint32_t ph = (it / kPStages) & 1;
           if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, lim)) { ok = false; break; }
           mbar_arrive_expect_tx(&full[s], C::kTx);
-          tma_load_2d(sB + s * kPB, &tmB, &full[s], kb * kBK, brow);
+          if (!C::kQ4) tma_load_2d(sB + s * kPB, &tmB, &full[s], kb * kBK, brow);
           if (!C::kGather) tma_load_2d(sA + s * kPA, &tmA, &full[s], kb * kBK, arow);
         }
         if (!ok) break;
@@ -184,11 +261,18 @@ __global__ void __launch_bounds__(PCfg<MODE>::kThreads, 1)
       // On abort, wait (bounded) for the copies this thread armed to land
       // before the CTA's shared memory is released.
       if (*abort_flag) {
-        for (int d = 0; d < kPStages && it > 0; ++d) {
+        for (int d = 0; d < kPStages && it > 0 && C::kProducerFull; ++d) {
           const uint32_t j = it - 1 - d;
           if ((int)j < 0) break;
           const long long t0 = clock64();
           while (!mbar_try_wait(&full[j % kPStages], (j / kPStages) & 1) && clock64() - t0 < lim) {
+          }
+        }
+        for (int d = 0; d < C::kRaw && C::kQ4; ++d) {
+          if ((int)raw_issued - 1 - d < 0) break;
+          const uint32_t j = raw_issued - 1 - d;
+          const long long t0 = clock64();
+          while (!mbar_try_wait(&raw_full[j % C::kRaw], (j / C::kRaw) & 1) && clock64() - t0 < lim) {
           }
         }
       }
@@ -256,9 +340,12 @@ __global__ void __launch_bounds__(PCfg<MODE>::kThreads, 1)
       tc_fence_after();
       const uint32_t tb = tmem_base + ((uint32_t)(warp * 32) << 16) + acc * kBN;
       const int row_w = tc.m2 * kPairRows + (int)rank * kBM + warp * 32;  // warp's first row in the group
-      epilogue_tile_staged<C::kGateUp>(
-          tb, a.out + ((size_t)__ldg(&G->row_begin) + row_w) * a.out_ld + tc.n * (C::kGateUp ? 128 : kBN),
-          a.out_ld, cnt - row_w, epi_stage + warp * 4096, lane);
+      __nv_bfloat16* row0 =
+          a.out + ((size_t)__ldg(&G->row_begin) + row_w) * a.out_ld + tc.n * (C::kGateUp ? 128 : kBN);
+      if (C::kQ4)
+        epilogue_tile_staged_lean<C::kGateUp>(tb, row0, a.out_ld, cnt - row_w, epi_stage + warp * 4096, lane);
+      else
+        epilogue_tile_staged<C::kGateUp>(tb, row0, a.out_ld, cnt - row_w, epi_stage + warp * 4096, lane);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive_remote(lead_tempty[acc]);
@@ -317,6 +404,57 @@ __global__ void __launch_bounds__(PCfg<MODE>::kThreads, 1)
       }
     }
     cp_async_wait<0>();
+  } else if (C::kQ4 && warp >= C::kDqWarp0) {
+    // ------------------------------------------------------------- q4 dequant
+    // a warp takes 8 rows, four lanes to a row: its code reads cover 256
+    // contiguous bytes and its SW128 writes hit distinct banks
+    const int d = (warp - C::kDqWarp0) * 8 + (lane >> 2);  // this CTA's B row, 0..127
+    const int qt = lane & 3;                                // codes 16 qt .. 16 qt + 15 of each stage
+    const uint32_t my_tiles = pair < total ? (uint32_t)((total - 1 - pair) / npairs + 1) : 0u;
+    const uint32_t nstages = my_tiles * (uint32_t)a.kblocks;
+    // this thread's scale row for tile ordinal j (shared-memory group table)
+    uint32_t srow_tile = 0xFFFFFFFFu;
+    const uint8_t* srow = nullptr;
+    auto scales_of = [&](uint32_t st) -> uint2 {  // stages st, st + 1 (st even)
+      const uint32_t j = st / a.kblocks;
+      if (j != srow_tile) {
+        const PairTile tc = decode_pair(a, s_pt, pair + (int)j * npairs);
+        const int row = C::kGateUp ? (rank ? a.up_off : 0) + tc.n * 128 + d
+                                   : tc.n * kBN + (int)rank * 128 + d;
+        srow = a.q4_pool + (unsigned long long)s_slot[tc.g] * a.q4_extent + a.q4_scale_off +
+               (size_t)row * a.q4_scale_ld;
+        srow_tile = j;
+      }
+      // 4 fp16 scales, 8-byte aligned (row stride K / 16 bytes, K a multiple of 128)
+      return __ldg(reinterpret_cast<const uint2*>(srow + (st % a.kblocks) * 4));
+    };
+    uint2 sc_cur = nstages > 0 ? scales_of(0) : make_uint2(0, 0);
+    uint2 sc_nxt = nstages > 2 ? scales_of(2) : make_uint2(0, 0);
+    for (uint32_t it = 0; it < nstages; ++it) {
+      if (it > 0 && (it & 1) == 0) {
+        sc_cur = sc_nxt;
+        if (it + 2 < nstages) sc_nxt = scales_of(it + 2);
+      }
+      const int r = it % C::kRaw;
+      if (!mbar_wait(&raw_full[r], (it / C::kRaw) & 1, abort_flag, lim)) break;
+      const int s = it % kPStages;
+      const uint32_t ph = (it / kPStages) & 1;
+      if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, lim)) break;
+      const uint2 cw = *reinterpret_cast<const uint2*>(raw_codes + r * (128 * kPRawRow) + d * kPRawRow + qt * 8);
+      const uint32_t sc = (it & 1) ? sc_cur.y : sc_cur.x;
+      const float sv = __half2float(__ushort_as_half((unsigned short)(qt >= 2 ? sc >> 16 : sc & 0xFFFFu)));
+      const uint64_t sx2 = f32x2(sv, sv), nx2 = f32x2(-136.0f * sv, -136.0f * sv);
+      uint8_t* dst_row = sB + s * kPB + d * 128;
+      const int c0 = qt * 2;  // 16-byte chunks c0, c0 + 1 of the 128-byte row
+      *reinterpret_cast<uint4*>(dst_row + ((c0 ^ (d & 7)) << 4)) = dequant8(cw.x, sx2, nx2);
+      *reinterpret_cast<uint4*>(dst_row + (((c0 + 1) ^ (d & 7)) << 4)) = dequant8(cw.y, sx2, nx2);
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(&full[s]);
+        mbar_arrive(&raw_empty[r]);  // the warp's rows of this code stage are consumed
+      }
+    }
   }
 
   tc_fence_before();
@@ -382,6 +520,8 @@ cudaError_t launch_gemm_pair(int mode, const CUtensorMap& tmA, const CUtensorMap
     case kGateUpGather: return launch_pair_mode<kGateUpGather>(tmA, tmB, a, max_pairs, s);
     case kGateUpTma: return launch_pair_mode<kGateUpTma>(tmA, tmB, a, max_pairs, s);
     case kDown: return launch_pair_mode<kDown>(tmA, tmB, a, max_pairs, s);
+    case kGateUpGatherQ4: return launch_pair_mode<kGateUpGatherQ4>(tmA, tmB, a, max_pairs, s);
+    case kDownQ4: return launch_pair_mode<kDownQ4>(tmA, tmB, a, max_pairs, s);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -511,6 +511,42 @@ __device__ __forceinline__ void epilogue_tile_staged(uint32_t tb, __nv_bfloat16*
   }
 }
 
+// ---------------------------------------------------------------------------
+// 4-bit weights (both GEMM kernels)
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint64_t f32x2(float lo, float hi) {
+  uint64_t v;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(v) : "r"(__float_as_uint(lo)), "r"(__float_as_uint(hi)));
+  return v;
+}
+
+// Eight 4-bit codes of one 32-bit word (code 2i in the low nibble of byte i,
+// code 2i+1 in its high nibble) -> eight bf16 weights scale * (q - 8), the
+// 16-byte chunk of one K-major row.  Each code becomes the float 128 + q by
+// placing its byte under the exponent byte 0x43 (one byte permute; q < 16
+// fills the top mantissa bits); one fused multiply-add per two values then
+// gives (128 + q) * s - 136 * s = (q - 8) * s exactly (the product needs at
+// most 8 + 11 bits and the fp16-exact scale times 136 is exact in fp32), and
+// each weight is rounded once to bf16.  nbias2 holds -136 * s twice.
+__device__ __forceinline__ uint4 dequant8(uint32_t w, uint64_t scale2, uint64_t nbias2) {
+  const uint32_t lo = w & 0x0F0F0F0Fu, hi = (w >> 4) & 0x0F0F0F0Fu;
+  uint32_t o[4];
+#pragma unroll
+  for (int b = 0; b < 4; ++b) {
+    uint32_t el, eh;
+    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(el) : "r"(lo), "r"(0x43000000u), "r"(0x7044u + (b << 8)));
+    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(eh) : "r"(hi), "r"(0x43000000u), "r"(0x7044u + (b << 8)));
+    uint64_t v;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(v) : "r"(el), "r"(eh));
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(v) : "l"(v), "l"(scale2), "l"(nbias2));
+    uint32_t vl, vh;
+    asm("mov.b64 {%0, %1}, %2;" : "=r"(vl), "=r"(vh) : "l"(v));
+    // the first operand lands in the upper half: (odd column, even column)
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(o[b]) : "r"(vh), "r"(vl));
+  }
+  return make_uint4(o[0], o[1], o[2], o[3]);
+}
+
 #endif  // __CUDACC__
 
 }  // namespace msi

@@ -814,10 +814,14 @@ bool pair_tiles(const FwdCtx& f, long long rows, int groups, long long min_rows 
   return !(f.flags & MSI_FWD_SINGLE_CTA) && groups > 0 && rows >= min_rows * groups;
 }
 
+// 4-bit weights: a pair CTA dequantises half the B rows of a single-CTA tile
+// per unit of tensor work, which pays once the groups fill 256-row tiles.
+constexpr long long kPairMinRowsQ4 = 512;
+
 msi_status routed_ffn(msi_plan* p, FwdCtx& f, int ng, int grid1, int grid2, long long rows) {
   const bool bf16 = p->d.wdtype == MSI_W_BF16;
-  const bool pair_up = bf16 && pair_tiles(f, rows, ng);
-  const bool pair_down = bf16 && pair_tiles(f, rows, ng, kPairMinRowsDown);
+  const bool pair_up = bf16 ? pair_tiles(f, rows, ng) : pair_tiles(f, rows, ng, kPairMinRowsQ4);
+  const bool pair_down = pair_tiles(f, rows, ng, bf16 ? kPairMinRowsDown : kPairMinRowsQ4);
   const auto& d = p->d;
   const Group* groups = at<Group>(f.ws, f.L.groups);
   const int* total = at<int>(f.ws, f.L.total);
@@ -840,8 +844,16 @@ msi_status routed_ffn(msi_plan* p, FwdCtx& f, int ng, int grid1, int grid2, long
     g2.q4_row_off = (int)(HI / (d.inter / 2));
     g2.q4_scale_off = 3 * HI / 2 + HI / 8;
     g2.q4_scale_ld = d.inter / 16;
-    LAUNCH(p, MSI_K_GATEUP, f.cs, launch_gemm(kGateUpGatherQ4, f.tm_h, p->tm_q13, g1, grid1, f.cs));
-    LAUNCH(p, MSI_K_DOWN, f.cs, launch_gemm(kDownQ4, f.tm_h, p->tm_q2, g2, grid2, f.cs));
+    if (pair_up)
+      LAUNCH(p, MSI_K_GATEUP, f.cs,
+             launch_gemm_pair(kGateUpGatherQ4, f.tm_h, p->tm_q13, g1, std::max(1, grid1 / 2), f.cs));
+    else
+      LAUNCH(p, MSI_K_GATEUP, f.cs, launch_gemm(kGateUpGatherQ4, f.tm_h, p->tm_q13, g1, grid1, f.cs));
+    if (pair_down)
+      LAUNCH(p, MSI_K_DOWN, f.cs,
+             launch_gemm_pair(kDownQ4, f.tm_h, p->tm_q2, g2, std::max(1, grid2 / 2), f.cs));
+    else
+      LAUNCH(p, MSI_K_DOWN, f.cs, launch_gemm(kDownQ4, f.tm_h, p->tm_q2, g2, grid2, f.cs));
     return MSI_OK;
   }
   if (pair_up)

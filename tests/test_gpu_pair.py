@@ -2,7 +2,9 @@
 pick them when a launch's groups average at least 1,024 rows.  Each case runs
 the same inputs through the pair kernels (default) and through the single-CTA
 kernels (MSI_FWD_SINGLE_CTA); both must match the fp64 oracle within the
-output tolerance, with route events exact, and agree with each other."""
+output tolerance, with route events exact, and agree with each other.  With
+4-bit experts the pair kernels take over from 512 rows per group, and each
+CTA dequantises only its own half of the B tile."""
 import numpy as np
 import pytest
 import torch
@@ -90,4 +92,43 @@ def test_pair_streamed_waves_full_oracle(tokens, top_k):
     torch.cuda.synchronize()
     assert case.plan.status() == N.MSI_OK
     compare_out(bf16_bits(out1), ref["out"])
+    case.close()
+
+
+@pytest.mark.parametrize("tokens", [4100, 2100])
+def test_pair_q4_resident_full_oracle(tokens):
+    """4-bit experts (group 32, fp16 scales): H 512, I 256, 16 experts, top-4,
+    shared expert; ~1,025 and ~525 rows per expert (pair tiles for both
+    projections, ragged last tiles)."""
+    cfg = synth.config("tiny", hidden=512, inter=256, n_experts=16, top_k=4, tokens=tokens,
+                       n_slots=16, has_shared=True, lru=False, wdtype=synth.W_Q4G32)
+    case = Case(cfg)
+    table, gens = case.stage_all()
+    x_bits = synth.hidden(cfg, 0, 14)
+    (op, ip, wp), (os_, is_, ws_) = _both(case, x_bits, table, gens)
+    ref = case.oracle_layer(x_bits)
+    compare_routes(ip, wp, oracle.router(x_bits, case.router_np[0], cfg.top_k))
+    assert np.array_equal(ip, is_)
+    ok = ~oracle.near_tie_tokens(ref["gap_k"])
+    compare_out(op, ref["out"], ok)
+    compare_out(os_, ref["out"], ok)
+    _agree(op, os_)
+    case.close()
+
+
+def test_pair_q4_qwen_shape_sampled_tokens():
+    """Qwen3-Next layer shape (H 2048, I 512, top-10) with 4-bit experts, 64
+    experts resident, 8,192 tokens: ~1,280 rows per expert."""
+    cfg = synth.config("prefill32k_q4_lru64", n_experts=64, tokens=8192, n_slots=64, lru=False)
+    case = Case(cfg)
+    table, gens = case.stage_all()
+    x_bits = synth.hidden(cfg, 0, 15)
+    (op, ip, wp), (os_, is_, ws_) = _both(case, x_bits, table, gens)
+    rng = np.random.default_rng(6)
+    toks = np.sort(rng.choice(cfg.tokens, 40, replace=False))
+    ref = case.oracle_layer(x_bits, tokens=toks)
+    compare_out(op[toks], ref["out"], ~oracle.near_tie_tokens(ref["gap_k"]))
+    compare_out(os_[toks], ref["out"], ~oracle.near_tie_tokens(ref["gap_k"]))
+    assert np.array_equal(ip, is_)
+    _agree(op, os_)
     case.close()
