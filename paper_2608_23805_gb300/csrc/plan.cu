@@ -876,7 +876,8 @@ msi_status shared_ffn(msi_plan* p, FwdCtx& f, cudaStream_t stream) {
   const int mt = (f.T + kBM - 1) / kBM;
   GemmArgs s1 = gateup_args(p, f, g, 1, total, at<__nv_bfloat16>(f.ws, f.L.hs));
   GemmArgs s2 = down_args(p, f, g, 1, total, at<__nv_bfloat16>(f.ws, f.L.ys));
-  if (p->d.wdtype == MSI_W_BF16 && pair_tiles(f, f.T, 1)) {
+  // the shared expert's weights are bf16 whatever the routed experts' format
+  if (pair_tiles(f, f.T, 1)) {
     const int pt = (f.T + 2 * kBM - 1) / (2 * kBM);
     LAUNCH(p, MSI_K_SHARED_GATEUP, stream,
            launch_gemm_pair(kGateUpTma, f.tm_x, p->tm_sh13, s1, pt * s1.nt, stream));
