@@ -445,22 +445,29 @@ __device__ __forceinline__ void epilogue_tile(uint32_t tb, __nv_bfloat16* dst, b
 // XOR-swizzled by row): read back eight lanes per 128 bytes of a row, so each
 // global store instruction covers whole rows (RB = 128: four rows of 128 B;
 // RB = 64: eight rows of 64 B) instead of one 16-32 B piece of 32 rows.
+// The swizzle key of row r is (r >> log2(8 / Q)) mod Q (Q chunks a row): the
+// eight lanes that share one 16-byte store wavefront then reach eight
+// different 16-byte bank groups, in the row-per-lane writes as in the
+// row-major reads.
 // Rows >= nvalid (past the expert's segment) are not stored.
 template <int RB>
 __device__ __forceinline__ void store_rows_staged(const uint32_t* p, uint8_t* stg,
                                                   __nv_bfloat16* row0, size_t ld, int nvalid,
                                                   int lane) {
   constexpr int Q = RB / 16;  // 16-byte chunks per row
+  static_assert(Q == 2 || Q == 4 || Q == 8, "staged rows of 32, 64 or 128 bytes");
+  constexpr int kShift = Q == 2 ? 2 : (Q == 4 ? 1 : 0);
+  const int key = (lane >> kShift) & (Q - 1);
 #pragma unroll
   for (int q = 0; q < Q; ++q)
-    *reinterpret_cast<uint4*>(stg + lane * RB + ((q ^ (lane & (Q - 1))) << 4)) =
+    *reinterpret_cast<uint4*>(stg + lane * RB + ((q ^ key) << 4)) =
         make_uint4(p[4 * q], p[4 * q + 1], p[4 * q + 2], p[4 * q + 3]);
   __syncwarp();
 #pragma unroll
   for (int it = 0; it < Q; ++it) {
     const int idx = it * 32 + lane;
     const int row = idx / Q, q = idx % Q;
-    const uint4 v = *reinterpret_cast<const uint4*>(stg + row * RB + ((q ^ (row & (Q - 1))) << 4));
+    const uint4 v = *reinterpret_cast<const uint4*>(stg + row * RB + ((q ^ ((row >> kShift) & (Q - 1))) << 4));
     if (row < nvalid)
       *reinterpret_cast<uint4*>(reinterpret_cast<uint8_t*>(row0 + (size_t)row * ld) + q * 16) = v;
   }
