@@ -20,7 +20,7 @@
 //     of all three planes, by TMA, feeding 12 MMAs), then each token's
 //     top-(k+1) candidates within the chunk by warp-shuffle argmax (logit
 //     desc, id asc) from shared memory, four rows at a time per warp.
-//  2. router_merge_kernel, one CTA per 32 tokens (eight warps, four tokens
+//  2. router_merge_kernel, one CTA per 32 tokens (sixteen warps, two tokens
 //     each): the top-(k+1) of the union of the chunks' candidates (it contains
 //     the global top-(k+1)), weights, gap, the block's expert histogram for
 //     the permutation and the shared-expert gate sigmoid(x . w_sg).
@@ -235,16 +235,17 @@ __global__ void __launch_bounds__(NTH, 1)
     // every warp: its 16 tokens' top k+1 in the chunk, four tokens at a time
     const float* L = reinterpret_cast<const float*>(smem);
     const int kp = a.kp;  // candidates per chunk: min(k + 1, chunk)
+    constexpr int NL = kRouterChunk / 32;  // logits per lane and token
     for (int q0 = warp * 16; q0 < warp * 16 + 16; q0 += 4) {
-      uint32_t kk[4][4];
-      int id[4][4];
+      uint32_t kk[4][NL];
+      int id[4][NL];
       float my_v[4];
       int my_i[4];
 #pragma unroll
       for (int u = 0; u < 4; ++u) {
         const float* row = L + (size_t)(q0 + u) * RT_LLD;
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
+        for (int i = 0; i < NL; ++i) {
           const int e = lane + 32 * i;
           kk[u][i] = e < ch ? logit_key(row[e]) : 0u;
           id[u][i] = e < ch ? e : 0x7fffffff;
@@ -287,24 +288,28 @@ __global__ void __launch_bounds__(NTH, 1)
   if (threadIdx.x == 0 && *abort_flag) atomicCAS(a.status, 0, (int)MSI_ERR_TIMEOUT);
 }
 
-// One CTA per 32-token block (eight warps, four tokens each, selected
+// One CTA per 32-token block (sixteen warps, two tokens each, selected
 // together): top-(k+1) of the union of the chunks' candidates, the route
 // event (ids, weights, gap), the block's expert histogram (one row of bcount
 // for the permutation) and, when the layer has a shared expert, its gate
 // sigmoid(x . w_sg).
-__global__ void __launch_bounds__(256) router_merge_kernel(const RouterTcArgs a) {
+constexpr int kMergeTPW = 2;                     // tokens per warp
+constexpr int kMergeThreads = 32 / kMergeTPW * 32;  // one CTA per 32-token block
+
+__global__ void __launch_bounds__(kMergeThreads) router_merge_kernel(const RouterTcArgs a) {
+  constexpr int U = kMergeTPW;
   __shared__ int hist[kMaxExperts];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int E = a.E, k = a.k;
   const int ncand = a.nchunk * a.kp;  // <= 160
   for (int e = threadIdx.x; e < E; e += blockDim.x) hist[e] = 0;
   __syncthreads();
-  const int tw = blockIdx.x * 32 + warp * 4;  // this warp's first token
+  const int tw = blockIdx.x * 32 + warp * U;  // this warp's first token
   {
-    uint32_t kk[4][5];
-    int id[4][5];
+    uint32_t kk[U][5];
+    int id[U][5];
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
+    for (int u = 0; u < U; ++u) {
       const int t = tw + u;
 #pragma unroll
       for (int i = 0; i < 5; ++i) {
@@ -317,10 +322,10 @@ __global__ void __launch_bounds__(256) router_merge_kernel(const RouterTcArgs a)
       }
       sort_desc(kk[u], id[u]);
     }
-    float my_v[4], next_v[4];
-    int my_i[4];
+    float my_v[U], next_v[U];
+    int my_i[U];
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
+    for (int u = 0; u < U; ++u) {
       my_v[u] = -INFINITY;
       next_v[u] = -INFINITY;
       my_i[u] = 0;
@@ -328,7 +333,7 @@ __global__ void __launch_bounds__(256) router_merge_kernel(const RouterTcArgs a)
     const int rounds = min(k + 1, E);
     for (int rr = 0; rr < rounds; ++rr) {
 #pragma unroll
-      for (int u = 0; u < 4; ++u) {
+      for (int u = 0; u < U; ++u) {
         uint32_t bk;
         int bi;
         take_best(kk[u], id[u], bk, bi);
@@ -341,7 +346,7 @@ __global__ void __launch_bounds__(256) router_merge_kernel(const RouterTcArgs a)
       }
     }
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
+    for (int u = 0; u < U; ++u) {
       const int t = tw + u;
       const float l0 = __shfl_sync(0xffffffffu, my_v[u], 0);
       const float ex = (lane < k) ? expf(my_v[u] - l0) : 0.f;
@@ -361,13 +366,16 @@ __global__ void __launch_bounds__(256) router_merge_kernel(const RouterTcArgs a)
     }
   }
   if (a.wsg != nullptr) {
-    // shared-expert gate of the warp's four tokens, dot products interleaved
-    float sum[4] = {0.f, 0.f, 0.f, 0.f};
+    // shared-expert gate of the warp's tokens, dot products interleaved
+    float sum[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) sum[u] = 0.f;
+#pragma unroll 4
     for (int h = lane * 8; h < a.H; h += 256) {
       const float4 w0 = __ldg(reinterpret_cast<const float4*>(a.wsg + h));
       const float4 w1 = __ldg(reinterpret_cast<const float4*>(a.wsg + h + 4));
 #pragma unroll
-      for (int u = 0; u < 4; ++u) {
+      for (int u = 0; u < U; ++u) {
         if (tw + u >= a.T) continue;
         const uint4 xv = __ldg(reinterpret_cast<const uint4*>(a.x + (size_t)(tw + u) * a.H + h));
         float s = sum[u];
@@ -383,7 +391,7 @@ __global__ void __launch_bounds__(256) router_merge_kernel(const RouterTcArgs a)
       }
     }
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
+    for (int u = 0; u < U; ++u) {
       float s = sum[u];
 #pragma unroll
       for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
@@ -416,7 +424,7 @@ cudaError_t launch_router_tc(const CUtensorMap& tmX, const CUtensorMap& tmW, con
   router_tc_kernel<<<dim3(nb, a.nchunk), NTH, RT_SMEM, s>>>(tmX, tmW, a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  router_merge_kernel<<<(a.T + 31) / 32, 256, 0, s>>>(a);
+  router_merge_kernel<<<(a.T + 31) / 32, kMergeThreads, 0, s>>>(a);
   return cudaGetLastError();
 }
 
