@@ -132,3 +132,56 @@ def test_pair_q4_qwen_shape_sampled_tokens():
     assert np.array_equal(ip, is_)
     _agree(op, os_)
     case.close()
+
+
+def test_pair_q4_streamed_waves_trace_and_oracle():
+    """4-bit experts in streamed LRU waves (32 experts, 16 slots, waves of 8),
+    8,192 tokens, top-4, shared expert: ~1,024 rows per expert, so both
+    projections run on pair tiles while slots are re-staged between waves.
+    Two calls: outputs match the oracle, the slot trace the oracle's simulator."""
+    cfg = synth.config("tiny", hidden=512, inter=256, n_experts=32, top_k=4, tokens=8192,
+                       n_slots=16, has_shared=True, wdtype=synth.W_Q4G32)
+    case = Case(cfg)
+    sim = oracle.LRUWaveSim(cfg.n_slots)
+    for call in range(2):
+        x_bits = synth.hidden(cfg, 0, 16 + call)
+        out, ev = case.plan.forward_streamed(0, bf16_tensor(x_bits), case.router[0])
+        torch.cuda.synchronize()
+        assert case.plan.status() == N.MSI_OK
+        ids = ev.ids.cpu().numpy()
+        ref = case.oracle_layer(x_bits)
+        compare_routes(ids, ev.weights.cpu().numpy(), ref)
+        sim.call(0, sorted(set(ids.reshape(-1).tolist())))
+        compare_out(bf16_bits(out), ref["out"], ~oracle.near_tie_tokens(ref["gap_k"]))
+    assert case.plan.trace() == sim.trace
+    case.close()
+
+
+@pytest.mark.parametrize("wdtype", [synth.W_BF16, synth.W_Q4G32])
+def test_pair_skewed_routing(wdtype):
+    """A heavily skewed routing in one launch: every hidden row carries the
+    constant 4.0 in feature 0 and the router's column 0 turns it into a
+    per-expert bias 4 * (0.25 - 0.04 e).  The first experts then take most
+    tokens (thousands of rows, many pair tiles), the last ones a row or two or
+    none.  Pair and single-CTA tiles both match the oracle."""
+    cfg = synth.config("tiny", hidden=512, inter=256, n_experts=16, top_k=4, tokens=6000,
+                       n_slots=16, has_shared=True, lru=False, wdtype=wdtype)
+    case = Case(cfg)
+    w = case.router_np[0].copy()
+    w[:, 0] = (0.25 - 0.04 * np.arange(cfg.n_experts)).astype(np.float32)
+    case.router_np[0] = w
+    case.router[0] = torch.from_numpy(w).cuda()
+    x_bits = synth.hidden(cfg, 0, 17).copy()
+    x_bits[:, 0] = 0x4080  # bf16 4.0
+    table, gens = case.stage_all()
+    (op, ip, wp), (os_, is_, ws_) = _both(case, x_bits, table, gens)
+    counts = np.bincount(ip.reshape(-1), minlength=cfg.n_experts)
+    assert counts.max() >= 3 * counts.mean() and (counts <= 2).any()
+    ref = case.oracle_layer(x_bits)
+    compare_routes(ip, wp, ref)
+    assert np.array_equal(ip, is_)
+    ok = ~oracle.near_tie_tokens(ref["gap_k"])
+    compare_out(op, ref["out"], ok)
+    compare_out(os_, ref["out"], ok)
+    _agree(op, os_)
+    case.close()
