@@ -71,13 +71,17 @@ struct ScatterArgs {
   int* perm;          // [T*k]
   int* inv;           // [T*k]
   int* offsets;       // [E+1]
-  // an extra last block writes the offsets and, for a resident call (table
-  // entries in the kernel's TableParams), re-checks the named slots'
-  // generations and builds the GEMM groups
+  // an extra last block writes the offsets and, for a resident call, re-checks
+  // the named slots' generations and builds the GEMM groups
   const GenWord* genwords;
   Group* groups;
   int* total_mtiles;   // [0]: 128-row tiles, [1]: 256-row pair tiles
   int* status;
+  // resident call: the call's table, copied to global memory by an earlier
+  // kernel of the forward (weight split or upload); null for a streamed call
+  const int* tab_slot;                    // [E]
+  const unsigned long long* tab_expected;  // [E]
+  int layer;
 };
 
 // Per-call tables uploaded by value (kernel parameters, < 32 KB).
@@ -133,13 +137,19 @@ struct CombineArgs {
 cudaError_t launch_router(const RouterArgs& a, cudaStream_t s);
 // Also begins the forward (its first kernel): clears the status word and,
 // when sh is not null, writes the shared-expert group of T rows in block
-// `shared_slot` and its tile counts.
+// `shared_slot` and its tile counts.  With tp not null it also copies the
+// call's slot table and expected generations to tab_slot / tab_expected
+// (the entries are read from the kernel argument by many blocks at once;
+// one block reading all of them serialises on its constant cache).
 cudaError_t launch_split3(const float* w, long long n, __nv_bfloat16* out, int* status, Group* sh,
-                          int* sh_total, int T, int shared_slot, cudaStream_t s);
+                          int* sh_total, int T, int shared_slot, const TableParams* tp,
+                          int* tab_slot, unsigned long long* tab_expected, cudaStream_t s);
 cudaError_t launch_router_tc(const CUtensorMap& tmX, const CUtensorMap& tmW, const RouterTcArgs& a,
                              cudaStream_t s);
 cudaError_t launch_colscan(const ScanArgs& a, cudaStream_t s);
-cudaError_t launch_scatter(const ScatterArgs& a, const TableParams& tp, cudaStream_t s);
+cudaError_t launch_scatter(const ScatterArgs& a, cudaStream_t s);
+// Copies the call's table to global memory and, when status is not null,
+// begins the forward (as the first kernel of a call without rows).
 cudaError_t launch_upload(const TableParams& p, int* table, unsigned long long* expected,
                           int* status, Group* shared_group, int* shared_total, cudaStream_t s);
 cudaError_t launch_setup_wave(const SetupArgs& a, const WaveParams& w, cudaStream_t s);

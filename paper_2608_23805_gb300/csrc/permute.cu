@@ -26,12 +26,14 @@ __global__ void __launch_bounds__(1024) colscan_kernel(const ScanArgs a) {
   const int b0 = min(a.nb, ty * sz), b1 = min(a.nb, b0 + sz);
   int sum = 0;
   if (e < a.E)
+#pragma unroll 8
     for (int b = b0; b < b1; ++b) sum += a.bcount[(size_t)b * a.E + e];
   part[ty][tx] = sum;
   __syncthreads();
   int run = 0;
   for (int y = 0; y < ty; ++y) run += part[y][tx];
   if (e < a.E) {
+#pragma unroll 8
     for (int b = b0; b < b1; ++b) {
       const int v = a.bcount[(size_t)b * a.E + e];
       a.bbase[(size_t)b * a.E + e] = run;
@@ -79,21 +81,24 @@ __device__ __forceinline__ int scan4(const int (&v)[4], int* wsum, int* total) {
 // Setup block of the scatter, resident call: the generation re-check of every
 // routed expert's slot (fail closed) and the GEMM groups with their 128- and
 // 256-row tile prefixes.
-__device__ void scatter_setup(const ScatterArgs& a, const TableParams& tp, const int* offs,
+__device__ void scatter_setup(const ScatterArgs& a, const int* offs,
                               const int* s_cnt) {
   __shared__ int wsum[kScatterWarps];
   __shared__ int kmin[kScatterWarps];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  if (tp.E == 0) return;  // streamed call: the groups are built per wave
+  if (a.tab_slot == nullptr) return;  // streamed call: the groups are built per wave
   int cnt[4], code[4], mt[4], pt[4];
   int key = 0x7fffffff;
+  int slot[4];
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
     const int e = tid * 4 + i;
     cnt[i] = code[i] = mt[i] = pt[i] = 0;
+    slot[i] = -1;
     if (e < a.E) {
       cnt[i] = s_cnt[e];
-      if (cnt[i] > 0) code[i] = check_code(a.genwords, tp.slot[e], tp.layer, e, tp.expected[e]);
+      slot[i] = a.tab_slot[e];
+      if (cnt[i] > 0) code[i] = check_code(a.genwords, slot[i], a.layer, e, a.tab_expected[e]);
       if (code[i] == 0) {
         mt[i] = (cnt[i] + kBM - 1) / kBM;
         pt[i] = (cnt[i] + 2 * kBM - 1) / (2 * kBM);
@@ -112,7 +117,7 @@ __device__ void scatter_setup(const ScatterArgs& a, const TableParams& tp, const
       Group g;
       g.row_begin = offs[e];
       g.row_count = cnt[i];
-      g.slot = tp.slot[e] < 0 ? 0 : tp.slot[e];
+      g.slot = slot[i] < 0 ? 0 : slot[i];
       g.mt_begin = mb;
       g.ok = code[i] == 0;
       g.expert = e;
@@ -136,8 +141,7 @@ __device__ void scatter_setup(const ScatterArgs& a, const TableParams& tp, const
   }
 }
 
-__global__ void __launch_bounds__(kScatterWarps * 32) scatter_kernel(const ScatterArgs a,
-                                                                     const TableParams tp) {
+__global__ void __launch_bounds__(kScatterWarps * 32) scatter_kernel(const ScatterArgs a) {
   __shared__ int offs[kMaxExperts + 1];
   __shared__ int s_cnt[kMaxExperts];
   __shared__ int run[kScatterWarps][kMaxExperts];
@@ -186,7 +190,7 @@ __global__ void __launch_bounds__(kScatterWarps * 32) scatter_kernel(const Scatt
     for (int e = tid; e <= a.E; e += blockDim.x) a.offsets[e] = offs[e];
     if (a.fuse_scan)
       for (int e = tid; e < a.E; e += blockDim.x) a.counts_out[e] = s_cnt[e];
-    scatter_setup(a, tp, offs, s_cnt);
+    scatter_setup(a, offs, s_cnt);
     return;
   }
 
@@ -197,26 +201,45 @@ __global__ void __launch_bounds__(kScatterWarps * 32) scatter_kernel(const Scatt
   const int f0 = b * a.tm * a.k;
   const int f1 = min(a.T, (b + 1) * a.tm) * a.k;
   const unsigned lt = (1u << lane) - 1u;
-  for (int f = f0 + lane; f - lane < f1; f += 32) {
-    const bool valid = f < f1;
-    const int e = valid ? a.ids[f] : -1;
-    const unsigned mask = __match_any_sync(0xffffffffu, e);
-    int before = 0;
-    if (valid) {
-      before = run[warp][e];
-      int pre = 0;  // this expert's ids in the router blocks before b
-      if (a.fuse_scan) {
-        for (int bb = 0; bb < b; ++bb) pre += a.bcount[(size_t)bb * a.E + e];
-      } else {
-        pre = a.bbase[(size_t)b * a.E + e];
-      }
-      const int pos = offs[e] + pre + before + __popc(mask & lt);
-      a.perm[pos] = f;
-      a.inv[f] = pos;
+  // eight steps of 32 ids at a time: their ids and block bases are loaded
+  // together (independent loads), then ranked in order
+  constexpr int kAhead = 8;
+  for (int fc = f0; fc < f1; fc += 32 * kAhead) {
+    int ev[kAhead], pre[kAhead];
+#pragma unroll
+    for (int j = 0; j < kAhead; ++j) {
+      const int f = fc + 32 * j + lane;
+      ev[j] = f < f1 ? a.ids[f] : -1;
     }
-    __syncwarp();
-    if (valid && lane == 31 - __clz(mask)) run[warp][e] = before + __popc(mask);
-    __syncwarp();
+#pragma unroll
+    for (int j = 0; j < kAhead; ++j) {
+      pre[j] = 0;  // this expert's ids in the router blocks before b
+      if (ev[j] >= 0) {
+        if (a.fuse_scan) {
+          for (int bb = 0; bb < b; ++bb) pre[j] += a.bcount[(size_t)bb * a.E + ev[j]];
+        } else {
+          pre[j] = a.bbase[(size_t)b * a.E + ev[j]];
+        }
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < kAhead; ++j) {
+      if (fc + 32 * j >= f1) break;  // uniform across the warp
+      const int f = fc + 32 * j + lane;
+      const int e = ev[j];
+      const bool valid = e >= 0;
+      const unsigned mask = __match_any_sync(0xffffffffu, e);
+      int before = 0;
+      if (valid) {
+        before = run[warp][e];
+        const int pos = offs[e] + pre[j] + before + __popc(mask & lt);
+        a.perm[pos] = f;
+        a.inv[f] = pos;
+      }
+      __syncwarp();
+      if (valid && lane == 31 - __clz(mask)) run[warp][e] = before + __popc(mask);
+      __syncwarp();
+    }
   }
 }
 
@@ -227,7 +250,7 @@ __global__ void upload_kernel(const TableParams p, int* table, unsigned long lon
     table[e] = p.slot[e];
     expected[e] = p.expected[e];
   }
-  if (threadIdx.x == 0) forward_begin(status, sh, sh_total, p.T, p.shared_slot);
+  if (threadIdx.x == 0 && status != nullptr) forward_begin(status, sh, sh_total, p.T, p.shared_slot);
 }
 
 // ---- generation re-check + GEMM groups (one block) ----
@@ -388,9 +411,9 @@ cudaError_t launch_colscan(const ScanArgs& a, cudaStream_t s) {
   return cudaGetLastError();
 }
 
-cudaError_t launch_scatter(const ScatterArgs& a, const TableParams& tp, cudaStream_t s) {
+cudaError_t launch_scatter(const ScatterArgs& a, cudaStream_t s) {
   const int grid = (a.nb + kScatterWarps - 1) / kScatterWarps + 1;  // + the setup block
-  scatter_kernel<<<grid, kScatterWarps * 32, 0, s>>>(a, tp);
+  scatter_kernel<<<grid, kScatterWarps * 32, 0, s>>>(a);
   return cudaGetLastError();
 }
 

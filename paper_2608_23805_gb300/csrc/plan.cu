@@ -640,10 +640,14 @@ msi_status route_rows(msi_plan* p, FwdCtx& f, const float* rw, const msi_route_e
                          : nullptr;
   if (tensor_router(d)) {
     __nv_bfloat16* w3 = at<__nv_bfloat16>(ws, L.w3);
+    // a resident call's table goes to the workspace here, for the scatter's
+    // generation re-check
+    const bool tab = first && tp.E > 0;
     LAUNCH(p, MSI_K_ROUTER, s,
            launch_split3(rw, (long long)E * H, w3, first ? at<int>(ws, L.status) : nullptr,
                          first && d.has_shared ? at<Group>(ws, L.sh_group) : nullptr,
-                         at<int>(ws, L.sh_total), f.T, tp.shared_slot, s));
+                         at<int>(ws, L.sh_total), f.T, tp.shared_slot, tab ? &tp : nullptr,
+                         at<int>(ws, L.table), at<unsigned long long>(ws, L.expected), s));
   }
   // host-buffer calls: every reader of the rows (router, shared expert) comes
   // after they have landed
@@ -754,7 +758,17 @@ msi_status front(msi_plan* p, FwdCtx& f, const TableParams& tp) {
   xa.groups = at<Group>(ws, L.groups);
   xa.total_mtiles = at<int>(ws, L.total);
   xa.status = at<int>(ws, L.status);
-  LAUNCH(p, MSI_K_SCATTER, f.cs, launch_scatter(xa, tp, f.cs));
+  if (tp.E > 0) {
+    // resident call: the scatter re-checks the table's slots from global
+    // memory (the weight split copied it; the FFMA router path copies it here)
+    if (!tensor_router(d))
+      LAUNCH(p, MSI_K_UPLOAD, f.cs, launch_upload(tp, at<int>(ws, L.table), at<unsigned long long>(ws, L.expected),
+                              nullptr, nullptr, nullptr, f.cs));
+    xa.tab_slot = at<int>(ws, L.table);
+    xa.tab_expected = at<unsigned long long>(ws, L.expected);
+    xa.layer = tp.layer;
+  }
+  LAUNCH(p, MSI_K_SCATTER, f.cs, launch_scatter(xa, f.cs));
   const size_t Tk = (size_t)f.T * k;
   if (f.ids_host != nullptr) {
     // the route ids go back beside the expert GEMMs

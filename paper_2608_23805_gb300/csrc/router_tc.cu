@@ -42,8 +42,9 @@ constexpr int RT_LLD = kRouterChunk + 1;             // padded logits row (float
 constexpr int RT_SMEM = 1024 + RT_STAGES * RT_STAGE + 256;
 static_assert(128 * RT_LLD * 4 <= RT_STAGES * RT_STAGE, "logits tile does not fit");
 
-__global__ void split3_kernel(const float* __restrict__ w, long long n, __nv_bfloat16* __restrict__ out,
-                              int* status, Group* sh, int* sh_total, int T, int shared_slot) {
+__device__ __forceinline__ void split3_body(const float* __restrict__ w, long long n,
+                                            __nv_bfloat16* __restrict__ out, int* status, Group* sh,
+                                            int* sh_total, int T, int shared_slot) {
   // the forward's first kernel (status null: a prediction pass)
   if (blockIdx.x == 0 && threadIdx.x == 0 && status != nullptr)
     forward_begin(status, sh, sh_total, T, shared_slot);
@@ -58,6 +59,28 @@ __global__ void split3_kernel(const float* __restrict__ w, long long n, __nv_bfl
     out[n + i] = mid;
     out[2 * n + i] = __float2bfloat16_rn(r2);
   }
+}
+
+__global__ void split3_kernel(const float* __restrict__ w, long long n, __nv_bfloat16* __restrict__ out,
+                              int* status, Group* sh, int* sh_total, int T, int shared_slot) {
+  split3_body(w, n, out, status, sh, sh_total, T, shared_slot);
+}
+
+// The same, plus the resident call's table copied to global memory: the
+// first warp of each block takes 32 entries, so the argument's entries are
+// read through many SMs' constant caches at once.
+__global__ void split3_table_kernel(const float* __restrict__ w, long long n,
+                                    __nv_bfloat16* __restrict__ out, int* status, Group* sh,
+                                    int* sh_total, int T, int shared_slot, const TableParams tp,
+                                    int* __restrict__ tab_slot,
+                                    unsigned long long* __restrict__ tab_expected) {
+  if (threadIdx.x < 32) {
+    for (int g = blockIdx.x * 32 + threadIdx.x; g < tp.E; g += gridDim.x * 32) {
+      tab_slot[g] = tp.slot[g];
+      tab_expected[g] = tp.expected[g];
+    }
+  }
+  split3_body(w, n, out, status, sh, sh_total, T, shared_slot);
 }
 
 // Selection order of the route event: logit descending, then expert id
@@ -405,10 +428,15 @@ __global__ void __launch_bounds__(kMergeThreads) router_merge_kernel(const Route
 }  // namespace
 
 cudaError_t launch_split3(const float* w, long long n, __nv_bfloat16* out, int* status, Group* sh,
-                          int* sh_total, int T, int shared_slot, cudaStream_t s) {
+                          int* sh_total, int T, int shared_slot, const TableParams* tp,
+                          int* tab_slot, unsigned long long* tab_expected, cudaStream_t s) {
   const long long want = (n + 255) / 256;
   const int grid = (int)(want < 152 * 8 ? want : 152 * 8);
-  split3_kernel<<<grid, 256, 0, s>>>(w, n, out, status, sh, sh_total, T, shared_slot);
+  if (tp != nullptr)
+    split3_table_kernel<<<grid, 256, 0, s>>>(w, n, out, status, sh, sh_total, T, shared_slot, *tp,
+                                             tab_slot, tab_expected);
+  else
+    split3_kernel<<<grid, 256, 0, s>>>(w, n, out, status, sh, sh_total, T, shared_slot);
   return cudaGetLastError();
 }
 
