@@ -148,10 +148,12 @@ __global__ void __launch_bounds__(NTH, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int E = a.E;
   const int ch = a.chunk;                 // experts per chunk
-  const int c = blockIdx.y;               // chunk index
+  // the chunks of one token tile are neighbours in launch order, so the x
+  // tile is read from HBM once and from L2 by the other chunks
+  const int c = blockIdx.x;               // chunk index
   const int kblocks = a.H / 64;
   const int nstage = kblocks;
-  const int m0 = blockIdx.x * 128;
+  const int m0 = blockIdx.y * 128;
   const long long lim = a.wait_limit;
 
   if (threadIdx.x == 0) {
@@ -449,7 +451,8 @@ cudaError_t launch_router_tc(const CUtensorMap& tmX, const CUtensorMap& tmW, con
   }
   const int nb = (a.T + 127) / 128;
   if (nb == 0) return cudaSuccess;
-  router_tc_kernel<<<dim3(nb, a.nchunk), NTH, RT_SMEM, s>>>(tmX, tmW, a);
+  if (nb > 65535) return cudaErrorInvalidConfiguration;  // token tiles index the grid's y
+  router_tc_kernel<<<dim3(a.nchunk, nb), NTH, RT_SMEM, s>>>(tmX, tmW, a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   router_merge_kernel<<<(a.T + 31) / 32, kMergeThreads, 0, s>>>(a);
