@@ -683,6 +683,7 @@ msi_status route_rows(msi_plan* p, FwdCtx& f, const float* rw, const msi_route_e
     ra.status = at<int>(ws, L.status);
     ra.wait_limit = kDeviceWaitCycles;
     LAUNCH(p, MSI_K_ROUTER, s, launch_router_tc(f.tm_x, tm_w3, ra, s));
+    p->launches++;  // launch_router_tc starts two kernels (logits + top-k, merge)
   } else {
     RouterArgs ra{};
     ra.x = static_cast<const __nv_bfloat16*>(f.x);
