@@ -150,10 +150,10 @@ __global__ void __launch_bounds__(NTH, 1)
   const int ch = a.chunk;                 // experts per chunk
   // the chunks of one token tile are neighbours in launch order, so the x
   // tile is read from HBM once and from L2 by the other chunks
-  const int c = blockIdx.x;               // chunk index
+  const int c = (int)(blockIdx.x % (unsigned)a.nchunk);  // chunk index
   const int kblocks = a.H / 64;
   const int nstage = kblocks;
-  const int m0 = blockIdx.y * 128;
+  const int m0 = (int)(blockIdx.x / (unsigned)a.nchunk) * 128;
   const long long lim = a.wait_limit;
 
   if (threadIdx.x == 0) {
@@ -451,8 +451,7 @@ cudaError_t launch_router_tc(const CUtensorMap& tmX, const CUtensorMap& tmW, con
   }
   const int nb = (a.T + 127) / 128;
   if (nb == 0) return cudaSuccess;
-  if (nb > 65535) return cudaErrorInvalidConfiguration;  // token tiles index the grid's y
-  router_tc_kernel<<<dim3(a.nchunk, nb), NTH, RT_SMEM, s>>>(tmX, tmW, a);
+  router_tc_kernel<<<(unsigned)nb * (unsigned)a.nchunk, NTH, RT_SMEM, s>>>(tmX, tmW, a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   router_merge_kernel<<<(a.T + 31) / 32, kMergeThreads, 0, s>>>(a);
