@@ -6,26 +6,36 @@ A step is one MoE layer forward over one batch of synthetic tokens: router
 (fp32 logits, softmax, top-k), histogram and permutation, expert staging into
 GPU slots (LRU waves, generation-fenced) where the workload streams, grouped
 SwiGLU expert FFN reading weights from slots, shared expert, combine.
-Default workload: the Qwen3-Next-shaped layer (hidden 2048, 512 experts,
-top-10, intermediate 512, shared expert) over 4,096 tokens with all 512
-experts resident in slots.  --workload prefill32k_lru64 runs the same layer
-at 32,768 tokens with a 64-slot pool: 448 of the 512 experts are staged from
-pinned host windows per call in LRU waves.  --workload decode48 runs one
+Default workload (prefill32k_lru64): the Qwen3-Next-shaped layer (hidden
+2048, 512 experts, top-10, intermediate 512, shared expert) over a
+32,768-token prefill with a 64-slot pool: 448 of the 512 experts are staged
+from pinned host windows per call in LRU waves of 32.  The same line carries
+a resident pass (`resident_32k`): the same 32,768 tokens with all 512 experts
+resident in a 512-slot pool, so the routed GEMMs' tensor fraction is also
+measured without waves.  --workload qwen3next_4k runs 4,096 tokens with all
+512 experts resident; qwen3next_32k the resident 32K step alone;
+prefill32k_q4_lru64 the staged 32K step with 4-bit experts.
+--workload decode48 runs one
 decode step through a stack of 48 layers of the tiny shape (hidden 256, 16
 experts, top-2, intermediate 128) over --batch rows, one 64-slot LRU pool
 shared by the 768 objects; --predict adds next-layer prediction with the
 two-bank prefetch (each call routes its rows through the next layer's router
 and stages the predicted objects after its last wave).
 
-Prints one JSON line (rank 0).  `value` is whole-job tokens/s over the timed
-steps (device time, CUDA events on the compute stream around each step, no
-per-kernel events inside it); a second timed pass of the same steps with an
+Prints one JSON line (rank 0).  `value` is whole-job tokens/s at the median
+timed step (device time, CUDA events on the compute stream around each step,
+no per-kernel events inside it; the mean is beside it); a second timed pass of the same steps with an
 event pair around every kernel launch gives `kernels_ms_per_step` and the
 roofline kernel's launch duration; `e2e` repeats the
 metric with the hidden rows copied from pinned host memory and the outputs
-read back inside the timed region; `roofline` is the dominant kernel's
-algorithmic work per launch over its event-timed duration; `cpu_baseline` is
-the fp64 oracle timed on a bounded sample on this host's cores.
+read back inside the timed region; `roofline` is the routed expert GEMMs'
+(gate-up and down together, the dominant pair) algorithmic work per launch
+pair over their event-timed duration, against the burst bf16 peak when
+tensor-bound (they run at full clock inside the step) or the copy bandwidth
+when HBM-bound; `h2d_roof` sets the staged bytes of a step against the
+host-to-device copy rate measured in the same run; `cpu_baseline` is the fp64
+oracle timed on a bounded sample on this host's cores, with the BLAS threads
+it actually ran on.
 Multi-GPU (torchrun): independent replicas, one per GPU, no collective in the
 data path; the timing is the max over ranks.
 """
@@ -183,7 +193,9 @@ class ClockSampler:
 # ---------------------------------------------------------------------------
 
 class Workload:
-    def __init__(self, name: str, batch: int | None = None, predict: bool = False):
+    def __init__(self, name: str, batch: int | None = None, predict: bool = False, windows=None):
+        """windows: pinned host windows of an earlier workload with the same
+        layer shape and weights (reused, not regenerated)."""
         import torch
 
         import synth
@@ -196,10 +208,14 @@ class Workload:
         self.L = L = cfg.n_layers
         self.predict = predict and L > 1
         E, H, I, eb = cfg.n_experts, cfg.hidden, cfg.inter, cfg.extent_bytes
-        self.windows = torch.empty(L * E * eb, dtype=torch.uint8, pin_memory=True)
-        wnp = self.windows.numpy()
-        for l in range(L):
-            synth.fill_extents(cfg, l, wnp[l * E * eb:(l + 1) * E * eb])
+        if windows is not None:
+            assert windows.numel() == L * E * eb
+            self.windows = windows
+        else:
+            self.windows = torch.empty(L * E * eb, dtype=torch.uint8, pin_memory=True)
+            wnp = self.windows.numpy()
+            for l in range(L):
+                synth.fill_extents(cfg, l, wnp[l * E * eb:(l + 1) * E * eb])
         self.routers_np = [synth.router_weight(cfg, l) for l in range(L)]
         self.routers = [torch.from_numpy(w).cuda() for w in self.routers_np]
         self.router_np, self.router = self.routers_np[0], self.routers[0]
@@ -264,14 +280,17 @@ def algorithmic(cfg, kind: str, units: dict):
     """Algorithmic work per step of one kernel kind: (bound, flops, bytes).
 
     rows = T*k routed rows; per routed row the gate-up GEMM does 2*H*2I flops
-    and the down GEMM 2*I*H; weights are read once per expert per step."""
+    and the down GEMM 2*I*H; weights are read once per expert per step; the
+    gate-up reads each token's row once (its re-reads for further experts are
+    L2 hits, not algorithmic HBM traffic) and writes h; the down reads h and
+    writes the expert outputs."""
     T, H, I, E, k = cfg.tokens, cfg.hidden, cfg.inter, cfg.n_experts, cfg.top_k
     rows = T * k
     wb = 2.0 if cfg.wdtype == 0 else 0.5625      # bytes per weight (bf16, or 4-bit + fp16 scale / 32)
     eb_w13 = 2 * I * H * wb
     eb_w2 = H * I * wb
     if kind == "gateup":
-        return 2.0 * rows * H * 2 * I, E * eb_w13 + rows * H * 2 + rows * I * 2
+        return 2.0 * rows * H * 2 * I, E * eb_w13 + T * H * 2 + rows * I * 2
     if kind == "down":
         return 2.0 * rows * I * H, E * eb_w2 + rows * I * 2 + rows * H * 2
     if kind == "shared_gateup":
@@ -287,40 +306,125 @@ def algorithmic(cfg, kind: str, units: dict):
     return 0.0, 0.0
 
 
-def roofline(cfg, kt: dict, steps: int, peaks: dict, clocks: dict, workload: str):
-    """Roofline object of the dominant (largest summed time) kernel kind."""
-    kind = max(kt, key=lambda k: kt[k][0])
-    ms, launches = kt[kind]
-    flops, nbytes = algorithmic(cfg, kind, {})
+def _bound_of(flops: float, nbytes: float, peaks: dict) -> str:
+    """tensor when the work's arithmetic intensity is at or above the ridge of
+    the burst bf16 peak over the copy bandwidth, else hbm."""
+    ridge = peaks["bf16_tflops"] * 1e12 / (peaks["hbm_gbs"] * 1e9)
+    return "tensor" if flops > 0 and flops / max(nbytes, 1.0) >= ridge else "hbm"
+
+
+def _part(flops_step: float, bytes_step: float, ms: float, launches: int, steps: int, peaks: dict,
+          bound: str) -> dict:
     per_launch_s = ms / 1e3 / max(launches, 1)
-    per_launch_flops = flops * steps / max(launches, 1)
-    per_launch_bytes = nbytes * steps / max(launches, 1)
-    ridge = peaks["bf16_tflops_sustained"] * 1e12 / (peaks["hbm_gbs"] * 1e9)
-    if kind == "router":
-        mhz = clocks.get("sm_mhz") or peaks.get("sm_max_mhz", 2070.0)
-        peak = N_SMS * FP32_LANES_PER_SM * 2 * mhz * 1e6 / 1e12
-        ach = per_launch_flops / per_launch_s / 1e12
-        r = {"bound": "alu", "achieved": ach, "peak": peak, "unit": "TFLOP/s",
-             "peak_source": "152 SMs x 128 FP32 lanes x 2 flop x median SM clock %.0f MHz" % mhz}
-    elif flops > 0 and flops / max(nbytes, 1) >= ridge:
-        ach = per_launch_flops / per_launch_s / 1e12
-        peak = peaks["bf16_tflops_sustained"]
-        r = {"bound": "tensor", "achieved": ach, "peak": peak, "unit": "TFLOP/s",
-             "peak_source": "bf16_tflops_sustained of measured (kernel timed inside the step)"}
+    if bound == "tensor":
+        ach = flops_step * steps / max(launches, 1) / per_launch_s / 1e12
+        return {"achieved": ach, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
+                "frac": ach / peaks["bf16_tflops"], "ms_per_launch": ms / max(launches, 1)}
+    ach = bytes_step * steps / max(launches, 1) / per_launch_s / 1e9
+    return {"achieved": ach, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+            "frac": ach / peaks["hbm_gbs"], "ms_per_launch": ms / max(launches, 1)}
+
+
+def roofline(cfg, kt: dict, steps: int, peaks: dict, clocks: dict, workload: str):
+    """Roofline object of the routed expert GEMMs, gate-up and down together
+    (the dominant pair of every step that routes rows): their algorithmic
+    flops (or bytes) per launch pair over the pair's summed event-timed
+    duration.  Tensor-bound work is set against the burst bf16 peak: the
+    kernels run at full SM clock inside steps of milliseconds, far from the
+    seconds-long power-capped loop the sustained figure comes from.  Without
+    routed GEMM time (a step with no rows) the dominant kernel kind alone."""
+    if "gateup" in kt and "down" in kt:
+        f1, b1 = algorithmic(cfg, "gateup", {})
+        f2, b2 = algorithmic(cfg, "down", {})
+        bound = _bound_of(f1 + f2, b1 + b2, peaks)
+        ms = kt["gateup"][0] + kt["down"][0]
+        launches = kt["gateup"][1]
+        r = {"bound": bound}
+        r.update(_part(f1 + f2, b1 + b2, ms, launches, steps, peaks, bound))
+        r["kernel"] = "gateup+down"
+        r["launches_per_step"] = launches / steps
+        r["parts"] = {
+            "gateup": dict(_part(f1, b1, kt["gateup"][0], kt["gateup"][1], steps, peaks, bound),
+                           flops_per_step=f1, bytes_per_step=b1),
+            "down": dict(_part(f2, b2, kt["down"][0], kt["down"][1], steps, peaks, bound),
+                         flops_per_step=f2, bytes_per_step=b2)}
+        kind = "gateup+down"
     else:
-        ach = per_launch_bytes / per_launch_s / 1e9
-        peak = peaks["hbm_gbs"]
-        r = {"bound": "hbm", "achieved": ach, "peak": peak, "unit": "GB/s",
-             "peak_source": "hbm_gbs of measured"}
-    r["frac"] = r["achieved"] / r["peak"]
-    r["kernel"] = kind
-    r["launches_per_step"] = launches / steps
-    r["ms_per_launch"] = ms / max(launches, 1)
+        kind = max(kt, key=lambda k: kt[k][0])
+        ms, launches = kt[kind]
+        flops, nbytes = algorithmic(cfg, kind, {})
+        if kind == "router":
+            mhz = clocks.get("sm_mhz") or peaks.get("sm_max_mhz", 2070.0)
+            peak = N_SMS * FP32_LANES_PER_SM * 2 * mhz * 1e6 / 1e12
+            per_launch_s = ms / 1e3 / max(launches, 1)
+            ach = flops * steps / max(launches, 1) / per_launch_s / 1e12
+            r = {"bound": "alu", "achieved": ach, "peak": peak, "unit": "TFLOP/s",
+                 "frac": ach / peak, "ms_per_launch": ms / max(launches, 1)}
+        else:
+            bound = _bound_of(flops, nbytes, peaks)
+            r = {"bound": bound}
+            r.update(_part(flops, nbytes, ms, launches, steps, peaks, bound))
+        r["kernel"] = kind
+        r["launches_per_step"] = launches / steps
+    if r["bound"] == "tensor":
+        r["peak_source"] = "bf16_tflops (burst) of measured"
+    elif r["bound"] == "hbm":
+        r["peak_source"] = "hbm_gbs of measured"
+    else:
+        r["peak_source"] = "152 SMs x 128 FP32 lanes x 2 flop x median SM clock"
     t = TRAFFIC.get((workload, kind))
     r["traffic"] = t["bytes_per_launch"] if (t and t.get("src_hash") == kernel_source_hash()) else None
     if r["traffic"] is not None:
         r["traffic_source"] = t["profile"]
     return r
+
+
+def blas_threads():
+    """(threads, how): the BLAS threads numpy's matrix products run on (the
+    oracle's time is almost all there), read from the loaded OpenBLAS."""
+    import ctypes
+    for var in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS"):
+        if os.environ.get(var, "").isdigit():
+            return int(os.environ[var]), var
+    np.ones((64, 64)) @ np.ones((64, 64))          # BLAS loaded
+    try:
+        paths = sorted({l.split()[-1] for l in open("/proc/self/maps") if "openblas" in l.lower()
+                        and l.split()[-1].startswith("/")})
+    except OSError:
+        paths = []
+    for path in paths:
+        try:
+            lib = ctypes.CDLL(path)
+        except OSError:
+            continue
+        for sym in ("scipy_openblas_get_num_threads64_", "openblas_get_num_threads64_",
+                    "openblas_get_num_threads"):
+            fn = getattr(lib, sym, None)
+            if fn is not None:
+                fn.restype = ctypes.c_int
+                return int(fn()), "%s from %s" % (sym, os.path.basename(path))
+    return os.cpu_count() or 1, "os.cpu_count() (no OpenBLAS found to ask)"
+
+
+def h2d_probe(nbytes: int = 192 << 20, reps: int = 4):
+    """Host-to-device copy rate (GB/s) of one staging run's size (32 extents
+    of 6 MiB) from pinned memory: best of `reps` copies, CUDA events."""
+    import torch
+    src = torch.empty(nbytes, dtype=torch.uint8, pin_memory=True)
+    dst = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
+    best = None
+    s = torch.cuda.Stream()
+    for _ in range(reps + 1):
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(s)
+        with torch.cuda.stream(s):
+            dst.copy_(src, non_blocking=True)
+        b.record(s)
+        b.synchronize()
+        t = a.elapsed_time(b) / 1e3
+        best = t if best is None else min(best, t)
+    return nbytes / best / 1e9
 
 
 def cpu_baseline(w: "Workload", tokens: int):
@@ -335,9 +439,9 @@ def cpu_baseline(w: "Workload", tokens: int):
         kw = dict(shared_extent=w.shared_np, w_sg=w.gate_np)
     if w.L > 1:
         dt = oracle_stack(cfg, w.x_bits[:tokens], w.routers_np, wnp)
-        cores = int(os.environ.get("OMP_NUM_THREADS", os.environ.get("OPENBLAS_NUM_THREADS",
-                                                                     os.cpu_count() or 1)))
-        return {"value": tokens / dt, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+        cores, how = blas_threads()
+        return {"value": tokens / dt, "unit": "tokens/s", "cores": cores, "cores_source": how,
+                "host_cpus": os.cpu_count(), "kind": "oracle",
                 "sample": "fp64 oracle of one decode step of %d rows through all %d layers (router, "
                           "expert FFNs, combine with residual, LRU-wave plan of the shared pool), "
                           "%.2f s" % (tokens, w.L, dt)}
@@ -348,8 +452,9 @@ def cpu_baseline(w: "Workload", tokens: int):
         sim = oracle.LRUWaveSim(cfg.n_slots)
         sim.call(0, range(cfg.n_experts))
     dt = time.perf_counter() - t0
-    cores = int(os.environ.get("OMP_NUM_THREADS", os.environ.get("OPENBLAS_NUM_THREADS", os.cpu_count() or 1)))
-    return {"value": tokens / dt, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+    cores, how = blas_threads()
+    return {"value": tokens / dt, "unit": "tokens/s", "cores": cores, "cores_source": how,
+            "host_cpus": os.cpu_count(), "kind": "oracle",
             "sample": "fp64 oracle forward of the first %d of %d tokens (router over all %d experts, "
                       "expert FFNs, shared expert, combine, LRU-wave plan), %.1f s" %
                       (tokens, cfg.tokens, cfg.n_experts, dt)}
@@ -376,7 +481,7 @@ def oracle_stack(cfg, x_bits, routers_np, wnp) -> float:
 
 
 SAMPLE_TOKENS = {"prefill32k_lru64": 4096, "prefill32k_q4_lru64": 4096, "qwen3next_4k": 4096,
-                 "tiny": 64}
+                 "qwen3next_32k": 4096, "tiny": 64}
 
 
 # ---------------------------------------------------------------------------
@@ -412,32 +517,39 @@ def run_ours(args):
     peaks, peak_kind = load_peaks()
 
     flush = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device="cuda")
+    # the host-to-device rate of this machine, before anything is timed
+    h2d_gbs = h2d_probe() if cfg.lru else None
     sampler = ClockSampler(local)
     sampler.start()
-    def flush_l2():
+    def flush_l2(wk=None):
         # on the compute stream, so that it is ordered before the step's start
         # event and never overlaps a timed step
-        with torch.cuda.stream(w.cs):
+        with torch.cuda.stream((wk or w).cs):
             flush.zero_()
 
-    # warm-up immediately precedes the timed steps (an idle GPU drops its clocks and link state)
-    for _ in range(args.warmup):
-        flush_l2()
-        w.step()
-    torch.cuda.synchronize()
-    flush_l2()                                       # one more untimed step right before timing
-    w.step()
-    torch.cuda.synchronize()
+    def warm(wk):
+        # warm-up immediately precedes the timed steps (an idle GPU drops its
+        # clocks and link state)
+        for _ in range(args.warmup):
+            flush_l2(wk)
+            wk.step()
+        torch.cuda.synchronize()
+        flush_l2(wk)                                 # one more untimed step right before timing
+        wk.step()
+        torch.cuda.synchronize()
 
-    def timed_steps():
+    warm(w)
+
+    def timed_steps(wk=None):
+        wk = wk or w
         evs = []
         for _ in range(args.steps):
-            flush_l2()                               # L2 flushed between timed steps (untimed)
+            flush_l2(wk)                             # L2 flushed between timed steps (untimed)
             a = torch.cuda.Event(enable_timing=True)
             b = torch.cuda.Event(enable_timing=True)
-            a.record(w.cs)
-            w.step()
-            b.record(w.cs)
+            a.record(wk.cs)
+            wk.step()
+            b.record(wk.cs)
             evs.append((a, b))
         torch.cuda.synchronize()
         return evs
@@ -453,7 +565,11 @@ def run_ours(args):
     wall = time.perf_counter() - wall0
     launches = w.plan.launches() - launches0
     staged = (w.plan.counters()["h2d_bytes"] - staged0) // args.steps
-    dev_s = sum(a.elapsed_time(b) for a, b in evs) / 1e3
+    step_ms = [a.elapsed_time(b) for a, b in evs]
+    # value at the median step (a staged step that meets one of the host
+    # link's periodic stalls would move a mean by tens of percent)
+    dev_s = float(np.median(step_ms)) * args.steps / 1e3
+    mean_ms = float(np.mean(step_ms))
     # (2) the same steps with an event pair around every kernel launch: the
     # per-kernel times and the roofline kernel's launch duration
     w.plan.timing(True)
@@ -487,7 +603,32 @@ def run_ours(args):
         b.record(w.cs)
         b.synchronize()
         e2e_evs.append((a, b))
-    e2e_s = sum(a.elapsed_time(b) for a, b in e2e_evs) / 1e3
+    e2e_s = float(np.median([a.elapsed_time(b) for a, b in e2e_evs])) * args.steps / 1e3
+
+    # the same 32K tokens with all 512 experts resident (no waves, no staging):
+    # the routed GEMMs' tensor fraction outside the LRU waves
+    resident = None
+    if args.workload == "prefill32k_lru64" and not args.no_resident_pass and world == 1:
+        rwk = Workload("qwen3next_32k", windows=w.windows)
+        warm(rwk)
+        revs = timed_steps(rwk)
+        rwk.plan.timing(True)
+        rwk.plan.timing_read(reset=True)
+        timed_steps(rwk)
+        rkt = rwk.plan.timing_read(reset=True)
+        rwk.plan.timing(False)
+        assert rwk.plan.status() == 0, "device status %d" % rwk.plan.status()
+        rms = float(np.median([a.elapsed_time(b) for a, b in revs]))
+        resident = {
+            "workload": "qwen3next_32k", "tokens": rwk.cfg.tokens, "slots": rwk.cfg.n_slots,
+            "residency": "all 512 experts resident", "ms_per_step": rms,
+            "value": rwk.cfg.tokens / rms * 1e3, "unit": "tokens/s",
+            "roofline": roofline(rwk.cfg, {k: v for k, v in rkt.items() if v[1] > 0}, args.steps, peaks,
+                                 {}, "qwen3next_32k"),
+            "kernels_ms_per_step": {k: round(v[0] / args.steps, 4) for k, v in rkt.items() if v[1] > 0},
+            "step_ms": [round(a.elapsed_time(b), 3) for a, b in revs]}
+        rwk.plan.close()
+        del rwk
     if backend:
         torch.distributed.barrier()
     clocks = sampler.stop()
@@ -502,7 +643,8 @@ def run_ours(args):
     line = {
         "metric": METRIC if w.L == 1 else METRIC_DECODE, "value": value, "unit": "tokens/s",
         "n_gpus": world, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": tmax / args.steps * 1e3, "higher_is_better": True,
+        "warmup": args.warmup, "ms_per_step": tmax / args.steps * 1e3, "ms_per_step_mean": mean_ms,
+        "step_statistic": "median of the timed steps", "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic: seeded N(0,1) bf16 hidden rows, N(0,0.02) bf16 expert weights, "
                 "N(0,0.02) fp32 router",
@@ -526,11 +668,20 @@ def run_ours(args):
         "clocks": clocks,
         "kernels_ms_per_step": {k: round(v[0] / args.steps, 4) for k, v in kt.items() if v[1] > 0},
         "wall_s_timed": wall,
-        "step_ms": [round(a.elapsed_time(b), 3) for a, b in evs],
+        "step_ms": [round(t, 3) for t in step_ms],
         "step_ms_kernel_timing": [round(a.elapsed_time(b), 3) for a, b in evs_k],
         "e2e_step_ms": [round(a.elapsed_time(b), 3) for a, b in e2e_evs],
         "peaks": peak_kind,
     }
+    if cfg.lru and h2d_gbs:
+        # the step's bytes from the host: the staged extents (and nothing else:
+        # the rows are already on the device in the device-timed step)
+        floor_ms = staged / (h2d_gbs * 1e9) * 1e3
+        line["h2d_roof"] = {"bytes_per_step": int(staged), "measured_gbs": h2d_gbs,
+                            "how": "pinned cudaMemcpyAsync of 192 MiB (one 32-extent run), best of 4",
+                            "floor_ms": floor_ms, "frac": floor_ms / (tmax / args.steps * 1e3)}
+    if resident is not None:
+        line["resident_32k"] = resident
     if src is not None:
         ss = src.stats()
         line["config"]["source"] = {
@@ -583,7 +734,8 @@ def run_reference(args):
             "ms_per_step": dt / args.steps * 1e3, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic (same seeded inputs)",
             "config": {"workload": args.workload, "tokens": cfg.tokens, "layers": cfg.n_layers},
-            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": os.cpu_count() or 1,
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": blas_threads()[0],
+                             "cores_source": blas_threads()[1], "host_cpus": os.cpu_count(),
                              "kind": "oracle", "sample": sample},
             "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0},
@@ -618,7 +770,7 @@ def run_reference(args):
         step()
     dt = time.perf_counter() - t0
     value = ntok * args.steps / dt
-    cores = os.cpu_count() or 1
+    cores, how = blas_threads()
     sample = ("fp64 oracle forward of %d of the %d tokens per step (router over all %d experts, "
               "expert FFNs, shared expert, combine, LRU-wave plan)" % (ntok, cfg.tokens, cfg.n_experts))
     print(json.dumps({
@@ -627,13 +779,14 @@ def run_reference(args):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic (same seeded inputs)",
         "config": {"workload": args.workload, "tokens": cfg.tokens, "sample_tokens": ntok},
-        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle",
-                         "sample": sample},
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "cores_source": how,
+                         "host_cpus": os.cpu_count(), "kind": "oracle", "sample": sample},
         "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }), flush=True)
 
 
-REF_TOKENS = {"prefill32k_lru64": 4096, "prefill32k_q4_lru64": 4096, "qwen3next_4k": 4096, "tiny": 64}
+REF_TOKENS = {"prefill32k_lru64": 4096, "prefill32k_q4_lru64": 4096, "qwen3next_4k": 4096,
+              "qwen3next_32k": 4096, "tiny": 64}
 
 
 def main():
@@ -641,9 +794,11 @@ def main():
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=10)
     ap.add_argument("--warmup", type=int, default=3)
-    ap.add_argument("--workload", default="qwen3next_4k",
-                    choices=["qwen3next_4k", "prefill32k_lru64", "prefill32k_q4_lru64", "tiny",
-                             "decode48"])
+    ap.add_argument("--workload", default="prefill32k_lru64",
+                    choices=["prefill32k_lru64", "qwen3next_4k", "qwen3next_32k", "prefill32k_q4_lru64",
+                             "tiny", "decode48"])
+    ap.add_argument("--no-resident-pass", action="store_true",
+                    help="prefill32k_lru64: skip the all-resident 32K pass")
     ap.add_argument("--batch", type=int, default=64, help="decode48: rows per decode step")
     ap.add_argument("--predict", action="store_true",
                     help="decode48: next-layer prediction with the two-bank prefetch")

@@ -147,6 +147,7 @@ CONFIGS = {
     "tiny": MoEConfig("tiny", 256, 16, 2, 128, 64, 8, False),
     "qwen3next_4k": MoEConfig("qwen3next_4k", 2048, 512, 10, 512, 4096, 512, True, lru=False),
     "prefill32k_lru64": MoEConfig("prefill32k_lru64", 2048, 512, 10, 512, 32768, 64, True),
+    "qwen3next_32k": MoEConfig("qwen3next_32k", 2048, 512, 10, 512, 32768, 512, True, lru=False),
     "decode48": MoEConfig("decode48", 256, 16, 2, 128, 64, 64, False, n_layers=48, steps=64),
     "prefill32k_q4_lru64": MoEConfig("prefill32k_q4_lru64", 2048, 512, 10, 512, 32768, 64, True,
                                      wdtype=W_Q4G32),
