@@ -85,9 +85,15 @@ enum {
   MSI_FAULT_WRONG_OBJECT = 3,      /* the object's next publication names another object */
   MSI_FAULT_IO_ERROR = 4,          /* with a source attached: the object's next read completes
                                       with an I/O error (EIO); its bundle is not published */
-  MSI_FAULT_STALE_EPOCH = 5        /* with a source attached: the object's next read carries the
+  MSI_FAULT_STALE_EPOCH = 5,       /* with a source attached: the object's next read carries the
                                       previous request epoch (a completion from before a reset);
                                       it is rejected at completion, its bundle not published */
+  MSI_FAULT_DEVICE_WAIT = 6        /* the next forward on `layer` (expert: any valid index,
+                                      ignored) runs its tensor-core kernels (router, expert
+                                      GEMMs) with one extra device wait on a barrier nothing
+                                      arrives at: it runs out after the plan's wait limit, the
+                                      kernel drains its copies and MMAs, frees TMEM and reports
+                                      MSI_ERR_TIMEOUT; the combine writes no `out` row */
 };
 
 /* Forward flags. */
@@ -160,7 +166,11 @@ uint64_t msi_extent_bytes(int hidden, int inter, int wdtype);
 
 /* Create a plan: validates the description, copies the manifest, creates the
  * per-slot generation words (all slots Vacant, generation 0) and the TMA
- * descriptors over the slot pool.  Needs a current CUDA device. */
+ * descriptors over the slot pool.  Needs a current CUDA device; the plan
+ * belongs to it.  Every call that enqueues work (staging, forwards, reset)
+ * must be made with that device current, else it returns
+ * MSI_ERR_INVALID_ARG with nothing enqueued; msi_plan_destroy makes it
+ * current itself while it releases the plan. */
 msi_status msi_plan_create(const msi_plan_desc* desc, msi_plan** out);
 
 /* Destroy a plan.  Fails with MSI_ERR_SLOT_BUSY (and destroys nothing) while a
@@ -218,10 +228,13 @@ msi_status msi_moe_forward(msi_plan* plan, int layer, const void* hidden, int T,
  * Same arguments and behaviour as msi_moe_forward minus the workspace, which
  * is a fixed 32 MiB device array inside the library, reserved on every GPU
  * that loads the library until exit.  Returns MSI_ERR_WORKSPACE, enqueueing
- * nothing, when msi_workspace_size(plan, T) exceeds 32 MiB.  The first call on
- * a device resolves the array's address (make it before any stream capture).
- * All calls share the array: calls whose kernels overlap on the GPU race, so
- * serialise them.  The call itself allocates nothing. */
+ * nothing, when msi_workspace_size(plan, T) exceeds 32 MiB (above 478 tokens
+ * at the Qwen3-Next layer shape: 512 experts, top-10, hidden 2048,
+ * intermediate 512, shared expert).  The first call on a device resolves the
+ * array's address (make it before any stream capture); after a device reset
+ * the process must restart before calling this again.  All calls share the
+ * array: calls whose kernels overlap on the GPU race, so serialise them.  The
+ * call itself allocates nothing. */
 msi_status msi_moe_forward_static(msi_plan* plan, int layer, const void* hidden, int T,
                                   const float* router_w, const int32_t* slot_table,
                                   const uint64_t* expected_generations, void* out,
@@ -333,6 +346,15 @@ msi_status msi_plan_reset(msi_plan* plan, uint64_t* new_epoch);
  * Errors: MSI_ERR_INVALID_ARG for a null plan, an unknown kind or an index
  * out of range.  Nothing is allocated; msi_plan_reset does not disarm. */
 msi_status msi_fault_inject(msi_plan* plan, int kind, int layer, int expert);
+
+/* Limit of every bounded device wait of the plan's kernels, in SM clock
+ * cycles (clock64); cycles <= 0 restores the default of 4e9 (~2 s at GB300
+ * clocks).  A wait that runs out raises MSI_ERR_TIMEOUT in the forward's
+ * status word (msi_forward_status); the kernel still waits, with its own
+ * ~10 ms bound, for the copies and MMAs it issued, frees its TMEM and returns,
+ * so the context stays usable.  Applies to forwards enqueued after the call.
+ * Library convenience (the paper's runtime has no device waits). */
+msi_status msi_plan_set_wait_cycles(msi_plan* plan, int64_t cycles);
 
 /* Host-side consumer tickets: a caller that reads slots outside a forward
  * holds the slot while reading.  Staging into a held slot waits, bounded. */

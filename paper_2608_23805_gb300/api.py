@@ -101,6 +101,10 @@ class Plan:
     def inject(self, kind: int, layer: int, expert: int):
         N.check(N.lib().msi_fault_inject(self.h, kind, layer, expert), "msi_fault_inject")
 
+    def set_wait_cycles(self, cycles: int):
+        """Limit of every bounded device wait (clock64 cycles); <= 0: default."""
+        N.check(N.lib().msi_plan_set_wait_cycles(self.h, int(cycles)), "msi_plan_set_wait_cycles")
+
     def set_source(self, src: "Source | None", file_off=None):
         """Stage missing extents from `src` (file offsets [L*E]); None detaches."""
         if src is None:

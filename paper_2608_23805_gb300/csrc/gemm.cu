@@ -155,6 +155,7 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
   uint64_t* raw_empty = raw_full + C::kRaw;  // q4: code stage converted by every dequant warp
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(raw_empty + C::kRaw);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  uint64_t* never = reinterpret_cast<uint64_t*>(tmem_slot + 2);  // no thread ever arrives here
   uint8_t* epi_stage = reinterpret_cast<uint8_t*>(full) + 256;  // kEpiWarps x 4 KB (bf16 modes)
   // group table after the epilogue staging (bf16 modes) or the barriers (q4)
   int* s_mt = reinterpret_cast<int*>(reinterpret_cast<uint8_t*>(full) + 256 +
@@ -174,6 +175,7 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
       mbar_init(&tempty[b], kEpiWarps);
     }
     mbar_init(drain, 1);
+    mbar_init(never, 1);
     for (int r = 0; r < C::kRaw && C::kQ4; ++r) {
       mbar_init(&raw_full[r], 1);
       mbar_init(&raw_empty[r], C::kDq);
@@ -254,14 +256,14 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
           const uint32_t j = it - 1 - d;
           if ((int)j < 0) break;
           const long long t0 = clock64();
-          while (!mbar_try_wait(&full[j % C::kStg], (j / C::kStg) & 1) && clock64() - t0 < lim) {
+          while (!mbar_try_wait(&full[j % C::kStg], (j / C::kStg) & 1) && clock64() - t0 < kDrainCycles) {
           }
         }
         for (int d = 0; d < C::kRaw && C::kQ4; ++d) {
           if ((int)raw_issued - 1 - d < 0) break;
           const uint32_t j = raw_issued - 1 - d;
           const long long t0 = clock64();
-          while (!mbar_try_wait(&raw_full[j % C::kRaw], (j / C::kRaw) & 1) && clock64() - t0 < lim) {
+          while (!mbar_try_wait(&raw_full[j % C::kRaw], (j / C::kRaw) & 1) && clock64() - t0 < kDrainCycles) {
           }
         }
       }
@@ -299,13 +301,14 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
       // every MMA this thread issued has completed before TMEM is released
       umma_commit(drain);
       const long long t0 = clock64();
-      while (!mbar_try_wait(drain, 0) && clock64() - t0 < lim) {
+      while (!mbar_try_wait(drain, 0) && clock64() - t0 < kDrainCycles) {
       }
     }
   } else if (warp < kEpiWarps) {
     // ------------------------------------------------------------- epilogue
     uint32_t jt = 0;
     const int r = warp * 32 + lane;
+    if (a.stall && threadIdx.x == 0) mbar_wait(never, 0, abort_flag, lim);  // runs out: abort
     for (int t = blockIdx.x; t < total; t += gridDim.x, ++jt) {
       const TileCoord tc = decode_tile(a, s_mt, t);
       const Group* G = &a.groups[tc.g];

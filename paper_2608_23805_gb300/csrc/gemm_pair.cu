@@ -171,6 +171,7 @@ __global__ void __launch_bounds__(PCfg<MODE>::kThreads, 1)
   uint64_t* raw_empty = raw_full + C::kRaw;  // q4: code stage converted by every dequant warp
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(raw_empty + C::kRaw);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  uint64_t* never = reinterpret_cast<uint64_t*>(tmem_slot + 2);  // no thread ever arrives here
   uint8_t* epi_stage = reinterpret_cast<uint8_t*>(full) + 256;  // 4 KB per epilogue warp
   int* s_pt = reinterpret_cast<int*>(epi_stage + kPEpiWarps * 4096);  // [num_groups + 1]
   int* s_slot = s_pt + kMaxExperts + 1;                               // [num_groups]
@@ -190,6 +191,7 @@ __global__ void __launch_bounds__(PCfg<MODE>::kThreads, 1)
       mbar_init(&tempty[b], 2 * kPEpiWarps);  // the epilogue warps of both CTAs
     }
     mbar_init(drain, 1);
+    mbar_init(never, 1);
     for (int r = 0; r < C::kRaw && C::kQ4; ++r) {
       mbar_init(&raw_full[r], 1);
       mbar_init(&raw_empty[r], C::kDq);
@@ -265,14 +267,14 @@ __global__ void __launch_bounds__(PCfg<MODE>::kThreads, 1)
           const uint32_t j = it - 1 - d;
           if ((int)j < 0) break;
           const long long t0 = clock64();
-          while (!mbar_try_wait(&full[j % kPStages], (j / kPStages) & 1) && clock64() - t0 < lim) {
+          while (!mbar_try_wait(&full[j % kPStages], (j / kPStages) & 1) && clock64() - t0 < kDrainCycles) {
           }
         }
         for (int d = 0; d < C::kRaw && C::kQ4; ++d) {
           if ((int)raw_issued - 1 - d < 0) break;
           const uint32_t j = raw_issued - 1 - d;
           const long long t0 = clock64();
-          while (!mbar_try_wait(&raw_full[j % C::kRaw], (j / C::kRaw) & 1) && clock64() - t0 < lim) {
+          while (!mbar_try_wait(&raw_full[j % C::kRaw], (j / C::kRaw) & 1) && clock64() - t0 < kDrainCycles) {
           }
         }
       }
@@ -323,7 +325,7 @@ __global__ void __launch_bounds__(PCfg<MODE>::kThreads, 1)
       // every pair MMA that reads this CTA's shared memory or writes its TMEM
       // has completed before either is released
       const long long t0 = clock64();
-      while (!mbar_try_wait(drain, 0) && clock64() - t0 < lim) {
+      while (!mbar_try_wait(drain, 0) && clock64() - t0 < kDrainCycles) {
       }
     }
   } else if (warp < kPEpiWarps) {
@@ -331,6 +333,7 @@ __global__ void __launch_bounds__(PCfg<MODE>::kThreads, 1)
     uint32_t jt = 0;
     const uint32_t lead_tempty[2] = {mapa_shared(smem_u32(&tempty[0]), 0),
                                      mapa_shared(smem_u32(&tempty[1]), 0)};
+    if (a.stall && threadIdx.x == 0) mbar_wait(never, 0, abort_flag, lim);  // runs out: abort
     for (int t = pair; t < total; t += npairs, ++jt) {
       const PairTile tc = decode_pair(a, s_pt, t);
       const Group* G = &a.groups[tc.g];

@@ -37,6 +37,12 @@ constexpr int kMaxExperts = 512;
 constexpr int kMaxTopK = 32;
 constexpr int kMaxWave = 256;
 
+// After an expired wait (abort), a CTA still waits for the TMA loads and MMAs
+// it issued before releasing shared memory and TMEM.  Those always complete
+// within microseconds, so that drain has its own bound (~10 ms at 2 GHz),
+// independent of the wait limit that expired (which may be short).
+constexpr long long kDrainCycles = 20000000LL;
+
 // ---------------------------------------------------------------------------
 // Device-side records
 // ---------------------------------------------------------------------------
@@ -84,6 +90,10 @@ struct GemmArgs {
   int top_k;
   int* status;
   long long wait_limit;     // clock64 cycles per bounded wait
+  // non-zero: the epilogue's first thread also waits on a barrier nothing
+  // arrives at (a host-armed test of the expiry path: the wait runs out after
+  // wait_limit, the CTA aborts, drains and reports MSI_ERR_TIMEOUT)
+  int stall;
   // 4-bit weights (q4 modes): codes and fp16 scales read from the slot pool
   const uint8_t* q4_pool;
   unsigned long long q4_extent;  // bytes per slot

@@ -12,6 +12,9 @@ constexpr int kRouterTM = 32;  // tokens per fp32 FFMA router block
 constexpr int kRouterChunk = 128;  // experts per tensor-core router CTA
 constexpr int kScatterWarps = 4;   // scatter warps per block, one per router block
 
+// The device that was current when the plan was created (plan.cu).
+int plan_device(const msi_plan* p);
+
 struct RouterArgs {
   const __nv_bfloat16* x;  // [T, H]
   const float* wr;         // [E, H]
@@ -47,6 +50,7 @@ struct RouterTcArgs {
   int* bcount;             // [ceil(T/32), E]
   int* status;
   long long wait_limit;
+  int stall;               // as GemmArgs::stall
 };
 
 struct ScanArgs {

@@ -12,11 +12,18 @@
 // Contract:
 //  - Scratch limit kStaticScratchBytes (32 MiB).  A call whose
 //    msi_workspace_size(plan, T) exceeds it returns MSI_ERR_WORKSPACE and
-//    enqueues nothing (about 580 tokens at the Qwen3-Next layer shape, about
-//    20,000 at hidden 256 / intermediate 128 / top-2).
+//    enqueues nothing: up to 478 tokens a call at the Qwen3-Next layer shape
+//    (512 experts, top-10, hidden 2048, intermediate 512, shared expert),
+//    21,502 at hidden 256 / intermediate 128 / 16 experts / top-2.
+//  - The call must be made with the plan's device current (the device that
+//    was current at msi_plan_create); otherwise MSI_ERR_INVALID_ARG, nothing
+//    enqueued.
 //  - The device address of the array is resolved with cudaGetSymbolAddress on
 //    the first call on each device (with that device current) and cached;
-//    make that first call before any stream capture.
+//    make that first call before any stream capture.  The cache is not
+//    invalidated: after a device reset (cudaDeviceReset, or the primary
+//    context released and re-created) the process must restart before it
+//    calls this entry point again.
 //  - Every call on a device shares the one array, which keeps the previous
 //    call's contents.  The forward writes every scratch word it reads before
 //    reading it (the status word is cleared by the forward's first kernel), so
@@ -50,8 +57,12 @@ extern "C" msi_status msi_moe_forward_static(msi_plan* plan, int layer, const vo
   msi_status st = msi_workspace_size(plan, T, &need);
   if (st != MSI_OK) return st;
   if (need > kStaticScratchBytes) return MSI_ERR_WORKSPACE;
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return MSI_ERR_CUDA;
+  // the scratch must be the plan's device's array: the plan's kernels run there
+  const int dev = msi::plan_device(plan);
+  int cur = -1;
+  if (cudaGetDevice(&cur) != cudaSuccess) return MSI_ERR_CUDA;
+  if (cur != dev) return MSI_ERR_INVALID_ARG;
+  if (dev < 0 || dev >= kMaxDevices) return MSI_ERR_CUDA;
   void* scratch = nullptr;
   {
     std::lock_guard<std::mutex> g(g_scratch_mu);

@@ -220,6 +220,10 @@ struct KernelTimer {
 
 struct msi_plan {
   msi_plan_desc d{};
+  // the device current at msi_plan_create: the plan's device memory, streams,
+  // events and tensor maps belong to it, and every call that enqueues work
+  // requires it to be current
+  int dev = -1;
   std::vector<uint64_t> off;
   int sms = 0;
   std::vector<Slot> slots;
@@ -264,6 +268,12 @@ struct msi_plan {
   // caller pins by object [L * E]: never a victim of the plan's waves/bundles
   std::vector<char> pinned_obj;
   int n_pins = 0;
+  // clock64 cycles each bounded device wait of the plan's kernels may take
+  // before it gives up (msi_plan_set_wait_cycles)
+  long long wait_cycles = kDeviceWaitCycles;
+  // MSI_FAULT_DEVICE_WAIT: the next forward on this layer runs its tensor-core
+  // kernels with one wait that nothing ends (-1: none armed)
+  int stall_layer = -1;
   std::mutex mu;
 
   explicit msi_plan(int S) : holds(S) {
@@ -283,6 +293,15 @@ bool tensor_router(const msi_plan_desc& d) {
   if (E <= 64 && (long long)E * d.hidden <= 32768) return false;
   return E % 16 == 0 && (E <= kRouterChunk || E % kRouterChunk == 0) && d.top_k <= 31 &&
          E / std::min(E, kRouterChunk) * std::min(d.top_k + 1, std::min(E, kRouterChunk)) <= 160;
+}
+
+// A call that enqueues work must be made with the plan's device current: its
+// kernels would otherwise launch on another GPU against this plan's memory.
+msi_status check_device(const msi_plan* p) {
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  return dev == p->dev ? MSI_OK : MSI_ERR_INVALID_ARG;
 }
 
 bool shape_ok(const msi_plan_desc& d) {
@@ -581,6 +600,7 @@ struct FwdCtx {
   void* ws;
   WsLayout L;
   unsigned flags;
+  int stall;  // MSI_FAULT_DEVICE_WAIT armed for this call
   cudaStream_t cs;
   CUtensorMap tm_h, tm_x, tm_hs;
   // host-buffer calls: the rows land on the copy stream (x_ready, recorded
@@ -610,6 +630,8 @@ msi_status validate_fwd(msi_plan* p, int layer, const void* x, int T, const floa
                         const msi_route_event* ev, void* ws, size_t ws_bytes) {
   if (p == nullptr || ev == nullptr) return MSI_ERR_INVALID_ARG;
   if (p->dying) return MSI_ERR_SHUT_DOWN;
+  msi_status dst = check_device(p);
+  if (dst != MSI_OK) return dst;
   if (layer < 0 || layer >= p->d.n_layers || T < 0) return MSI_ERR_INVALID_ARG;
   if (T > 0 && (x == nullptr || rw == nullptr || out == nullptr || ev->ids == nullptr ||
                 ev->weights == nullptr))
@@ -681,7 +703,8 @@ msi_status route_rows(msi_plan* p, FwdCtx& f, const float* rw, const msi_route_e
     ra.sg = at<float>(ws, L.sg);
     ra.bcount = at<int>(ws, L.bcount);
     ra.status = at<int>(ws, L.status);
-    ra.wait_limit = kDeviceWaitCycles;
+    ra.wait_limit = p->wait_cycles;
+    ra.stall = f.stall;
     LAUNCH(p, MSI_K_ROUTER, s, launch_router_tc(f.tm_x, tm_w3, ra, s));
     p->launches++;  // launch_router_tc starts two kernels (logits + top-k, merge)
   } else {
@@ -800,7 +823,8 @@ GemmArgs gateup_args(msi_plan* p, FwdCtx& f, const Group* groups, int ng, const 
   g.perm = at<int>(f.ws, f.L.perm);
   g.top_k = d.top_k;
   g.status = at<int>(f.ws, f.L.status);
-  g.wait_limit = kDeviceWaitCycles;
+  g.wait_limit = p->wait_cycles;
+  g.stall = f.stall;
   return g;
 }
 
@@ -1033,6 +1057,7 @@ msi_status msi_plan_create(const msi_plan_desc* desc, msi_plan** out) {
   };
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
+  p->dev = dev;
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&p->sms, cudaDevAttrMultiProcessorCount, dev);
   if (e == cudaSuccess) e = cudaMalloc(&p->d_gen, sizeof(GenWord) * d.n_slots);
   if (e == cudaSuccess) e = cudaMemset(p->d_gen, 0, sizeof(GenWord) * d.n_slots);
@@ -1071,6 +1096,10 @@ msi_status msi_plan_destroy(msi_plan* p) {
     for (auto& h : p->holds)
       if (h.load() > 0) return MSI_ERR_SLOT_BUSY;
     p->dying = true;
+    // release everything with the plan's device current (the caller's current
+    // device is restored afterwards)
+    int cur = -1;
+    const bool swap = cudaGetDevice(&cur) == cudaSuccess && cur != p->dev && cudaSetDevice(p->dev) == cudaSuccess;
     // drain: every readiness, consumer and forward event still referenced
     for (auto& s : p->slots) {
       if (s.ready >= 0) cudaEventSynchronize(p->pool.ev[s.ready]);
@@ -1099,10 +1128,17 @@ msi_status msi_plan_destroy(msi_plan* p) {
     }
     if (p->ev_io_a) cudaEventDestroy(p->ev_io_a);
     if (p->ev_io_b) cudaEventDestroy(p->ev_io_b);
+    if (swap) cudaSetDevice(cur);
   }
   delete p;
   return MSI_OK;
 }
+
+}  // extern "C"
+
+int msi::plan_device(const msi_plan* p) { return p->dev; }
+
+extern "C" {
 
 msi_status msi_workspace_size(const msi_plan* p, int T, size_t* bytes) {
   if (p == nullptr || bytes == nullptr || T < 0) return MSI_ERR_INVALID_ARG;
@@ -1115,6 +1151,8 @@ msi_status msi_slot_stage(msi_plan* p, int slot, int layer, int expert, msi_stre
   if (p == nullptr) return MSI_ERR_INVALID_ARG;
   std::lock_guard<std::mutex> g(p->mu);
   if (p->dying) return MSI_ERR_SHUT_DOWN;
+  msi_status dst = check_device(p);
+  if (dst != MSI_OK) return dst;
   const auto& d = p->d;
   if (slot < 0 || slot >= d.n_slots || layer < 0 || layer >= d.n_layers || expert < 0 ||
       expert >= d.n_experts)
@@ -1216,6 +1254,8 @@ msi_status forward_resident(msi_plan* p, int layer, const void* x, int T, const 
   f.ws = ws;
   f.L = layout(p, T);
   f.flags = flags;
+  f.stall = p->stall_layer == layer;
+  if (f.stall) p->stall_layer = -1;  // one-shot
   f.cs = reinterpret_cast<cudaStream_t>(compute);
   apply_io(f, hio);
   // readiness: the compute stream waits for every pending publication it reads
@@ -1382,6 +1422,8 @@ msi_status forward_streamed(msi_plan* p, int layer, const void* x, int T, const 
   f.ws = ws;
   f.L = layout(p, T);
   f.flags = flags;
+  f.stall = p->stall_layer == layer;
+  if (f.stall) p->stall_layer = -1;  // one-shot
   f.cs = reinterpret_cast<cudaStream_t>(compute);
   apply_io(f, hio);
   cudaStream_t ss = reinterpret_cast<cudaStream_t>(stage);
@@ -1612,6 +1654,8 @@ msi_status host_begin(msi_plan* p, int T, const void* hidden_host, void* out_hos
                       size_t ws_bytes, cudaStream_t cs, HostIO* h, void** x_dev, void** out_dev) {
   if (T < 0 || (T > 0 && (hidden_host == nullptr || out_host == nullptr))) return MSI_ERR_INVALID_ARG;
   if (p->dying) return MSI_ERR_SHUT_DOWN;
+  msi_status dst = check_device(p);
+  if (dst != MSI_OK) return dst;
   const size_t base = layout(p, T).bytes, rb = rows_bytes(p, T);
   if (ws == nullptr || (uintptr_t)ws % 256 || ws_bytes < base + 2 * rb) return MSI_ERR_WORKSPACE;
   if (p->io == nullptr) {
@@ -1723,6 +1767,8 @@ msi_status msi_plan_reset(msi_plan* p, uint64_t* new_epoch) {
   if (p == nullptr) return MSI_ERR_INVALID_ARG;
   std::lock_guard<std::mutex> g(p->mu);
   if (p->dying) return MSI_ERR_SHUT_DOWN;
+  msi_status dst = check_device(p);
+  if (dst != MSI_OK) return dst;
   for (auto& h : p->holds)
     if (h.load() > 0) return MSI_ERR_SLOT_BUSY;
   // drain: every outstanding stage, consumer and forward
@@ -1774,10 +1820,21 @@ msi_status msi_fault_inject(msi_plan* p, int kind, int layer, int expert) {
       expert >= p->d.n_experts)
     return MSI_ERR_INVALID_ARG;
   if (kind != MSI_FAULT_SHORT_READ && kind != MSI_FAULT_STALE_COMPLETION &&
-      kind != MSI_FAULT_WRONG_OBJECT && kind != MSI_FAULT_IO_ERROR && kind != MSI_FAULT_STALE_EPOCH)
+      kind != MSI_FAULT_WRONG_OBJECT && kind != MSI_FAULT_IO_ERROR && kind != MSI_FAULT_STALE_EPOCH &&
+      kind != MSI_FAULT_DEVICE_WAIT)
     return MSI_ERR_INVALID_ARG;
   std::lock_guard<std::mutex> g(p->mu);
-  p->faults[obj_key(layer, expert)] = kind;
+  if (kind == MSI_FAULT_DEVICE_WAIT)
+    p->stall_layer = layer;
+  else
+    p->faults[obj_key(layer, expert)] = kind;
+  return MSI_OK;
+}
+
+msi_status msi_plan_set_wait_cycles(msi_plan* p, int64_t cycles) {
+  if (p == nullptr) return MSI_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> g(p->mu);
+  p->wait_cycles = cycles > 0 ? (long long)cycles : kDeviceWaitCycles;
   return MSI_OK;
 }
 

@@ -144,6 +144,7 @@ __global__ void __launch_bounds__(NTH, 1)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   int* ready_flag = const_cast<int*>(abort_flag) + 1;
+  uint64_t* never = reinterpret_cast<uint64_t*>(tmem_slot + 4);  // no thread ever arrives here
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int E = a.E;
@@ -163,6 +164,7 @@ __global__ void __launch_bounds__(NTH, 1)
     }
     mbar_init(tfull, 1);
     mbar_init(drain, 1);
+    mbar_init(never, 1);
     *abort_flag = 0;
     mbar_fence_init();
   }
@@ -199,7 +201,7 @@ __global__ void __launch_bounds__(NTH, 1)
         for (int d = 0; d < RT_STAGES && it - 1 - d >= 0; ++d) {
           const int j = it - 1 - d;
           const long long t0 = clock64();
-          while (!mbar_try_wait(&full[j % RT_STAGES], (j / RT_STAGES) & 1) && clock64() - t0 < lim) {
+          while (!mbar_try_wait(&full[j % RT_STAGES], (j / RT_STAGES) & 1) && clock64() - t0 < kDrainCycles) {
           }
         }
       }
@@ -228,7 +230,7 @@ __global__ void __launch_bounds__(NTH, 1)
       if (ok) umma_commit(tfull);
       umma_commit(drain);
       const long long t0 = clock64();
-      while (!mbar_try_wait(drain, 0) && clock64() - t0 < lim) {
+      while (!mbar_try_wait(drain, 0) && clock64() - t0 < kDrainCycles) {
       }
     }
   } else if (warp < 4) {
@@ -236,7 +238,8 @@ __global__ void __launch_bounds__(NTH, 1)
     // Chunk logits TMEM -> shared memory (the stage buffers are free once the
     // MMA loop is done; rows padded so the 32 lanes' column writes fall into
     // distinct banks).
-    const bool ready = __all_sync(0xffffffffu, mbar_wait(tfull, 0, abort_flag, lim));
+    if (a.stall && threadIdx.x == 0) mbar_wait(never, 0, abort_flag, lim);  // runs out: abort
+    const bool ready = __all_sync(0xffffffffu, mbar_wait(tfull, 0, abort_flag, lim)) && !*abort_flag;
     tc_fence_after();
     float* L = reinterpret_cast<float*>(smem);
     if (ready) {
@@ -381,10 +384,14 @@ __global__ void __launch_bounds__(kMergeThreads) router_merge_kernel(const Route
       const float lk1 = __shfl_sync(0xffffffffu, my_v[u], k - 1);
       if (t < a.T) {
         if (lane < k) {
+          // an aborted router leaves no valid candidate: expert 0 stands in,
+          // counted like any id, so that the permutation stays a bijection
+          // (the status word already fails the call)
           const bool real = my_i[u] >= 0 && my_i[u] < E;
-          a.ids[(size_t)t * k + lane] = real ? my_i[u] : 0;
+          const int id = real ? my_i[u] : 0;
+          a.ids[(size_t)t * k + lane] = id;
           a.weights[(size_t)t * k + lane] = ex / sum;
-          if (real) atomicAdd(&hist[my_i[u]], 1);
+          atomicAdd(&hist[id], 1);
         }
         if (a.gap != nullptr && lane == 0) a.gap[t] = (k < E) ? (lk1 - next_v[u]) : INFINITY;
       }

@@ -24,7 +24,7 @@ MSI_ERR_UNSUPPORTED = 9
 MSI_ERR_WORKSPACE = 10
 MSI_ERR_SOURCE = 11
 (MSI_FAULT_SHORT_READ, MSI_FAULT_STALE_COMPLETION, MSI_FAULT_WRONG_OBJECT, MSI_FAULT_IO_ERROR,
- MSI_FAULT_STALE_EPOCH) = 1, 2, 3, 4, 5
+ MSI_FAULT_STALE_EPOCH, MSI_FAULT_DEVICE_WAIT) = 1, 2, 3, 4, 5, 6
 MSI_MAX_WINDOWS = 64
 
 MSI_W_BF16 = 0
@@ -113,6 +113,7 @@ _SIGS = {
     "msi_forward_status": (ctypes.c_int, [_P, ctypes.POINTER(ctypes.c_int)]),
     "msi_plan_reset": (ctypes.c_int, [_P, ctypes.POINTER(ctypes.c_uint64)]),
     "msi_fault_inject": (ctypes.c_int, [_P, ctypes.c_int, ctypes.c_int, ctypes.c_int]),
+    "msi_plan_set_wait_cycles": (ctypes.c_int, [_P, ctypes.c_int64]),
     "msi_source_open": (ctypes.c_int, [ctypes.POINTER(msi_source_desc), ctypes.POINTER(_P)]),
     "msi_source_close": (ctypes.c_int, [_P]),
     "msi_source_stats_read": (ctypes.c_int, [_P, ctypes.POINTER(msi_source_stats)]),
