@@ -333,21 +333,26 @@ def roofline(cfg, kt: dict, steps: int, peaks: dict, clocks: dict, workload: str
     kernels run at full SM clock inside steps of milliseconds, far from the
     seconds-long power-capped loop the sustained figure comes from.  Without
     routed GEMM time (a step with no rows) the dominant kernel kind alone."""
-    if "gateup" in kt and "down" in kt:
+    if "ffn" in kt or ("gateup" in kt and "down" in kt):
+        # separate launches (gateup, down) and fused wave launches (ffn: both
+        # projections of one wave in one kernel) may both appear in a step
         f1, b1 = algorithmic(cfg, "gateup", {})
         f2, b2 = algorithmic(cfg, "down", {})
         bound = _bound_of(f1 + f2, b1 + b2, peaks)
-        ms = kt["gateup"][0] + kt["down"][0]
-        launches = kt["gateup"][1]
+        ms = sum(kt[k][0] for k in ("gateup", "down", "ffn") if k in kt)
+        launches = kt["ffn"][1] if "ffn" in kt else kt["gateup"][1]
         r = {"bound": bound}
         r.update(_part(f1 + f2, b1 + b2, ms, launches, steps, peaks, bound))
         r["kernel"] = "gateup+down"
         r["launches_per_step"] = launches / steps
-        r["parts"] = {
-            "gateup": dict(_part(f1, b1, kt["gateup"][0], kt["gateup"][1], steps, peaks, bound),
-                           flops_per_step=f1, bytes_per_step=b1),
-            "down": dict(_part(f2, b2, kt["down"][0], kt["down"][1], steps, peaks, bound),
-                         flops_per_step=f2, bytes_per_step=b2)}
+        r["parts"] = {}
+        if "gateup" in kt and "down" in kt:
+            r["parts"]["gateup"] = dict(_part(f1, b1, kt["gateup"][0], kt["gateup"][1], steps, peaks, bound),
+                                        flops_per_step=f1, bytes_per_step=b1)
+            r["parts"]["down"] = dict(_part(f2, b2, kt["down"][0], kt["down"][1], steps, peaks, bound),
+                                      flops_per_step=f2, bytes_per_step=b2)
+        if "ffn" in kt:
+            r["fused_waves"] = True
         kind = "gateup+down"
     else:
         kind = max(kt, key=lambda k: kt[k][0])

@@ -103,9 +103,14 @@ enum {
                              bf16 launches whose groups average >= 1,024 rows use CTA-pair
                              256-row tiles (both accumulate in fp32 over the same K order
                              and meet the same output tolerance) */
-  MSI_FWD_SHARED_UNGATED = 4 /* the shared expert's output is added with gate 1 instead of
-                                sigmoid(x . w_sg) (the other reading of its gate; no effect
-                                without a shared expert) */
+  MSI_FWD_SHARED_UNGATED = 4, /* the shared expert's output is added with gate 1 instead of
+                                 sigmoid(x . w_sg) (the other reading of its gate; no effect
+                                 without a shared expert) */
+  MSI_FWD_SPLIT_WAVES = 8     /* streamed calls: launch each bf16 wave's gate-up and down GEMMs
+                                 as two kernels; by default a wave whose gate-up takes
+                                 single-CTA tiles runs both in one launch, the down tiles
+                                 after the gate-up tiles they read (same tiles, same K order,
+                                 bit-identical results) */
 };
 
 /* Plan description (copied by msi_plan_create; pointers must outlive the plan). */
@@ -454,7 +459,8 @@ enum {
   MSI_K_SHARED_DOWN = 8,   /* shared-expert down GEMM */
   MSI_K_COMBINE = 9,       /* weighted combine */
   MSI_K_PUBLISH = 10,      /* slot generation publication (staging stream) */
-  MSI_K_COUNT = 11
+  MSI_K_FFN = 11,          /* one wave's gate-up and down GEMMs in one launch */
+  MSI_K_COUNT = 12
 };
 
 /* Per-kernel timing: when enabled, every launch is bracketed by CUDA events on

@@ -18,9 +18,10 @@ def _ptr(t) -> int | None:
     return None if t is None else t.data_ptr()
 
 
-def _flags(residual: bool, single_cta: bool, shared_gate: bool = True) -> int:
+def _flags(residual: bool, single_cta: bool, shared_gate: bool = True, split_waves: bool = False) -> int:
     return ((N.MSI_FWD_RESIDUAL if residual else 0) | (N.MSI_FWD_SINGLE_CTA if single_cta else 0)
-            | (0 if shared_gate else N.MSI_FWD_SHARED_UNGATED))
+            | (0 if shared_gate else N.MSI_FWD_SHARED_UNGATED)
+            | (N.MSI_FWD_SPLIT_WAVES if split_waves else 0))
 
 
 def _stream(s) -> int | None:
@@ -150,7 +151,7 @@ class Plan:
 
     def forward_streamed(self, layer, x, router_w, out=None, ev=None, residual=False, stream=None,
                          stage_stream=None, check=True, single_cta=False, next_router_w=None,
-                         next_ev=None):
+                         next_ev=None, split_waves=False):
         """Streamed layer forward.  With next_router_w (layer + 1's router), the
         rows are also routed through it and layer + 1's predicted objects are
         prefetched after the last wave; the predicted route event is written to
@@ -162,8 +163,8 @@ class Plan:
         if next_router_w is None:
             rc = N.lib().msi_moe_forward_streamed(self.h, layer, _ptr(x), T, _ptr(router_w), _ptr(out),
                                                   ctypes.byref(ev.c), _ptr(ws), ws.numel(),
-                                                  _flags(residual, single_cta), _stream(stream),
-                                                  _stream(stage_stream))
+                                                  _flags(residual, single_cta, True, split_waves),
+                                                  _stream(stream), _stream(stage_stream))
             where = "msi_moe_forward_streamed"
         else:
             next_ev = RouteEvent(T, self.k, self.E) if next_ev is None else next_ev
@@ -171,7 +172,7 @@ class Plan:
             rc = N.lib().msi_moe_forward_streamed_next(
                 self.h, layer, _ptr(x), T, _ptr(router_w), _ptr(out), ctypes.byref(ev.c),
                 _ptr(next_router_w), ctypes.byref(next_ev.c), _ptr(ws), ws.numel(),
-                _flags(residual, single_cta), _stream(stream), _stream(stage_stream))
+                _flags(residual, single_cta, True, split_waves), _stream(stream), _stream(stage_stream))
             where = "msi_moe_forward_streamed_next"
         if check:
             N.check(rc, where)

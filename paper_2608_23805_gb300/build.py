@@ -18,8 +18,8 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libmsi.so")
-SOURCES = ["plan.cu", "router.cu", "router_tc.cu", "permute.cu", "gemm.cu", "gemm_pair.cu", "noalloc.cu",
-           "source.cpp"]
+SOURCES = ["plan.cu", "router.cu", "router_tc.cu", "permute.cu", "gemm.cu", "gemm_pair.cu", "gemm_fused.cu",
+           "noalloc.cu", "source.cpp"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -105,6 +105,31 @@ struct GemmArgs {
 
 enum GemmMode { kGateUpGather = 0, kGateUpTma = 1, kDown = 2, kGateUpGatherQ4 = 3, kDownQ4 = 4 };
 
+// One wave's gate-up and down projections in one launch (gemm_fused.cu).
+struct FusedArgs {
+  const Group* groups;
+  int num_groups;
+  const int* total_mtiles;  // device: [0] 128-row tiles
+  int nt_up, nt_dn;         // column tiles: I / 128 (h), H / 256 (y)
+  int kb_up, kb_dn;         // K blocks: H / 64, I / 64
+  int w13_rows_per_slot;    // rows of one slot in the W13 map (3 I); gate rows at n * 128
+  int w13_up_off;           // up rows after the gate rows (I)
+  int w2_rows_per_slot;     // rows of one slot in the W2 map (3 H)
+  int w2_row_off;           // W2 after W13 inside a slot (2 H rows of I)
+  __nv_bfloat16* h;         // [T k, I]
+  int h_ld;
+  __nv_bfloat16* y;         // [T k, H]
+  int y_ld;
+  const __nv_bfloat16* x;   // [T, H]
+  int x_ld;
+  const int* perm;          // permuted row -> t k + j
+  int top_k;
+  int* ready;               // [m-tiles] finished gate-up tiles per 128-row tile (zeroed per wave)
+  int* status;
+  long long wait_limit;
+  int stall;                // as GemmArgs::stall
+};
+
 // ---------------------------------------------------------------------------
 // Launchers (return cudaError_t of the launch)
 // ---------------------------------------------------------------------------
@@ -114,6 +139,10 @@ cudaError_t launch_gemm(int mode, const CUtensorMap& tmA, const CUtensorMap& tmB
 // kGateUpTma and kDown; `max_pairs` bounds the pairs launched.
 cudaError_t launch_gemm_pair(int mode, const CUtensorMap& tmA, const CUtensorMap& tmB,
                              const GemmArgs& a, int max_pairs, cudaStream_t s);
+// Gate-up and down of one wave in one cooperative launch of `grid` CTAs
+// (at most one per SM); tmW13 / tmW2 as the pool maps of the two projections.
+cudaError_t launch_fused_wave(const CUtensorMap& tmW13, const CUtensorMap& tmW2, const FusedArgs& a,
+                              int grid, cudaStream_t s);
 
 // GEMM tiling
 constexpr int kBM = 128;

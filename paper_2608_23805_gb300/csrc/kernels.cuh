@@ -121,6 +121,8 @@ struct SetupArgs {
   Group* groups;
   int* total_mtiles;   // [0]: 128-row tiles, [1]: 256-row pair tiles
   int* status;
+  int* ready;          // fused wave: per-m-tile counters, zeroed here (or nullptr)
+  int n_ready;
 };
 
 struct CombineArgs {

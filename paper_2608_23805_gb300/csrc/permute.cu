@@ -317,6 +317,8 @@ __global__ void __launch_bounds__(kMaxExperts) setup_kernel(const SetupArgs a, c
     g.pad1 = 0;
     a.groups[i] = g;
   }
+  if (a.ready != nullptr)
+    for (int r = i; r < a.n_ready; r += blockDim.x) a.ready[r] = 0;
   const int key = code ? (e << 4) | code : 0x7fffffff;
   const int m = block_min(key, tmp);
   if (i == 0) {

@@ -173,7 +173,7 @@ struct WaveEntry {
 
 struct WsLayout {
   size_t status, table, expected, groups, total, sh_group, sh_total, w3, cand_v, cand_i, bcount,
-      bbase, offsets, perm, inv, sg, h, yp, hs, ys, bytes;
+      bbase, offsets, perm, inv, sg, h, yp, hs, ys, ready, bytes;
   int tm;  // tokens per router block
 };
 
@@ -344,6 +344,7 @@ WsLayout layout(const msi_plan* p, int T) {
   L.sg = take(4 * (size_t)T);
   L.h = take(2 * Tk * I);
   L.yp = take(2 * Tk * H);
+  L.ready = take(4 * (Tk / kBM + E + 1));  // fused waves: a counter per 128-row tile
   if (p->d.has_shared) {
     L.hs = take(2 * (size_t)T * I);
     L.ys = take(2 * (size_t)T * H);
@@ -857,7 +858,15 @@ bool pair_tiles(const FwdCtx& f, long long rows, int groups, long long min_rows 
 // per unit of tensor work, which pays once the groups fill 256-row tiles.
 constexpr long long kPairMinRowsQ4 = 512;
 
-msi_status routed_ffn(msi_plan* p, FwdCtx& f, int ng, int grid1, int grid2, long long rows) {
+// A streamed bf16 wave whose gate-up takes single-CTA tiles runs its gate-up
+// and down in one launch (gemm_fused.cu): the wave is too small to fill the
+// SMs' last round of gate-up tiles, and the down tiles fill it.
+bool fused_wave(const msi_plan* p, const FwdCtx& f, long long rows, int ng) {
+  return p->d.wdtype == MSI_W_BF16 && !(f.flags & MSI_FWD_SPLIT_WAVES) && !pair_tiles(f, rows, ng);
+}
+
+msi_status routed_ffn(msi_plan* p, FwdCtx& f, int ng, int grid1, int grid2, long long rows,
+                      int wave_mtiles = -1) {
   const bool bf16 = p->d.wdtype == MSI_W_BF16;
   const bool pair_up = bf16 ? pair_tiles(f, rows, ng) : pair_tiles(f, rows, ng, kPairMinRowsQ4);
   const bool pair_down = pair_tiles(f, rows, ng, bf16 ? kPairMinRowsDown : kPairMinRowsQ4);
@@ -893,6 +902,38 @@ msi_status routed_ffn(msi_plan* p, FwdCtx& f, int ng, int grid1, int grid2, long
              launch_gemm_pair(kDownQ4, f.tm_h, p->tm_q2, g2, std::max(1, grid2 / 2), f.cs));
     else
       LAUNCH(p, MSI_K_DOWN, f.cs, launch_gemm(kDownQ4, f.tm_h, p->tm_q2, g2, grid2, f.cs));
+    return MSI_OK;
+  }
+  if (wave_mtiles >= 0 && fused_wave(p, f, rows, ng)) {
+    // one launch: the wave's gate-up tiles, then its down tiles (the setup
+    // kernel zeroed the per-m-tile counters)
+    FusedArgs fa{};
+    fa.groups = groups;
+    fa.num_groups = ng;
+    fa.total_mtiles = total;
+    fa.nt_up = d.inter / 128;
+    fa.nt_dn = d.hidden / kBN;
+    fa.kb_up = d.hidden / kBK;
+    fa.kb_dn = d.inter / kBK;
+    fa.w13_rows_per_slot = 3 * d.inter;
+    fa.w13_up_off = d.inter;
+    fa.w2_rows_per_slot = 3 * d.hidden;
+    fa.w2_row_off = 2 * d.hidden;
+    fa.h = at<__nv_bfloat16>(f.ws, f.L.h);
+    fa.h_ld = d.inter;
+    fa.y = at<__nv_bfloat16>(f.ws, f.L.yp);
+    fa.y_ld = d.hidden;
+    fa.x = static_cast<const __nv_bfloat16*>(f.x);
+    fa.x_ld = d.hidden;
+    fa.perm = at<int>(f.ws, f.L.perm);
+    fa.top_k = d.top_k;
+    fa.ready = at<int>(f.ws, f.L.ready);
+    fa.status = at<int>(f.ws, f.L.status);
+    fa.wait_limit = p->wait_cycles;
+    fa.stall = f.stall;
+    const long long tiles = (long long)wave_mtiles * (fa.nt_up + fa.nt_dn);
+    const int grid = (int)std::min<long long>(p->sms, std::max<long long>(1, tiles));
+    LAUNCH(p, MSI_K_FFN, f.cs, launch_fused_wave(p->tm_w13, p->tm_w2, fa, grid, f.cs));
     return MSI_OK;
   }
   if (pair_up)
@@ -1595,10 +1636,14 @@ msi_status forward_streamed(msi_plan* p, int layer, const void* x, int T, const 
     sa.groups = at<Group>(ws, f.L.groups);
     sa.total_mtiles = at<int>(ws, f.L.total);
     sa.status = at<int>(ws, f.L.status);
+    if (fused_wave(p, f, wave_rows, wp.n)) {
+      sa.ready = at<int>(ws, f.L.ready);
+      sa.n_ready = mtiles;
+    }
     LAUNCH(p, MSI_K_SETUP, f.cs, launch_setup_wave(sa, wp, f.cs));
     const int g1 = std::max(1, std::min(p->sms, mtiles * (d.inter / 128)));
     const int g2 = std::max(1, std::min(p->sms, mtiles * (d.hidden / kBN)));
-    st = routed_ffn(p, f, wp.n, g1, g2, wave_rows);
+    st = routed_ffn(p, f, wp.n, g1, g2, wave_rows, mtiles);
     if (st != MSI_OK) return st;
     st = consumer_record(p, used, f.cs);
     if (st != MSI_OK) return st;

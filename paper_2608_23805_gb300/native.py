@@ -34,8 +34,9 @@ MSI_SLOT_VACANT, MSI_SLOT_LOADING, MSI_SLOT_DEVICE_READY, MSI_SLOT_IN_USE, MSI_S
 MSI_FWD_RESIDUAL = 1
 MSI_FWD_SINGLE_CTA = 2
 MSI_FWD_SHARED_UNGATED = 4
+MSI_FWD_SPLIT_WAVES = 8
 KERNEL_KINDS = ["upload", "router", "scan", "scatter", "setup", "gateup", "down", "shared_gateup",
-                "shared_down", "combine", "publish"]
+                "shared_down", "combine", "publish", "ffn"]
 
 
 class msi_plan_desc(ctypes.Structure):

@@ -71,3 +71,15 @@ def test_router_roof_is_the_fp32_alu_rate():
     r = bench.roofline(cfg, {"router": (1.0, 10)}, 10, PEAKS, {"sm_mhz": 2000.0}, "x")
     assert r["bound"] == "alu"
     assert r["peak"] == pytest.approx(152 * 128 * 2 * 2000e6 / 1e12)
+
+
+def test_roofline_of_fused_wave_launches():
+    """Fused wave launches (one kernel per wave for both projections) carry
+    the pair's flops over their own time."""
+    cfg = synth.config("prefill32k_lru64")
+    kt = {"ffn": (2.0 * 4, 64)}
+    r = bench.roofline(cfg, kt, 4, PEAKS, {}, "no-such-workload")
+    flops_step = 1_374_389_534_720 + 687_194_767_360
+    assert r["bound"] == "tensor" and r["fused_waves"]
+    assert r["achieved"] == pytest.approx(flops_step / 2.0e-3 / 1e12)
+    assert r["launches_per_step"] == 16

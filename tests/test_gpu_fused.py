@@ -1,0 +1,82 @@
+"""Fused wave GEMMs: a streamed call runs each bf16 wave's gate-up and down
+projections in one launch, the down tiles after the gate-up tiles whose h rows
+they read (per-m-tile counters).  The same tiles with the same K order run as
+two launches under MSI_FWD_SPLIT_WAVES with single-CTA tiles, so the two must
+agree bit for bit; both match the fp64 oracle, with route events exact and
+the slot trace equal to the simulator's."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+from gpu_case import Case, bf16_bits, bf16_tensor, compare_out, compare_routes
+from paper_2608_23805_gb300 import native as N
+
+pytestmark = pytest.mark.gpu
+
+
+def _run(case, x, split):
+    case.plan.trace(clear=True)
+    out, ev = case.plan.forward_streamed(0, x, case.router[0], split_waves=split, single_cta=split)
+    torch.cuda.synchronize()
+    assert case.plan.status() == N.MSI_OK
+    return bf16_bits(out), ev.ids.cpu().numpy(), ev.weights.cpu().numpy(), case.plan.trace()
+
+
+@pytest.mark.parametrize("tokens,top_k", [(2048, 4), (333, 3)])
+def test_fused_waves_small_shape_full_oracle(tokens, top_k):
+    """H 512, I 256, 32 experts, 16 slots (waves of 8): ~256 and ~31 rows per
+    expert (several m-tiles per expert; ragged and single-tile groups)."""
+    cfg = synth.config("tiny", hidden=512, inter=256, n_experts=32, top_k=top_k, tokens=tokens,
+                       n_slots=16)
+    case = Case(cfg)
+    x_bits = synth.hidden(cfg, 0, 21)
+    x = bf16_tensor(x_bits)
+    of, idf, wf, trf = _run(case, x, split=False)
+    case2 = Case(cfg)
+    os_, ids_, ws_, trs = _run(case2, x, split=True)
+    assert np.array_equal(of, os_)                    # bit-identical to the split launches
+    assert np.array_equal(idf, ids_) and np.array_equal(wf, ws_)
+    assert trf == trs
+    ref = case.oracle_layer(x_bits)
+    compare_routes(idf, wf, ref)
+    compare_out(of, ref["out"])
+    case.close()
+    case2.close()
+
+
+def test_fused_waves_qwen_shape_sampled():
+    """Qwen3-Next shape, 8,192 tokens, 64 slots (waves of 32): ~160 rows per
+    expert, two m-tiles each (a full and a ragged one)."""
+    cfg = synth.config("prefill32k_lru64", tokens=8192)
+    case = Case(cfg)
+    x_bits = synth.hidden(cfg, 0, 22)
+    x = bf16_tensor(x_bits)
+    of, idf, wf, _ = _run(case, x, split=False)
+    os_, ids_, _, _ = _run(case, x, split=True)       # same plan: the second call's waves differ,
+    assert np.array_equal(idf, ids_)                  # the expert work does not
+    assert np.array_equal(of, os_)
+    rng = np.random.default_rng(9)
+    toks = np.sort(rng.choice(cfg.tokens, 40, replace=False))
+    ref = case.oracle_layer(x_bits, tokens=toks)
+    compare_out(of[toks], ref["out"])
+    assert case.plan.launches() > 0
+    case.close()
+
+
+def test_fused_waves_launch_count():
+    """One expert-FFN launch per wave instead of two."""
+    cfg = synth.config("tiny", hidden=512, inter=256, n_experts=32, top_k=4, tokens=1024, n_slots=16)
+    case = Case(cfg)
+    x = bf16_tensor(synth.hidden(cfg, 0, 23))
+    case.plan.timing(True)
+    case.plan.timing_read(reset=True)
+    case.plan.forward_streamed(0, x, case.router[0])
+    torch.cuda.synchronize()
+    kt = case.plan.timing_read(reset=True)
+    case.plan.timing(False)
+    n_waves = len({r[6] for r in case.plan.trace() if r[5] in ("hit", "stage")})
+    assert kt["ffn"][1] == n_waves
+    assert kt["gateup"][1] == 0 and kt["down"][1] == 0
+    case.close()
