@@ -66,12 +66,9 @@ L2_BYTES = 129 * 1024 * 1024
 # (the summaries under profiles/), keyed by (workload, kernel kind); reported
 # only while the GEMM source still hashes to the value the capture was taken at.
 TRAFFIC = {
-    ("qwen3next_4k", "gateup"): {"bytes_per_launch": 2267939328 + 42387968, "src_hash": "51698327c3146b09",
-                                 "profile": "profiles/gemm_gateup_qwen3next_4k.md"},
-    ("prefill32k_lru64", "gateup"): {"bytes_per_launch": 205885440 + 14321920, "src_hash": "51698327c3146b09",
-                                     "profile": "profiles/gemm_gateup_prefill32k_lru64.md"},
-    ("prefill32k_q4_lru64", "gateup"): {"bytes_per_launch": 106187008 + 10726400, "src_hash": "51698327c3146b09",
-                                        "profile": "profiles/gemm_gateup_q4_prefill32k_q4_lru64.md"},
+    # one fused wave launch (gate-up + down of 32 experts, ~20,480 routed rows)
+    ("prefill32k_lru64", "gateup+down"): {"bytes_per_launch": 293111552 + 59264000, "src_hash": "17e10c6ea83bf188",
+                                          "profile": "profiles/gemm_fused_wave_prefill32k_lru64.md"},
 }
 
 
@@ -89,7 +86,7 @@ def kernel_source_hash() -> str:
     and blank lines left out: a capture stays valid until the code changes."""
     import re
     h = hashlib.sha256()
-    for name in ("gemm.cu", "gemm_pair.cu", "internal.cuh"):
+    for name in ("gemm.cu", "gemm_pair.cu", "gemm_fused.cu", "gemm_fused_pair.cu", "internal.cuh"):
         with open(os.path.join(ROOT, "paper_2608_23805_gb300", "csrc", name)) as f:
             src = re.sub(r"/\*.*?\*/", "", f.read(), flags=re.S)
         for line in src.splitlines():

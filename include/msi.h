@@ -107,10 +107,11 @@ enum {
                                  sigmoid(x . w_sg) (the other reading of its gate; no effect
                                  without a shared expert) */
   MSI_FWD_SPLIT_WAVES = 8     /* streamed calls: launch each bf16 wave's gate-up and down GEMMs
-                                 as two kernels; by default a wave whose gate-up takes
-                                 single-CTA tiles runs both in one launch, the down tiles
-                                 after the gate-up tiles they read (same tiles, same K order,
-                                 bit-identical results) */
+                                 as two kernels; by default both run in one launch, the down
+                                 tiles after the gate-up tiles they read, on 256-row CTA-pair
+                                 tiles once the wave's groups average >= 1,024 rows (else, or
+                                 with MSI_FWD_SINGLE_CTA, 128-row tiles: then bit-identical
+                                 to the split launches with MSI_FWD_SINGLE_CTA) */
 };
 
 /* Plan description (copied by msi_plan_create; pointers must outlive the plan). */

@@ -133,7 +133,7 @@ class Plan:
         return ws
 
     def forward(self, layer, x, router_w, slot_table, expected, out=None, ev=None, residual=False,
-                stream=None, check=True, single_cta=False, shared_gate=True):
+                stream=None, check=True, single_cta=False, shared_gate=True, split_waves=False):
         T = x.shape[0]
         out = torch.empty_like(x) if out is None else out
         ev = RouteEvent(T, self.k, self.E) if ev is None else ev
@@ -142,7 +142,7 @@ class Plan:
         ex = np.ascontiguousarray(expected, dtype=np.uint64)
         rc = N.lib().msi_moe_forward(self.h, layer, _ptr(x), T, _ptr(router_w), st.ctypes.data,
                                      ex.ctypes.data, _ptr(out), ctypes.byref(ev.c), _ptr(ws),
-                                     ws.numel(), _flags(residual, single_cta, shared_gate),
+                                     ws.numel(), _flags(residual, single_cta, shared_gate, split_waves),
                                      _stream(stream))
         if check:
             N.check(rc, "msi_moe_forward")

@@ -19,7 +19,7 @@ CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libmsi.so")
 SOURCES = ["plan.cu", "router.cu", "router_tc.cu", "permute.cu", "gemm.cu", "gemm_pair.cu", "gemm_fused.cu",
-           "noalloc.cu", "source.cpp"]
+           "gemm_fused_pair.cu", "noalloc.cu", "source.cpp"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -143,6 +143,10 @@ cudaError_t launch_gemm_pair(int mode, const CUtensorMap& tmA, const CUtensorMap
 // (at most one per SM); tmW13 / tmW2 as the pool maps of the two projections.
 cudaError_t launch_fused_wave(const CUtensorMap& tmW13, const CUtensorMap& tmW2, const FusedArgs& a,
                               int grid, cudaStream_t s);
+// The same on CTA pairs (256-row tiles, gemm_fused_pair.cu); at most
+// `max_pairs` pairs, never more than can be resident at once.
+cudaError_t launch_fused_wave_pair(const CUtensorMap& tmW13, const CUtensorMap& tmW2,
+                                   const FusedArgs& a, int max_pairs, cudaStream_t s);
 
 // GEMM tiling
 constexpr int kBM = 128;

@@ -86,6 +86,9 @@ struct ScatterArgs {
   const int* tab_slot;                    // [E]
   const unsigned long long* tab_expected;  // [E]
   int layer;
+  // fused resident GEMMs: per-m-tile counters zeroed by the setup block (or nullptr)
+  int* ready;
+  int n_ready;
 };
 
 // Per-call tables uploaded by value (kernel parameters, < 32 KB).

@@ -87,6 +87,8 @@ __device__ void scatter_setup(const ScatterArgs& a, const int* offs,
   __shared__ int kmin[kScatterWarps];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   if (a.tab_slot == nullptr) return;  // streamed call: the groups are built per wave
+  if (a.ready != nullptr)
+    for (int r = tid; r < a.n_ready; r += blockDim.x) a.ready[r] = 0;
   int cnt[4], code[4], mt[4], pt[4];
   int key = 0x7fffffff;
   int slot[4];
@@ -351,8 +353,9 @@ __device__ __forceinline__ void fma8(float (&acc)[8], float w, const uint4& y) {
 }
 
 // One block per token; the token's k row indices and weights are read once
-// into shared memory, and four expert rows are loaded before they are summed
-// (still in j order, fp32).
+// into shared memory, and up to eight expert rows are loaded before they are
+// summed (still in j order, fp32), so each thread keeps eight 16-byte loads
+// in flight.
 __global__ void __launch_bounds__(256) combine_kernel(const CombineArgs a) {
   if (*a.status != 0) return;  // fail closed: nothing stale becomes visible
   __shared__ int s_row[kMaxTopK];
@@ -369,13 +372,22 @@ __global__ void __launch_bounds__(256) combine_kernel(const CombineArgs a) {
 #pragma unroll
     for (int i = 0; i < 8; ++i) acc[i] = 0.f;
     int j = 0;
-    for (; j + 4 <= a.k; j += 4) {
+    for (; j + 8 <= a.k; j += 8) {
+      uint4 y[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u)
+        y[u] = __ldg(reinterpret_cast<const uint4*>(a.yp + (size_t)s_row[j + u] * a.H) + c);
+#pragma unroll
+      for (int u = 0; u < 8; ++u) fma8(acc, s_w[j + u], y[u]);
+    }
+    if (j + 4 <= a.k) {
       uint4 y[4];
 #pragma unroll
       for (int u = 0; u < 4; ++u)
         y[u] = __ldg(reinterpret_cast<const uint4*>(a.yp + (size_t)s_row[j + u] * a.H) + c);
 #pragma unroll
       for (int u = 0; u < 4; ++u) fma8(acc, s_w[j + u], y[u]);
+      j += 4;
     }
     for (; j < a.k; ++j)
       fma8(acc, s_w[j], __ldg(reinterpret_cast<const uint4*>(a.yp + (size_t)s_row[j] * a.H) + c));

@@ -737,6 +737,22 @@ msi_status route_rows(msi_plan* p, FwdCtx& f, const float* rw, const msi_route_e
   return MSI_OK;
 }
 
+// A streamed bf16 wave runs its gate-up and down in one launch
+// (gemm_fused.cu, gemm_fused_pair.cu): a wave is too small to fill the SMs'
+// last round of gate-up tiles, and the down tiles fill it.
+bool fused_wave(const msi_plan* p, const FwdCtx& f, long long, int) {
+  return p->d.wdtype == MSI_W_BF16 && !(f.flags & MSI_FWD_SPLIT_WAVES);
+}
+
+// A resident bf16 forward fuses its two projections while neither would take
+// pair tiles (groups averaging < 512 rows, e.g. 4,096 tokens over 512
+// experts): there the down projection's first tiles then overlap the
+// gate-up's last round.  Longer calls keep the pair-tile down projection.
+bool fused_resident(const msi_plan* p, const FwdCtx& f, long long rows, int ng) {
+  return p->d.wdtype == MSI_W_BF16 && !(f.flags & MSI_FWD_SPLIT_WAVES) && ng > 0 &&
+         !(!(f.flags & MSI_FWD_SINGLE_CTA) && rows >= 512LL * ng);
+}
+
 // Forward begin + router + histogram + permutation.
 msi_status front(msi_plan* p, FwdCtx& f, const TableParams& tp) {
   const auto& d = p->d;
@@ -792,6 +808,10 @@ msi_status front(msi_plan* p, FwdCtx& f, const TableParams& tp) {
     xa.tab_slot = at<int>(ws, L.table);
     xa.tab_expected = at<unsigned long long>(ws, L.expected);
     xa.layer = tp.layer;
+    if (fused_resident(p, f, (long long)f.T * k, E)) {
+      xa.ready = at<int>(ws, L.ready);
+      xa.n_ready = (int)((size_t)f.T * k / kBM + E + 1);
+    }
   }
   LAUNCH(p, MSI_K_SCATTER, f.cs, launch_scatter(xa, f.cs));
   const size_t Tk = (size_t)f.T * k;
@@ -857,13 +877,13 @@ bool pair_tiles(const FwdCtx& f, long long rows, int groups, long long min_rows 
 // 4-bit weights: a pair CTA dequantises half the B rows of a single-CTA tile
 // per unit of tensor work, which pays once the groups fill 256-row tiles.
 constexpr long long kPairMinRowsQ4 = 512;
+// A fused wave (gate-up and down in one launch) takes 256-row pair tiles
+// once its groups average >= 1,024 rows: at ~640 rows per group their row
+// padding (a 256-row tile per ~128-row remainder) outweighs the smaller
+// operand feed per SM (measured at 32K, waves of 32: 2.14 ms per step on
+// pairs against 2.10 ms on single-CTA tiles).
+constexpr long long kPairMinRowsFused = 1024;
 
-// A streamed bf16 wave whose gate-up takes single-CTA tiles runs its gate-up
-// and down in one launch (gemm_fused.cu): the wave is too small to fill the
-// SMs' last round of gate-up tiles, and the down tiles fill it.
-bool fused_wave(const msi_plan* p, const FwdCtx& f, long long rows, int ng) {
-  return p->d.wdtype == MSI_W_BF16 && !(f.flags & MSI_FWD_SPLIT_WAVES) && !pair_tiles(f, rows, ng);
-}
 
 msi_status routed_ffn(msi_plan* p, FwdCtx& f, int ng, int grid1, int grid2, long long rows,
                       int wave_mtiles = -1) {
@@ -932,6 +952,11 @@ msi_status routed_ffn(msi_plan* p, FwdCtx& f, int ng, int grid1, int grid2, long
     fa.wait_limit = p->wait_cycles;
     fa.stall = f.stall;
     const long long tiles = (long long)wave_mtiles * (fa.nt_up + fa.nt_dn);
+    if (pair_tiles(f, rows, ng, kPairMinRowsFused)) {
+      const int pairs = (int)std::min<long long>(p->sms / 2, std::max<long long>(1, tiles));
+      LAUNCH(p, MSI_K_FFN, f.cs, launch_fused_wave_pair(p->tm_w13, p->tm_w2, fa, pairs, f.cs));
+      return MSI_OK;
+    }
     const int grid = (int)std::min<long long>(p->sms, std::max<long long>(1, tiles));
     LAUNCH(p, MSI_K_FFN, f.cs, launch_fused_wave(p->tm_w13, p->tm_w2, fa, grid, f.cs));
     return MSI_OK;
@@ -1329,7 +1354,8 @@ msi_status forward_resident(msi_plan* p, int layer, const void* x, int T, const 
     const long long mt_max = ((long long)T * d.top_k + kBM - 1) / kBM + E;
     const int g1 = (int)std::min<long long>(p->sms, mt_max * (d.inter / 128));
     const int g2 = (int)std::min<long long>(p->sms, mt_max * (d.hidden / kBN));
-    st = routed_ffn(p, f, E, g1, g2, (long long)T * d.top_k);
+    st = routed_ffn(p, f, E, g1, g2, (long long)T * d.top_k,
+                    fused_resident(p, f, (long long)T * d.top_k, E) ? (int)mt_max : -1);
     if (st != MSI_OK) return st;
     st = consumer_record(p, used, f.cs);
     if (st != MSI_OK) return st;
