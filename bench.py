@@ -59,7 +59,10 @@ METRIC_DECODE = "MoE decode tokens/s through a 48-layer stack"
 PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
                   "sm_max_mhz": 2070.0}
 N_SMS = 152
-FP32_LANES_PER_SM = 128
+# FP32 FFMA throughput measured on this machine's GB300 at 2,070 MHz
+# (profiles/ffma_roof.md): the roof of the SIMT router
+FFMA_TFLOPS_MEASURED = 82.6
+FFMA_MHZ = 2070.0
 L2_BYTES = 129 * 1024 * 1024
 
 # dram__bytes_read.sum + dram__bytes_write.sum per launch from one ncu capture
@@ -357,7 +360,7 @@ def roofline(cfg, kt: dict, steps: int, peaks: dict, clocks: dict, workload: str
         flops, nbytes = algorithmic(cfg, kind, {})
         if kind == "router":
             mhz = clocks.get("sm_mhz") or peaks.get("sm_max_mhz", 2070.0)
-            peak = N_SMS * FP32_LANES_PER_SM * 2 * mhz * 1e6 / 1e12
+            peak = FFMA_TFLOPS_MEASURED * mhz / FFMA_MHZ
             per_launch_s = ms / 1e3 / max(launches, 1)
             ach = flops * steps / max(launches, 1) / per_launch_s / 1e12
             r = {"bound": "alu", "achieved": ach, "peak": peak, "unit": "TFLOP/s",
@@ -373,7 +376,7 @@ def roofline(cfg, kt: dict, steps: int, peaks: dict, clocks: dict, workload: str
     elif r["bound"] == "hbm":
         r["peak_source"] = "hbm_gbs of measured"
     else:
-        r["peak_source"] = "152 SMs x 128 FP32 lanes x 2 flop x median SM clock"
+        r["peak_source"] = "measured FP32 FFMA rate (profiles/ffma_roof.md) x median SM clock / 2070 MHz"
     t = TRAFFIC.get((workload, kind))
     r["traffic"] = t["bytes_per_launch"] if (t and t.get("src_hash") == kernel_source_hash()) else None
     if r["traffic"] is not None:

@@ -70,7 +70,7 @@ def test_router_roof_is_the_fp32_alu_rate():
     cfg = synth.config("qwen3next_4k")
     r = bench.roofline(cfg, {"router": (1.0, 10)}, 10, PEAKS, {"sm_mhz": 2000.0}, "x")
     assert r["bound"] == "alu"
-    assert r["peak"] == pytest.approx(152 * 128 * 2 * 2000e6 / 1e12)
+    assert r["peak"] == pytest.approx(82.6 * 2000.0 / 2070.0)
 
 
 def test_roofline_of_fused_wave_launches():
