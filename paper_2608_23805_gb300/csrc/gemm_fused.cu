@@ -48,8 +48,9 @@ constexpr int kFThreads = (kFGatherWarp0 + kFGatherWarps) * 32;
 constexpr int kFStages = kStages;
 constexpr int kFFullCount = 1 + kFGatherWarps * 32;  // producer (expect_tx) + each gather thread
 constexpr uint32_t kFIdesc = idesc_bf16(kBM, kBN);
+// + the group table: tile prefix, slot, first row, rows, scan scratch
 constexpr int kFSmem = 1024 + kFStages * (kABytes + kBBytes) + 256 + kFEpiWarps * 4096 +
-                       (2 * kMaxExperts + 2) * 4;
+                       (4 * kMaxExperts + 1 + 64) * 4;
 
 struct FTile {
   int up;  // 1: gate-up tile, 0: down tile
@@ -58,13 +59,13 @@ struct FTile {
 
 // Tile t -> (kind, group, 128-row tile, column tile) from the shared-memory
 // table of the groups' 128-row tile prefix (s_mt[num_groups] = m-tiles).
-__device__ __forceinline__ FTile fdecode(const FusedArgs& a, const int* s_mt, int t) {
-  const int n_up = s_mt[a.num_groups] * a.nt_up;
+__device__ __forceinline__ FTile fdecode(const FusedArgs& a, int ng, const int* s_mt, int t) {
+  const int n_up = s_mt[ng] * a.nt_up;
   FTile c;
   c.up = t < n_up;
   const int nt = c.up ? a.nt_up : a.nt_dn;
   const int tt = c.up ? t : t - n_up;
-  int lo = 0, hi = a.num_groups - 1;
+  int lo = 0, hi = ng - 1;
   while (lo < hi) {
     const int mid = (lo + hi + 1) >> 1;
     if (s_mt[mid] * nt <= tt) lo = mid; else hi = mid - 1;
@@ -94,7 +95,8 @@ __device__ __forceinline__ void epilogue_bar() { asm volatile("bar.sync 1, 128;"
 
 __global__ void __launch_bounds__(kFThreads, 1)
     fused_wave_kernel(const __grid_constant__ CUtensorMap tmW13,
-                      const __grid_constant__ CUtensorMap tmW2, const FusedArgs a) {
+                      const __grid_constant__ CUtensorMap tmW2, const FusedArgs a,
+                      const __grid_constant__ WaveParams w) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -109,8 +111,11 @@ __global__ void __launch_bounds__(kFThreads, 1)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(never + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   uint8_t* epi_stage = reinterpret_cast<uint8_t*>(full) + 256;  // 4 KB per epilogue warp
-  int* s_mt = reinterpret_cast<int*>(epi_stage + kFEpiWarps * 4096);  // [num_groups + 1]
-  int* s_slot = s_mt + kMaxExperts + 1;                                // [num_groups]
+  int* s_mt = reinterpret_cast<int*>(epi_stage + kFEpiWarps * 4096);  // [groups + 1] tile prefix
+  int* s_slot = s_mt + kMaxExperts + 1;                                // [groups]
+  int* s_rb = s_slot + kMaxExperts;                                    // [groups] first row
+  int* s_cnt = s_rb + kMaxExperts;                                     // [groups] rows
+  int* s_tmp = s_cnt + kMaxExperts;                                    // [64]
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -137,16 +142,15 @@ __global__ void __launch_bounds__(kFThreads, 1)
     tma_prefetch(&tmW13);
     tma_prefetch(&tmW2);
   }
-  for (int g = threadIdx.x; g < a.num_groups; g += blockDim.x) {
-    s_mt[g] = __ldg(&a.groups[g].mt_begin);
-    s_slot[g] = __ldg(&a.groups[g].slot);
-  }
-  if (threadIdx.x == 0) s_mt[a.num_groups] = __ldg(a.total_mtiles);
+  // the previous wave's counters, zeroed for the next wave
+  for (int r = blockIdx.x * blockDim.x + threadIdx.x; r < a.n_ready_clear; r += gridDim.x * blockDim.x)
+    a.ready_clear[r] = 0;
+  const int ng = fused_group_table(a, w, kBM, blockIdx.x == 0, s_mt, s_slot, s_rb, s_cnt, s_tmp);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  const int total = s_mt[a.num_groups] * (a.nt_up + a.nt_dn);
+  const int total = s_mt[ng] * (a.nt_up + a.nt_dn);
   const long long lim = a.wait_limit;
 
   if (warp == 5) {
@@ -154,7 +158,7 @@ __global__ void __launch_bounds__(kFThreads, 1)
     if (lane == 0) {
       uint32_t it = 0;
       for (int t = blockIdx.x; t < total; t += gridDim.x) {
-        const FTile tc = fdecode(a, s_mt, t);
+        const FTile tc = fdecode(a, ng, s_mt, t);
         const int kb_n = tc.up ? a.kb_up : a.kb_dn;
         const int r0 = tc.up ? s_slot[tc.g] * a.w13_rows_per_slot + tc.n * 128
                              : s_slot[tc.g] * a.w2_rows_per_slot + a.w2_row_off + tc.n * kBN;
@@ -189,7 +193,7 @@ __global__ void __launch_bounds__(kFThreads, 1)
     if (lane == 0) {
       uint32_t it = 0, jt = 0;
       for (int t = blockIdx.x; t < total; t += gridDim.x, ++jt) {
-        const FTile tc = fdecode(a, s_mt, t);
+        const FTile tc = fdecode(a, ng, s_mt, t);
         const int kb_n = tc.up ? a.kb_up : a.kb_dn;
         const uint32_t acc = jt & 1, aph = (jt >> 1) & 1;
         if (!mbar_wait(&tempty[acc], aph ^ 1, abort_flag, lim)) break;
@@ -224,10 +228,9 @@ __global__ void __launch_bounds__(kFThreads, 1)
     uint32_t jt = 0;
     if (a.stall && threadIdx.x == 0) mbar_wait(never, 0, abort_flag, lim);  // runs out: abort
     for (int t = blockIdx.x; t < total; t += gridDim.x, ++jt) {
-      const FTile tc = fdecode(a, s_mt, t);
-      const Group* G = &a.groups[tc.g];
-      const int cnt = __ldg(&G->row_count);
-      const size_t rb = (size_t)__ldg(&G->row_begin);
+      const FTile tc = fdecode(a, ng, s_mt, t);
+      const int cnt = s_cnt[tc.g];
+      const size_t rb = (size_t)s_rb[tc.g];
       const uint32_t acc = jt & 1, aph = (jt >> 1) & 1;
       if (!mbar_wait(&tfull[acc], aph, abort_flag, lim)) break;
       tc_fence_after();
@@ -260,10 +263,9 @@ __global__ void __launch_bounds__(kFThreads, 1)
     // gate-up tile, h rows for a down tile; -1 past the group's segment),
     // loaded one tile ahead
     auto tile_rows = [&](int t, int (&pr)[8]) {
-      const FTile tc = fdecode(a, s_mt, t);
-      const Group* G = &a.groups[tc.g];
-      const int cnt = __ldg(&G->row_count);
-      const int rb = __ldg(&G->row_begin);
+      const FTile tc = fdecode(a, ng, s_mt, t);
+      const int cnt = s_cnt[tc.g];
+      const int rb = s_rb[tc.g];
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
         const int rr = tc.m * kBM + r0 + 16 * i;
@@ -275,7 +277,7 @@ __global__ void __launch_bounds__(kFThreads, 1)
     for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
       const bool has_next = t + (int)gridDim.x < total;
       if (has_next) tile_rows(t + gridDim.x, pr_next);
-      const FTile tc = fdecode(a, s_mt, t);
+      const FTile tc = fdecode(a, ng, s_mt, t);
       const int kb_n = tc.up ? a.kb_up : a.kb_dn;
       if (!tc.up) {
         // every gate-up tile of this m-tile has published its h columns
@@ -341,7 +343,7 @@ __global__ void __launch_bounds__(kFThreads, 1)
 }
 
 cudaError_t launch_fused_wave(const CUtensorMap& tmW13, const CUtensorMap& tmW2, const FusedArgs& a,
-                              int grid, cudaStream_t s) {
+                              const WaveParams& w, int grid, cudaStream_t s) {
   static std::atomic<unsigned long long> attr_done{0};
   cudaError_t e = smem_attr_once(fused_wave_kernel, kFSmem, attr_done);
   if (e != cudaSuccess) return e;
@@ -358,7 +360,7 @@ cudaError_t launch_fused_wave(const CUtensorMap& tmW13, const CUtensorMap& tmW2,
   cfg.stream = s;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, fused_wave_kernel, tmW13, tmW2, a);
+  return cudaLaunchKernelEx(&cfg, fused_wave_kernel, tmW13, tmW2, a, w);
 }
 
 }  // namespace msi

@@ -53,7 +53,8 @@ constexpr int kQGatherWarps = 4;
 constexpr int kQGatherWarp0 = 6;
 constexpr int kQThreads = (kQGatherWarp0 + kQGatherWarps) * 32;
 constexpr int kQFullLocal = 1 + kQGatherWarps * 32;  // own producer (expect_tx) + own gather threads
-constexpr int kQSmem = 1024 + kQStages * (kQA + kQB) + 256 + kQEpiWarps * 4096 + (2 * kMaxExperts + 2) * 4;
+// + the group table: tile prefix, slot, first row, rows, scan scratch
+constexpr int kQSmem = 1024 + kQStages * (kQA + kQB) + 256 + kQEpiWarps * 4096 + (4 * kMaxExperts + 1 + 64) * 4;
 
 struct QTile {
   int up;  // 1: gate-up tile, 0: down tile
@@ -62,13 +63,13 @@ struct QTile {
 
 // Pair tile t -> (kind, group, 256-row tile, column tile) from the
 // shared-memory table of the groups' 256-row tile prefix.
-__device__ __forceinline__ QTile qdecode(const FusedArgs& a, const int* s_pt, int t) {
-  const int n_up = s_pt[a.num_groups] * a.nt_up;
+__device__ __forceinline__ QTile qdecode(const FusedArgs& a, int ng, const int* s_pt, int t) {
+  const int n_up = s_pt[ng] * a.nt_up;
   QTile c;
   c.up = t < n_up;
   const int nt = c.up ? a.nt_up : a.nt_dn;
   const int tt = c.up ? t : t - n_up;
-  int lo = 0, hi = a.num_groups - 1;
+  int lo = 0, hi = ng - 1;
   while (lo < hi) {
     const int mid = (lo + hi + 1) >> 1;
     if (s_pt[mid] * nt <= tt) lo = mid; else hi = mid - 1;
@@ -97,7 +98,8 @@ __device__ __forceinline__ void epilogue_bar() { asm volatile("bar.sync 1, 128;"
 
 __global__ void __launch_bounds__(kQThreads, 1)
     fused_wave_pair_kernel(const __grid_constant__ CUtensorMap tmW13,
-                           const __grid_constant__ CUtensorMap tmW2, const FusedArgs a) {
+                           const __grid_constant__ CUtensorMap tmW2, const FusedArgs a,
+                           const __grid_constant__ WaveParams w) {
   extern __shared__ uint8_t smem_raw[];
   // the same offsets in both CTAs: the pair MMA addresses the peer's operands
   // through the even CTA's descriptors
@@ -114,8 +116,11 @@ __global__ void __launch_bounds__(kQThreads, 1)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(never + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   uint8_t* epi_stage = reinterpret_cast<uint8_t*>(full) + 256;  // 4 KB per epilogue warp
-  int* s_pt = reinterpret_cast<int*>(epi_stage + kQEpiWarps * 4096);  // [num_groups + 1]
-  int* s_slot = s_pt + kMaxExperts + 1;                               // [num_groups]
+  int* s_pt = reinterpret_cast<int*>(epi_stage + kQEpiWarps * 4096);  // [groups + 1] tile prefix
+  int* s_slot = s_pt + kMaxExperts + 1;                               // [groups]
+  int* s_rb = s_slot + kMaxExperts;                                   // [groups] first row
+  int* s_cnt = s_rb + kMaxExperts;                                    // [groups] rows
+  int* s_tmp = s_cnt + kMaxExperts;                                   // [64]
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -144,16 +149,15 @@ __global__ void __launch_bounds__(kQThreads, 1)
     tma_prefetch(&tmW13);
     tma_prefetch(&tmW2);
   }
-  for (int g = threadIdx.x; g < a.num_groups; g += blockDim.x) {
-    s_pt[g] = __ldg(&a.groups[g].pt_begin);
-    s_slot[g] = __ldg(&a.groups[g].slot);
-  }
-  if (threadIdx.x == 0) s_pt[a.num_groups] = __ldg(a.total_mtiles + 1);
+  // the previous wave's counters, zeroed for the next wave
+  for (int r = blockIdx.x * blockDim.x + threadIdx.x; r < a.n_ready_clear; r += gridDim.x * blockDim.x)
+    a.ready_clear[r] = 0;
+  const int ng = fused_group_table(a, w, kQRows, blockIdx.x == 0, s_pt, s_slot, s_rb, s_cnt, s_tmp);
   tc_fence_before();
   cluster_sync_all();  // both CTAs' barriers initialised before any cross-CTA arrival
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  const int total = s_pt[a.num_groups] * (a.nt_up + a.nt_dn);
+  const int total = s_pt[ng] * (a.nt_up + a.nt_dn);
   const int pair = blockIdx.x >> 1;
   const int npairs = gridDim.x >> 1;
   const long long lim = a.wait_limit;
@@ -163,7 +167,7 @@ __global__ void __launch_bounds__(kQThreads, 1)
     if (lane == 0) {
       uint32_t it = 0;
       for (int t = pair; t < total; t += npairs) {
-        const QTile tc = qdecode(a, s_pt, t);
+        const QTile tc = qdecode(a, ng, s_pt, t);
         const int kb_n = tc.up ? a.kb_up : a.kb_dn;
         // gate-up: the even CTA holds 128 gate rows, the odd CTA the matching
         // up rows; down: CTA r holds W2 rows 256 n + 128 r .. + 128
@@ -197,7 +201,7 @@ __global__ void __launch_bounds__(kQThreads, 1)
       // ----------------------------------------------------------- MMA issuer
       uint32_t it = 0, jt = 0;
       for (int t = pair; t < total; t += npairs, ++jt) {
-        const QTile tc = qdecode(a, s_pt, t);
+        const QTile tc = qdecode(a, ng, s_pt, t);
         const int kb_n = tc.up ? a.kb_up : a.kb_dn;
         const uint32_t acc = jt & 1, aph = (jt >> 1) & 1;
         if (!mbar_wait(&tempty[acc], aph ^ 1, abort_flag, lim)) break;
@@ -227,7 +231,7 @@ __global__ void __launch_bounds__(kQThreads, 1)
       uint32_t it = 0;
       bool ok = true;
       for (int t = pair; t < total && ok; t += npairs) {
-        const QTile tc = qdecode(a, s_pt, t);
+        const QTile tc = qdecode(a, ng, s_pt, t);
         const int kb_n = tc.up ? a.kb_up : a.kb_dn;
         for (int kb = 0; kb < kb_n; ++kb, ++it) {
           const int s = it % kQStages;
@@ -252,10 +256,9 @@ __global__ void __launch_bounds__(kQThreads, 1)
                                      mapa_shared(smem_u32(&tempty[1]), 0)};
     if (a.stall && threadIdx.x == 0) mbar_wait(never, 0, abort_flag, lim);  // runs out: abort
     for (int t = pair; t < total; t += npairs, ++jt) {
-      const QTile tc = qdecode(a, s_pt, t);
-      const Group* G = &a.groups[tc.g];
-      const int cnt = __ldg(&G->row_count);
-      const size_t rb = (size_t)__ldg(&G->row_begin);
+      const QTile tc = qdecode(a, ng, s_pt, t);
+      const int cnt = s_cnt[tc.g];
+      const size_t rb = (size_t)s_rb[tc.g];
       const uint32_t acc = jt & 1, aph = (jt >> 1) & 1;
       if (!mbar_wait(&tfull[acc], aph, abort_flag, lim)) break;
       tc_fence_after();
@@ -285,10 +288,9 @@ __global__ void __launch_bounds__(kQThreads, 1)
     uint32_t it = 0;
     bool ok = true;
     auto tile_rows = [&](int t, int (&pr)[8]) {
-      const QTile tc = qdecode(a, s_pt, t);
-      const Group* G = &a.groups[tc.g];
-      const int cnt = __ldg(&G->row_count);
-      const int rb = __ldg(&G->row_begin);
+      const QTile tc = qdecode(a, ng, s_pt, t);
+      const int cnt = s_cnt[tc.g];
+      const int rb = s_rb[tc.g];
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
         const int rr = tc.m2 * kQRows + (int)rank * kBM + r0 + 16 * i;
@@ -300,7 +302,7 @@ __global__ void __launch_bounds__(kQThreads, 1)
     for (int t = pair; t < total && ok; t += npairs) {
       const bool has_next = t + npairs < total;
       if (has_next) tile_rows(t + npairs, pr_next);
-      const QTile tc = qdecode(a, s_pt, t);
+      const QTile tc = qdecode(a, ng, s_pt, t);
       const int kb_n = tc.up ? a.kb_up : a.kb_dn;
       if (!tc.up) {
         // both CTAs of every gate-up tile of this 256-row tile have published
@@ -367,7 +369,7 @@ __global__ void __launch_bounds__(kQThreads, 1)
 }
 
 cudaError_t launch_fused_wave_pair(const CUtensorMap& tmW13, const CUtensorMap& tmW2,
-                                   const FusedArgs& a, int max_pairs, cudaStream_t s) {
+                                   const FusedArgs& a, const WaveParams& w, int max_pairs, cudaStream_t s) {
   static std::atomic<unsigned long long> attr_done{0};
   static std::atomic<int> max_clusters[64] = {};
   cudaError_t e = smem_attr_once(fused_wave_pair_kernel, kQSmem, attr_done);
@@ -399,7 +401,7 @@ cudaError_t launch_fused_wave_pair(const CUtensorMap& tmW13, const CUtensorMap& 
   }
   const int pairs = std::max(1, std::min(mc, max_pairs));
   cfg.gridDim = dim3(2 * pairs, 1, 1);
-  return cudaLaunchKernelEx(&cfg, fused_wave_pair_kernel, tmW13, tmW2, a);
+  return cudaLaunchKernelEx(&cfg, fused_wave_pair_kernel, tmW13, tmW2, a, w);
 }
 
 }  // namespace msi

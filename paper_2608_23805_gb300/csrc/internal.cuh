@@ -105,6 +105,16 @@ struct GemmArgs {
 
 enum GemmMode { kGateUpGather = 0, kGateUpTma = 1, kDown = 2, kGateUpGatherQ4 = 3, kDownQ4 = 4 };
 
+// One LRU wave's experts: slot, expert id and the generation each must hold
+// (kernel parameter, by value).
+struct WaveParams {
+  int n;
+  int layer;
+  int slot[kMaxWave];
+  int expert[kMaxWave];
+  unsigned long long expected[kMaxWave];
+};
+
 // One wave's gate-up and down projections in one launch (gemm_fused.cu).
 struct FusedArgs {
   const Group* groups;
@@ -124,10 +134,20 @@ struct FusedArgs {
   int x_ld;
   const int* perm;          // permuted row -> t k + j
   int top_k;
-  int* ready;               // [m-tiles] finished gate-up tiles per 128-row tile (zeroed per wave)
+  int* ready;               // [m-tiles] finished gate-up tiles per 128-row tile (zero at launch)
   int* status;
   long long wait_limit;
   int stall;                // as GemmArgs::stall
+  // wave mode (wave != 0): the kernel builds the wave's groups itself from the
+  // call's counts and offsets and the WaveParams (the generation re-check of
+  // every slot, fail closed), and zeroes ready_clear[0, n_ready_clear) for the
+  // next wave (the counters of the previous one); groups / total_mtiles unused
+  int wave;
+  const int* counts;        // [E] rows per expert
+  const int* offsets;       // [E + 1] first permuted row per expert
+  const GenWord* genwords;  // published (generation, object) per slot
+  int* ready_clear;
+  int n_ready_clear;
 };
 
 // ---------------------------------------------------------------------------
@@ -142,11 +162,11 @@ cudaError_t launch_gemm_pair(int mode, const CUtensorMap& tmA, const CUtensorMap
 // Gate-up and down of one wave in one cooperative launch of `grid` CTAs
 // (at most one per SM); tmW13 / tmW2 as the pool maps of the two projections.
 cudaError_t launch_fused_wave(const CUtensorMap& tmW13, const CUtensorMap& tmW2, const FusedArgs& a,
-                              int grid, cudaStream_t s);
+                              const WaveParams& w, int grid, cudaStream_t s);
 // The same on CTA pairs (256-row tiles, gemm_fused_pair.cu); at most
 // `max_pairs` pairs, never more than can be resident at once.
 cudaError_t launch_fused_wave_pair(const CUtensorMap& tmW13, const CUtensorMap& tmW2,
-                                   const FusedArgs& a, int max_pairs, cudaStream_t s);
+                                   const FusedArgs& a, const WaveParams& w, int max_pairs, cudaStream_t s);
 
 // GEMM tiling
 constexpr int kBM = 128;
@@ -595,6 +615,80 @@ __device__ __forceinline__ uint4 dequant8(uint32_t w, uint64_t scale2, uint64_t 
     asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(o[b]) : "r"(vh), "r"(vl));
   }
   return make_uint4(o[0], o[1], o[2], o[3]);
+}
+
+// Shared-memory group table of a fused launch, read by every role: tile
+// prefix s_mt[0..ng] (s_mt[ng] = tiles), slot, first permuted row and rows
+// per group.  Wave mode builds it from the wave (the generation re-check of
+// each slot: a group whose slot does not hold the expected object and
+// version gets no tiles, and CTA 0 records the lowest such expert's status,
+// fail closed); otherwise it is read from the groups in global memory.
+// tile_rows: 128 (single-CTA tiles) or 256 (pair tiles).  Every thread of the
+// CTA calls it (blockDim >= kMaxWave); returns the number of groups.
+__device__ __forceinline__ int fused_group_table(const FusedArgs& a, const WaveParams& w, int tile_rows,
+                                                 bool record, int* s_mt, int* s_slot, int* s_rb,
+                                                 int* s_cnt, int* s_tmp) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  if (!a.wave) {
+    for (int g = tid; g < a.num_groups; g += blockDim.x) {
+      const Group G = a.groups[g];
+      s_mt[g] = tile_rows == kBM ? G.mt_begin : G.pt_begin;
+      s_slot[g] = G.slot;
+      s_rb[g] = G.row_begin;
+      s_cnt[g] = G.row_count;
+    }
+    if (tid == 0) s_mt[a.num_groups] = __ldg(a.total_mtiles + (tile_rows == kBM ? 0 : 1));
+    return a.num_groups;
+  }
+  const int n = w.n;
+  int e = 0, cnt = 0, slot = 0, code = 0;
+  if (tid < n) {
+    e = w.expert[tid];
+    cnt = __ldg(&a.counts[e]);
+    slot = w.slot[tid];
+    if (cnt > 0) {
+      if (slot < 0) {
+        code = MSI_ERR_NOT_RESIDENT;
+      } else {
+        const unsigned long long obj = a.genwords[slot].obj;
+        const unsigned long long gen = a.genwords[slot].gen;
+        if (obj != obj_key(w.layer, e)) code = MSI_ERR_WRONG_OBJECT;
+        else if (gen != w.expected[tid]) code = MSI_ERR_STALE_GENERATION;
+      }
+    }
+  }
+  const int mt = (tid < n && code == 0) ? (cnt + tile_rows - 1) / tile_rows : 0;
+  // exclusive scan of mt over the block; lowest failing expert
+  int incl = mt;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const int o = __shfl_up_sync(0xffffffffu, incl, off);
+    if (lane >= off) incl += o;
+  }
+  int key = code ? (e << 4) | code : 0x7fffffff;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) key = min(key, __shfl_xor_sync(0xffffffffu, key, off));
+  if (lane == 31) s_tmp[warp] = incl;
+  if (lane == 0) s_tmp[32 + warp] = key;
+  __syncthreads();
+  const int nw = blockDim.x >> 5;
+  int base = 0, total = 0, kmin = 0x7fffffff;
+  for (int q = 0; q < nw; ++q) {
+    if (q < warp) base += s_tmp[q];
+    total += s_tmp[q];
+    kmin = min(kmin, s_tmp[32 + q]);
+  }
+  if (tid < n) {
+    s_mt[tid] = base + incl - mt;
+    s_slot[tid] = slot < 0 ? 0 : slot;
+    s_rb[tid] = __ldg(&a.offsets[e]);
+    s_cnt[tid] = code == 0 ? cnt : 0;
+  }
+  if (tid == 0) {
+    s_mt[n] = total;
+    if (record && kmin != 0x7fffffff) atomicCAS(a.status, 0, kmin & 15);
+  }
+  return n;
 }
 
 #endif  // __CUDACC__

@@ -101,14 +101,6 @@ struct TableParams {
   unsigned long long expected[kMaxExperts];
 };
 
-struct WaveParams {
-  int n;
-  int layer;
-  int slot[kMaxWave];
-  int expert[kMaxWave];
-  unsigned long long expected[kMaxWave];
-};
-
 struct PublishParams {
   int n;
   int slot[kMaxWave];

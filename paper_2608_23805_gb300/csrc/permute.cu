@@ -86,9 +86,9 @@ __device__ void scatter_setup(const ScatterArgs& a, const int* offs,
   __shared__ int wsum[kScatterWarps];
   __shared__ int kmin[kScatterWarps];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  if (a.tab_slot == nullptr) return;  // streamed call: the groups are built per wave
-  if (a.ready != nullptr)
+  if (a.ready != nullptr)  // fused GEMMs: counters of the call's first launch
     for (int r = tid; r < a.n_ready; r += blockDim.x) a.ready[r] = 0;
+  if (a.tab_slot == nullptr) return;  // streamed call: the groups are built per wave
   int cnt[4], code[4], mt[4], pt[4];
   int key = 0x7fffffff;
   int slot[4];

@@ -173,7 +173,7 @@ struct WaveEntry {
 
 struct WsLayout {
   size_t status, table, expected, groups, total, sh_group, sh_total, w3, cand_v, cand_i, bcount,
-      bbase, offsets, perm, inv, sg, h, yp, hs, ys, ready, bytes;
+      bbase, offsets, perm, inv, sg, h, yp, hs, ys, ready, ready_n, bytes;
   int tm;  // tokens per router block
 };
 
@@ -344,7 +344,10 @@ WsLayout layout(const msi_plan* p, int T) {
   L.sg = take(4 * (size_t)T);
   L.h = take(2 * Tk * I);
   L.yp = take(2 * Tk * H);
-  L.ready = take(4 * (Tk / kBM + E + 1));  // fused waves: a counter per 128-row tile
+  // fused GEMMs: a counter per 128-row tile, two banks (consecutive waves
+  // alternate; each wave's kernel zeroes the other bank for the next)
+  L.ready_n = Tk / kBM + E + 1;
+  L.ready = take(2 * 4 * L.ready_n);
   if (p->d.has_shared) {
     L.hs = take(2 * (size_t)T * I);
     L.ys = take(2 * (size_t)T * H);
@@ -753,6 +756,9 @@ bool fused_resident(const msi_plan* p, const FwdCtx& f, long long rows, int ng) 
          !(!(f.flags & MSI_FWD_SINGLE_CTA) && rows >= 512LL * ng);
 }
 
+// Counters in one bank of the fused GEMMs' per-m-tile counters.
+int ready_bank(const FwdCtx& f) { return (int)(f.L.ready_n); }
+
 // Forward begin + router + histogram + permutation.
 msi_status front(msi_plan* p, FwdCtx& f, const TableParams& tp) {
   const auto& d = p->d;
@@ -810,8 +816,13 @@ msi_status front(msi_plan* p, FwdCtx& f, const TableParams& tp) {
     xa.layer = tp.layer;
     if (fused_resident(p, f, (long long)f.T * k, E)) {
       xa.ready = at<int>(ws, L.ready);
-      xa.n_ready = (int)((size_t)f.T * k / kBM + E + 1);
+      xa.n_ready = ready_bank(f);
     }
+  } else if (fused_wave(p, f, 0, 0)) {
+    // streamed call: the first wave's bank (later waves' banks are zeroed by
+    // the wave before them)
+    xa.ready = at<int>(ws, L.ready);
+    xa.n_ready = ready_bank(f);
   }
   LAUNCH(p, MSI_K_SCATTER, f.cs, launch_scatter(xa, f.cs));
   const size_t Tk = (size_t)f.T * k;
@@ -885,8 +896,10 @@ constexpr long long kPairMinRowsQ4 = 512;
 constexpr long long kPairMinRowsFused = 1024;
 
 
+// wave_mtiles >= 0: the expert FFN of one wave (wp, index wave) or of a
+// resident call (wp null) may run fused; -1: split launches.
 msi_status routed_ffn(msi_plan* p, FwdCtx& f, int ng, int grid1, int grid2, long long rows,
-                      int wave_mtiles = -1) {
+                      int wave_mtiles = -1, const WaveParams* wp = nullptr, int wave = 0) {
   const bool bf16 = p->d.wdtype == MSI_W_BF16;
   const bool pair_up = bf16 ? pair_tiles(f, rows, ng) : pair_tiles(f, rows, ng, kPairMinRowsQ4);
   const bool pair_down = pair_tiles(f, rows, ng, bf16 ? kPairMinRowsDown : kPairMinRowsQ4);
@@ -947,18 +960,32 @@ msi_status routed_ffn(msi_plan* p, FwdCtx& f, int ng, int grid1, int grid2, long
     fa.x_ld = d.hidden;
     fa.perm = at<int>(f.ws, f.L.perm);
     fa.top_k = d.top_k;
-    fa.ready = at<int>(f.ws, f.L.ready);
+    int* bank0 = at<int>(f.ws, f.L.ready);
+    int* bank1 = bank0 + f.L.ready_n;
+    fa.ready = (wave & 1) ? bank1 : bank0;
     fa.status = at<int>(f.ws, f.L.status);
     fa.wait_limit = p->wait_cycles;
     fa.stall = f.stall;
+    static const WaveParams no_wave{};
+    if (wp != nullptr) {
+      // the kernel re-checks the wave's slots and builds its groups itself,
+      // and zeroes the other bank for the next wave
+      fa.wave = 1;
+      fa.counts = f.ev->counts;
+      fa.offsets = at<int>(f.ws, f.L.offsets);
+      fa.genwords = p->d_gen;
+      fa.ready_clear = (wave & 1) ? bank0 : bank1;
+      fa.n_ready_clear = (int)f.L.ready_n;
+    }
+    const WaveParams& wv = wp != nullptr ? *wp : no_wave;
     const long long tiles = (long long)wave_mtiles * (fa.nt_up + fa.nt_dn);
     if (pair_tiles(f, rows, ng, kPairMinRowsFused)) {
       const int pairs = (int)std::min<long long>(p->sms / 2, std::max<long long>(1, tiles));
-      LAUNCH(p, MSI_K_FFN, f.cs, launch_fused_wave_pair(p->tm_w13, p->tm_w2, fa, pairs, f.cs));
+      LAUNCH(p, MSI_K_FFN, f.cs, launch_fused_wave_pair(p->tm_w13, p->tm_w2, fa, wv, pairs, f.cs));
       return MSI_OK;
     }
     const int grid = (int)std::min<long long>(p->sms, std::max<long long>(1, tiles));
-    LAUNCH(p, MSI_K_FFN, f.cs, launch_fused_wave(p->tm_w13, p->tm_w2, fa, grid, f.cs));
+    LAUNCH(p, MSI_K_FFN, f.cs, launch_fused_wave(p->tm_w13, p->tm_w2, fa, wv, grid, f.cs));
     return MSI_OK;
   }
   if (pair_up)
@@ -1653,23 +1680,24 @@ msi_status forward_streamed(msi_plan* p, int layer, const void* x, int T, const 
     }
     st = wait_ready(p, used, f.cs);
     if (st != MSI_OK) return st;
-    SetupArgs sa{};
-    sa.counts = ev->counts;
-    sa.offsets = at<int>(ws, f.L.offsets);
-    sa.genwords = p->d_gen;
-    sa.E = E;
-    sa.layer = layer;
-    sa.groups = at<Group>(ws, f.L.groups);
-    sa.total_mtiles = at<int>(ws, f.L.total);
-    sa.status = at<int>(ws, f.L.status);
-    if (fused_wave(p, f, wave_rows, wp.n)) {
-      sa.ready = at<int>(ws, f.L.ready);
-      sa.n_ready = mtiles;
+    const bool fused = fused_wave(p, f, wave_rows, wp.n);
+    if (!fused) {
+      // split launches: the setup kernel re-checks the wave's slots and
+      // builds its groups (a fused wave's kernel does both itself)
+      SetupArgs sa{};
+      sa.counts = ev->counts;
+      sa.offsets = at<int>(ws, f.L.offsets);
+      sa.genwords = p->d_gen;
+      sa.E = E;
+      sa.layer = layer;
+      sa.groups = at<Group>(ws, f.L.groups);
+      sa.total_mtiles = at<int>(ws, f.L.total);
+      sa.status = at<int>(ws, f.L.status);
+      LAUNCH(p, MSI_K_SETUP, f.cs, launch_setup_wave(sa, wp, f.cs));
     }
-    LAUNCH(p, MSI_K_SETUP, f.cs, launch_setup_wave(sa, wp, f.cs));
     const int g1 = std::max(1, std::min(p->sms, mtiles * (d.inter / 128)));
     const int g2 = std::max(1, std::min(p->sms, mtiles * (d.hidden / kBN)));
-    st = routed_ffn(p, f, wp.n, g1, g2, wave_rows, mtiles);
+    st = routed_ffn(p, f, wp.n, g1, g2, wave_rows, fused ? mtiles : -1, fused ? &wp : nullptr, (int)w);
     if (st != MSI_OK) return st;
     st = consumer_record(p, used, f.cs);
     if (st != MSI_OK) return st;
