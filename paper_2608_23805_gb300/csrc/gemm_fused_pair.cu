@@ -35,7 +35,17 @@
 // relay (odd CTA) and TMEM allocation, warp 5 TMA producer (B), warps 6-9 the
 // CTA's 128 A rows by cp.async (x rows through the permutation for gate-up
 // tiles, h rows for down tiles).
+//
+// 4-bit weights (Q4): the producer loads each stage's packed codes of the
+// CTA's 128 B rows (one 128 x 32-byte box of the code maps over the slot
+// pool) into a three-stage ring, and sixteen dequant warps convert them into
+// the bf16 B stage as in gemm_pair.cu (a quarter row per thread: 16 codes
+// under one fp16 scale, w = s * (q - 8) exact in fp32, rounded once to bf16),
+// with the W13 or W2 scales of the tile's rows.  The epilogue reads TMEM 16
+// columns at a time so that the 832 threads fit the register file.
 #include <algorithm>
+
+#include <cuda_fp16.h>
 
 #include "internal.cuh"
 
@@ -51,10 +61,22 @@ constexpr uint32_t kQIdesc = idesc_bf16(kQRows, kBN);
 constexpr int kQEpiWarps = 4;
 constexpr int kQGatherWarps = 4;
 constexpr int kQGatherWarp0 = 6;
-constexpr int kQThreads = (kQGatherWarp0 + kQGatherWarps) * 32;
-constexpr int kQFullLocal = 1 + kQGatherWarps * 32;  // own producer (expect_tx) + own gather threads
-// + the group table: tile prefix, slot, first row, rows, scan scratch
-constexpr int kQSmem = 1024 + kQStages * (kQA + kQB) + 256 + kQEpiWarps * 4096 + (4 * kMaxExperts + 1 + 64) * 4;
+constexpr int kQRawRow = 32;          // 64 codes of one B row per stage (one TMA box row)
+constexpr int kQRaw = 3;              // 4-bit: code stages in flight
+constexpr int kQDq = 16;              // 4-bit: dequant warps
+
+template <bool Q4>
+struct QCfg {
+  static constexpr int kThreads = (kQGatherWarp0 + kQGatherWarps + (Q4 ? kQDq : 0)) * 32;
+  // own gather threads + (bf16) the producer's expect_tx or (4-bit) each dequant warp
+  static constexpr int kFullLocal = kQGatherWarps * 32 + (Q4 ? kQDq : 1);
+  static constexpr int kRawBytes = Q4 ? kQRaw * 128 * kQRawRow : 0;
+  // group table: tile prefix, slot, first row, rows, scan scratch (4-bit
+  // launches are waves only, at most kMaxWave groups)
+  static constexpr int kGroups = Q4 ? kMaxWave : kMaxExperts;
+  static constexpr int kSmem = 1024 + kQStages * (kQA + kQB) + kRawBytes + 256 + kQEpiWarps * 4096 +
+                               (4 * kGroups + 1 + 64) * 4;
+};
 
 struct QTile {
   int up;  // 1: gate-up tile, 0: down tile
@@ -96,10 +118,12 @@ __device__ __forceinline__ void epilogue_bar() { asm volatile("bar.sync 1, 128;"
 
 }  // namespace
 
-__global__ void __launch_bounds__(kQThreads, 1)
+template <bool Q4>
+__global__ void __launch_bounds__(QCfg<Q4>::kThreads, 1)
     fused_wave_pair_kernel(const __grid_constant__ CUtensorMap tmW13,
                            const __grid_constant__ CUtensorMap tmW2, const FusedArgs a,
                            const __grid_constant__ WaveParams w) {
+  using C = QCfg<Q4>;
   extern __shared__ uint8_t smem_raw[];
   // the same offsets in both CTAs: the pair MMA addresses the peer's operands
   // through the even CTA's descriptors
@@ -107,20 +131,23 @@ __global__ void __launch_bounds__(kQThreads, 1)
                                              ~static_cast<uintptr_t>(1023));
   uint8_t* sA = smem;
   uint8_t* sB = smem + kQStages * kQA;
-  uint64_t* full = reinterpret_cast<uint64_t*>(sB + kQStages * kQB);
+  uint8_t* raw_codes = sB + kQStages * kQB;  // 4-bit: [kQRaw][128][32]
+  uint64_t* full = reinterpret_cast<uint64_t*>(raw_codes + C::kRawBytes);
   uint64_t* empty = full + kQStages;
   uint64_t* tfull = empty + kQStages;
   uint64_t* tempty = tfull + 2;
   uint64_t* drain = tempty + 2;
   uint64_t* never = drain + 1;  // no thread ever arrives here
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(never + 1);
+  uint64_t* raw_full = never + 1;            // 4-bit: code stage landed (TMA bytes)
+  uint64_t* raw_empty = raw_full + kQRaw;    // 4-bit: code stage converted by every dequant warp
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(raw_empty + kQRaw);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   uint8_t* epi_stage = reinterpret_cast<uint8_t*>(full) + 256;  // 4 KB per epilogue warp
   int* s_pt = reinterpret_cast<int*>(epi_stage + kQEpiWarps * 4096);  // [groups + 1] tile prefix
-  int* s_slot = s_pt + kMaxExperts + 1;                               // [groups]
-  int* s_rb = s_slot + kMaxExperts;                                   // [groups] first row
-  int* s_cnt = s_rb + kMaxExperts;                                    // [groups] rows
-  int* s_tmp = s_cnt + kMaxExperts;                                   // [64]
+  int* s_slot = s_pt + C::kGroups + 1;                                // [groups]
+  int* s_rb = s_slot + C::kGroups;                                    // [groups] first row
+  int* s_cnt = s_rb + C::kGroups;                                     // [groups] rows
+  int* s_tmp = s_cnt + C::kGroups;                                    // [64]
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -129,7 +156,7 @@ __global__ void __launch_bounds__(kQThreads, 1)
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kQStages; ++s) {
-      mbar_init(&full[s], kQFullLocal + (leader ? 1 : 0));  // + the peer's relay
+      mbar_init(&full[s], C::kFullLocal + (leader ? 1 : 0));  // + the peer's relay
       mbar_init(&empty[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
@@ -138,6 +165,10 @@ __global__ void __launch_bounds__(kQThreads, 1)
     }
     mbar_init(drain, 1);
     mbar_init(never, 1);
+    for (int r = 0; r < kQRaw && Q4; ++r) {
+      mbar_init(&raw_full[r], 1);
+      mbar_init(&raw_empty[r], kQDq);
+    }
     *abort_flag = 0;
     mbar_fence_init();
   }
@@ -164,7 +195,7 @@ __global__ void __launch_bounds__(kQThreads, 1)
 
   if (warp == 5) {
     // ------------------------------------------------------------- TMA producer (B)
-    if (lane == 0) {
+    if (lane == 0 && !Q4) {
       uint32_t it = 0;
       for (int t = pair; t < total; t += npairs) {
         const QTile tc = qdecode(a, ng, s_pt, t);
@@ -192,6 +223,35 @@ __global__ void __launch_bounds__(kQThreads, 1)
           if ((int)j < 0) break;
           const long long t0 = clock64();
           while (!mbar_try_wait(&full[j % kQStages], (j / kQStages) & 1) && clock64() - t0 < kDrainCycles) {
+          }
+        }
+      }
+    } else if (lane == 0) {
+      // 4-bit: the CTA's 128 code rows of each stage into the raw ring
+      // (gate-up: gate rows in the even CTA, up rows in the odd one; down:
+      // W2 rows 256 n + 128 r)
+      uint32_t it = 0;
+      for (int t = pair; t < total; t += npairs) {
+        const QTile tc = qdecode(a, ng, s_pt, t);
+        const int kb_n = tc.up ? a.kb_up : a.kb_dn;
+        const int qrow = tc.up ? s_slot[tc.g] * a.q13_rows_per_slot + (rank ? a.w13_up_off : 0) + tc.n * 128
+                               : s_slot[tc.g] * a.q2_rows_per_slot + a.q2_row_off + tc.n * kBN + (int)rank * 128;
+        const CUtensorMap* map = tc.up ? &tmW13 : &tmW2;
+        bool ok = true;
+        for (int kb = 0; kb < kb_n; ++kb, ++it) {
+          const int r = it % kQRaw;
+          if (!mbar_wait(&raw_empty[r], ((it / kQRaw) & 1) ^ 1, abort_flag, lim)) { ok = false; break; }
+          mbar_arrive_expect_tx(&raw_full[r], 128 * kQRawRow);
+          tma_load_2d(raw_codes + r * (128 * kQRawRow), map, &raw_full[r], kb * kQRawRow, qrow);
+        }
+        if (!ok) break;
+      }
+      if (*abort_flag) {
+        for (int d = 0; d < kQRaw && it > 0; ++d) {
+          const uint32_t j = it - 1 - d;
+          if ((int)j < 0) break;
+          const long long t0 = clock64();
+          while (!mbar_try_wait(&raw_full[j % kQRaw], (j / kQRaw) & 1) && clock64() - t0 < kDrainCycles) {
           }
         }
       }
@@ -265,13 +325,20 @@ __global__ void __launch_bounds__(kQThreads, 1)
       const uint32_t tb = tmem_base + ((uint32_t)(warp * 32) << 16) + acc * kBN;
       const int row_w = tc.m2 * kQRows + (int)rank * kBM + warp * 32;  // warp's first row in the group
       if (tc.up) {
-        epilogue_tile_staged<true>(tb, a.h + (rb + row_w) * a.h_ld + tc.n * 128, a.h_ld, cnt - row_w,
-                                   epi_stage + warp * 4096, lane);
+        if (Q4)
+          epilogue_tile_staged_lean<true>(tb, a.h + (rb + row_w) * a.h_ld + tc.n * 128, a.h_ld, cnt - row_w,
+                                          epi_stage + warp * 4096, lane);
+        else
+          epilogue_tile_staged<true>(tb, a.h + (rb + row_w) * a.h_ld + tc.n * 128, a.h_ld, cnt - row_w,
+                                     epi_stage + warp * 4096, lane);
         // publish this CTA's half of the tile: every epilogue thread's h
         // stores, then one release add on the 256-row tile's counter
         __threadfence();
         epilogue_bar();
         if (threadIdx.x == 0) red_release_gpu_add(&a.ready[s_pt[tc.g] + tc.m2], 1);
+      } else if (Q4) {
+        epilogue_tile_staged_lean<false>(tb, a.y + (rb + row_w) * a.y_ld + tc.n * kBN, a.y_ld, cnt - row_w,
+                                         epi_stage + warp * 4096, lane);
       } else {
         epilogue_tile_staged<false>(tb, a.y + (rb + row_w) * a.y_ld + tc.n * kBN, a.y_ld, cnt - row_w,
                                     epi_stage + warp * 4096, lane);
@@ -280,7 +347,7 @@ __global__ void __launch_bounds__(kQThreads, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive_remote(lead_tempty[acc]);
     }
-  } else {
+  } else if (warp < kQGatherWarp0 + kQGatherWarps) {
     // ------------------------------------------------------------- A rows
     const int gt = threadIdx.x - kQGatherWarp0 * 32;  // 0..127
     const int chunk = gt & 7;                         // 16-byte chunk of a 128-byte row slice
@@ -355,6 +422,58 @@ __global__ void __launch_bounds__(kQThreads, 1)
       }
     }
     cp_async_wait<0>();
+  } else if (Q4) {
+    // ------------------------------------------------------------- 4-bit dequant
+    // a warp takes 8 of the CTA's 128 B rows, four lanes to a row (a quarter
+    // row of 16 codes under one scale); its code reads cover 256 contiguous
+    // bytes and its SW128 writes reach every bank group once per 8 lanes
+    const int d = (warp - kQGatherWarp0 - kQGatherWarps) * 8 + (lane >> 2);  // B row, 0..127
+    const int qt = lane & 3;                                                 // codes 16 qt .. 16 qt + 15
+    // this thread's scale row of tile t (W13 rows for a gate-up tile, W2
+    // rows for a down tile); scales of a stage pair are one 8-byte load
+    auto scale_row = [&](int t) -> const uint8_t* {
+      const QTile tc = qdecode(a, ng, s_pt, t);
+      const uint8_t* ext = a.q4_pool + (unsigned long long)s_slot[tc.g] * a.q4_extent;
+      return tc.up ? ext + a.q13_scale_off + (size_t)((rank ? a.w13_up_off : 0) + tc.n * 128 + d) * a.q13_scale_ld
+                   : ext + a.q2_scale_off + (size_t)(tc.n * kBN + (int)rank * 128 + d) * a.q2_scale_ld;
+    };
+    uint32_t it = 0;
+    bool ok = true;
+    // the next stage pair's scales are loaded one pair ahead, across tiles
+    uint2 nxt = pair < total ? __ldg(reinterpret_cast<const uint2*>(scale_row(pair))) : make_uint2(0, 0);
+    for (int t = pair; t < total && ok; t += npairs) {
+      const QTile tc = qdecode(a, ng, s_pt, t);
+      const int kb_n = tc.up ? a.kb_up : a.kb_dn;  // even (K a multiple of 128)
+      const uint8_t* srow = scale_row(t);
+      const uint8_t* srow_next = t + npairs < total ? scale_row(t + npairs) : nullptr;
+      uint2 cur = make_uint2(0, 0);
+      for (int kb = 0; kb < kb_n; ++kb, ++it) {
+        if ((kb & 1) == 0) {
+          cur = nxt;
+          if (kb + 2 < kb_n) nxt = __ldg(reinterpret_cast<const uint2*>(srow + (kb + 2) * 4));
+          else if (srow_next != nullptr) nxt = __ldg(reinterpret_cast<const uint2*>(srow_next));
+        }
+        const int r = it % kQRaw;
+        if (!mbar_wait(&raw_full[r], (it / kQRaw) & 1, abort_flag, lim)) { ok = false; break; }
+        const int s = it % kQStages;
+        const uint32_t ph = (it / kQStages) & 1;
+        if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, lim)) { ok = false; break; }
+        const uint2 cw = *reinterpret_cast<const uint2*>(raw_codes + r * (128 * kQRawRow) + d * kQRawRow + qt * 8);
+        const uint32_t sc = (kb & 1) ? cur.y : cur.x;
+        const float sv = __half2float(__ushort_as_half((unsigned short)(qt >= 2 ? sc >> 16 : sc & 0xFFFFu)));
+        const uint64_t sx2 = f32x2(sv, sv), nx2 = f32x2(-136.0f * sv, -136.0f * sv);
+        uint8_t* dst_row = sB + s * kQB + d * 128;
+        const int c0 = qt * 2;  // 16-byte chunks c0, c0 + 1 of the 128-byte row
+        *reinterpret_cast<uint4*>(dst_row + ((c0 ^ (d & 7)) << 4)) = dequant8(cw.x, sx2, nx2);
+        *reinterpret_cast<uint4*>(dst_row + (((c0 + 1) ^ (d & 7)) << 4)) = dequant8(cw.y, sx2, nx2);
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          mbar_arrive(&full[s]);
+          mbar_arrive(&raw_empty[r]);  // the warp's rows of this code stage are consumed
+        }
+      }
+    }
   }
 
   tc_fence_before();
@@ -368,11 +487,13 @@ __global__ void __launch_bounds__(kQThreads, 1)
   if (threadIdx.x == 0 && *abort_flag) atomicCAS(a.status, 0, (int)MSI_ERR_TIMEOUT);
 }
 
-cudaError_t launch_fused_wave_pair(const CUtensorMap& tmW13, const CUtensorMap& tmW2,
-                                   const FusedArgs& a, const WaveParams& w, int max_pairs, cudaStream_t s) {
+template <bool Q4>
+static cudaError_t launch_pair(const CUtensorMap& tmW13, const CUtensorMap& tmW2, const FusedArgs& a,
+                               const WaveParams& w, int max_pairs, cudaStream_t s) {
   static std::atomic<unsigned long long> attr_done{0};
   static std::atomic<int> max_clusters[64] = {};
-  cudaError_t e = smem_attr_once(fused_wave_pair_kernel, kQSmem, attr_done);
+  auto kernel = fused_wave_pair_kernel<Q4>;
+  cudaError_t e = smem_attr_once(kernel, QCfg<Q4>::kSmem, attr_done);
   if (e != cudaSuccess) return e;
   if (max_pairs < 1) return cudaSuccess;
   cudaLaunchConfig_t cfg = {};
@@ -381,8 +502,8 @@ cudaError_t launch_fused_wave_pair(const CUtensorMap& tmW13, const CUtensorMap& 
   attr[0].val.clusterDim.x = 2;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
-  cfg.blockDim = dim3(kQThreads, 1, 1);
-  cfg.dynamicSmemBytes = kQSmem;
+  cfg.blockDim = dim3(QCfg<Q4>::kThreads, 1, 1);
+  cfg.dynamicSmemBytes = QCfg<Q4>::kSmem;
   cfg.stream = s;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
@@ -394,14 +515,25 @@ cudaError_t launch_fused_wave_pair(const CUtensorMap& tmW13, const CUtensorMap& 
   int mc = dev < 64 ? max_clusters[dev].load() : 0;
   if (mc <= 0) {
     cfg.gridDim = dim3(2, 1, 1);
-    e = cudaOccupancyMaxActiveClusters(&mc, fused_wave_pair_kernel, &cfg);
+    e = cudaOccupancyMaxActiveClusters(&mc, kernel, &cfg);
     if (e != cudaSuccess) return e;
     if (mc <= 0) return cudaErrorInvalidConfiguration;
     if (dev < 64) max_clusters[dev].store(mc);
   }
   const int pairs = std::max(1, std::min(mc, max_pairs));
   cfg.gridDim = dim3(2 * pairs, 1, 1);
-  return cudaLaunchKernelEx(&cfg, fused_wave_pair_kernel, tmW13, tmW2, a, w);
+  return cudaLaunchKernelEx(&cfg, kernel, tmW13, tmW2, a, w);
+}
+
+cudaError_t launch_fused_wave_pair(const CUtensorMap& tmW13, const CUtensorMap& tmW2,
+                                   const FusedArgs& a, const WaveParams& w, int max_pairs, cudaStream_t s) {
+  return launch_pair<false>(tmW13, tmW2, a, w, max_pairs, s);
+}
+
+cudaError_t launch_fused_wave_pair_q4(const CUtensorMap& tmQ13, const CUtensorMap& tmQ2,
+                                      const FusedArgs& a, const WaveParams& w, int max_pairs, cudaStream_t s) {
+  if (!a.wave) return cudaErrorInvalidValue;  // 4-bit fused launches are waves (group table of kMaxWave)
+  return launch_pair<true>(tmQ13, tmQ2, a, w, max_pairs, s);
 }
 
 }  // namespace msi

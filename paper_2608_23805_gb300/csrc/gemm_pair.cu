@@ -89,43 +89,6 @@ struct PCfg {
                                (2 * kMaxExperts + 2) * 4;
 };
 
-// The staged epilogue of one warp's 32 rows, TMEM read 16 columns at a time
-// (the 4-bit modes' thread count leaves 72 registers a thread).
-template <bool GATEUP>
-__device__ __forceinline__ void epilogue_tile_staged_lean(uint32_t tb, __nv_bfloat16* row0, size_t ld,
-                                                          int nvalid, uint8_t* stg, int lane) {
-  if (GATEUP) {
-#pragma unroll 1
-    for (int c = 0; c < 128; c += 16) {
-      uint32_t g[16], u[16];
-      tmem_ld16(tb + c, g);
-      tmem_ld16(tb + 128 + c, u);
-      tmem_ld_wait(g);
-      tmem_ld_wait(u);
-      uint32_t p[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        const float g0 = __uint_as_float(g[2 * i]), g1 = __uint_as_float(g[2 * i + 1]);
-        const float u0 = __uint_as_float(u[2 * i]), u1 = __uint_as_float(u[2 * i + 1]);
-        p[i] = pack_bf16x2(__fdividef(g0 * u0, 1.0f + __expf(-g0)),
-                           __fdividef(g1 * u1, 1.0f + __expf(-g1)));
-      }
-      store_rows_staged<32>(p, stg, row0 + c, ld, nvalid, lane);
-    }
-  } else {
-#pragma unroll 1
-    for (int c = 0; c < kBN; c += 16) {
-      uint32_t v[16];
-      tmem_ld16(tb + c, v);
-      tmem_ld_wait(v);
-      uint32_t p[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) p[i] = pack_bf16x2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1]));
-      store_rows_staged<32>(p, stg, row0 + c, ld, nvalid, lane);
-    }
-  }
-}
-
 struct PairTile {
   int g, m2, n;
 };

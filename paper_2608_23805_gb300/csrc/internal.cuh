@@ -148,6 +148,17 @@ struct FusedArgs {
   const GenWord* genwords;  // published (generation, object) per slot
   int* ready_clear;
   int n_ready_clear;
+  // 4-bit waves (gemm_fused_pair.cu, Q4): codes by TMA through the code maps,
+  // fp16 scales read from the slot pool
+  const uint8_t* q4_pool;
+  unsigned long long q4_extent;   // bytes per slot
+  int q13_rows_per_slot;          // W13 code rows (H / 2 bytes each) per slot
+  int q2_rows_per_slot;           // W2 code rows (I / 2 bytes each) per slot
+  int q2_row_off;                 // first W2 code row inside a slot
+  long long q13_scale_off;        // byte offset of the W13 scales in an extent
+  int q13_scale_ld;               // bytes of scales per W13 row (H / 16)
+  long long q2_scale_off;         // byte offset of the W2 scales in an extent
+  int q2_scale_ld;                // bytes of scales per W2 row (I / 16)
 };
 
 // ---------------------------------------------------------------------------
@@ -167,6 +178,9 @@ cudaError_t launch_fused_wave(const CUtensorMap& tmW13, const CUtensorMap& tmW2,
 // `max_pairs` pairs, never more than can be resident at once.
 cudaError_t launch_fused_wave_pair(const CUtensorMap& tmW13, const CUtensorMap& tmW2,
                                    const FusedArgs& a, const WaveParams& w, int max_pairs, cudaStream_t s);
+// 4-bit waves on CTA pairs (tmQ13 / tmQ2: the byte-granular code maps).
+cudaError_t launch_fused_wave_pair_q4(const CUtensorMap& tmQ13, const CUtensorMap& tmQ2,
+                                      const FusedArgs& a, const WaveParams& w, int max_pairs, cudaStream_t s);
 
 // GEMM tiling
 constexpr int kBM = 128;
@@ -577,6 +591,44 @@ __device__ __forceinline__ void epilogue_tile_staged(uint32_t tb, __nv_bfloat16*
         p[16 + i] = pack_bf16x2(__uint_as_float(w[2 * i]), __uint_as_float(w[2 * i + 1]));
       }
       store_rows_staged<128>(p, stg, row0 + c, ld, nvalid, lane);
+    }
+  }
+}
+
+// The staged epilogue of one warp's 32 rows, TMEM read 16 columns at a time
+// (the 4-bit modes' thread count leaves 72 registers a thread;
+// CTA-pair kernels).
+template <bool GATEUP>
+__device__ __forceinline__ void epilogue_tile_staged_lean(uint32_t tb, __nv_bfloat16* row0, size_t ld,
+                                                          int nvalid, uint8_t* stg, int lane) {
+  if (GATEUP) {
+#pragma unroll 1
+    for (int c = 0; c < 128; c += 16) {
+      uint32_t g[16], u[16];
+      tmem_ld16(tb + c, g);
+      tmem_ld16(tb + 128 + c, u);
+      tmem_ld_wait(g);
+      tmem_ld_wait(u);
+      uint32_t p[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const float g0 = __uint_as_float(g[2 * i]), g1 = __uint_as_float(g[2 * i + 1]);
+        const float u0 = __uint_as_float(u[2 * i]), u1 = __uint_as_float(u[2 * i + 1]);
+        p[i] = pack_bf16x2(__fdividef(g0 * u0, 1.0f + __expf(-g0)),
+                           __fdividef(g1 * u1, 1.0f + __expf(-g1)));
+      }
+      store_rows_staged<32>(p, stg, row0 + c, ld, nvalid, lane);
+    }
+  } else {
+#pragma unroll 1
+    for (int c = 0; c < kBN; c += 16) {
+      uint32_t v[16];
+      tmem_ld16(tb + c, v);
+      tmem_ld_wait(v);
+      uint32_t p[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) p[i] = pack_bf16x2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1]));
+      store_rows_staged<32>(p, stg, row0 + c, ld, nvalid, lane);
     }
   }
 }

@@ -456,6 +456,13 @@ msi_status wait_ready(msi_plan* p, const std::vector<int>& slots, cudaStream_t s
   return MSI_OK;
 }
 
+// Write the slots' published words (generation, object) on `stage`, in
+// stream order (the publication kernel).
+msi_status write_words(msi_plan* p, const PublishParams& w, cudaStream_t stage) {
+  LAUNCH(p, MSI_K_PUBLISH, stage, launch_publish(w, p->d_gen, stage));
+  return MSI_OK;
+}
+
 // Enqueue the copies of `misses` on `stage` and publish them with one event.
 msi_status stage_enqueue(msi_plan* p, int layer, const std::vector<WaveEntry>& misses,
                          cudaStream_t stage) {
@@ -484,7 +491,8 @@ msi_status stage_enqueue(msi_plan* p, int layer, const std::vector<WaveEntry>& m
       p->faults.erase(f);
     }
   }
-  LAUNCH(p, MSI_K_PUBLISH, stage, launch_publish(inv, p->d_gen, stage));
+  st = write_words(p, inv, stage);
+  if (st != MSI_OK) return st;
   const uint64_t eb = p->d.extent_bytes;
   auto src_of = [&](const WaveEntry& m) {
     return static_cast<const char*>(p->d.host_windows) +
@@ -565,7 +573,8 @@ msi_status stage_enqueue(msi_plan* p, int layer, const std::vector<WaveEntry>& m
     i = j;
   }
   }
-  LAUNCH(p, MSI_K_PUBLISH, stage, launch_publish(pub, p->d_gen, stage));
+  st = write_words(p, pub, stage);
+  if (st != MSI_OK) return st;
   int ev;
   st = p->pool.acquire(&ev);
   if (st != MSI_OK) return st;
@@ -740,11 +749,15 @@ msi_status route_rows(msi_plan* p, FwdCtx& f, const float* rw, const msi_route_e
   return MSI_OK;
 }
 
-// A streamed bf16 wave runs its gate-up and down in one launch
-// (gemm_fused.cu, gemm_fused_pair.cu): a wave is too small to fill the SMs'
-// last round of gate-up tiles, and the down tiles fill it.
-bool fused_wave(const msi_plan* p, const FwdCtx& f, long long, int) {
-  return p->d.wdtype == MSI_W_BF16 && !(f.flags & MSI_FWD_SPLIT_WAVES);
+// A streamed wave runs its gate-up and down in one launch (gemm_fused.cu,
+// gemm_fused_pair.cu): a wave is too small to fill the SMs' last round of
+// gate-up tiles, and the down tiles fill it.  bf16 waves always; 4-bit waves
+// on CTA pairs, once their groups average >= 512 rows (smaller 4-bit waves
+// keep the split single-CTA launches).
+bool fused_wave(const msi_plan* p, const FwdCtx& f, long long rows, int ng) {
+  if (f.flags & MSI_FWD_SPLIT_WAVES) return false;
+  if (p->d.wdtype == MSI_W_BF16) return true;
+  return !(f.flags & MSI_FWD_SINGLE_CTA) && ng > 0 && rows >= 512LL * ng;
 }
 
 // A resident bf16 forward fuses its two projections while neither would take
@@ -818,9 +831,9 @@ msi_status front(msi_plan* p, FwdCtx& f, const TableParams& tp) {
       xa.ready = at<int>(ws, L.ready);
       xa.n_ready = ready_bank(f);
     }
-  } else if (fused_wave(p, f, 0, 0)) {
-    // streamed call: the first wave's bank (later waves' banks are zeroed by
-    // the wave before them)
+  } else if (!(f.flags & MSI_FWD_SPLIT_WAVES)) {
+    // streamed call: the first fused wave's bank (later waves' banks are
+    // zeroed by the wave before them)
     xa.ready = at<int>(ws, L.ready);
     xa.n_ready = ready_bank(f);
   }
@@ -906,40 +919,15 @@ msi_status routed_ffn(msi_plan* p, FwdCtx& f, int ng, int grid1, int grid2, long
   const auto& d = p->d;
   const Group* groups = at<Group>(f.ws, f.L.groups);
   const int* total = at<int>(f.ws, f.L.total);
-  GemmArgs g1 = gateup_args(p, f, groups, ng, total, at<__nv_bfloat16>(f.ws, f.L.h));
-  GemmArgs g2 = down_args(p, f, groups, ng, total, at<__nv_bfloat16>(f.ws, f.L.yp));
-  if (d.wdtype == MSI_W_Q4G32) {
-    // 4-bit extent: W13 codes [2I, H/2] | W2 codes [H, I/2] | W13 scales [2I, H/32] | W2 scales [H, I/32]
-    const long long HI = (long long)d.hidden * d.inter;
-    for (GemmArgs* g : {&g1, &g2}) {
-      g->q4_pool = static_cast<const uint8_t*>(d.slot_pool);
-      g->q4_extent = d.extent_bytes;
-    }
-    // code rows through the byte maps: W13 rows of H/2 bytes, W2 rows of I/2
-    // bytes; an extent is a whole number of either (27 I / 8 and 27 H / 8)
-    g1.q4_rows_per_slot = (int)(d.extent_bytes / (d.hidden / 2));
-    g1.q4_row_off = 0;
-    g1.q4_scale_off = 3 * HI / 2;
-    g1.q4_scale_ld = d.hidden / 16;
-    g2.q4_rows_per_slot = (int)(d.extent_bytes / (d.inter / 2));
-    g2.q4_row_off = (int)(HI / (d.inter / 2));
-    g2.q4_scale_off = 3 * HI / 2 + HI / 8;
-    g2.q4_scale_ld = d.inter / 16;
-    if (pair_up)
-      LAUNCH(p, MSI_K_GATEUP, f.cs,
-             launch_gemm_pair(kGateUpGatherQ4, f.tm_h, p->tm_q13, g1, std::max(1, grid1 / 2), f.cs));
-    else
-      LAUNCH(p, MSI_K_GATEUP, f.cs, launch_gemm(kGateUpGatherQ4, f.tm_h, p->tm_q13, g1, grid1, f.cs));
-    if (pair_down)
-      LAUNCH(p, MSI_K_DOWN, f.cs,
-             launch_gemm_pair(kDownQ4, f.tm_h, p->tm_q2, g2, std::max(1, grid2 / 2), f.cs));
-    else
-      LAUNCH(p, MSI_K_DOWN, f.cs, launch_gemm(kDownQ4, f.tm_h, p->tm_q2, g2, grid2, f.cs));
-    return MSI_OK;
-  }
+  // 4-bit extent: W13 codes [2I, H/2] | W2 codes [H, I/2] | W13 scales [2I, H/32] | W2 scales [H, I/32];
+  // code rows through the byte maps: W13 rows of H/2 bytes, W2 rows of I/2
+  // bytes (an extent is a whole number of either: 27 I / 8 and 27 H / 8)
+  const long long HI = (long long)d.hidden * d.inter;
+  const int q13_rows = (int)(d.extent_bytes / (d.hidden / 2));
+  const int q2_rows = (int)(d.extent_bytes / (d.inter / 2));
+  const int q2_off = (int)(HI / (d.inter / 2));
   if (wave_mtiles >= 0 && fused_wave(p, f, rows, ng)) {
-    // one launch: the wave's gate-up tiles, then its down tiles (the setup
-    // kernel zeroed the per-m-tile counters)
+    // one launch: the wave's gate-up tiles, then its down tiles
     FusedArgs fa{};
     fa.groups = groups;
     fa.num_groups = ng;
@@ -979,13 +967,60 @@ msi_status routed_ffn(msi_plan* p, FwdCtx& f, int ng, int grid1, int grid2, long
     }
     const WaveParams& wv = wp != nullptr ? *wp : no_wave;
     const long long tiles = (long long)wave_mtiles * (fa.nt_up + fa.nt_dn);
+    // a wave's launch leaves one SM (a pair: two) to the staging stream: the
+    // next wave's invalidation and publication kernels run there at once
+    // instead of waiting for this persistent launch to end, which would hold
+    // back the next wave's copies (measured at 32K: 14.5 against 16.0 ms per
+    // step)
+    const int spare = wp != nullptr ? 1 : 0;
+    const int pairs = (int)std::min<long long>(p->sms / 2 - spare, std::max<long long>(1, tiles));
+    if (!bf16) {
+      // 4-bit waves: CTA pairs (fused_wave admits them from 512 rows per group)
+      fa.q4_pool = static_cast<const uint8_t*>(d.slot_pool);
+      fa.q4_extent = d.extent_bytes;
+      fa.q13_rows_per_slot = q13_rows;
+      fa.q2_rows_per_slot = q2_rows;
+      fa.q2_row_off = q2_off;
+      fa.q13_scale_off = 3 * HI / 2;
+      fa.q13_scale_ld = d.hidden / 16;
+      fa.q2_scale_off = 3 * HI / 2 + HI / 8;
+      fa.q2_scale_ld = d.inter / 16;
+      LAUNCH(p, MSI_K_FFN, f.cs, launch_fused_wave_pair_q4(p->tm_q13, p->tm_q2, fa, wv, pairs, f.cs));
+      return MSI_OK;
+    }
     if (pair_tiles(f, rows, ng, kPairMinRowsFused)) {
-      const int pairs = (int)std::min<long long>(p->sms / 2, std::max<long long>(1, tiles));
       LAUNCH(p, MSI_K_FFN, f.cs, launch_fused_wave_pair(p->tm_w13, p->tm_w2, fa, wv, pairs, f.cs));
       return MSI_OK;
     }
-    const int grid = (int)std::min<long long>(p->sms, std::max<long long>(1, tiles));
+    const int grid = (int)std::min<long long>(p->sms - spare, std::max<long long>(1, tiles));
     LAUNCH(p, MSI_K_FFN, f.cs, launch_fused_wave(p->tm_w13, p->tm_w2, fa, wv, grid, f.cs));
+    return MSI_OK;
+  }
+  GemmArgs g1 = gateup_args(p, f, groups, ng, total, at<__nv_bfloat16>(f.ws, f.L.h));
+  GemmArgs g2 = down_args(p, f, groups, ng, total, at<__nv_bfloat16>(f.ws, f.L.yp));
+  if (d.wdtype == MSI_W_Q4G32) {
+    for (GemmArgs* g : {&g1, &g2}) {
+      g->q4_pool = static_cast<const uint8_t*>(d.slot_pool);
+      g->q4_extent = d.extent_bytes;
+    }
+    g1.q4_rows_per_slot = q13_rows;
+    g1.q4_row_off = 0;
+    g1.q4_scale_off = 3 * HI / 2;
+    g1.q4_scale_ld = d.hidden / 16;
+    g2.q4_rows_per_slot = q2_rows;
+    g2.q4_row_off = q2_off;
+    g2.q4_scale_off = 3 * HI / 2 + HI / 8;
+    g2.q4_scale_ld = d.inter / 16;
+    if (pair_up)
+      LAUNCH(p, MSI_K_GATEUP, f.cs,
+             launch_gemm_pair(kGateUpGatherQ4, f.tm_h, p->tm_q13, g1, std::max(1, grid1 / 2), f.cs));
+    else
+      LAUNCH(p, MSI_K_GATEUP, f.cs, launch_gemm(kGateUpGatherQ4, f.tm_h, p->tm_q13, g1, grid1, f.cs));
+    if (pair_down)
+      LAUNCH(p, MSI_K_DOWN, f.cs,
+             launch_gemm_pair(kDownQ4, f.tm_h, p->tm_q2, g2, std::max(1, grid2 / 2), f.cs));
+    else
+      LAUNCH(p, MSI_K_DOWN, f.cs, launch_gemm(kDownQ4, f.tm_h, p->tm_q2, g2, grid2, f.cs));
     return MSI_OK;
   }
   if (pair_up)

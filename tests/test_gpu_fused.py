@@ -124,3 +124,33 @@ def test_fused_resident_equals_split_launches(tokens):
     ref = case.oracle_layer(x_bits, tokens=toks)
     compare_out(outs[0][0][toks], ref["out"])
     case.close()
+
+
+@pytest.mark.parametrize("tokens", [5120, 2600])
+def test_fused_q4_waves_equal_split_launches(tokens):
+    """4-bit experts: waves whose groups average >= 512 rows (~640 and ~325
+    rows per expert here; the smaller one keeps the split single-CTA
+    launches) run both projections in one CTA-pair launch with the codes
+    dequantised in the kernel; bit-identical to the split pair launches and
+    within the output tolerance of the oracle."""
+    cfg = synth.config("tiny", hidden=512, inter=256, n_experts=32, top_k=4, tokens=tokens,
+                       n_slots=16, wdtype=synth.W_Q4G32)
+    case = Case(cfg)
+    x_bits = synth.hidden(cfg, 0, 25)
+    x = bf16_tensor(x_bits)
+    case.plan.timing(True)
+    case.plan.timing_read(reset=True)
+    of, idf, wf, trf = _run(case, x, split=False)
+    kt = case.plan.timing_read(reset=True)
+    case.plan.timing(False)
+    assert (kt["ffn"][1] > 0) == (tokens * 4 // 32 >= 512)
+    case2 = Case(cfg)
+    os_, ids_, _, trs = _run(case2, x, split=True)
+    assert np.array_equal(idf, ids_)
+    assert trf == trs
+    assert np.array_equal(of, os_)
+    ref = case.oracle_layer(x_bits)
+    compare_routes(idf, wf, ref)
+    compare_out(of, ref["out"])
+    case.close()
+    case2.close()
