@@ -20,8 +20,9 @@
 //       A rows read from h.
 // A down tile needs every gate-up tile of its m-tile (the whole h row): the
 // gate-up epilogue publishes each finished tile on a per-m-tile counter
-// (stores, a gpu-scope fence, a release add) and the gather warps of a down
-// tile acquire that counter before they read h.
+// (stores, a gpu-scope fence, a release add), and the producer acquires that
+// counter, orders the h writes before its async-proxy reads
+// (fence.proxy.async.global) and loads the down tile's A rows from h by TMA.
 //
 // Progress: tiles are taken in a static round-robin (t = blockIdx.x +
 // i * gridDim.x), so every CTA processes its tiles in increasing order and
@@ -31,9 +32,11 @@
 // sequence).  The launch is cooperative, so every CTA is resident.
 //
 // Roles: warps 0-3 epilogue, warp 4 MMA issue + TMEM allocation, warp 5 TMA
-// producer (B: W13 or W2 rows of the group's slot), warps 6-9 A rows by
-// cp.async into the 128-byte-swizzled layout (arriving on the stage barrier
-// as their copies land).  Every wait is bounded; on expiry the CTA raises its
+// producer (B: W13 or W2 rows of the group's slot; A of a down tile: h
+// rows), warps 6-9 the gate-up tiles' A rows (x rows through the
+// permutation) by cp.async into the 128-byte-swizzled layout, arriving on the
+// stage barrier as their copies land (on a down tile's stages they only
+// arrive).  Every wait is bounded; on expiry the CTA raises its
 // abort flag, all roles drain and the kernel reports MSI_ERR_TIMEOUT.
 #include "internal.cuh"
 
@@ -88,6 +91,17 @@ __device__ __forceinline__ void red_release_gpu_add(int* p, int v) {
   asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
 }
 
+// Generic-proxy writes to global memory (observed through an acquire) before
+// this thread's later async-proxy (TMA) reads.
+__device__ __forceinline__ void fence_proxy_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
+// One arrival counting for `count` expected arrivals.
+__device__ __forceinline__ void mbar_arrive_n(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+
 // The four epilogue warps (128 threads) only.
 __device__ __forceinline__ void epilogue_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
 
@@ -95,8 +109,8 @@ __device__ __forceinline__ void epilogue_bar() { asm volatile("bar.sync 1, 128;"
 
 __global__ void __launch_bounds__(kFThreads, 1)
     fused_wave_kernel(const __grid_constant__ CUtensorMap tmW13,
-                      const __grid_constant__ CUtensorMap tmW2, const FusedArgs a,
-                      const __grid_constant__ WaveParams w) {
+                      const __grid_constant__ CUtensorMap tmW2, const __grid_constant__ CUtensorMap tmH,
+                      const FusedArgs a, const __grid_constant__ WaveParams w) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -141,6 +155,7 @@ __global__ void __launch_bounds__(kFThreads, 1)
   if (warp == 5 && lane == 0) {
     tma_prefetch(&tmW13);
     tma_prefetch(&tmW2);
+    tma_prefetch(&tmH);
   }
   // the previous wave's counters, zeroed for the next wave
   for (int r = blockIdx.x * blockDim.x + threadIdx.x; r < a.n_ready_clear; r += gridDim.x * blockDim.x)
@@ -165,14 +180,34 @@ __global__ void __launch_bounds__(kFThreads, 1)
         const int r1 = tc.up ? r0 + a.w13_up_off : r0 + 128;
         const CUtensorMap* map = tc.up ? &tmW13 : &tmW2;
         bool ok = true;
+        if (!tc.up) {
+          // every gate-up tile of this m-tile has published its h columns
+          const int* rdy = a.ready + s_mt[tc.g] + tc.m;
+          const long long t0 = clock64();
+          while (ld_acquire_gpu(rdy) < a.nt_up) {
+            if (*abort_flag) { ok = false; break; }
+            if (clock64() - t0 > lim) {
+              *abort_flag = 1;
+              ok = false;
+              break;
+            }
+          }
+          if (!ok) break;
+          fence_proxy_async_global();
+        }
+        // the down tile's A: its 128 h rows (rows past the group's segment
+        // are the next group's or the tensor's zero fill; their outputs are
+        // not stored)
+        const int arow = s_rb[tc.g] + tc.m * kBM;
         for (int kb = 0; kb < kb_n; ++kb, ++it) {
           const int s = it % kFStages;
           const uint32_t ph = (it / kFStages) & 1;
           if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, lim)) { ok = false; break; }
-          mbar_arrive_expect_tx(&full[s], kBBytes);
+          mbar_arrive_expect_tx(&full[s], tc.up ? kBBytes : kBBytes + kABytes);
           uint8_t* b = sB + s * kBBytes;
           tma_load_2d(b, map, &full[s], kb * kBK, r0);
           tma_load_2d(b + kBBytes / 2, map, &full[s], kb * kBK, r1);
+          if (!tc.up) tma_load_2d(sA + s * kABytes, &tmH, &full[s], kb * kBK, arow);
         }
         if (!ok) break;
       }
@@ -259,9 +294,8 @@ __global__ void __launch_bounds__(kFThreads, 1)
     const int r0 = gt >> 3;                           // rows r0 + 16 i
     uint32_t it = 0;
     bool ok = true;
-    // this thread's eight source rows of tile t (x rows by token for a
-    // gate-up tile, h rows for a down tile; -1 past the group's segment),
-    // loaded one tile ahead
+    // this thread's eight x rows of gate-up tile t (by token; -1 past the
+    // group's segment), loaded one tile ahead
     auto tile_rows = [&](int t, int (&pr)[8]) {
       const FTile tc = fdecode(a, ng, s_mt, t);
       const int cnt = s_cnt[tc.g];
@@ -269,7 +303,7 @@ __global__ void __launch_bounds__(kFThreads, 1)
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
         const int rr = tc.m * kBM + r0 + 16 * i;
-        pr[i] = rr >= cnt ? -1 : (tc.up ? __ldg(&a.perm[rb + rr]) / a.top_k : rb + rr);
+        pr[i] = (!tc.up || rr >= cnt) ? -1 : __ldg(&a.perm[rb + rr]) / a.top_k;
       }
     };
     int pr[8], pr_next[8];
@@ -280,49 +314,43 @@ __global__ void __launch_bounds__(kFThreads, 1)
       const FTile tc = fdecode(a, ng, s_mt, t);
       const int kb_n = tc.up ? a.kb_up : a.kb_dn;
       if (!tc.up) {
-        // every gate-up tile of this m-tile has published its h columns
-        const int* rdy = a.ready + s_mt[tc.g] + tc.m;
-        bool seen = true;
-        if (lane == 0) {
-          const long long t0 = clock64();
-          while (ld_acquire_gpu(rdy) < a.nt_up) {
-            if (*abort_flag) { seen = false; break; }
-            if (clock64() - t0 > lim) {
-              *abort_flag = 1;
-              seen = false;
-              break;
-            }
-          }
+        // the producer loads a down tile's A by TMA: each warp only arrives
+        // (for its 32 threads) once the stage is free
+        for (int kb = 0; kb < kb_n; ++kb, ++it) {
+          const int s = it % kFStages;
+          const uint32_t ph = (it / kFStages) & 1;
+          bool free_stage = true;
+          if (lane == 0) free_stage = mbar_wait(&empty[s], ph ^ 1, abort_flag, lim);
+          free_stage = __shfl_sync(0xffffffffu, free_stage, 0);
+          if (!free_stage) { ok = false; break; }
+          if (lane == 0) mbar_arrive_n(&full[s], 32);
+          __syncwarp();
         }
-        seen = __shfl_sync(0xffffffffu, seen, 0);
-        __syncwarp();
-        if (!seen) { ok = false; break; }
-      }
-      const __nv_bfloat16* src_base = tc.up ? a.x : a.h;
-      const size_t ld = tc.up ? (size_t)a.x_ld : (size_t)a.h_ld;
-      const __nv_bfloat16* src[8];
-      uint32_t nbytes[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        if (pr[i] >= 0) {
-          src[i] = src_base + (size_t)pr[i] * ld + chunk * 8;
-          nbytes[i] = 16;
-        } else {
-          src[i] = src_base;
-          nbytes[i] = 0;  // zero-fill rows past the group's segment
-        }
-      }
-      for (int kb = 0; kb < kb_n; ++kb, ++it) {
-        const int s = it % kFStages;
-        const uint32_t ph = (it / kFStages) & 1;
-        if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, lim)) { ok = false; break; }
-        uint8_t* dstA = sA + s * kABytes;
+      } else {
+        const __nv_bfloat16* src[8];
+        uint32_t nbytes[8];
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
-          const int rr = r0 + 16 * i;
-          cp_async16(dstA + rr * 128 + ((chunk ^ (rr & 7)) << 4), src[i] + kb * kBK, nbytes[i]);
+          if (pr[i] >= 0) {
+            src[i] = a.x + (size_t)pr[i] * a.x_ld + chunk * 8;
+            nbytes[i] = 16;
+          } else {
+            src[i] = a.x;
+            nbytes[i] = 0;  // zero-fill rows past the group's segment
+          }
         }
-        cp_async_arrive_noinc(&full[s]);  // arrives when this thread's copies land
+        for (int kb = 0; kb < kb_n; ++kb, ++it) {
+          const int s = it % kFStages;
+          const uint32_t ph = (it / kFStages) & 1;
+          if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, lim)) { ok = false; break; }
+          uint8_t* dstA = sA + s * kABytes;
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const int rr = r0 + 16 * i;
+            cp_async16(dstA + rr * 128 + ((chunk ^ (rr & 7)) << 4), src[i] + kb * kBK, nbytes[i]);
+          }
+          cp_async_arrive_noinc(&full[s]);  // arrives when this thread's copies land
+        }
       }
       if (has_next) {
 #pragma unroll
@@ -342,8 +370,8 @@ __global__ void __launch_bounds__(kFThreads, 1)
   if (threadIdx.x == 0 && *abort_flag) atomicCAS(a.status, 0, (int)MSI_ERR_TIMEOUT);
 }
 
-cudaError_t launch_fused_wave(const CUtensorMap& tmW13, const CUtensorMap& tmW2, const FusedArgs& a,
-                              const WaveParams& w, int grid, cudaStream_t s) {
+cudaError_t launch_fused_wave(const CUtensorMap& tmW13, const CUtensorMap& tmW2, const CUtensorMap& tmH,
+                              const FusedArgs& a, const WaveParams& w, int grid, cudaStream_t s) {
   static std::atomic<unsigned long long> attr_done{0};
   cudaError_t e = smem_attr_once(fused_wave_kernel, kFSmem, attr_done);
   if (e != cudaSuccess) return e;
@@ -360,7 +388,7 @@ cudaError_t launch_fused_wave(const CUtensorMap& tmW13, const CUtensorMap& tmW2,
   cfg.stream = s;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, fused_wave_kernel, tmW13, tmW2, a, w);
+  return cudaLaunchKernelEx(&cfg, fused_wave_kernel, tmW13, tmW2, tmH, a, w);
 }
 
 }  // namespace msi

@@ -172,8 +172,8 @@ cudaError_t launch_gemm_pair(int mode, const CUtensorMap& tmA, const CUtensorMap
                              const GemmArgs& a, int max_pairs, cudaStream_t s);
 // Gate-up and down of one wave in one cooperative launch of `grid` CTAs
 // (at most one per SM); tmW13 / tmW2 as the pool maps of the two projections.
-cudaError_t launch_fused_wave(const CUtensorMap& tmW13, const CUtensorMap& tmW2, const FusedArgs& a,
-                              const WaveParams& w, int grid, cudaStream_t s);
+cudaError_t launch_fused_wave(const CUtensorMap& tmW13, const CUtensorMap& tmW2, const CUtensorMap& tmH,
+                              const FusedArgs& a, const WaveParams& w, int grid, cudaStream_t s);
 // The same on CTA pairs (256-row tiles, gemm_fused_pair.cu); at most
 // `max_pairs` pairs, never more than can be resident at once.
 cudaError_t launch_fused_wave_pair(const CUtensorMap& tmW13, const CUtensorMap& tmW2,

@@ -993,7 +993,7 @@ msi_status routed_ffn(msi_plan* p, FwdCtx& f, int ng, int grid1, int grid2, long
       return MSI_OK;
     }
     const int grid = (int)std::min<long long>(p->sms - spare, std::max<long long>(1, tiles));
-    LAUNCH(p, MSI_K_FFN, f.cs, launch_fused_wave(p->tm_w13, p->tm_w2, fa, wv, grid, f.cs));
+    LAUNCH(p, MSI_K_FFN, f.cs, launch_fused_wave(p->tm_w13, p->tm_w2, f.tm_h, fa, wv, grid, f.cs));
     return MSI_OK;
   }
   GemmArgs g1 = gateup_args(p, f, groups, ng, total, at<__nv_bfloat16>(f.ws, f.L.h));
