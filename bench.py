@@ -199,9 +199,11 @@ class ClockSampler:
 # ---------------------------------------------------------------------------
 
 class Workload:
-    def __init__(self, name: str, batch: int | None = None, predict: bool = False, windows=None):
+    def __init__(self, name: str, batch: int | None = None, predict: bool = False, windows=None,
+                 early_staging: bool = False):
         """windows: pinned host windows of an earlier workload with the same
-        layer shape and weights (reused, not regenerated)."""
+        layer shape and weights (reused, not regenerated); early_staging:
+        streamed calls copy their first misses while they route."""
         import torch
 
         import synth
@@ -238,7 +240,7 @@ class Workload:
         self.plan = api.Plan(n_layers=L, n_experts=E, top_k=cfg.top_k, hidden=H, inter=I,
                              n_slots=cfg.n_slots, host_windows=self.windows,
                              has_shared=cfg.has_shared, shared_w=shared_w, shared_gate_w=gate_w,
-                             wdtype=cfg.wdtype)
+                             wdtype=cfg.wdtype, early_staging=early_staging)
         self.cs = torch.cuda.Stream()
         self.ss = torch.cuda.Stream()
         self.out = torch.empty_like(self.x)
@@ -512,7 +514,8 @@ def run_ours(args):
         torch.cuda.set_device(0)
     import __graft_entry__
     __graft_entry__.build()
-    w = Workload(args.workload, args.batch, args.predict)
+    early = not args.no_early_staging and args.source == "none"
+    w = Workload(args.workload, args.batch, args.predict, early_staging=early)
     cfg = w.cfg
     src = None
     if args.source != "none":
@@ -662,7 +665,9 @@ def run_ours(args):
         "config": {"workload": args.workload, "tokens": cfg.tokens, "hidden": cfg.hidden,
                    "experts": cfg.n_experts, "top_k": cfg.top_k, "inter": cfg.inter,
                    "shared_expert": cfg.has_shared, "slots": cfg.n_slots,
-                   "residency": "LRU waves of %d, staged from pinned host windows" % (cfg.n_slots // 2)
+                   "residency": "LRU waves of %d, staged from pinned host windows%s" % (
+                       cfg.n_slots // 2, "; first misses copied early, while the call routes"
+                       if early and cfg.lru and cfg.n_layers == 1 else "")
                    if cfg.lru else "all experts resident",
                    "layers": w.L,
                    "weights": "bf16" if cfg.wdtype == 0 else "q4g32",
@@ -813,6 +818,9 @@ def main():
     ap.add_argument("--batch", type=int, default=64, help="decode48: rows per decode step")
     ap.add_argument("--predict", action="store_true",
                     help="decode48: next-layer prediction with the two-bank prefetch")
+    ap.add_argument("--no-early-staging", action="store_true",
+                    help="staged workloads: no early-staging buffer (misses copied only after "
+                         "the call's plan)")
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--source", default="none", choices=["none", "buffered", "direct"],

@@ -353,6 +353,22 @@ msi_status msi_plan_reset(msi_plan* plan, uint64_t* new_epoch);
  * out of range.  Nothing is allocated; msi_plan_reset does not disarm. */
 msi_status msi_fault_inject(msi_plan* plan, int kind, int layer, int expert);
 
+/* Optional early-staging buffer for streamed calls (a library convenience;
+ * the paper's runtime copies each miss after its plan).  buf: caller-owned
+ * device memory, 16-byte aligned, bytes >= extent_bytes (at most
+ * wave_capacity extents of it are used); NULL detaches (after waiting for
+ * the calls that used it).  A streamed call whose T * top_k >= 8 * n_experts
+ * (every expert then almost surely needed) copies, on its stage stream and
+ * while it routes, the extents of the layer's non-resident experts in
+ * ascending order (the order the LRU-wave plan stages misses) into the
+ * buffer (in a host-buffer call, after its rows have crossed); its waves
+ * then copy those extents device to device into their slots instead of from
+ * the host windows.  Victims, generations, publication and the slot trace
+ * are those of a call without the buffer; outputs are bit-identical.  Not
+ * used with a source attached.  The buffer must stay allocated until it is
+ * detached or the plan destroyed. */
+msi_status msi_plan_set_bounce(msi_plan* plan, void* buf, size_t bytes);
+
 /* Limit of every bounded device wait of the plan's kernels, in SM clock
  * cycles (clock64); cycles <= 0 restores the default of 4e9 (~2 s at GB300
  * clocks).  A wait that runs out raises MSI_ERR_TIMEOUT in the forward's

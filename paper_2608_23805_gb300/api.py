@@ -46,7 +46,10 @@ class Plan:
 
     def __init__(self, *, n_layers, n_experts, top_k, hidden, inter, n_slots, host_windows,
                  has_shared=False, shared_w=None, shared_gate_w=None, wdtype=N.MSI_W_BF16,
-                 slot_pool=None, extent_off=None, wave_capacity=0, wait_timeout_s=0.0):
+                 slot_pool=None, extent_off=None, wave_capacity=0, wait_timeout_s=0.0,
+                 early_staging=False):
+        """early_staging: give streamed calls an early-staging buffer of one
+        wave of extents (msi_plan_set_bounce)."""
         lib = N.lib()
         self.E, self.k, self.H, self.I = n_experts, top_k, hidden, inter
         self.n_layers, self.S = n_layers, n_slots
@@ -75,6 +78,12 @@ class Plan:
         N.check(lib.msi_plan_create(ctypes.byref(d), ctypes.byref(h)), "msi_plan_create")
         self.h = h
         self._ws = {}
+        self.bounce = None
+        if early_staging:
+            C = wave_capacity if wave_capacity > 0 else n_slots // 2
+            self.bounce = torch.empty(C * self.extent_bytes, dtype=torch.uint8, device="cuda")
+            N.check(lib.msi_plan_set_bounce(self.h, self.bounce.data_ptr(), self.bounce.numel()),
+                    "msi_plan_set_bounce")
 
     # -- residency ---------------------------------------------------------
     def stage(self, slot: int, layer: int, expert: int, stream=None) -> int:

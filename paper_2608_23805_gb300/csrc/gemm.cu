@@ -437,17 +437,16 @@ __global__ void __launch_bounds__(Cfg<MODE>::kThreads, 1)
       const uint32_t ph = (it / C::kStg) & 1;
       if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, lim)) { ok = false; break; }
       // this thread's half row: 32 codes (16 bytes) under one group scale
-      const uint4 cw = *reinterpret_cast<const uint4*>(raw_codes + r * (kBN * kRawRowBytes) +
-                                                        d * kRawRowBytes + half * 16);
+      const uint4 cw = ld_shared_v4(smem_u32(raw_codes + r * (kBN * kRawRowBytes) + d * kRawRowBytes + half * 16));
       const uint32_t sc = (it & 1) ? sc_cur.y : sc_cur.x;
       const float sv = __half2float(__ushort_as_half((unsigned short)(half ? sc >> 16 : sc & 0xFFFFu)));
       const uint64_t sx2 = f32x2(sv, sv), nx2 = f32x2(-136.0f * sv, -136.0f * sv);
-      uint8_t* dst_row = sB + s * kBBytes + d * 128;
+      const uint32_t dst_row = smem_u32(sB + s * kBBytes + d * 128);
       const uint32_t words[4] = {cw.x, cw.y, cw.z, cw.w};
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
         const int c = half * 4 + j;  // 16-byte chunk of the 128-byte row
-        *reinterpret_cast<uint4*>(dst_row + ((c ^ (d & 7)) << 4)) = dequant8(words[j], sx2, nx2);
+        st_shared_v4(dst_row + ((c ^ (d & 7)) << 4), dequant8(words[j], sx2, nx2));
       }
       fence_proxy_async_smem();
       __syncwarp();

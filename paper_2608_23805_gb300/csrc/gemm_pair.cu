@@ -406,14 +406,14 @@ __global__ void __launch_bounds__(PCfg<MODE>::kThreads, 1)
       const int s = it % kPStages;
       const uint32_t ph = (it / kPStages) & 1;
       if (!mbar_wait(&empty[s], ph ^ 1, abort_flag, lim)) break;
-      const uint2 cw = *reinterpret_cast<const uint2*>(raw_codes + r * (128 * kPRawRow) + d * kPRawRow + qt * 8);
+      const uint2 cw = ld_shared_v2(smem_u32(raw_codes + r * (128 * kPRawRow) + d * kPRawRow + qt * 8));
       const uint32_t sc = (it & 1) ? sc_cur.y : sc_cur.x;
       const float sv = __half2float(__ushort_as_half((unsigned short)(qt >= 2 ? sc >> 16 : sc & 0xFFFFu)));
       const uint64_t sx2 = f32x2(sv, sv), nx2 = f32x2(-136.0f * sv, -136.0f * sv);
-      uint8_t* dst_row = sB + s * kPB + d * 128;
+      const uint32_t dst_row = smem_u32(sB + s * kPB + d * 128);
       const int c0 = qt * 2;  // 16-byte chunks c0, c0 + 1 of the 128-byte row
-      *reinterpret_cast<uint4*>(dst_row + ((c0 ^ (d & 7)) << 4)) = dequant8(cw.x, sx2, nx2);
-      *reinterpret_cast<uint4*>(dst_row + (((c0 + 1) ^ (d & 7)) << 4)) = dequant8(cw.y, sx2, nx2);
+      st_shared_v4(dst_row + ((c0 ^ (d & 7)) << 4), dequant8(cw.x, sx2, nx2));
+      st_shared_v4(dst_row + (((c0 + 1) ^ (d & 7)) << 4), dequant8(cw.y, sx2, nx2));
       fence_proxy_async_smem();
       __syncwarp();
       if (lane == 0) {

@@ -274,6 +274,15 @@ struct msi_plan {
   // MSI_FAULT_DEVICE_WAIT: the next forward on this layer runs its tensor-core
   // kernels with one wait that nothing ends (-1: none armed)
   int stall_layer = -1;
+  // early staging (msi_plan_set_bounce): a caller-owned device buffer of
+  // bounce_cap extents; during a streamed call, the extents copied into it
+  // while the call routes (spec_idx[e]: index in the buffer, -1 if none; for
+  // layer spec_layer only), and an event after the call's last read of it
+  char* bounce = nullptr;
+  int bounce_cap = 0;
+  int spec_layer = -1;
+  std::vector<int> spec_idx;
+  cudaEvent_t ev_bounce = nullptr;
   std::mutex mu;
 
   explicit msi_plan(int S) : holds(S) {
@@ -557,19 +566,29 @@ msi_status stage_enqueue(msi_plan* p, int layer, const std::vector<WaveEntry>& m
       return fail == MSI_ERR_SOURCE ? MSI_ERR_SOURCE : fail;
     }
   } else {
-  // one copy per run of extents that continue each other in both the host
-  // window and the slot pool (consecutive experts into consecutive slots):
-  // large copies reach the host link's rate, per-extent copies fall short
+  // one copy per run of extents that continue each other in both the source
+  // and the slot pool (consecutive experts into consecutive slots): large
+  // copies reach the host link's rate, per-extent copies fall short.  An
+  // extent already copied into the early-staging buffer during this call's
+  // routing comes from there, device to device.
+  auto early = [&](const WaveEntry& m) {
+    return p->spec_layer == layer && p->spec_idx[m.expert] >= 0;
+  };
+  auto from_of = [&](const WaveEntry& m) -> const char* {
+    return early(m) ? p->bounce + (size_t)p->spec_idx[m.expert] * eb : src_of(m);
+  };
   for (size_t i = 0; i < misses.size();) {
-    const char* src = src_of(misses[i]);
+    const bool dev = early(misses[i]);
+    const char* src = from_of(misses[i]);
     char* dst = dst_of(misses[i]);
     uint64_t bytes = eb;
     size_t j = i + 1;
-    while (j < misses.size() && src_of(misses[j]) == src + bytes && dst_of(misses[j]) == dst + bytes) {
+    while (j < misses.size() && early(misses[j]) == dev && from_of(misses[j]) == src + bytes &&
+           dst_of(misses[j]) == dst + bytes) {
       bytes += eb;
       ++j;
     }
-    CK(cudaMemcpyAsync(dst, src, bytes, cudaMemcpyHostToDevice, stage));
+    CK(cudaMemcpyAsync(dst, src, bytes, dev ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice, stage));
     i = j;
   }
   }
@@ -1256,6 +1275,10 @@ msi_status msi_plan_destroy(msi_plan* p) {
     }
     if (p->ev_io_a) cudaEventDestroy(p->ev_io_a);
     if (p->ev_io_b) cudaEventDestroy(p->ev_io_b);
+    if (p->ev_bounce) {
+      cudaEventSynchronize(p->ev_bounce);
+      cudaEventDestroy(p->ev_bounce);
+    }
     if (swap) cudaSetDevice(cur);
   }
   delete p;
@@ -1556,6 +1579,52 @@ msi_status forward_streamed(msi_plan* p, int layer, const void* x, int T, const 
   f.cs = reinterpret_cast<cudaStream_t>(compute);
   apply_io(f, hio);
   cudaStream_t ss = reinterpret_cast<cudaStream_t>(stage);
+  // Early staging: when the call is long enough that every expert is almost
+  // surely needed (T k >= 8 E), the extents of the first misses the waves
+  // would stage (the non-resident experts, ascending, as the LRU-wave plan
+  // orders misses) are copied into the caller's early-staging buffer while
+  // the call routes; the waves then copy them device to device.  Residency,
+  // victims, publication and the trace are decided by the plan as always;
+  // an extent copied early but not needed is simply not used.
+  struct SpecEnd {
+    msi_plan* p;
+    cudaStream_t ss;
+    bool on = false;
+    ~SpecEnd() {
+      if (!on) return;
+      cudaEventRecord(p->ev_bounce, ss);  // after every read of the buffer in this call
+      p->spec_layer = -1;
+    }
+  } spec_end{p, ss};
+  if (p->bounce != nullptr && p->src == nullptr && T > 0 && (long long)T * d.top_k >= 8LL * E) {
+    std::fill(p->spec_idx.begin(), p->spec_idx.end(), -1);
+    CK(cudaStreamWaitEvent(ss, p->ev_bounce, 0));  // the previous call's reads of the buffer
+    // a host-buffer call's rows cross the host link first (routing waits on them)
+    if (f.x_ready != nullptr) CK(cudaStreamWaitEvent(ss, f.x_ready, 0));
+    const uint64_t eb = d.extent_bytes;
+    int n = 0;
+    for (int e = 0; e < E && n < p->bounce_cap; ++e)
+      if (p->where[(size_t)layer * E + e] < 0) p->spec_idx[e] = n++;
+    for (int e = 0; e < E;) {
+      if (p->spec_idx[e] < 0) {
+        ++e;
+        continue;
+      }
+      // runs of experts that continue each other in the host windows
+      const char* src = static_cast<const char*>(d.host_windows) + p->off[(size_t)layer * E + e];
+      uint64_t bytes = eb;
+      int j = e + 1;
+      while (j < E && p->spec_idx[j] == p->spec_idx[j - 1] + 1 &&
+             static_cast<const char*>(d.host_windows) + p->off[(size_t)layer * E + j] == src + bytes) {
+        bytes += eb;
+        ++j;
+      }
+      CK(cudaMemcpyAsync(p->bounce + (size_t)p->spec_idx[e] * eb, src, bytes, cudaMemcpyHostToDevice, ss));
+      e = j;
+    }
+    p->spec_layer = layer;
+    spec_end.on = true;
+  }
   static thread_local TableParams tp;
   tp.E = 0;
   tp.layer = layer;
@@ -1962,6 +2031,33 @@ msi_status msi_fault_inject(msi_plan* p, int kind, int layer, int expert) {
     p->stall_layer = layer;
   else
     p->faults[obj_key(layer, expert)] = kind;
+  return MSI_OK;
+}
+
+msi_status msi_plan_set_bounce(msi_plan* p, void* buf, size_t bytes) {
+  if (p == nullptr) return MSI_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> g(p->mu);
+  if (p->dying) return MSI_ERR_SHUT_DOWN;
+  if (buf == nullptr) {
+    // the caller may free the buffer once the calls that used it completed
+    if (p->ev_bounce != nullptr) CK(cudaEventSynchronize(p->ev_bounce));
+    p->bounce = nullptr;
+    p->bounce_cap = 0;
+    return MSI_OK;
+  }
+  if ((uintptr_t)buf % 16 || bytes < p->d.extent_bytes) return MSI_ERR_INVALID_ARG;
+  msi_status dst = check_device(p);
+  if (dst != MSI_OK) return dst;
+  if (p->ev_bounce == nullptr) {
+    cudaEvent_t e = nullptr;
+    CK(cudaEventCreateWithFlags(&e, cudaEventDisableTiming));
+    p->ev_bounce = e;
+  } else {
+    CK(cudaEventSynchronize(p->ev_bounce));
+  }
+  p->bounce = static_cast<char*>(buf);
+  p->bounce_cap = (int)std::min<uint64_t>(bytes / p->d.extent_bytes, (uint64_t)p->C);
+  p->spec_idx.assign(p->d.n_experts, -1);
   return MSI_OK;
 }
 

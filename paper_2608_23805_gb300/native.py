@@ -115,6 +115,7 @@ _SIGS = {
     "msi_plan_reset": (ctypes.c_int, [_P, ctypes.POINTER(ctypes.c_uint64)]),
     "msi_fault_inject": (ctypes.c_int, [_P, ctypes.c_int, ctypes.c_int, ctypes.c_int]),
     "msi_plan_set_wait_cycles": (ctypes.c_int, [_P, ctypes.c_int64]),
+    "msi_plan_set_bounce": (ctypes.c_int, [_P, _P, ctypes.c_size_t]),
     "msi_source_open": (ctypes.c_int, [ctypes.POINTER(msi_source_desc), ctypes.POINTER(_P)]),
     "msi_source_close": (ctypes.c_int, [_P]),
     "msi_source_stats_read": (ctypes.c_int, [_P, ctypes.POINTER(msi_source_stats)]),
