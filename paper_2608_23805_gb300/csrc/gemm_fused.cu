@@ -24,10 +24,10 @@
 // counter, orders the h writes before its async-proxy reads
 // (fence.proxy.async.global) and loads the down tile's A rows from h by TMA.
 //
-// Progress: tiles are taken in a static round-robin (t = blockIdx.x +
-// i * gridDim.x), so every CTA processes its tiles in increasing order and
-// all gate-up tiles precede all down tiles.  A CTA waiting on a down tile
-// waits for gate-up tiles of lower index, which their CTAs reach without
+// Progress: tiles follow a static schedule (FusedSched: gate-up tiles
+// round-robin, down tiles weighted to even out the CTAs' work), in which
+// every CTA runs its gate-up tiles before its down tiles.  A CTA waiting on
+// a down tile waits for gate-up tiles, which their CTAs reach without
 // waiting on anything (no down tile comes before a gate-up tile in any CTA's
 // sequence).  The launch is cooperative, so every CTA is resident.
 //
@@ -165,14 +165,14 @@ __global__ void __launch_bounds__(kFThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  const int total = s_mt[ng] * (a.nt_up + a.nt_dn);
+  const FusedSched sc(s_mt[ng] * a.nt_up, s_mt[ng] * a.nt_dn, gridDim.x, blockIdx.x, a.sched_w);
   const long long lim = a.wait_limit;
 
   if (warp == 5) {
     // ------------------------------------------------------------- TMA producer (B)
     if (lane == 0) {
       uint32_t it = 0;
-      for (int t = blockIdx.x; t < total; t += gridDim.x) {
+      for (int t = sc.first(); t >= 0; t = sc.next(t)) {
         const FTile tc = fdecode(a, ng, s_mt, t);
         const int kb_n = tc.up ? a.kb_up : a.kb_dn;
         const int r0 = tc.up ? s_slot[tc.g] * a.w13_rows_per_slot + tc.n * 128
@@ -227,7 +227,7 @@ __global__ void __launch_bounds__(kFThreads, 1)
     // ------------------------------------------------------------- MMA issuer
     if (lane == 0) {
       uint32_t it = 0, jt = 0;
-      for (int t = blockIdx.x; t < total; t += gridDim.x, ++jt) {
+      for (int t = sc.first(); t >= 0; t = sc.next(t), ++jt) {
         const FTile tc = fdecode(a, ng, s_mt, t);
         const int kb_n = tc.up ? a.kb_up : a.kb_dn;
         const uint32_t acc = jt & 1, aph = (jt >> 1) & 1;
@@ -262,7 +262,7 @@ __global__ void __launch_bounds__(kFThreads, 1)
     // ------------------------------------------------------------- epilogue
     uint32_t jt = 0;
     if (a.stall && threadIdx.x == 0) mbar_wait(never, 0, abort_flag, lim);  // runs out: abort
-    for (int t = blockIdx.x; t < total; t += gridDim.x, ++jt) {
+    for (int t = sc.first(); t >= 0; t = sc.next(t), ++jt) {
       const FTile tc = fdecode(a, ng, s_mt, t);
       const int cnt = s_cnt[tc.g];
       const size_t rb = (size_t)s_rb[tc.g];
@@ -307,10 +307,12 @@ __global__ void __launch_bounds__(kFThreads, 1)
       }
     };
     int pr[8], pr_next[8];
-    if (blockIdx.x < total) tile_rows(blockIdx.x, pr);
-    for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
-      const bool has_next = t + (int)gridDim.x < total;
-      if (has_next) tile_rows(t + gridDim.x, pr_next);
+    const int t_first = sc.first();
+    if (t_first >= 0) tile_rows(t_first, pr);
+    for (int t = t_first; t >= 0 && ok; t = sc.next(t)) {
+      const int t_next = sc.next(t);
+      const bool has_next = t_next >= 0;
+      if (has_next) tile_rows(t_next, pr_next);
       const FTile tc = fdecode(a, ng, s_mt, t);
       const int kb_n = tc.up ? a.kb_up : a.kb_dn;
       if (!tc.up) {

@@ -9,7 +9,8 @@
 // each holding 128 of its A rows and 128 of its B rows, so per unit of tensor
 // work an SM receives a third less operand data than with single-CTA tiles.
 //
-// Tile order (static round-robin over pairs, t = pair + i * npairs):
+// Tiles (FusedSched over the pairs: gate-up tiles round-robin, down tiles
+// weighted to even out the pairs' work):
 //   t <  n_up: gate-up pair tile (g, m2, n): h[256 rows, 128 n .. 128 n + 128)
 //              (the even CTA holds the gate rows of B, the odd CTA the up rows);
 //   t >= n_up: down pair tile (g, m2, n): y[256 rows, 256 n .. 256 n + 256)
@@ -18,10 +19,10 @@
 // epilogues of both CTAs of every gate-up tile of that m-tile: each publishes
 // on the m-tile's counter (stores, a gpu-scope fence, a release add) and the
 // down tile's A loads wait until the counter reaches 2 * (I / 128).  Every
-// pair processes its tiles in increasing order with all gate-up tiles first,
-// so a pair waiting on a down tile waits only for gate-up tiles of lower
-// index, which their pairs reach without waiting; the grid never exceeds the
-// clusters that can be resident at once.
+// pair processes all its gate-up tiles before its down tiles, so a pair
+// waiting on a down tile waits only for gate-up tiles, which their pairs
+// reach without waiting; the grid never exceeds the clusters that can be
+// resident at once.
 //
 // Synchronisation within a pair is that of gemm_pair.cu: each CTA's loads
 // complete on its own `full` barrier, the odd CTA's relay forwards completed
@@ -188,16 +189,16 @@ __global__ void __launch_bounds__(QCfg<Q4>::kThreads, 1)
   cluster_sync_all();  // both CTAs' barriers initialised before any cross-CTA arrival
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  const int total = s_pt[ng] * (a.nt_up + a.nt_dn);
   const int pair = blockIdx.x >> 1;
   const int npairs = gridDim.x >> 1;
+  const FusedSched sc(s_pt[ng] * a.nt_up, s_pt[ng] * a.nt_dn, npairs, pair, a.sched_w);
   const long long lim = a.wait_limit;
 
   if (warp == 5) {
     // ------------------------------------------------------------- TMA producer (B)
     if (lane == 0 && !Q4) {
       uint32_t it = 0;
-      for (int t = pair; t < total; t += npairs) {
+      for (int t = sc.first(); t >= 0; t = sc.next(t)) {
         const QTile tc = qdecode(a, ng, s_pt, t);
         const int kb_n = tc.up ? a.kb_up : a.kb_dn;
         // gate-up: the even CTA holds 128 gate rows, the odd CTA the matching
@@ -231,7 +232,7 @@ __global__ void __launch_bounds__(QCfg<Q4>::kThreads, 1)
       // (gate-up: gate rows in the even CTA, up rows in the odd one; down:
       // W2 rows 256 n + 128 r)
       uint32_t it = 0;
-      for (int t = pair; t < total; t += npairs) {
+      for (int t = sc.first(); t >= 0; t = sc.next(t)) {
         const QTile tc = qdecode(a, ng, s_pt, t);
         const int kb_n = tc.up ? a.kb_up : a.kb_dn;
         const int qrow = tc.up ? s_slot[tc.g] * a.q13_rows_per_slot + (rank ? a.w13_up_off : 0) + tc.n * 128
@@ -260,7 +261,7 @@ __global__ void __launch_bounds__(QCfg<Q4>::kThreads, 1)
     if (lane == 0 && leader) {
       // ----------------------------------------------------------- MMA issuer
       uint32_t it = 0, jt = 0;
-      for (int t = pair; t < total; t += npairs, ++jt) {
+      for (int t = sc.first(); t >= 0; t = sc.next(t), ++jt) {
         const QTile tc = qdecode(a, ng, s_pt, t);
         const int kb_n = tc.up ? a.kb_up : a.kb_dn;
         const uint32_t acc = jt & 1, aph = (jt >> 1) & 1;
@@ -290,7 +291,7 @@ __global__ void __launch_bounds__(QCfg<Q4>::kThreads, 1)
       // ------------------------------------------------------ stage relay (odd)
       uint32_t it = 0;
       bool ok = true;
-      for (int t = pair; t < total && ok; t += npairs) {
+      for (int t = sc.first(); t >= 0 && ok; t = sc.next(t)) {
         const QTile tc = qdecode(a, ng, s_pt, t);
         const int kb_n = tc.up ? a.kb_up : a.kb_dn;
         for (int kb = 0; kb < kb_n; ++kb, ++it) {
@@ -315,7 +316,7 @@ __global__ void __launch_bounds__(QCfg<Q4>::kThreads, 1)
     const uint32_t lead_tempty[2] = {mapa_shared(smem_u32(&tempty[0]), 0),
                                      mapa_shared(smem_u32(&tempty[1]), 0)};
     if (a.stall && threadIdx.x == 0) mbar_wait(never, 0, abort_flag, lim);  // runs out: abort
-    for (int t = pair; t < total; t += npairs, ++jt) {
+    for (int t = sc.first(); t >= 0; t = sc.next(t), ++jt) {
       const QTile tc = qdecode(a, ng, s_pt, t);
       const int cnt = s_cnt[tc.g];
       const size_t rb = (size_t)s_rb[tc.g];
@@ -365,10 +366,12 @@ __global__ void __launch_bounds__(QCfg<Q4>::kThreads, 1)
       }
     };
     int pr[8], pr_next[8];
-    if (pair < total) tile_rows(pair, pr);
-    for (int t = pair; t < total && ok; t += npairs) {
-      const bool has_next = t + npairs < total;
-      if (has_next) tile_rows(t + npairs, pr_next);
+    const int t_first = sc.first();
+    if (t_first >= 0) tile_rows(t_first, pr);
+    for (int t = t_first; t >= 0 && ok; t = sc.next(t)) {
+      const int t_next = sc.next(t);
+      const bool has_next = t_next >= 0;
+      if (has_next) tile_rows(t_next, pr_next);
       const QTile tc = qdecode(a, ng, s_pt, t);
       const int kb_n = tc.up ? a.kb_up : a.kb_dn;
       if (!tc.up) {
@@ -440,12 +443,14 @@ __global__ void __launch_bounds__(QCfg<Q4>::kThreads, 1)
     uint32_t it = 0;
     bool ok = true;
     // the next stage pair's scales are loaded one pair ahead, across tiles
-    uint2 nxt = pair < total ? __ldg(reinterpret_cast<const uint2*>(scale_row(pair))) : make_uint2(0, 0);
-    for (int t = pair; t < total && ok; t += npairs) {
+    const int t_first = sc.first();
+    uint2 nxt = t_first >= 0 ? __ldg(reinterpret_cast<const uint2*>(scale_row(t_first))) : make_uint2(0, 0);
+    for (int t = t_first; t >= 0 && ok; t = sc.next(t)) {
       const QTile tc = qdecode(a, ng, s_pt, t);
       const int kb_n = tc.up ? a.kb_up : a.kb_dn;  // even (K a multiple of 128)
       const uint8_t* srow = scale_row(t);
-      const uint8_t* srow_next = t + npairs < total ? scale_row(t + npairs) : nullptr;
+      const int t_next = sc.next(t);
+      const uint8_t* srow_next = t_next >= 0 ? scale_row(t_next) : nullptr;
       uint2 cur = make_uint2(0, 0);
       for (int kb = 0; kb < kb_n; ++kb, ++it) {
         if ((kb & 1) == 0) {

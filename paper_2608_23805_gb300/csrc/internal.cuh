@@ -148,6 +148,7 @@ struct FusedArgs {
   const GenWord* genwords;  // published (generation, object) per slot
   int* ready_clear;
   int n_ready_clear;
+  int sched_w;              // FusedSched: down tiles one gate-up tile is worth (>= 1)
   // 4-bit waves (gemm_fused_pair.cu, Q4): codes by TMA through the code maps,
   // fp16 scales read from the slot pool
   const uint8_t* q4_pool;
@@ -221,6 +222,41 @@ __device__ __forceinline__ uint4 ld_shared_v4(uint32_t addr) {
                : "memory");
   return v;
 }
+
+// Static tile schedule of the fused kernels.  U gate-up tiles (indices
+// 0..U-1) then D down tiles (U..U+D-1) over P workers (CTAs, or CTA pairs).
+// Gate-up tiles go round-robin: worker c takes c, c + P, ...; the first
+// U mod P workers get one more than the rest.  A gate-up tile is worth w
+// down tiles, so the down tiles first make up that difference (phase A: the
+// first w * (P - U mod P) down tiles round-robin over the workers with one
+// gate-up tile fewer), then go round-robin over all workers (phase B).
+// Every tile has exactly one worker, and every worker runs its gate-up
+// tiles first and then its down tiles, each in increasing index order.
+struct FusedSched {
+  int U, D, P, c, n_hi, n_lo, DA;
+  __device__ __forceinline__ FusedSched(int U_, int D_, int P_, int c_, int w) : U(U_), D(D_), P(P_), c(c_) {
+    n_hi = U % P;
+    n_lo = P - n_hi;
+    DA = n_hi > 0 ? min(D, w * n_lo) : 0;
+  }
+  // the worker's first down tile, or -1
+  __device__ __forceinline__ int down_first() const {
+    if (c >= n_hi && c - n_hi < DA) return U + (c - n_hi);
+    const int i = DA + c;
+    return i < D ? U + i : -1;
+  }
+  __device__ __forceinline__ int first() const { return c < U ? c : down_first(); }
+  // the worker's tile after t, or -1
+  __device__ __forceinline__ int next(int t) const {
+    if (t < U) return t + P < U ? t + P : down_first();
+    const int i = t - U;
+    if (i < DA) {
+      if (i + n_lo < DA) return t + n_lo;
+      return DA + c < D ? U + DA + c : -1;
+    }
+    return i + P < D ? t + P : -1;
+  }
+};
 
 __device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");

@@ -955,6 +955,7 @@ msi_status routed_ffn(msi_plan* p, FwdCtx& f, int ng, int grid1, int grid2, long
     fa.nt_dn = d.hidden / kBN;
     fa.kb_up = d.hidden / kBK;
     fa.kb_dn = d.inter / kBK;
+    fa.sched_w = std::max(1, fa.kb_up / fa.kb_dn);  // a gate-up tile's K blocks per down tile's
     fa.w13_rows_per_slot = 3 * d.inter;
     fa.w13_up_off = d.inter;
     fa.w2_rows_per_slot = 3 * d.hidden;
