@@ -294,8 +294,10 @@ __global__ void __launch_bounds__(kFThreads, 1)
     const int r0 = gt >> 3;                           // rows r0 + 16 i
     uint32_t it = 0;
     bool ok = true;
-    // this thread's eight x rows of gate-up tile t (by token; -1 past the
-    // group's segment), loaded one tile ahead
+    // this thread's eight permutation entries of gate-up tile t (routed row
+    // token * k + j; -1 past the group's segment), loaded one tile ahead and
+    // first used at that tile's start, so the loads' latency is not waited
+    // for at the start of the current tile
     auto tile_rows = [&](int t, int (&pr)[8]) {
       const FTile tc = fdecode(a, ng, s_mt, t);
       const int cnt = s_cnt[tc.g];
@@ -303,7 +305,7 @@ __global__ void __launch_bounds__(kFThreads, 1)
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
         const int rr = tc.m * kBM + r0 + 16 * i;
-        pr[i] = (!tc.up || rr >= cnt) ? -1 : __ldg(&a.perm[rb + rr]) / a.top_k;
+        pr[i] = (!tc.up || rr >= cnt) ? -1 : __ldg(&a.perm[rb + rr]);
       }
     };
     int pr[8], pr_next[8];
@@ -334,7 +336,7 @@ __global__ void __launch_bounds__(kFThreads, 1)
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
           if (pr[i] >= 0) {
-            src[i] = a.x + (size_t)pr[i] * a.x_ld + chunk * 8;
+            src[i] = a.x + (size_t)(pr[i] / a.top_k) * a.x_ld + chunk * 8;
             nbytes[i] = 16;
           } else {
             src[i] = a.x;

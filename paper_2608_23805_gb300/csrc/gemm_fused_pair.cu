@@ -355,6 +355,9 @@ __global__ void __launch_bounds__(QCfg<Q4>::kThreads, 1)
     const int r0 = gt >> 3;                           // rows r0 + 16 i of this CTA's 128
     uint32_t it = 0;
     bool ok = true;
+    // this thread's eight A rows of tile t: a gate-up tile's permutation
+    // entries (token * k + j), a down tile's h rows; -1 past the group's
+    // segment.  Loaded one tile ahead and first used at that tile's start.
     auto tile_rows = [&](int t, int (&pr)[8]) {
       const QTile tc = qdecode(a, ng, s_pt, t);
       const int cnt = s_cnt[tc.g];
@@ -362,7 +365,7 @@ __global__ void __launch_bounds__(QCfg<Q4>::kThreads, 1)
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
         const int rr = tc.m2 * kQRows + (int)rank * kBM + r0 + 16 * i;
-        pr[i] = rr >= cnt ? -1 : (tc.up ? __ldg(&a.perm[rb + rr]) / a.top_k : rb + rr);
+        pr[i] = rr >= cnt ? -1 : (tc.up ? __ldg(&a.perm[rb + rr]) : rb + rr);
       }
     };
     int pr[8], pr_next[8];
@@ -400,7 +403,7 @@ __global__ void __launch_bounds__(QCfg<Q4>::kThreads, 1)
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
         if (pr[i] >= 0) {
-          src[i] = src_base + (size_t)pr[i] * ld + chunk * 8;
+          src[i] = src_base + (size_t)(tc.up ? pr[i] / a.top_k : pr[i]) * ld + chunk * 8;
           nbytes[i] = 16;
         } else {
           src[i] = src_base;
