@@ -1664,8 +1664,21 @@ msi_status forward_streamed(msi_plan* p, int layer, const void* x, int T, const 
       if (ev != nullptr) cudaStreamWaitEvent(cs, ev, 0);
     }
   } pred_join{f.cs, predict ? p->ev_pjoin : nullptr};
-  st = shared_ffn(p, f, f.cs);  // overlaps the host planning and the first wave's copies
-  if (st != MSI_OK) return st;
+  // The shared expert needs no residency.  A call that will stage at least
+  // two waves of misses (T k >= 8 E: every expert almost surely needed)
+  // runs it on the compute stream right after its first miss wave's GEMMs,
+  // where that stream would otherwise wait for the next wave's copies;
+  // ahead of the hit waves it would hold back their GEMMs and with them the
+  // consumer tickets the next copies wait for.  Other calls run it here,
+  // beside the host's planning.
+  int resident_now = 0;
+  for (int e = 0; e < E; ++e) resident_now += p->where[(size_t)layer * E + e] >= 0;
+  bool late_shared = d.has_shared && T > 0 && (long long)T * d.top_k >= 8LL * E &&
+                           E - resident_now >= 2 * p->C;
+  if (!late_shared) {
+    st = shared_ffn(p, f, f.cs);
+    if (st != MSI_OK) return st;
+  }
   const cudaError_t se = cudaEventSynchronize(p->pool.ev[cev]);
   p->pool.unref(cev);
   if (se != cudaSuccess) return cuda_fail(se, "counts readback");
@@ -1806,6 +1819,15 @@ msi_status forward_streamed(msi_plan* p, int layer, const void* x, int T, const 
     if (st != MSI_OK) return st;
     st = consumer_record(p, used, f.cs);
     if (st != MSI_OK) return st;
+    if (late_shared) {
+      bool any_miss = false;
+      for (const auto& we : waves[w]) any_miss = any_miss || we.miss;
+      if (any_miss || w + 1 == n_waves) {
+        st = shared_ffn(p, f, f.cs);
+        if (st != MSI_OK) return st;
+        late_shared = false;
+      }
+    }
   }
   if (predict) {
     // the predicted counts (the prediction ran beside the waves' GEMMs), then
