@@ -62,6 +62,101 @@ __device__ __forceinline__ void load_stage(const RouterArgs& a, uint8_t* st, int
   }
 }
 
+// Top-k, softmax weights, gap and shared gate of the block's tokens from the
+// logits L[TM][lld] in shared memory (each warp TM / warps tokens), then the
+// block's expert histogram.  ids_s: shared scratch [TM * k].  NV: logits per
+// lane (E <= 32 NV).
+template <int NV>
+__device__ __forceinline__ void select_and_count(const RouterArgs& a, const float* L, int lld, int* ids_s,
+                                                 int t0) {
+  const int tid = threadIdx.x;
+  // top-k: warp w handles tokens w*tpw .. w*tpw+tpw-1
+  const int warp = tid >> 5, lane = tid & 31;
+  const int nvalid = min(TM, a.T - t0);
+  const int k = a.k;
+  const int per_lane = (a.E + 31) >> 5;  // <= 16
+  const int tpw = TM / (int)(blockDim.x >> 5);  // tokens per warp
+  for (int q = 0; q < tpw; ++q) {
+    const int tok = warp * tpw + q;
+    if (tok >= nvalid) break;
+    float v[NV];
+#pragma unroll
+    for (int i = 0; i < NV; ++i) {
+      const int e = lane + 32 * i;
+      v[i] = (i < per_lane && e < a.E) ? L[tok * lld + e] : -INFINITY;
+    }
+    uint32_t removed = 0;
+    float my_v = -INFINITY;
+    int my_i = 0;
+    float next_v = -INFINITY;  // logit of rank k (when k < E)
+    const int rounds = min(k + 1, a.E);
+    for (int r = 0; r < rounds; ++r) {
+      float bv = -INFINITY;
+      int bi = 0x7fffffff;
+#pragma unroll
+      for (int i = 0; i < NV; ++i) {
+        const int e = lane + 32 * i;
+        if (i < per_lane && e < a.E && !((removed >> i) & 1u)) {
+          if (v[i] > bv || (v[i] == bv && e < bi)) { bv = v[i]; bi = e; }
+        }
+      }
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) {
+        const float ov = __shfl_xor_sync(0xffffffffu, bv, off);
+        const int oi = __shfl_xor_sync(0xffffffffu, bi, off);
+        if (ov > bv || (ov == bv && oi < bi)) { bv = ov; bi = oi; }
+      }
+      if ((bi & 31) == lane) removed |= 1u << (bi >> 5);
+      if (r == lane) { my_v = bv; my_i = bi; }
+      if (r == k) next_v = bv;
+    }
+    const float l0 = __shfl_sync(0xffffffffu, my_v, 0);
+    float ex = (lane < k) ? expf(my_v - l0) : 0.f;
+    float sum = ex;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
+    const size_t t = (size_t)t0 + tok;
+    if (lane < k) {
+      a.ids[t * k + lane] = my_i;
+      a.weights[t * k + lane] = ex / sum;
+      ids_s[tok * k + lane] = my_i;
+    }
+    if (a.gap != nullptr) {
+      const float lk1 = __shfl_sync(0xffffffffu, my_v, k - 1);
+      if (lane == 0) a.gap[t] = (k < a.E) ? (lk1 - next_v) : INFINITY;
+    }
+    if (a.wsg != nullptr) {
+      const __nv_bfloat16* xr = a.x + t * a.H;
+      float s = 0.f;
+      for (int h = lane * 8; h < a.H; h += 256) {
+        const uint4 xv = *reinterpret_cast<const uint4*>(xr + h);
+        const float4 w0 = *reinterpret_cast<const float4*>(a.wsg + h);
+        const float4 w1 = *reinterpret_cast<const float4*>(a.wsg + h + 4);
+        s = fmaf(bf16_lo(xv.x), w0.x, s);
+        s = fmaf(bf16_hi(xv.x), w0.y, s);
+        s = fmaf(bf16_lo(xv.y), w0.z, s);
+        s = fmaf(bf16_hi(xv.y), w0.w, s);
+        s = fmaf(bf16_lo(xv.z), w1.x, s);
+        s = fmaf(bf16_hi(xv.z), w1.y, s);
+        s = fmaf(bf16_lo(xv.w), w1.z, s);
+        s = fmaf(bf16_hi(xv.w), w1.w, s);
+      }
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+      if (lane == 0) a.sg[t] = 1.0f / (1.0f + expf(-s));
+    }
+  }
+  __syncthreads();
+
+  // per-block histogram of the routed ids (deterministic, no atomics)
+  const int nids = nvalid * k;
+  for (int e = tid; e < a.E; e += NTH) {
+    int c = 0;
+    for (int i = 0; i < nids; ++i) c += (ids_s[i] == e);
+    a.bcount[(size_t)blockIdx.x * a.E + e] = c;
+  }
+}
+
 template <int EP>
 __global__ void __launch_bounds__(NTH, 1) router_kernel(const RouterArgs a) {
   using C = RCfg<EP>;
@@ -131,91 +226,67 @@ __global__ void __launch_bounds__(NTH, 1) router_kernel(const RouterArgs a) {
     for (int j = 0; j < J; ++j) L[(tg * 8 + i) * LLD + el + 64 * j] = acc[i][j];
   __syncthreads();
 
-  // top-k: warp w handles tokens w*4 .. w*4+3
-  const int warp = tid >> 5, lane = tid & 31;
-  const int nvalid = min(TM, a.T - t0);
-  const int k = a.k;
-  const int per_lane = (a.E + 31) >> 5;  // <= 16
-  for (int q = 0; q < TM / 8; ++q) {
-    const int tok = warp * (TM / 8) + q;
-    if (tok >= nvalid) break;
-    float v[16];
-#pragma unroll
-    for (int i = 0; i < 16; ++i) {
-      const int e = lane + 32 * i;
-      v[i] = (i < per_lane && e < a.E) ? L[tok * LLD + e] : -INFINITY;
-    }
-    uint32_t removed = 0;
-    float my_v = -INFINITY;
-    int my_i = 0;
-    float next_v = -INFINITY;  // logit of rank k (when k < E)
-    const int rounds = min(k + 1, a.E);
-    for (int r = 0; r < rounds; ++r) {
-      float bv = -INFINITY;
-      int bi = 0x7fffffff;
-#pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        const int e = lane + 32 * i;
-        if (i < per_lane && e < a.E && !((removed >> i) & 1u)) {
-          if (v[i] > bv || (v[i] == bv && e < bi)) { bv = v[i]; bi = e; }
-        }
-      }
-#pragma unroll
-      for (int off = 16; off > 0; off >>= 1) {
-        const float ov = __shfl_xor_sync(0xffffffffu, bv, off);
-        const int oi = __shfl_xor_sync(0xffffffffu, bi, off);
-        if (ov > bv || (ov == bv && oi < bi)) { bv = ov; bi = oi; }
-      }
-      if ((bi & 31) == lane) removed |= 1u << (bi >> 5);
-      if (r == lane) { my_v = bv; my_i = bi; }
-      if (r == k) next_v = bv;
-    }
-    const float l0 = __shfl_sync(0xffffffffu, my_v, 0);
-    float ex = (lane < k) ? expf(my_v - l0) : 0.f;
-    float sum = ex;
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
-    const size_t t = (size_t)t0 + tok;
-    if (lane < k) {
-      a.ids[t * k + lane] = my_i;
-      a.weights[t * k + lane] = ex / sum;
-      ids_s[tok * k + lane] = my_i;
-    }
-    if (a.gap != nullptr) {
-      const float lk1 = __shfl_sync(0xffffffffu, my_v, k - 1);
-      if (lane == 0) a.gap[t] = (k < a.E) ? (lk1 - next_v) : INFINITY;
-    }
-    if (a.wsg != nullptr) {
-      const __nv_bfloat16* xr = a.x + t * a.H;
-      float s = 0.f;
-      for (int h = lane * 8; h < a.H; h += 256) {
-        const uint4 xv = *reinterpret_cast<const uint4*>(xr + h);
-        const float4 w0 = *reinterpret_cast<const float4*>(a.wsg + h);
-        const float4 w1 = *reinterpret_cast<const float4*>(a.wsg + h + 4);
-        s = fmaf(bf16_lo(xv.x), w0.x, s);
-        s = fmaf(bf16_hi(xv.x), w0.y, s);
-        s = fmaf(bf16_lo(xv.y), w0.z, s);
-        s = fmaf(bf16_hi(xv.y), w0.w, s);
-        s = fmaf(bf16_lo(xv.z), w1.x, s);
-        s = fmaf(bf16_hi(xv.z), w1.y, s);
-        s = fmaf(bf16_lo(xv.w), w1.z, s);
-        s = fmaf(bf16_hi(xv.w), w1.w, s);
-      }
-#pragma unroll
-      for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
-      if (lane == 0) a.sg[t] = 1.0f / (1.0f + expf(-s));
-    }
-  }
-  __syncthreads();
-
-  // per-block histogram of the routed ids (deterministic, no atomics)
-  const int nids = nvalid * k;
-  for (int e = tid; e < a.E; e += NTH) {
-    int c = 0;
-    for (int i = 0; i < nids; ++i) c += (ids_s[i] == e);
-    a.bcount[(size_t)blockIdx.x * a.E + e] = c;
-  }
+  select_and_count<16>(a, L, LLD, ids_s, t0);
 }
+
+// Layers of at most 32 experts: one lane per expert and one warp per token
+// (32 warps, the block's 32 tokens at once).  Lane e of warp t computes the
+// logit of token t and expert e as one fp32 fmaf chain over h in ascending
+// order (the tiled kernel's value), from a chunk of Wr staged transposed in
+// shared memory (rows padded to 33 words: conflict-free stores and reads)
+// and the token's x row (read as broadcasts).  The tiled kernel would spend
+// a block of 256 threads and 64 expert columns on them.
+constexpr int kSmallThreads = 1024;
+constexpr int kSmallHC = 256;                  // h per staged chunk
+constexpr int kSmallWLD = 33;                  // Wr^T row stride (floats)
+constexpr int kSmallWT = kSmallHC * kSmallWLD * 4;
+constexpr int kSmallXS = TM * kSmallHC * 2;
+constexpr int kSmallLLD = 36;                  // logits row stride (floats)
+constexpr int kSmallSmem = kSmallWT + kSmallXS + TM * kSmallLLD * 4 + TM * kMaxTopK * 4;
+static_assert(kSmallThreads / 32 == TM, "one warp per token");
+
+__global__ void __launch_bounds__(kSmallThreads, 1) router_small_kernel(const RouterArgs a) {
+  // the forward's first kernel (status null: a prediction pass)
+  if (blockIdx.x == 0 && threadIdx.x == 0 && a.status != nullptr)
+    forward_begin(a.status, a.sh, a.sh_total, a.T, a.shared_slot);
+  extern __shared__ __align__(128) uint8_t smem[];
+  float* wt = reinterpret_cast<float*>(smem);
+  __nv_bfloat16* xs = reinterpret_cast<__nv_bfloat16*>(smem + kSmallWT);
+  float* L = reinterpret_cast<float*>(smem + kSmallWT + kSmallXS);
+  int* ids_s = reinterpret_cast<int*>(smem + kSmallWT + kSmallXS + TM * kSmallLLD * 4);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int t0 = blockIdx.x * TM;
+  const int nvalid = min(TM, a.T - t0);
+  float acc = 0.f;
+  for (int h0 = 0; h0 < a.H; h0 += kSmallHC) {
+    const int hc = min(kSmallHC, a.H - h0);
+    for (int i = tid; i < a.E * hc; i += kSmallThreads) {
+      const int e = i / hc, h = i - e * hc;
+      wt[h * kSmallWLD + e] = __ldg(&a.wr[(size_t)e * a.H + h0 + h]);
+    }
+    const int nc = hc / 8;  // 16-byte chunks of a token's row in this chunk
+    for (int i = tid; i < TM * nc; i += kSmallThreads) {
+      const int tok = i / nc, c = i - tok * nc;
+      uint4 v = make_uint4(0u, 0u, 0u, 0u);
+      if (tok < nvalid) v = __ldg(reinterpret_cast<const uint4*>(a.x + (size_t)(t0 + tok) * a.H + h0) + c);
+      reinterpret_cast<uint4*>(xs + tok * kSmallHC)[c] = v;
+    }
+    __syncthreads();
+    if (lane < a.E) {
+      const __nv_bfloat16* xr = xs + warp * kSmallHC;
+      for (int h = 0; h < hc; h += 2) {
+        const uint32_t xv = *reinterpret_cast<const uint32_t*>(xr + h);
+        acc = fmaf(bf16_lo(xv), wt[h * kSmallWLD + lane], acc);
+        acc = fmaf(bf16_hi(xv), wt[(h + 1) * kSmallWLD + lane], acc);
+      }
+    }
+    __syncthreads();
+  }
+  L[warp * kSmallLLD + lane] = acc;
+  __syncthreads();
+  select_and_count<1>(a, L, kSmallLLD, ids_s, t0);
+}
+
 }  // namespace
 
 template <int EP>
@@ -231,7 +302,20 @@ static cudaError_t launch_ep(const RouterArgs& a, cudaStream_t s) {
   return cudaGetLastError();
 }
 
+static cudaError_t launch_small(const RouterArgs& a, cudaStream_t s) {
+  static std::atomic<unsigned long long> attr_done{0};
+  {
+    cudaError_t e = smem_attr_once(router_small_kernel, kSmallSmem, attr_done);
+    if (e != cudaSuccess) return e;
+  }
+  const int nb = (a.T + TM - 1) / TM;
+  if (nb == 0) return cudaSuccess;
+  router_small_kernel<<<nb, kSmallThreads, kSmallSmem, s>>>(a);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_router(const RouterArgs& a, cudaStream_t s) {
+  if (a.E <= 32) return launch_small(a, s);
   return a.E <= 64 ? launch_ep<64>(a, s) : launch_ep<512>(a, s);
 }
 

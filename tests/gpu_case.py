@@ -30,7 +30,7 @@ class Case:
     """Inputs of one workload (all layers), host windows filled, plan created."""
 
     def __init__(self, cfg: synth.MoEConfig, n_slots=None, wave_capacity=0, layers=None,
-                 wait_timeout_s=0.0):
+                 wait_timeout_s=0.0, early_staging=False):
         self.cfg = cfg
         L = cfg.n_layers if layers is None else layers
         self.L = L
@@ -53,7 +53,8 @@ class Case:
                              n_slots=cfg.n_slots if n_slots is None else n_slots,
                              host_windows=self.windows, has_shared=cfg.has_shared,
                              shared_w=shared_w, shared_gate_w=gate_w, wdtype=cfg.wdtype,
-                             wave_capacity=wave_capacity, wait_timeout_s=wait_timeout_s)
+                             wave_capacity=wave_capacity, wait_timeout_s=wait_timeout_s,
+                             early_staging=early_staging)
 
     def extent(self, layer, e):
         eb = self.cfg.extent_bytes

@@ -1,6 +1,6 @@
 """The 32K-token single-layer prefills at their full size, in the launch
 configuration the bench times (msi_moe_forward_streamed, default flags, a
-side stage stream): 32,768 tokens, 512 experts, top-10, a 64-slot pool in
+side stage stream, an early-staging buffer of one wave): 32,768 tokens, 512 experts, top-10, a 64-slot pool in
 LRU waves of 32, bf16 and 4-bit experts.  Every route event is compared with
 the oracle router, the slot trace with the oracle's simulator (bit-exact),
 and the outputs on sampled tokens (the first, the last and random ones)
@@ -27,7 +27,7 @@ def _needed(ids):
 def test_prefill32k_full_size(name, samples):
     cfg = synth.config(name)
     assert cfg.tokens == 32768 and cfg.n_experts == 512 and cfg.n_slots == 64
-    case = Case(cfg)
+    case = Case(cfg, early_staging=True)
     sim = oracle.LRUWaveSim(cfg.n_slots)
     stage = torch.cuda.Stream()
     rng = np.random.default_rng(7)
