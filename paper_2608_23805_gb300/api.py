@@ -78,6 +78,7 @@ class Plan:
         N.check(lib.msi_plan_create(ctypes.byref(d), ctypes.byref(h)), "msi_plan_create")
         self.h = h
         self._ws = {}
+        self._ws_bytes = {}
         self.bounce = None
         if early_staging:
             C = wave_capacity if wave_capacity > 0 else n_slots // 2
@@ -133,11 +134,14 @@ class Plan:
 
     # -- forward -------------------------------------------------------------
     def workspace(self, T: int) -> torch.Tensor:
-        n = ctypes.c_size_t()
-        N.check(N.lib().msi_workspace_size(self.h, T, ctypes.byref(n)), "msi_workspace_size")
+        need = self._ws_bytes.get(T)
+        if need is None:  # a pure function of the plan's shape and T
+            n = ctypes.c_size_t()
+            N.check(N.lib().msi_workspace_size(self.h, T, ctypes.byref(n)), "msi_workspace_size")
+            need = self._ws_bytes[T] = n.value
         ws = self._ws.get("buf")
-        if ws is None or ws.numel() < n.value:
-            ws = torch.empty(max(n.value, 256), dtype=torch.uint8, device="cuda")
+        if ws is None or ws.numel() < need:
+            ws = torch.empty(max(need, 256), dtype=torch.uint8, device="cuda")
             self._ws["buf"] = ws
         return ws
 
