@@ -70,13 +70,13 @@ L2_BYTES = 129 * 1024 * 1024
 # only while the GEMM source still hashes to the value the capture was taken at.
 TRAFFIC = {
     # one fused wave launch (gate-up + down of 32 experts, ~20,480 routed rows)
-    ("prefill32k_lru64", "gateup+down"): {"bytes_per_launch": 293416192 + 58992128, "src_hash": "61d39743f2721403",
+    ("prefill32k_lru64", "gateup+down"): {"bytes_per_launch": 293416192 + 58992128, "src_hash": "aabc8aa52af9bf27",
                                           "profile": "profiles/gemm_fused_wave_prefill32k_lru64.md"},
     # the fused launch of a 4K resident call
-    ("qwen3next_4k", "gateup+down"): {"bytes_per_launch": 3388257536 + 196642816, "src_hash": "61d39743f2721403",
+    ("qwen3next_4k", "gateup+down"): {"bytes_per_launch": 3388257536 + 196642816, "src_hash": "aabc8aa52af9bf27",
                                       "profile": "profiles/gemm_fused_qwen3next_4k.md"},
     # one fused 4-bit wave launch
-    ("prefill32k_q4_lru64", "gateup+down"): {"bytes_per_launch": 144022272 + 54480128, "src_hash": "61d39743f2721403",
+    ("prefill32k_q4_lru64", "gateup+down"): {"bytes_per_launch": 144022272 + 54480128, "src_hash": "aabc8aa52af9bf27",
                                              "profile": "profiles/gemm_fused_wave_q4_prefill32k_q4_lru64.md"},
 }
 

@@ -234,20 +234,21 @@ __device__ __forceinline__ uint4 ld_shared_v4(uint32_t addr) {
 // tiles first and then its down tiles, each in increasing index order.
 struct FusedSched {
   int U, D, P, c, n_hi, n_lo, DA;
-  __device__ __forceinline__ FusedSched(int U_, int D_, int P_, int c_, int w) : U(U_), D(D_), P(P_), c(c_) {
+  __host__ __device__ __forceinline__ FusedSched(int U_, int D_, int P_, int c_, int w)
+      : U(U_), D(D_), P(P_), c(c_) {
     n_hi = U % P;
     n_lo = P - n_hi;
-    DA = n_hi > 0 ? min(D, w * n_lo) : 0;
+    DA = n_hi > 0 ? (D < w * n_lo ? D : w * n_lo) : 0;
   }
   // the worker's first down tile, or -1
-  __device__ __forceinline__ int down_first() const {
+  __host__ __device__ __forceinline__ int down_first() const {
     if (c >= n_hi && c - n_hi < DA) return U + (c - n_hi);
     const int i = DA + c;
     return i < D ? U + i : -1;
   }
-  __device__ __forceinline__ int first() const { return c < U ? c : down_first(); }
+  __host__ __device__ __forceinline__ int first() const { return c < U ? c : down_first(); }
   // the worker's tile after t, or -1
-  __device__ __forceinline__ int next(int t) const {
+  __host__ __device__ __forceinline__ int next(int t) const {
     if (t < U) return t + P < U ? t + P : down_first();
     const int i = t - U;
     if (i < DA) {
