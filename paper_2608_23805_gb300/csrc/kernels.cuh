@@ -155,6 +155,21 @@ cudaError_t launch_upload(const TableParams& p, int* table, unsigned long long* 
                           int* status, Group* shared_group, int* shared_total, cudaStream_t s);
 cudaError_t launch_setup_wave(const SetupArgs& a, const WaveParams& w, cudaStream_t s);
 cudaError_t launch_publish(const PublishParams& p, GenWord* genwords, cudaStream_t s);
+// One launch for a wave whose extents all come from the early-staging buffer:
+// each slot's published word is invalidated before any byte of its extent is
+// copied (device to device), and the last block to finish publishes the
+// wave's words.  ticket counts finished blocks across launches; target is its
+// value once this launch's blocks have finished.
+struct StageCopyArgs {
+  PublishParams pub;
+  const char* src[kMaxWave];     // extents in the early-staging buffer
+  char* pool;                    // slot pool base
+  unsigned long long bytes;      // extent bytes (a multiple of 16)
+  unsigned long long* ticket;
+  unsigned long long target;
+  int parts;                     // blocks per extent
+};
+cudaError_t launch_stage_copy(const StageCopyArgs& a, GenWord* genwords, cudaStream_t s);
 cudaError_t launch_combine(const CombineArgs& a, cudaStream_t s);
 cudaError_t launch_zero_counts(int* counts, int E, cudaStream_t s);
 

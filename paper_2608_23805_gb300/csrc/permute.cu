@@ -340,6 +340,40 @@ __global__ void publish_kernel(const PublishParams p, GenWord* gw) {
   }
 }
 
+// Block b copies part b % parts of extent b / parts.  Its first thread
+// invalidates the extent's slot word and makes that visible before the
+// block's copies; every block makes its copies visible before it takes a
+// ticket, and the block that takes the launch's last ticket publishes.
+__global__ void stage_copy_kernel(const StageCopyArgs a, GenWord* gw) {
+  const int i = blockIdx.x / a.parts, part = blockIdx.x % a.parts;
+  const int slot = a.pub.slot[i];
+  if (threadIdx.x == 0) {
+    GenWord z;
+    z.gen = 0;
+    z.obj = 0;
+    gw[slot] = z;
+    __threadfence();
+  }
+  __syncthreads();
+  const uint4* src = reinterpret_cast<const uint4*>(a.src[i]);
+  uint4* dst = reinterpret_cast<uint4*>(a.pool + (size_t)slot * a.bytes);
+  const unsigned long long n16 = a.bytes / 16;
+  const unsigned long long per = (n16 + a.parts - 1) / a.parts;
+  const unsigned long long b0 = per * part, b1 = min(n16, b0 + per);
+  for (unsigned long long k = b0 + threadIdx.x; k < b1; k += blockDim.x) dst[k] = __ldg(src + k);
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0 && atomicAdd(a.ticket, 1ull) + 1ull == a.target) {
+    __threadfence();
+    for (int j = 0; j < a.pub.n; ++j) {
+      GenWord g;
+      g.gen = a.pub.gen[j];
+      g.obj = a.pub.obj[j];
+      gw[a.pub.slot[j]] = g;
+    }
+  }
+}
+
 // ---- combine: out[t] = sum_j w[t,j] yp[inv[t*k+j]] (+ sg[t] ys[t]) (+ x[t]) ----
 __device__ __forceinline__ void fma8(float (&acc)[8], float w, const uint4& y) {
   acc[0] = fmaf(w, bf16_lo(y.x), acc[0]);
@@ -446,6 +480,12 @@ cudaError_t launch_setup_wave(const SetupArgs& a, const WaveParams& w, cudaStrea
 cudaError_t launch_publish(const PublishParams& p, GenWord* genwords, cudaStream_t s) {
   if (p.n == 0) return cudaSuccess;
   publish_kernel<<<1, kMaxWave, 0, s>>>(p, genwords);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_stage_copy(const StageCopyArgs& a, GenWord* genwords, cudaStream_t s) {
+  if (a.pub.n == 0) return cudaSuccess;
+  stage_copy_kernel<<<a.pub.n * a.parts, 256, 0, s>>>(a, genwords);
   return cudaGetLastError();
 }
 

@@ -230,6 +230,10 @@ struct msi_plan {
   std::vector<int> where;  // [L * E]: slot holding (l, e) or -1
   std::vector<std::atomic<int>> holds;
   GenWord* d_gen = nullptr;
+  // blocks finished by the one-launch staging of early-staged waves (device
+  // counter, never reset) and the host's running total of blocks launched
+  unsigned long long* d_ticket = nullptr;
+  unsigned long long ticket_total = 0;
   int* h_status = nullptr;
   int* h_counts = nullptr;
   EventPool pool;
@@ -472,6 +476,9 @@ msi_status write_words(msi_plan* p, const PublishParams& w, cudaStream_t stage) 
   return MSI_OK;
 }
 
+// Largest wave (bytes) staged by one launch from the early-staging buffer
+constexpr uint64_t kStageCopyMaxBytes = 8ull << 20;
+
 // Enqueue the copies of `misses` on `stage` and publish them with one event.
 msi_status stage_enqueue(msi_plan* p, int layer, const std::vector<WaveEntry>& misses,
                          cudaStream_t stage) {
@@ -500,9 +507,29 @@ msi_status stage_enqueue(msi_plan* p, int layer, const std::vector<WaveEntry>& m
       p->faults.erase(f);
     }
   }
+  const uint64_t eb = p->d.extent_bytes;
+  // A small wave whose extents were all copied early (decode-sized waves):
+  // invalidation, device-to-device copies and publication in one launch.  A
+  // large wave keeps the copy engine: a copy kernel would contend for the
+  // SMs the waves' GEMMs hold.
+  bool one_launch = p->src == nullptr && p->spec_layer == layer &&
+                    (uint64_t)misses.size() * eb <= kStageCopyMaxBytes && eb % 16 == 0;
+  for (size_t i = 0; i < misses.size() && one_launch; ++i) one_launch = p->spec_idx[misses[i].expert] >= 0;
+  if (one_launch) {
+    StageCopyArgs sa{};
+    sa.pub = pub;
+    for (size_t i = 0; i < misses.size(); ++i)
+      sa.src[i] = p->bounce + (size_t)p->spec_idx[misses[i].expert] * eb;
+    sa.pool = static_cast<char*>(p->d.slot_pool);
+    sa.bytes = eb;
+    sa.parts = (int)std::max<uint64_t>(1, std::min<uint64_t>(64, eb / 32768));
+    sa.ticket = p->d_ticket;
+    sa.target = p->ticket_total + (unsigned long long)misses.size() * (unsigned long long)sa.parts;
+    LAUNCH(p, MSI_K_PUBLISH, stage, launch_stage_copy(sa, p->d_gen, stage));
+    p->ticket_total = sa.target;
+  } else {
   st = write_words(p, inv, stage);
   if (st != MSI_OK) return st;
-  const uint64_t eb = p->d.extent_bytes;
   auto src_of = [&](const WaveEntry& m) {
     return static_cast<const char*>(p->d.host_windows) +
            p->off[(size_t)layer * p->d.n_experts + m.expert];
@@ -594,6 +621,7 @@ msi_status stage_enqueue(msi_plan* p, int layer, const std::vector<WaveEntry>& m
   }
   st = write_words(p, pub, stage);
   if (st != MSI_OK) return st;
+  }
   int ev;
   st = p->pool.acquire(&ev);
   if (st != MSI_OK) return st;
@@ -1195,6 +1223,7 @@ msi_status msi_plan_create(const msi_plan_desc* desc, msi_plan** out) {
   p->pinned_obj.assign(nobj, 0);
   auto fail = [&](msi_status s) {
     if (p->d_gen) cudaFree(p->d_gen);
+    if (p->d_ticket) cudaFree(p->d_ticket);
     if (p->h_status) cudaFreeHost(p->h_status);
     if (p->h_counts) cudaFreeHost(p->h_counts);
     if (p->side) cudaStreamDestroy(p->side);
@@ -1209,6 +1238,8 @@ msi_status msi_plan_create(const msi_plan_desc* desc, msi_plan** out) {
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&p->sms, cudaDevAttrMultiProcessorCount, dev);
   if (e == cudaSuccess) e = cudaMalloc(&p->d_gen, sizeof(GenWord) * d.n_slots);
   if (e == cudaSuccess) e = cudaMemset(p->d_gen, 0, sizeof(GenWord) * d.n_slots);
+  if (e == cudaSuccess) e = cudaMalloc(&p->d_ticket, sizeof(unsigned long long));
+  if (e == cudaSuccess) e = cudaMemset(p->d_ticket, 0, sizeof(unsigned long long));
   if (e == cudaSuccess) e = cudaMallocHost(&p->h_status, sizeof(int));
   if (e == cudaSuccess) e = cudaMallocHost(&p->h_counts, sizeof(int) * d.n_experts);
   if (e == cudaSuccess && d.has_shared) e = cudaStreamCreateWithFlags(&p->side, cudaStreamNonBlocking);
@@ -1261,6 +1292,7 @@ msi_status msi_plan_destroy(msi_plan* p) {
     p->timer.destroy();
     for (auto ev : p->pool.ev) cudaEventDestroy(ev);
     cudaFree(p->d_gen);
+    cudaFree(p->d_ticket);
     cudaFreeHost(p->h_status);
     cudaFreeHost(p->h_counts);
     if (p->side) cudaStreamDestroy(p->side);

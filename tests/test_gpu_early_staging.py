@@ -91,3 +91,29 @@ def test_early_staging_with_unneeded_experts():
         assert np.array_equal(oa, ob)
     a.close()
     b.close()
+
+
+def test_early_staging_decode_stack_equals_plain_staging():
+    """The decode stack at batch 64 (48 layers of the tiny shape, one 64-slot
+    pool; T k = 8 E, so every layer call copies its first misses early and
+    stages a wave drawn wholly from the early-staging buffer in one launch:
+    invalidation, device copies, publication): route ids, outputs and slot
+    traces equal those of a plan without the buffer, over four steps."""
+    cfg = synth.config("decode48", tokens=64)
+    b = Case(cfg)
+    a = _Twin(b)
+    stage_a, stage_b = torch.cuda.Stream(), torch.cuda.Stream()
+    for step in range(4):
+        xa = xb = bf16_tensor(synth.hidden(cfg, 0, 2000 + step, tokens=64))
+        for l in range(cfg.n_layers):
+            oa, eva = a.plan.forward_streamed(l, xa, a.router[l], residual=True, stage_stream=stage_a)
+            ob, evb = b.plan.forward_streamed(l, xb, b.router[l], residual=True, stage_stream=stage_b)
+            torch.cuda.synchronize()
+            assert a.plan.status() == N.MSI_OK and b.plan.status() == N.MSI_OK
+            assert torch.equal(eva.ids, evb.ids)
+            assert torch.equal(oa.view(torch.int16), ob.view(torch.int16))
+            xa, xb = oa, ob
+    assert a.plan.trace() == b.plan.trace()
+    assert a.plan.counters()["stages"] == b.plan.counters()["stages"]
+    a.close()
+    b.close()
