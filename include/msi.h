@@ -363,7 +363,9 @@ msi_status msi_fault_inject(msi_plan* plan, int kind, int layer, int expert);
  * ascending order (the order the LRU-wave plan stages misses) into the
  * buffer (in a host-buffer call, after its rows have crossed); its waves
  * then copy those extents device to device into their slots instead of from
- * the host windows.  Victims, generations, publication and the slot trace
+ * the host windows (a wave of at most 8 MB drawn wholly from the buffer in
+ * one launch that also invalidates and publishes its slots' words).
+ * Victims, generations, publication and the slot trace
  * are those of a call without the buffer; outputs are bit-identical.  Not
  * used with a source attached.  The buffer must stay allocated until it is
  * detached or the plan destroyed. */
