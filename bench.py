@@ -259,6 +259,11 @@ class Workload:
 
     def step(self, x=None):
         x = self.x if x is None else x
+        if self.L > 1 and not self.predict:
+            # the whole stack in one call (msi_moe_forward_streamed_stack)
+            self.plan.forward_streamed_stack(0, x, self.routers, self.outs[0], self.outs[1], self.evs,
+                                             residual=True, stream=self.cs, stage_stream=self.ss)
+            return
         if self.L > 1:
             for l in range(self.L):
                 nxt = self.routers[l + 1] if self.predict and l + 1 < self.L else None

@@ -259,6 +259,24 @@ msi_status msi_moe_forward_streamed(msi_plan* plan, int layer, const void* hidde
                                     void* workspace, size_t workspace_bytes, unsigned flags,
                                     msi_stream compute, msi_stream stage);
 
+/* msi_moe_forward_streamed over a stack of layers layer0 .. layer0 + n - 1
+ * in one call (a decode step): layer i (from 0) reads the previous layer's
+ * output (`hidden` for i = 0) and writes out_a when i is even, out_b when i
+ * is odd, so the stack's output is in out_a when n is odd and in out_b when
+ * it is even; both [T, H] bf16, device, 16-byte aligned, distinct from
+ * `hidden` and from each other.  router_w: n device pointers (host array),
+ * the layers' routers; evs: n route events (host array of structs with
+ * device buffers).  flags apply to every layer (a stack normally passes
+ * MSI_FWD_RESIDUAL).  Each layer is exactly one msi_moe_forward_streamed
+ * call, made by the library without returning to the caller in between.
+ * Stops at the first layer that fails and returns its status; *done (may be
+ * NULL) receives the number of layers completed. */
+msi_status msi_moe_forward_streamed_stack(msi_plan* plan, int layer0, int n, const void* hidden, int T,
+                                          const float* const* router_w, void* out_a, void* out_b,
+                                          const msi_route_event* evs, void* workspace,
+                                          size_t workspace_bytes, unsigned flags, msi_stream compute,
+                                          msi_stream stage, int* done);
+
 /* msi_moe_forward_streamed plus next-layer prediction and a two-bank prefetch
  * (the paper's protected LRU with two-bank next-layer prefetch, Sec.
  * "Evaluation", "Cache and storage state"; prediction and pinning share the

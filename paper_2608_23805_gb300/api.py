@@ -192,6 +192,30 @@ class Plan:
             return out, ev
         return rc, out, ev
 
+    def forward_streamed_stack(self, layer0, x, routers, out_a, out_b, evs, residual=False,
+                               stream=None, stage_stream=None, check=True):
+        """Streamed forwards of layers layer0 .. layer0 + len(routers) - 1 in
+        one call (msi_moe_forward_streamed_stack): layer i reads the previous
+        output (x for i = 0) and writes out_a for even i, out_b for odd i.
+        evs: one RouteEvent per layer.  Returns the tensor holding the last
+        layer's output."""
+        n = len(routers)
+        assert len(evs) == n
+        T = x.shape[0]
+        ws = self.workspace(T)
+        rw = (ctypes.c_void_p * max(n, 1))(*[r.data_ptr() for r in routers])
+        ea = (N.msi_route_event * max(n, 1))(*[e.c for e in evs])
+        done = ctypes.c_int()
+        rc = N.lib().msi_moe_forward_streamed_stack(
+            self.h, layer0, n, _ptr(x), T, ctypes.cast(rw, ctypes.c_void_p), _ptr(out_a), _ptr(out_b),
+            ctypes.cast(ea, ctypes.c_void_p), _ptr(ws), ws.numel(), _flags(residual, False),
+            _stream(stream), _stream(stage_stream), ctypes.byref(done))
+        last = out_a if n % 2 == 1 else out_b
+        if check:
+            N.check(rc, "msi_moe_forward_streamed_stack")
+            return last
+        return rc, done.value, last
+
     def workspace_host(self, T: int) -> torch.Tensor:
         n = ctypes.c_size_t()
         N.check(N.lib().msi_workspace_size_host(self.h, T, ctypes.byref(n)), "msi_workspace_size_host")

@@ -1889,6 +1889,28 @@ msi_status msi_moe_forward_streamed(msi_plan* p, int layer, const void* x, int T
                           stage);
 }
 
+msi_status msi_moe_forward_streamed_stack(msi_plan* p, int layer0, int n, const void* x, int T,
+                                          const float* const* rw, void* out_a, void* out_b,
+                                          const msi_route_event* evs, void* ws, size_t ws_bytes,
+                                          unsigned flags, msi_stream compute, msi_stream stage, int* done) {
+  if (done != nullptr) *done = 0;
+  if (p == nullptr || n < 0 || (n > 0 && (rw == nullptr || evs == nullptr)) || out_a == nullptr ||
+      out_b == nullptr || out_a == out_b || out_a == x || out_b == x)
+    return MSI_ERR_INVALID_ARG;
+  if (layer0 < 0 || (long long)layer0 + n > p->d.n_layers) return MSI_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> g(p->mu);
+  const void* in = x;
+  for (int i = 0; i < n; ++i) {
+    void* out = (i & 1) ? out_b : out_a;
+    const msi_status st = forward_streamed(p, layer0 + i, in, T, rw[i], out, &evs[i], nullptr, nullptr, ws,
+                                           ws_bytes, flags, compute, stage);
+    if (st != MSI_OK) return st;
+    if (done != nullptr) *done = i + 1;
+    in = out;
+  }
+  return MSI_OK;
+}
+
 msi_status msi_moe_forward_streamed_next(msi_plan* p, int layer, const void* x, int T, const float* rw,
                                          void* out, const msi_route_event* ev, const float* next_rw,
                                          const msi_route_event* next_ev, void* ws, size_t ws_bytes,

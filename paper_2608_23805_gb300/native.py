@@ -116,6 +116,9 @@ _SIGS = {
     "msi_fault_inject": (ctypes.c_int, [_P, ctypes.c_int, ctypes.c_int, ctypes.c_int]),
     "msi_plan_set_wait_cycles": (ctypes.c_int, [_P, ctypes.c_int64]),
     "msi_plan_set_bounce": (ctypes.c_int, [_P, _P, ctypes.c_size_t]),
+    "msi_moe_forward_streamed_stack": (ctypes.c_int, [_P, ctypes.c_int, ctypes.c_int, _P, ctypes.c_int,
+                                                      _P, _P, _P, _P, _P, ctypes.c_size_t, ctypes.c_uint,
+                                                      _P, _P, ctypes.POINTER(ctypes.c_int)]),
     "msi_source_open": (ctypes.c_int, [ctypes.POINTER(msi_source_desc), ctypes.POINTER(_P)]),
     "msi_source_close": (ctypes.c_int, [_P]),
     "msi_source_stats_read": (ctypes.c_int, [_P, ctypes.POINTER(msi_source_stats)]),

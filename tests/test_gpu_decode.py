@@ -60,3 +60,39 @@ def test_decode48_stack(batch, steps):
           "%d stages, %d hits" % (batch, steps * cfg.n_layers, near_total, set_diverged,
                                   c["stages"], c["hits"]))
     case.close()
+
+
+def test_decode_stack_call_equals_layer_calls():
+    """msi_moe_forward_streamed_stack over the 48-layer decode stack (batch 64,
+    with the early-staging buffer the bench uses) equals 48 separate
+    streamed calls on a twin plan: every layer's route ids, the stack's
+    output bit for bit, and the slot traces, over three steps."""
+    cfg = synth.config("decode48", tokens=64)
+    a = Case(cfg, early_staging=True)
+    b = Case(cfg, early_staging=True)
+    E, L = cfg.n_experts, cfg.n_layers
+    from paper_2608_23805_gb300 import api
+    evs = [api.RouteEvent(64, cfg.top_k, E) for _ in range(L)]
+    bufs = [torch.empty((64, cfg.hidden), dtype=torch.bfloat16, device="cuda") for _ in range(2)]
+    stage_a, stage_b = torch.cuda.Stream(), torch.cuda.Stream()
+    for step in range(3):
+        x = bf16_tensor(synth.hidden(cfg, 0, 3000 + step, tokens=64))
+        last = a.plan.forward_streamed_stack(0, x, a.router, bufs[0], bufs[1], evs, residual=True,
+                                             stage_stream=stage_a)
+        xb = x
+        ids_b = []
+        for l in range(L):
+            xb, evb = b.plan.forward_streamed(l, xb, b.router[l], residual=True, stage_stream=stage_b)
+            ids_b.append(evb.ids)
+        torch.cuda.synchronize()
+        assert a.plan.status() == N.MSI_OK and b.plan.status() == N.MSI_OK
+        for l in range(L):
+            assert torch.equal(evs[l].ids, ids_b[l]), l
+        assert torch.equal(last.view(torch.int16), xb.view(torch.int16))
+    assert a.plan.trace() == b.plan.trace()
+    # argument checks: a stack past the last layer is refused, nothing enqueued
+    rc, done, _ = a.plan.forward_streamed_stack(L - 1, x, a.router[:2], bufs[0], bufs[1], evs[:2],
+                                                residual=True, check=False)
+    assert rc == N.MSI_ERR_INVALID_ARG and done == 0
+    a.close()
+    b.close()
