@@ -360,7 +360,20 @@ __global__ void stage_copy_kernel(const StageCopyArgs a, GenWord* gw) {
   const unsigned long long n16 = a.bytes / 16;
   const unsigned long long per = (n16 + a.parts - 1) / a.parts;
   const unsigned long long b0 = per * part, b1 = min(n16, b0 + per);
-  for (unsigned long long k = b0 + threadIdx.x; k < b1; k += blockDim.x) dst[k] = __ldg(src + k);
+  // four 16-byte loads in flight per thread before their stores
+  for (unsigned long long k = b0 + threadIdx.x; k < b1; k += 4ull * blockDim.x) {
+    uint4 v[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const unsigned long long kk = k + (unsigned long long)u * blockDim.x;
+      if (kk < b1) v[u] = __ldg(src + kk);
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const unsigned long long kk = k + (unsigned long long)u * blockDim.x;
+      if (kk < b1) dst[kk] = v[u];
+    }
+  }
   __threadfence();
   __syncthreads();
   if (threadIdx.x == 0 && atomicAdd(a.ticket, 1ull) + 1ull == a.target) {

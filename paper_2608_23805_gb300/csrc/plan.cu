@@ -522,7 +522,7 @@ msi_status stage_enqueue(msi_plan* p, int layer, const std::vector<WaveEntry>& m
       sa.src[i] = p->bounce + (size_t)p->spec_idx[misses[i].expert] * eb;
     sa.pool = static_cast<char*>(p->d.slot_pool);
     sa.bytes = eb;
-    sa.parts = (int)std::max<uint64_t>(1, std::min<uint64_t>(64, eb / 32768));
+    sa.parts = (int)std::max<uint64_t>(1, std::min<uint64_t>(256, eb / 16384));  // 16 KB a block
     sa.ticket = p->d_ticket;
     sa.target = p->ticket_total + (unsigned long long)misses.size() * (unsigned long long)sa.parts;
     LAUNCH(p, MSI_K_PUBLISH, stage, launch_stage_copy(sa, p->d_gen, stage));

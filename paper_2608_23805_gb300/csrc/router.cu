@@ -229,60 +229,70 @@ __global__ void __launch_bounds__(NTH, 1) router_kernel(const RouterArgs a) {
   select_and_count<16>(a, L, LLD, ids_s, t0);
 }
 
-// Layers of at most 32 experts: one lane per expert and one warp per token
-// (32 warps, the block's 32 tokens at once).  Lane e of warp t computes the
-// logit of token t and expert e as one fp32 fmaf chain over h in ascending
-// order (the tiled kernel's value), from a chunk of Wr staged transposed in
-// shared memory (rows padded to 33 words: conflict-free stores and reads)
-// and the token's x row (read as broadcasts).  The tiled kernel would spend
-// a block of 256 threads and 64 expert columns on them.
-constexpr int kSmallThreads = 1024;
+// Layers of at most 32 experts: one lane per expert, EL lanes per token
+// (EL = 16 for at most 16 experts, two tokens a warp; else 32), the block's
+// 32 tokens at once.  A lane computes its (token, expert) logit as one fp32
+// fmaf chain over h in ascending order (the tiled kernel's value), four h at
+// a time from a chunk of Wr staged in shared memory as [h / 4][EL][4] (one
+// 16-byte read per lane) and the token's x row (one 8-byte broadcast).  The
+// tiled kernel would spend a block of 256 threads and 64 expert columns on
+// them.
 constexpr int kSmallHC = 256;                  // h per staged chunk
-constexpr int kSmallWLD = 33;                  // Wr^T row stride (floats)
-constexpr int kSmallWT = kSmallHC * kSmallWLD * 4;
-constexpr int kSmallXS = TM * kSmallHC * 2;
 constexpr int kSmallLLD = 36;                  // logits row stride (floats)
-constexpr int kSmallSmem = kSmallWT + kSmallXS + TM * kSmallLLD * 4 + TM * kMaxTopK * 4;
-static_assert(kSmallThreads / 32 == TM, "one warp per token");
+template <int EL>
+struct SmallCfg {
+  static constexpr int kWarps = TM * EL / 32;
+  static constexpr int kThreads = kWarps * 32;
+  static constexpr int kWT = kSmallHC * EL * 4;    // Wr chunk [HC / 4][EL][4] fp32
+  static constexpr int kXS = TM * kSmallHC * 2;    // x chunk [TM][HC] bf16
+  static constexpr int kSmem = kWT + kXS + TM * kSmallLLD * 4 + TM * kMaxTopK * 4;
+};
 
-__global__ void __launch_bounds__(kSmallThreads, 1) router_small_kernel(const RouterArgs a) {
+template <int EL>
+__global__ void __launch_bounds__(SmallCfg<EL>::kThreads, 1) router_small_kernel(const RouterArgs a) {
+  using C = SmallCfg<EL>;
   // the forward's first kernel (status null: a prediction pass)
   if (blockIdx.x == 0 && threadIdx.x == 0 && a.status != nullptr)
     forward_begin(a.status, a.sh, a.sh_total, a.T, a.shared_slot);
   extern __shared__ __align__(128) uint8_t smem[];
-  float* wt = reinterpret_cast<float*>(smem);
-  __nv_bfloat16* xs = reinterpret_cast<__nv_bfloat16*>(smem + kSmallWT);
-  float* L = reinterpret_cast<float*>(smem + kSmallWT + kSmallXS);
-  int* ids_s = reinterpret_cast<int*>(smem + kSmallWT + kSmallXS + TM * kSmallLLD * 4);
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  float4* wt = reinterpret_cast<float4*>(smem);
+  __nv_bfloat16* xs = reinterpret_cast<__nv_bfloat16*>(smem + C::kWT);
+  float* L = reinterpret_cast<float*>(smem + C::kWT + C::kXS);
+  int* ids_s = reinterpret_cast<int*>(smem + C::kWT + C::kXS + TM * kSmallLLD * 4);
+  const int tid = threadIdx.x;
+  const int tok = tid / EL, e = tid % EL;  // this lane's token (in the block) and expert
   const int t0 = blockIdx.x * TM;
   const int nvalid = min(TM, a.T - t0);
   float acc = 0.f;
   for (int h0 = 0; h0 < a.H; h0 += kSmallHC) {
     const int hc = min(kSmallHC, a.H - h0);
-    for (int i = tid; i < a.E * hc; i += kSmallThreads) {
-      const int e = i / hc, h = i - e * hc;
-      wt[h * kSmallWLD + e] = __ldg(&a.wr[(size_t)e * a.H + h0 + h]);
+    const int nq = hc / 4;  // h quads of this chunk
+    for (int i = tid; i < a.E * nq; i += C::kThreads) {
+      const int ee = i % a.E, q = i / a.E;
+      wt[q * EL + ee] = __ldg(reinterpret_cast<const float4*>(a.wr + (size_t)ee * a.H + h0) + q);
     }
     const int nc = hc / 8;  // 16-byte chunks of a token's row in this chunk
-    for (int i = tid; i < TM * nc; i += kSmallThreads) {
-      const int tok = i / nc, c = i - tok * nc;
+    for (int i = tid; i < TM * nc; i += C::kThreads) {
+      const int tk = i / nc, c = i - tk * nc;
       uint4 v = make_uint4(0u, 0u, 0u, 0u);
-      if (tok < nvalid) v = __ldg(reinterpret_cast<const uint4*>(a.x + (size_t)(t0 + tok) * a.H + h0) + c);
-      reinterpret_cast<uint4*>(xs + tok * kSmallHC)[c] = v;
+      if (tk < nvalid) v = __ldg(reinterpret_cast<const uint4*>(a.x + (size_t)(t0 + tk) * a.H + h0) + c);
+      reinterpret_cast<uint4*>(xs + tk * kSmallHC)[c] = v;
     }
     __syncthreads();
-    if (lane < a.E) {
-      const __nv_bfloat16* xr = xs + warp * kSmallHC;
-      for (int h = 0; h < hc; h += 2) {
-        const uint32_t xv = *reinterpret_cast<const uint32_t*>(xr + h);
-        acc = fmaf(bf16_lo(xv), wt[h * kSmallWLD + lane], acc);
-        acc = fmaf(bf16_hi(xv), wt[(h + 1) * kSmallWLD + lane], acc);
+    if (e < a.E) {
+      const uint2* xr = reinterpret_cast<const uint2*>(xs + tok * kSmallHC);
+      for (int q = 0; q < nq; ++q) {
+        const float4 w = wt[q * EL + e];
+        const uint2 xv = xr[q];
+        acc = fmaf(bf16_lo(xv.x), w.x, acc);
+        acc = fmaf(bf16_hi(xv.x), w.y, acc);
+        acc = fmaf(bf16_lo(xv.y), w.z, acc);
+        acc = fmaf(bf16_hi(xv.y), w.w, acc);
       }
     }
     __syncthreads();
   }
-  L[warp * kSmallLLD + lane] = acc;
+  L[tok * kSmallLLD + e] = acc;
   __syncthreads();
   select_and_count<1>(a, L, kSmallLLD, ids_s, t0);
 }
@@ -302,20 +312,23 @@ static cudaError_t launch_ep(const RouterArgs& a, cudaStream_t s) {
   return cudaGetLastError();
 }
 
+template <int EL>
 static cudaError_t launch_small(const RouterArgs& a, cudaStream_t s) {
+  using C = SmallCfg<EL>;
   static std::atomic<unsigned long long> attr_done{0};
   {
-    cudaError_t e = smem_attr_once(router_small_kernel, kSmallSmem, attr_done);
+    cudaError_t e = smem_attr_once(router_small_kernel<EL>, C::kSmem, attr_done);
     if (e != cudaSuccess) return e;
   }
   const int nb = (a.T + TM - 1) / TM;
   if (nb == 0) return cudaSuccess;
-  router_small_kernel<<<nb, kSmallThreads, kSmallSmem, s>>>(a);
+  router_small_kernel<EL><<<nb, C::kThreads, C::kSmem, s>>>(a);
   return cudaGetLastError();
 }
 
 cudaError_t launch_router(const RouterArgs& a, cudaStream_t s) {
-  if (a.E <= 32) return launch_small(a, s);
+  if (a.E <= 16) return launch_small<16>(a, s);
+  if (a.E <= 32) return launch_small<32>(a, s);
   return a.E <= 64 ? launch_ep<64>(a, s) : launch_ep<512>(a, s);
 }
 
