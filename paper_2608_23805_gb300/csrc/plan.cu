@@ -1109,9 +1109,10 @@ msi_status finish(msi_plan* p, FwdCtx& f) {
   const auto& d = p->d;
   if (f.T > 0) {
     // host-buffer calls combine in row chunks; each chunk's rows go back
-    // while the next chunk is combined
+    // while the next chunk is combined (only the last chunk's copy is left
+    // after the combine: eight chunks from 8,192 rows)
     const int H = d.hidden, k = d.top_k;
-    const int nc = (f.out_host != nullptr && f.T >= 1024) ? 4 : 1;
+    const int nc = f.out_host == nullptr || f.T < 1024 ? 1 : (f.T < 8192 ? 4 : 8);
     for (int ci = 0; ci < nc; ++ci) {
       const long long t0 = (long long)f.T * ci / nc, t1 = (long long)f.T * (ci + 1) / nc;
       CombineArgs c{};

@@ -94,9 +94,10 @@ def test_streamed_host_call_with_early_staging_equals_device_call():
     """The bench's end-to-end configuration: a host-buffer streamed call on
     a plan with an early-staging buffer (copied after the call's rows have
     crossed) and T k >= 8 E, at the Qwen3-Next layer shape with 64 experts
-    and 16 slots (waves of 8, the shared expert after the first miss wave):
-    outputs, ids and slot traces equal those of the device-buffer call."""
-    cfg = synth.config("prefill32k_lru64", tokens=2048, n_experts=64, n_slots=16)
+    and 16 slots (waves of 8, the shared expert after the first miss wave;
+    8,200 rows, so eight uneven combine chunks): outputs, ids and slot
+    traces equal those of the device-buffer call."""
+    cfg = synth.config("prefill32k_lru64", tokens=8200, n_experts=64, n_slots=16)
     a, b = Case(cfg, early_staging=True), Case(cfg, early_staging=True)
     for call in range(2):
         x_bits = synth.hidden(cfg, 0, 150 + call)
@@ -108,7 +109,7 @@ def test_streamed_host_call_with_early_staging_equals_device_call():
         assert torch.equal(ob.view(torch.int16), oa.cpu().view(torch.int16))
         assert torch.equal(ids_host, eva.ids.cpu())
     assert a.plan.trace() == b.plan.trace()
-    toks = np.arange(0, cfg.tokens, 61)
+    toks = np.arange(0, cfg.tokens, 241)
     compare_out(bf16_bits(ob)[toks], a.oracle_layer(x_bits, tokens=toks)["out"])
     a.close()
     b.close()
